@@ -1,0 +1,378 @@
+"""Pins for the CPU oracle: each test checks the oracle against something the
+paper or the mathematics fixes, never against the oracle itself."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2609_05228_gb300 import synth
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _load(name):
+    with open(os.path.join(GOLD, name)) as f:
+        return json.load(f)
+
+
+class _W:
+    """Minimal layer holder for the oracle (fp64 weights)."""
+
+    def __init__(self, spec, router_w, router_b, w_gate, w_up, w_down, gamma, a_gsp, a_rcr):
+        self.spec = spec
+        self.router_w, self.router_b = router_w, router_b
+        self.w_gate, self.w_up, self.w_down, self.gamma = w_gate, w_up, w_down, gamma
+        self.extra = {"a_gsp": a_gsp, "a_rcr": a_rcr}
+
+
+def _tiny_layer(seed=0, d=24, n=6, k=3, m=10, eps=1e-6, m_min=1, bias=True):
+    g = np.random.Generator(np.random.PCG64(seed))
+    spec = synth.LayerSpec(d, n, k, m, dtype="f32", eps=eps, min_active=m_min)
+    rw = g.standard_normal((n, d)) * 0.3
+    rb = g.standard_normal(n) * 0.3 if bias else np.zeros(n)
+    wg = g.standard_normal((n, m, d)) * 0.3
+    wu = g.standard_normal((n, m, d)) * 0.3
+    wd = g.standard_normal((n, d, m)) * 0.3
+    gam = 1 + g.uniform(-0.1, 0.1, d)
+    a_gsp = np.abs(1 + 0.4 * g.standard_normal(n))
+    a_rcr = np.abs(1 + 0.4 * g.standard_normal(n))
+    return _W(spec, rw, rb, wg, wu, wd, gam, a_gsp, a_rcr)
+
+
+# ---------------------------------------------------------------- golden
+
+
+def test_alg4_worked_example_fp64():
+    ex = _load("alg4_worked.json")
+    ids = np.array([ex["ids"]])
+    g = np.array([ex["g"]])
+    for case in ex["cases"]:
+        skip, g_hat, c, _, _ = O.ace_skip(ids, g, np.array(ex["a_gsp"]), np.array(ex["a_rcr"]),
+                                          case["tau"], case["m_min"], ex["eps"])
+        np.testing.assert_allclose(c[0], ex["c"], rtol=1e-15)
+        assert skip[0].astype(int).tolist() == case["skip"], case
+        np.testing.assert_allclose(g_hat[0], case["g_hat"], rtol=1e-15, atol=0)
+
+
+def test_alg4_worked_example_fp32_spec():
+    ex = _load("alg4_worked.json")
+    ids = np.array([ex["ids"]], dtype=np.int32)
+    g = np.array([ex["g"]], dtype=np.float32)
+    for case in ex["cases"]:
+        d = O.decide_fp32(ids, g, ex["a_gsp"], ex["a_rcr"], "threshold", case["tau"],
+                          case["m_min"], ex["eps"])
+        assert d["skip"][0].astype(int).tolist() == case["skip"], case
+        np.testing.assert_allclose(d["g_hat"][0], case["g_hat"], rtol=2e-7, atol=0)
+
+
+@pytest.mark.parametrize("fp32", [False, True])
+def test_tau_ties_worked_example(fp32):
+    ex = _load("tau_ties_worked.json")
+    c = np.array(ex["c"], dtype=np.float32 if fp32 else np.float64)
+    prot = np.array(ex["protected"], dtype=bool)
+    for case in ex["cases"]:
+        fn = O.tau_from_ratio_fp32 if fp32 else O.tau_from_ratio
+        tau, m_q, cnt = fn(c, prot, case["q"])
+        assert m_q == case["m_q"], case
+        cand = c[~prot]
+        assert int(np.sum(cand < tau)) == case["count"] == cnt, case
+        ftype = np.float32 if fp32 else np.float64
+        want = case["tau"]
+        if want == "inf":
+            assert math.isinf(tau)
+        elif want == "0":
+            assert tau == 0
+        elif want.startswith("above"):
+            v = ftype(float(want.split()[1]))
+            assert tau == np.nextafter(v, ftype(np.inf))
+        else:
+            assert tau == ftype(float(want))
+
+
+def test_tables_worked_example():
+    ex = _load("tables_worked.json")
+    gs = ex["gsp"]
+    a = O.gsp_table(np.array(gs["gamma"]), np.array(gs["w_gate"]), np.array(gs["w_up"]),
+                    np.array(gs["w_down"]), eps=0.0)
+    np.testing.assert_allclose(a, gs["expected"], rtol=1e-14)
+    rc = ex["rcr"]
+    a = O.rcr_table(np.array(rc["router_w"]), np.array(rc["gamma"]), np.array(rc["w_gate"]),
+                    np.array(rc["w_up"]), np.array(rc["w_down"]), eps=0.0)
+    np.testing.assert_allclose(a, rc["expected"], rtol=1e-14)
+
+
+# ---------------------------------------------------------------- layer identities
+
+
+def _torch_topk_moe(x, w):
+    """Ordinary top-k MoE from library routines: RMSNorm, nn.Linear router,
+    torch.softmax over all experts, torch.topk, renormalised gates,
+    F.silu SwiGLU experts."""
+    xt = torch.tensor(x, dtype=torch.float64)
+    h = xt * torch.rsqrt(xt.pow(2).mean(-1, keepdim=True) + w.spec.rms_eps)
+    h = h * torch.tensor(w.gamma, dtype=torch.float64)
+    z = torch.nn.functional.linear(h, torch.tensor(w.router_w), torch.tensor(w.router_b))
+    probs = torch.softmax(z, dim=-1)
+    top, idx = torch.topk(probs, w.spec.top_k, dim=-1)
+    top = top / top.sum(-1, keepdim=True)
+    y = torch.zeros_like(h)
+    for t in range(h.shape[0]):
+        for i in range(w.spec.top_k):
+            e = int(idx[t, i])
+            u = torch.nn.functional.linear(h[t], torch.tensor(w.w_gate[e]))
+            v = torch.nn.functional.linear(h[t], torch.tensor(w.w_up[e]))
+            f = torch.nn.functional.linear(torch.nn.functional.silu(u) * v, torch.tensor(w.w_down[e]))
+            y[t] += top[t, i] * f
+    return y.numpy()
+
+
+def test_skip_ratio_zero_is_topk_moe():
+    w = _tiny_layer(1)
+    x = np.random.Generator(np.random.PCG64(7)).standard_normal((40, w.spec.hidden))
+    ref = _torch_topk_moe(x, w)
+    for mode, val in [("threshold", 0.0), ("ratio", 0.0)]:
+        y = O.moe_forward(x, w, mode, val)
+        # tau = 0 keeps every slot; g_hat = g / (1 + eps)
+        np.testing.assert_allclose(y * (1 + w.spec.eps), ref, rtol=1e-11, atol=1e-12)
+
+
+def test_sparse_equals_dense_bruteforce():
+    w = _tiny_layer(2, m_min=2)
+    x = np.random.Generator(np.random.PCG64(8)).standard_normal((30, w.spec.hidden))
+    for tau in [0.05, 0.2, 0.4, 1.0]:
+        y, dec = O.moe_forward(x, w, "threshold", tau, return_decision=True)
+        h = O.rmsnorm(x, w.gamma, w.spec.rms_eps)
+        # evaluate every expert on every token, then weight by the kept g_hat
+        dense = np.stack([
+            np.stack([
+                (lambda u, v: (u / (1 + np.exp(-u)) * v) @ w.w_down[e].T)(h[t] @ w.w_gate[e].T, h[t] @ w.w_up[e].T)
+                for e in range(w.spec.n_experts)]) for t in range(h.shape[0])])
+        wts = np.zeros((h.shape[0], w.spec.n_experts))
+        for t in range(h.shape[0]):
+            for i in range(w.spec.top_k):
+                if not dec["skip"][t, i]:
+                    wts[t, dec["ids"][t, i]] += dec["g_hat"][t, i]
+        ref = np.einsum("te,ted->td", wts, dense)
+        np.testing.assert_allclose(y, ref, rtol=1e-12, atol=1e-13)
+
+
+def test_top1_always_kept():
+    w = _tiny_layer(3)
+    x = np.random.Generator(np.random.PCG64(9)).standard_normal((25, w.spec.hidden))
+    y, dec = O.moe_forward(x, w, "threshold", math.inf, return_decision=True)
+    assert not dec["skip"][:, 0].any()
+    assert dec["skip"][:, 1:].all()
+    h = O.rmsnorm(x, w.gamma, w.spec.rms_eps)
+    z = O.router_logits(h, w.router_w, w.router_b)
+    top1 = np.argmax(z, axis=1)
+    assert (dec["ids"][:, 0] == top1).all()
+    for t in range(h.shape[0]):
+        e = top1[t]
+        g0 = dec["g"][t, 0]
+        f = O.swiglu_expert(h[t:t + 1], w.w_gate[e], w.w_up[e], w.w_down[e])[0]
+        np.testing.assert_allclose(y[t], g0 / (g0 + w.spec.eps) * f, rtol=1e-12)
+
+
+def test_skip_requires_both_views_and_mass_ordering():
+    rng = np.random.Generator(np.random.PCG64(4))
+    T, N, k = 400, 16, 6
+    z = rng.standard_normal((T, N))
+    ids, g = O.topk_gates(z, k)
+    a_gsp = np.abs(1 + 0.5 * rng.standard_normal(N))
+    a_rcr = np.abs(1 + 0.5 * rng.standard_normal(N))
+    for tau in [0.05, 0.1, 0.15, 0.25]:
+        skip, g_hat, c, pg, pr = O.ace_skip(ids, g, a_gsp, a_rcr, tau, 1, 1e-6)
+        assert (pg[skip] < tau).all() and (pr[skip] < tau).all()
+        low_g = pg < tau
+        low_r = pr < tau
+        low_g[:, 0] = low_r[:, 0] = False
+        alpha = (g * skip).sum(1)
+        assert (alpha <= (g * low_g).sum(1) + 1e-15).all()
+        assert (alpha <= (g * low_r).sum(1) + 1e-15).all()
+        # a slot flagged by exactly one view is never skipped
+        assert not (skip & (low_g ^ low_r)).any()
+    # constructed disagreement: expert 5 huge in GSP, tiny in RCR -> never skipped
+    a_gsp2 = np.ones(N)
+    a_rcr2 = np.ones(N)
+    a_gsp2[5], a_rcr2[5] = 50.0, 1e-3
+    skip, *_ = O.ace_skip(ids, g, a_gsp2, a_rcr2, 0.3, 1, 1e-6)
+    assert not skip[ids == 5].any()
+    assert skip.any()
+
+
+def test_perturbation_identity_and_bound():
+    w = _tiny_layer(5, eps=0.0)
+    x = np.random.Generator(np.random.PCG64(10)).standard_normal((20, w.spec.hidden))
+    y_full, _ = O.moe_forward(x, w, "threshold", 0.0, return_decision=True)
+    y_ace, dec = O.moe_forward(x, w, "threshold", 0.3, return_decision=True)
+    h = O.rmsnorm(x, w.gamma, w.spec.rms_eps)
+    checked = 0
+    for t in range(h.shape[0]):
+        f = np.stack([O.swiglu_expert(h[t:t + 1], w.w_gate[e], w.w_up[e], w.w_down[e])[0]
+                      for e in dec["ids"][t]])
+        g = dec["g"][t]
+        S = dec["skip"][t]
+        alpha = g[S].sum()
+        if alpha == 0:
+            np.testing.assert_allclose(y_ace[t], y_full[t], rtol=1e-13)
+            continue
+        mu_s = (g[S, None] * f[S]).sum(0) / alpha
+        mu_i = (g[~S, None] * f[~S]).sum(0) / (1 - alpha)
+        lhs = np.linalg.norm(y_full[t] - y_ace[t])
+        np.testing.assert_allclose(lhs, alpha * np.linalg.norm(mu_s - mu_i), rtol=1e-10)
+        assert lhs <= 2 * alpha * np.linalg.norm(f, axis=1).max() * (1 + 1e-12)
+        checked += 1
+    assert checked > 5
+
+
+def test_swiglu_output_bound():
+    rng = np.random.Generator(np.random.PCG64(11))
+    d, m = 16, 12
+    wg = rng.standard_normal((m, d))
+    wu = rng.standard_normal((m, d))
+    wd = rng.standard_normal((d, m))
+    gam = 1 + rng.uniform(-0.5, 0.5, d)
+    for _ in range(50):
+        xbar = rng.standard_normal(d)
+        f = O.swiglu_expert((xbar * gam)[None], wg, wu, wd)[0]
+        bound = (np.linalg.norm(xbar) ** 2 * np.linalg.norm(gam[:, None] * wg.T, 2)
+                 * np.linalg.norm(gam[:, None] * wu.T, 2) * np.linalg.norm(wd.T, 2))
+        assert np.linalg.norm(f) <= bound * (1 + 1e-12)
+
+
+def test_router_translation_invariance():
+    w = _tiny_layer(6)
+    x = np.random.Generator(np.random.PCG64(12)).standard_normal((30, w.spec.hidden))
+    h = O.rmsnorm(x, w.gamma, w.spec.rms_eps)
+    shift = np.random.Generator(np.random.PCG64(13)).standard_normal(w.spec.hidden)
+    ids1, g1 = O.topk_gates(O.router_logits(h, w.router_w, w.router_b), w.spec.top_k)
+    ids2, g2 = O.topk_gates(O.router_logits(h, w.router_w + shift, w.router_b + 0.7), w.spec.top_k)
+    assert (ids1 == ids2).all()
+    np.testing.assert_allclose(g1, g2, rtol=1e-12)
+    r1 = O.rcr_table(w.router_w, w.gamma, w.w_gate, w.w_up, w.w_down)
+    r2 = O.rcr_table(w.router_w + shift, w.gamma, w.w_gate, w.w_up, w.w_down)
+    np.testing.assert_allclose(r1, r2, rtol=1e-12)
+
+
+def test_table_means_scaling_and_identical_experts():
+    w = _tiny_layer(7)
+    args = (w.gamma, w.w_gate, w.w_up, w.w_down)
+    a = O.gsp_table(*args, eps=0.0)
+    r = O.rcr_table(w.router_w, *args, eps=0.0)
+    assert abs(a.mean() - 1) < 1e-14 and abs(r.mean() - 1) < 1e-14
+    # scaling expert 2's down projection by s scales its raw score by s
+    s = 3.0
+    wd = w.w_down.copy()
+    wd[2] *= s
+    a2 = O.gsp_table(w.gamma, w.w_gate, w.w_up, wd, eps=0.0)
+    r2 = O.rcr_table(w.router_w, w.gamma, w.w_gate, w.w_up, wd, eps=0.0)
+    for t_old, t_new in [(a, a2), (r, r2)]:
+        np.testing.assert_allclose(t_new[2] / t_new[0], s * t_old[2] / t_old[0], rtol=1e-12)
+        np.testing.assert_allclose(t_new[1] / t_new[0], t_old[1] / t_old[0], rtol=1e-12)
+    # scaling expert 1's gate projection by s scales its GSP score by s
+    wg = w.w_gate.copy()
+    wg[1] *= s
+    a3 = O.gsp_table(w.gamma, wg, w.w_up, w.w_down, eps=0.0)
+    np.testing.assert_allclose(a3[1] / a3[0], s * a[1] / a[0], rtol=1e-12)
+    # global scale of all W_down leaves the normalised tables unchanged
+    np.testing.assert_allclose(O.gsp_table(w.gamma, w.w_gate, w.w_up, w.w_down * 5, eps=0.0), a, rtol=1e-12)
+    # identical experts -> every entry equals mu / (mu + eps)
+    same = lambda arr: np.repeat(arr[:1], arr.shape[0], axis=0)
+    eps = 1e-6
+    a4 = O.gsp_table(w.gamma, same(w.w_gate), same(w.w_up), same(w.w_down), eps=eps)
+    assert np.ptp(a4) < 1e-15
+    raw = O.gsp_table(w.gamma, same(w.w_gate), same(w.w_up), same(w.w_down), eps=0.0)
+    assert np.allclose(raw, 1.0, rtol=1e-15)
+
+
+def test_rmsnorm_closed_form():
+    d = 64
+    gam = np.linspace(0.9, 1.1, d)
+    for cval in [0.5, -3.0, 1e-4]:
+        x = np.full((1, d), cval)
+        h = O.rmsnorm(x, gam, 1e-6)
+        np.testing.assert_allclose(h[0], cval / math.sqrt(cval * cval + 1e-6) * gam, rtol=1e-14)
+
+
+# ---------------------------------------------------------------- ratio mode
+
+
+def test_realised_ratio_matches_request():
+    rng = np.random.Generator(np.random.PCG64(14))
+    T, N, k = 300, 32, 8
+    z = rng.standard_normal((T, N))
+    a_gsp = np.abs(1 + 0.3 * rng.standard_normal(N))
+    a_rcr = np.abs(1 + 0.3 * rng.standard_normal(N))
+    for m_min in [1, 3]:
+        for q in [0.0, 0.125, 0.25, 0.5, 0.625, 0.9]:
+            dec = O.ace_decide(z, k, a_gsp, a_rcr, "ratio", q, m_min)
+            n_cand = T * (k - m_min)
+            m_q = min(int(math.floor(q * T * k + 0.5)), n_cand)
+            assert dec["m_q"] == m_q
+            assert int(dec["skip"].sum()) == m_q, (q, m_min)
+            assert (k - dec["skip"].sum(1) >= m_min).all()
+
+
+def test_decide_fp32_matches_fp64_off_boundary():
+    z32 = synth.make_logits(2000, 128, seed=3)
+    a_gsp, a_rcr = synth.make_tables(128, seed=4, spread=0.2)
+    k = 8
+    ids32, g32 = O.route_fp32(z32, k)
+    ids64, g64 = O.topk_gates(z32.astype(np.float64), k)
+    zs = np.sort(z32.astype(np.float64), axis=1)[:, ::-1]
+    clear = (zs[:, k - 1] - zs[:, k]) > 1e-5
+    assert (ids32[clear] == ids64[clear]).all()
+    np.testing.assert_allclose(g32, g64, rtol=3e-6)
+    for tau in [0.08, 0.11, 0.13]:
+        d32 = O.decide_fp32(ids32, g32, a_gsp, a_rcr, "threshold", tau)
+        _, _, c64, _, _ = O.ace_skip(ids64, g64, a_gsp.astype(np.float64), a_rcr.astype(np.float64), 0.0, 1, 1e-6)
+        s64, gh64, *_ = O.ace_skip(ids64, g64, a_gsp.astype(np.float64), a_rcr.astype(np.float64), tau, 1, 1e-6)
+        margin = np.abs(c64 - tau) > 1e-5 * tau
+        ok = clear[:, None] & margin
+        assert (d32["skip"][ok] == s64[ok]).all()
+        rows = ok.all(1)
+        np.testing.assert_allclose(d32["g_hat"][rows], gh64[rows], rtol=5e-6, atol=1e-7)
+
+
+def test_exp32_error_bound():
+    x = np.linspace(-87.0, 0.0, 400001).astype(np.float32)
+    x = np.concatenate([x, -np.abs(np.random.Generator(np.random.PCG64(0)).standard_normal(100000)).astype(np.float32),
+                        np.array([0.0, -0.0, -1e-30, -1e-8], dtype=np.float32)])
+    y = O.exp32(x).astype(np.float64)
+    ref = np.exp(x.astype(np.float64))
+    ulp = np.spacing(ref.astype(np.float32)).astype(np.float64)
+    err = np.abs(y - ref) / ulp
+    assert err.max() <= 2.0, err.max()
+    assert O.exp32(np.array([0.0], np.float32))[0] == np.float32(1.0)
+    assert O.exp32(np.array([-90.0], np.float32))[0] == 0.0
+
+
+def test_permutation_bruteforce():
+    rng = np.random.Generator(np.random.PCG64(15))
+    T, N, k = 50, 12, 4
+    ids = np.stack([rng.permutation(N)[:k] for _ in range(T)])
+    skip = rng.random((T, k)) < 0.4
+    skip[:, 0] = False
+    off, perm = O.permutation(ids, skip, N)
+    want = sorted((int(ids[t, i]), t, t * k + i) for t in range(T) for i in range(k) if not skip[t, i])
+    assert perm.tolist() == [s for _, _, s in want]
+    counts = np.bincount([e for e, _, _ in want], minlength=N)
+    assert off.tolist() == [0] + np.cumsum(counts).tolist()
+
+
+def test_zipf_router_bias_slope():
+    spec = synth.spec_qwen(zipf=True)
+    n, d, k = spec.n_experts, spec.hidden, spec.top_k
+    w = synth.make_layer(synth.LayerSpec(d, n, k, 64, dtype="bf16", zipf=True), seed=0)
+    x = synth.make_tokens(spec, 4096, seed=1)
+    h = O.rmsnorm(x, w.gamma, 1e-6)
+    z = O.router_logits(h, w.router_w, w.router_b)
+    ids, _ = O.topk_gates(z, k)
+    counts = np.sort(np.bincount(ids.ravel(), minlength=n))[::-1].astype(np.float64)
+    r = np.arange(1, n // 2 + 1)
+    slope = np.polyfit(np.log(r), np.log(np.maximum(counts[: n // 2], 1)), 1)[0]
+    assert -1.2 < slope < -1.0, slope
