@@ -1,0 +1,366 @@
+#!/usr/bin/env python3
+"""Benchmark of the ACE MoE-layer forward (token-adaptive expert skipping) on
+GB300, one process per GPU.
+
+Default workload: the Qwen3-30B-A3B-shaped MoE layer (hidden 2048, 128
+experts, top-8, expert FFN 768, bf16) decoding a batch of 64 tokens at target
+skip ratio 0.5 (per-batch threshold, App. B.1). A step is one full layer
+forward: RMSNorm, router, top-k, skip decision, threshold, compaction,
+experts and combine. Inputs are synthetic (seeded N(0,1) tokens, N(0, 0.02^2)
+weights) and resident in HBM; the forward is replayed from a CUDA graph and
+each step is timed with CUDA events; L2 is flushed (a 512 MB write) between
+steps, outside the timed events.
+
+Prints one JSON line (rank 0). `--impl reference` times the CPU oracle
+instead, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+WORKLOADS = {
+    "decode": dict(zipf=False, T=64, q=0.5,
+                   name="ACE MoE layer decode: d=2048 N=128 top-8 m=768 bf16, batch 64 tokens, skip ratio 0.5"),
+    "prefill": dict(zipf=True, T=4096, q=0.5,
+                    name="ACE MoE layer prefill: d=2048 N=128 top-8 m=768 bf16, 4096 tokens Zipf(1.1) routing, "
+                         "skip ratio 0.5"),
+}
+METRIC = "ACE MoE-layer tokens/s (prefill, decode) + speedup vs skip=0; % of roofline"
+L2_FLUSH_BYTES = 512 << 20
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.gpu = gpu_index
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={gpu_index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            return None
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def build_layer(wl, max_tokens):
+    from paper_2609_05228_gb300 import ace, offline, synth
+    spec = synth.spec_qwen(zipf=wl["zipf"])
+    w = synth.make_layer(spec, seed=0)
+    a_gsp, a_rcr = offline.tables(w)
+    w.extra["a_gsp"], w.extra["a_rcr"] = a_gsp, a_rcr
+    layer = ace.AceLayer(w, a_gsp, a_rcr, max_tokens=max_tokens)
+    return w, layer
+
+
+def time_point(torch, layer, x, out, T, q, steps, warmup, flush, profile=False):
+    """Device time per step (ms) of a graph-replayed forward; optional stage times."""
+    from paper_2609_05228_gb300 import ace
+    s = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    ace.ace_layer_set_profiling(layer.handle, profile)
+    # warm the path once eagerly (outside capture)
+    with torch.cuda.stream(s):
+        ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q, s)
+    s.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q, torch.cuda.current_stream())
+    stages = []
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    with torch.cuda.stream(s):
+        for _ in range(warmup):
+            flush.zero_()
+            g.replay()
+        s.synchronize()
+        for i in range(steps):
+            flush.zero_()
+            starts[i].record(s)
+            g.replay()
+            ends[i].record(s)
+            if profile:
+                stages.append(ace.ace_last_stage_times(layer.handle))
+    s.synchronize()
+    ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
+    ace.ace_layer_set_profiling(layer.handle, False)
+    return ms, stages
+
+
+def algorithmic(w, T, R, D):
+    """Algorithmic bytes and flops of one forward (retained work only) and of
+    the gate/up expert kernel. D = distinct experts with >= 1 retained slot."""
+    s = w.spec
+    d, m, N = s.hidden, s.ffn, s.n_experts
+    e = 2
+    w_bytes = 3 * d * m * e * D
+    total_bytes = w_bytes + N * d * e + 2 * T * d * e
+    flops = 6 * d * m * R + 2 * d * N * T
+    gate_up_bytes = 2 * d * m * e * D + R * d * e + R * m * 4
+    return total_bytes, flops, gate_up_bytes
+
+
+def run_ours(args, rank, world, torch, dist):
+    from paper_2609_05228_gb300 import ace, synth
+    wl = WORKLOADS[args.workload]
+    T, q = wl["T"], wl["q"]
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    w, layer = build_layer(wl, max_tokens=max(T, 64))
+    spec = w.spec
+    xh = synth.make_tokens(spec, T, seed=1 + rank)
+    x = torch.from_numpy(xh.view(np.int16)).view(torch.bfloat16).to(dev)
+    out = torch.empty_like(x)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    # decision statistics of this batch (R, distinct experts)
+    ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q)
+    skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, spec.top_k)
+    off, _ = ace.ace_last_permutation(layer.handle, spec.n_experts, R)
+    D = int((np.diff(off) > 0).sum())
+
+    # timed region
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(dev.index)
+    t_wall = time.perf_counter()
+    ms, stages = time_point(torch, layer, x, out, T, q, args.steps, args.warmup, flush, profile=True)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t_wall
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    step_ms = float(np.mean(ms))
+    tmax = torch.tensor([step_ms], device=dev)
+    if world > 1:
+        dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
+    step_ms_max = float(tmax.item())
+
+    # skip ratio 0 with the same kernels, for the speedup
+    ms0, _ = time_point(torch, layer, x, out, T, 0.0, max(10, args.steps // 2), 3, flush)
+    t0 = float(np.mean(ms0))
+
+    # end to end through the host-buffer C call (pinned buffers, copies included)
+    xp = torch.from_numpy(xh.view(np.int16)).pin_memory()
+    op = torch.empty_like(xp).pin_memory()
+    for _ in range(3):
+        ace.ace_moe_forward_host(layer.handle, xp, op, T, "ratio", q)
+    e2e_steps = max(10, args.steps)
+    t = time.perf_counter()
+    for _ in range(e2e_steps):
+        ace.ace_moe_forward_host(layer.handle, xp, op, T, "ratio", q)
+    e2e_s = (time.perf_counter() - t) / e2e_steps
+
+    hbm, bf16, peak_kind = _peaks()
+    total_bytes, flops, gu_bytes = algorithmic(w, T, R, D)
+    gu_ms = float(np.mean([st["gate_up"] for st in stages])) if stages else float("nan")
+    achieved = gu_bytes / (gu_ms * 1e-3) / 1e9
+    stage_avg = {k: round(float(np.mean([st[k] for st in stages])) * 1e3, 2) for k in stages[0]} if stages else {}
+
+    result = {
+        "metric": METRIC,
+        "value": round(world * T / (step_ms_max * 1e-3), 1),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(step_ms_max, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) tokens, N(0,0.02^2) weights, offline GSP/RCR tables)",
+        "config": {"workload": wl["name"], "tokens_per_step": T, "skip_ratio": q,
+                   "parallelism": f"replicas{world}" if world > 1 else "single GPU",
+                   "l2": "flushed (512 MB write) between timed steps", "graph": "CUDA graph replay"},
+        "realised_skip_ratio": round((T * spec.top_k - R) / (T * spec.top_k), 6),
+        "retained_slots": R,
+        "distinct_experts": D,
+        "speedup_vs_q0": round(t0 / step_ms, 4),
+        "q0_ms_per_step": round(t0, 5),
+        "stage_us": stage_avg,
+        "wall_s": round(wall, 3),
+        "roofline": {"bound": "hbm", "kernel": "k_gemv_gateup", "achieved": round(achieved, 1),
+                     "peak": hbm, "unit": "GB/s", "frac": round(achieved / hbm, 4),
+                     "peak_source": peak_kind, "traffic": None,
+                     "algorithmic_bytes": gu_bytes, "kernel_us": round(gu_ms * 1e3, 2)},
+        "layer_roofline": {"bytes": total_bytes, "flops": flops,
+                           "hbm_frac": round(total_bytes / (step_ms * 1e-3) / 1e9 / hbm, 4),
+                           "tensor_frac": round(flops / (step_ms * 1e-3) / 1e12 / bf16, 5)},
+        "e2e": {"value": round(T / e2e_s, 1), "unit": "tokens/s",
+                "h2d_bytes_per_step": int(T * spec.hidden * 2), "d2h_bytes_per_step": int(T * spec.hidden * 2)},
+        "gpu_launches": args.steps * (10 if 0 < q < 1 else 8),
+        "clocks": clk,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(w, wl, budget_s=args.cpu_seconds)
+    if rank == 0 and args.sweep:
+        result["sweep"] = sweep(torch, args)
+    layer.close()
+    return result
+
+
+def sweep(torch, args):
+    """Tokens/s and speedup vs q=0 over the decode batches and prefill ratios."""
+    from paper_2609_05228_gb300 import synth
+    pts = []
+    for wlname, Ts, qs in [("decode", [1, 8, 32, 64], [0.0, 0.25, 0.5]),
+                           ("prefill", [4096], [0.0, 0.25, 0.5, 0.625])]:
+        wl = WORKLOADS[wlname]
+        w, layer = build_layer(wl, max_tokens=max(Ts))
+        flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+        for T in Ts:
+            xh = synth.make_tokens(w.spec, T, seed=1)
+            x = torch.from_numpy(xh.view(np.int16)).view(torch.bfloat16).cuda()
+            out = torch.empty_like(x)
+            base = None
+            for q in qs:
+                ms, _ = time_point(torch, layer, x, out, T, q, 20, 3, flush)
+                t = float(np.median(ms))
+                base = t if q == 0.0 else base
+                pts.append({"workload": wlname, "T": T, "q": q, "us": round(t * 1e3, 2),
+                            "tokens_per_s": round(T / (t * 1e-3), 1),
+                            "speedup_vs_q0": round(base / t, 4) if base else None})
+        layer.close()
+    return pts
+
+
+def cpu_baseline(w, wl, budget_s=12.0):
+    """The CPU oracle (fp64) on a bounded sample of the same workload."""
+    import oracle as O
+    from paper_2609_05228_gb300 import synth
+    T = wl["T"] if wl["T"] <= 64 else 256
+    x = synth.make_tokens(w.spec, T, seed=1)
+    n = 0
+    t0 = time.perf_counter()
+    while True:
+        O.moe_forward(x, w, "ratio", wl["q"])
+        n += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return {"value": round(n * T / dt, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n} forwards of {T} tokens ({dt:.1f} s), numpy fp64 with its default BLAS threads"}
+
+
+def run_reference(args):
+    """The reference arm: the CPU oracle on a bounded sample, per step."""
+    import oracle as O
+    from paper_2609_05228_gb300 import offline, synth
+    wl = WORKLOADS[args.workload]
+    spec = synth.spec_qwen(zipf=wl["zipf"])
+    w = synth.make_layer(spec, seed=0)
+    w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables(w)
+    T = wl["T"] if wl["T"] <= 64 else 256
+    x = synth.make_tokens(spec, T, seed=1)
+    for _ in range(args.warmup):
+        O.moe_forward(x, w, "ratio", wl["q"])
+    times = []
+    for _ in range(args.steps):
+        t = time.perf_counter()
+        O.moe_forward(x, w, "ratio", wl["q"])
+        times.append(time.perf_counter() - t)
+    step = float(np.mean(times))
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    val = round(T / step, 2)
+    return {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": wl["name"], "tokens_per_step": T, "skip_ratio": wl["q"],
+                                            "sample": f"{T} tokens per step"},
+            "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{args.steps} steps of {T} tokens"},
+            "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="decode", choices=sorted(WORKLOADS))
+    ap.add_argument("--sweep", action="store_true", help="add decode/prefill sweep points")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args)), flush=True)
+        return
+
+    import torch
+    import torch.distributed as dist
+    if world > 1:
+        dist.init_process_group("nccl")
+    try:
+        res = run_ours(args, rank, world, torch, dist)
+        if rank == 0:
+            print(json.dumps(res), flush=True)
+    finally:
+        if world > 1:
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

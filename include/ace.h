@@ -1,0 +1,202 @@
+/*
+ * ace.h — C ABI of libace.so: the ACE MoE-layer forward with token-adaptive
+ * expert skipping, on one GB300 GPU (sm_103a).
+ *
+ * Method: ACE, "Adaptive Calibration-Free Expert Skipping for MoE-based LLMs".
+ *   - router top-k and gates:            §3.1 (routed set {(e_i, g_i)}), Algorithm 1
+ *   - per-slot skip decision:            §3.1-3.2 Eqs. gsp_contribution, gsp_probability,
+ *                                        rcr_contribution, rcr_probability, ace_contribution,
+ *                                        ace_candidate_intersection; Algorithm 4
+ *   - target skip ratio -> threshold:    App. B.1 (budget-to-threshold mapping)
+ *   - expert FFN:                        Eq. swiglu_expert
+ *   - sparse output:                     Eq. ace_sparse_output
+ *
+ * Conventions common to every call
+ *   - Pointers are plain device or host pointers as stated per argument. No
+ *     call takes ownership of a caller pointer.
+ *   - Weight layouts follow nn.Linear ([out_features, in_features]), row
+ *     major: the paper's row-vector W_gate in R^{d x m} is w_gate[e] transposed.
+ *   - `stream` is a cudaStream_t (a CUstream) passed as void*; NULL is the
+ *     legacy default stream. All device work of a call is ordered on it.
+ *   - Every call returns an ace_status; on failure ace_last_error_message()
+ *     (thread-local) describes it. No call aborts the process.
+ *   - Errors found by kernels (non-finite router logits, a bounded device wait
+ *     that ran out) are recorded in a per-layer device word and reported by the
+ *     next call that synchronises (ace_last_skip_mask, ace_layer_sync).
+ *   - One forward may be in flight per layer at a time; calls on different
+ *     layers are independent.
+ */
+#ifndef ACE_H
+#define ACE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum ace_status {
+    ACE_OK = 0,
+    ACE_ERR_INVALID_ARG = 1,   /* bad pointer, size or mode */
+    ACE_ERR_UNSUPPORTED = 2,   /* shape outside what the kernels support */
+    ACE_ERR_OOM = 3,           /* device allocation failed at create time */
+    ACE_ERR_CUDA = 4,          /* a CUDA runtime call failed */
+    ACE_ERR_TIMEOUT = 5,       /* a bounded device wait ran out */
+    ACE_ERR_NUMERIC = 6,       /* non-finite router logits were seen */
+    ACE_ERR_STATE = 7          /* call out of order (e.g. no forward yet) */
+} ace_status;
+
+typedef enum ace_dtype { ACE_BF16 = 0, ACE_F32 = 1 } ace_dtype;
+
+typedef enum ace_skip_mode {
+    ACE_SKIP_THRESHOLD = 0,    /* value = tau (Algorithm 4 input tau_q) */
+    ACE_SKIP_RATIO = 1         /* value = q in [0,1]; tau derived per batch (App. B.1) */
+} ace_skip_mode;
+
+typedef struct ace_layer_desc {
+    int hidden;          /* d */
+    int n_experts;       /* N, 1..1024 */
+    int top_k;           /* k, 1..min(N, 16) */
+    int ffn;             /* m, expert FFN width */
+    int max_tokens;      /* largest T a forward may pass; sizes the workspace */
+    int dtype;           /* ace_dtype of x, out, weights and gamma */
+    float eps;           /* the paper's epsilon (Eqs. gsp_probability, rcr_probability,
+                            Algorithm 4 gate renormalisation); 1e-6 if <= 0 */
+    float rms_eps;       /* RMSNorm epsilon; 1e-6 if <= 0 */
+    float router_temp;   /* logits are divided by it; 1 if <= 0 */
+    int min_active;      /* m_min of Algorithm 4 (1 = only the top-1 safeguard) */
+    int has_router_bias; /* router_b is read when non-zero */
+} ace_layer_desc;
+
+typedef struct ace_skip_ctl {
+    int mode;            /* ace_skip_mode */
+    float value;         /* tau (>= 0, may be +inf) or q (in [0,1]) */
+} ace_skip_ctl;
+
+typedef struct ace_layer ace_layer;   /* opaque */
+
+/*
+ * ace_layer_create — build one MoE layer on the current CUDA device.
+ *   router_w  [N, d]      device, dtype        router weight rows w_e (§3.2 logit z_e = x.w_e + b_e)
+ *   router_b  [N]         device, float32      router bias b_e; read only if has_router_bias
+ *   w_gate    [N, m, d]   device, dtype        per-expert W_gate^T
+ *   w_up      [N, m, d]   device, dtype        per-expert W_up^T
+ *   w_down    [N, d, m]   device, dtype        per-expert W_down^T
+ *   rms_gamma [d]         device, dtype        RMSNorm scale gamma (Gamma = Diag(gamma), §3.1)
+ *   a_gsp     [N]         host,   float32      GSP table A^GSP (Algorithm 2), finite, >= 0
+ *   a_rcr     [N]         host,   float32      RCR table A^RCR (Algorithm 3), finite, >= 0
+ * The weights are copied and repacked into layer-owned device memory; the
+ * caller may free its buffers once the call returns (it synchronises
+ * `stream`). The workspace for max_tokens is allocated here; the forward
+ * allocates nothing.
+ * Errors: INVALID_ARG for NULL pointers, non-positive sizes, k > N, tables
+ * that are negative or non-finite; UNSUPPORTED for d or m not a multiple of
+ * 64 (bf16) or 4 (f32), N > 1024, k > 16; OOM; CUDA.
+ */
+ace_status ace_layer_create(const ace_layer_desc* desc,
+                            const void* router_w, const float* router_b,
+                            const void* w_gate, const void* w_up, const void* w_down,
+                            const void* rms_gamma,
+                            const float* a_gsp, const float* a_rcr,
+                            void* stream, ace_layer** out_layer);
+
+/* Frees everything the layer owns. NULL is a no-op. Synchronises the device. */
+void ace_layer_destroy(ace_layer* layer);
+
+/*
+ * ace_moe_forward — y_t = sum_{i in I_t} g^_i f_{e_i}(x_t) for t < T
+ * (Eq. ace_sparse_output), with RMSNorm, router, top-k, the skip decision of
+ * Algorithm 4, compaction of the retained slots and the SwiGLU experts all on
+ * the GPU. No residual is added.
+ *   x    [T, d]  device, dtype     layer input (pre-RMSNorm hidden states)
+ *   out  [T, d]  device, dtype     layer output; must not alias x
+ *   T    0..max_tokens             T = 0 is a no-op
+ * Stream-ordered and asynchronous; allocates nothing; the sequence of
+ * launches depends only on (T, ctl.mode), so it can be captured in a CUDA graph.
+ * Errors: INVALID_ARG (NULL, T out of range, ratio outside [0,1], negative
+ * or NaN tau), CUDA.
+ */
+ace_status ace_moe_forward(ace_layer* layer, const void* x, void* out, int T,
+                           ace_skip_ctl ctl, void* stream);
+
+/*
+ * ace_moe_forward_host — the same forward from HOST buffers: copies x to a
+ * layer-owned device buffer, runs ace_moe_forward, copies the result back
+ * and synchronises `stream` before returning.
+ *   x_host   [T, d] host, dtype (pinned memory gives the fastest copies)
+ *   out_host [T, d] host, dtype
+ */
+ace_status ace_moe_forward_host(ace_layer* layer, const void* x_host, void* out_host, int T,
+                                ace_skip_ctl ctl, void* stream);
+
+/*
+ * ace_route_logits — run only the decision steps (top-k + gates, the
+ * Algorithm 4 skip decision, App. B.1 threshold in ratio mode, and the
+ * compaction) on caller-supplied float32 router logits, as ace_moe_forward
+ * does after its router. Results are read with ace_last_skip_mask and
+ * ace_last_permutation.
+ *   logits [T, N] device, float32
+ */
+ace_status ace_route_logits(ace_layer* layer, const float* logits, int T, ace_skip_ctl ctl,
+                            void* stream);
+
+/*
+ * ace_last_skip_mask — results of the last forward / route call, copied to
+ * host buffers the caller owns. Synchronises the stream of that call. Any
+ * output pointer may be NULL.
+ *   skip      [T, k] uint8    1 = slot skipped; slot i is rank i (logit-descending)
+ *   ids       [T, k] int32    routed expert e_i
+ *   gates_hat [T, k] float32  renormalised gate g^_i (0 where skipped)
+ *   tau       [1]   float32   threshold used (derived per batch in ratio mode)
+ *   retained  [1]   int32     R, the number of retained slots
+ * Errors: STATE before any forward; NUMERIC / TIMEOUT from the device word.
+ */
+ace_status ace_last_skip_mask(ace_layer* layer, uint8_t* skip, int32_t* ids, float* gates_hat,
+                              float* tau, int32_t* retained);
+
+/* Router logits z [T, N] float32 (host) of the last ace_moe_forward. */
+ace_status ace_last_router_logits(ace_layer* layer, float* logits);
+
+/*
+ * Retained slots grouped by expert, of the last call (host buffers):
+ *   offsets [N+1] int32  exclusive scan of per-expert retained counts
+ *   perm    [R]   int32  slot ids t*k+i, sorted by (expert, token)
+ */
+ace_status ace_last_permutation(ace_layer* layer, int32_t* offsets, int32_t* perm);
+
+/* Waits for the layer's last stream and reports any device-side error word. */
+ace_status ace_layer_sync(ace_layer* layer);
+
+/*
+ * ace_debug_exp32 — the float32 exp used for the gates (x <= 0), applied
+ * element-wise on the device: y[i] = exp(x[i]). Exposed so its bits can be
+ * checked against an independent implementation.
+ *   x, y [n] device float32
+ */
+ace_status ace_debug_exp32(const float* x, float* y, int n, void* stream);
+
+/*
+ * Stage timing (instrumentation; the paper has no counterpart). When enabled,
+ * each ace_moe_forward records CUDA events on its stream around its stages:
+ *   0 RMSNorm, 1 router logits, 2 top-k + decision + threshold + compaction,
+ *   3 expert gate/up, 4 expert down, 5 combine.
+ * ace_last_stage_times synchronises the last stream and writes up to n_max
+ * stage durations in milliseconds (host float32) of the last forward; it
+ * returns the stage count in *n_out. Enabling it is not allowed while the
+ * stream is being captured.
+ */
+ace_status ace_layer_set_profiling(ace_layer* layer, int enable);
+ace_status ace_last_stage_times(ace_layer* layer, float* ms, int n_max, int* n_out);
+
+/* Fills *desc with the layer's descriptor (after defaults were applied). */
+ace_status ace_layer_get_desc(const ace_layer* layer, ace_layer_desc* desc);
+
+const char* ace_status_string(ace_status status);
+const char* ace_last_error_message(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ACE_H */

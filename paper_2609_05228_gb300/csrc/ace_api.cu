@@ -1,0 +1,363 @@
+// ace_api.cu — the C ABI of libace.so (include/ace.h): argument checks,
+// layer-owned weights and workspace, and the launch sequence of the forward.
+#include <math.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <string>
+#include <vector>
+
+#include "ace_internal.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+ace_status fail(ace_status st, const std::string& msg) {
+    g_last_error = msg;
+    return st;
+}
+
+ace_status cuda_fail(cudaError_t e, const char* where) {
+    std::string m = std::string(where) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")";
+    return fail(ACE_ERR_CUDA, m);
+}
+
+#define ACE_CUDA(call, where)                              \
+    do {                                                   \
+        cudaError_t e_ = (call);                           \
+        if (e_ != cudaSuccess) return cuda_fail(e_, where); \
+    } while (0)
+
+template <typename P>
+cudaError_t dalloc(P** p, size_t bytes) {
+    void* q = nullptr;
+    cudaError_t e = cudaMalloc(&q, bytes < 16 ? 16 : bytes);
+    *p = static_cast<P*>(q);
+    return e;
+}
+
+void free_layer(ace_layer* L) {
+    if (!L) return;
+    void* ptrs[] = {L->router_w, L->router_b, L->w_gate, L->w_up, L->w_down, L->gamma, L->a_gsp, L->a_rcr,
+                    L->ws.h, L->ws.logits, L->ws.ids, L->ws.gates, L->ws.cval, L->ws.keys, L->ws.skip,
+                    L->ws.ghat, L->ws.tau, L->ws.chunk_counts, L->ws.offsets, L->ws.dlist, L->ws.perm,
+                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.err, L->ws.x_stage,
+                    L->ws.out_stage};
+    for (void* p : ptrs)
+        if (p) cudaFree(p);
+    for (cudaEvent_t e : L->ev)
+        if (e) cudaEventDestroy(e);
+    delete L;
+}
+
+bool tables_ok(const float* t, int n) {
+    for (int i = 0; i < n; ++i)
+        if (!(t[i] >= 0.0f) || !isfinite(t[i])) return false;
+    return true;
+}
+
+ace_status check_device_word(ace_layer* L) {
+    int err = 0;
+    ACE_CUDA(cudaMemcpy(&err, L->ws.err, sizeof(int), cudaMemcpyDeviceToHost), "read device error word");
+    if (err) {
+        ACE_CUDA(cudaMemset(L->ws.err, 0, sizeof(int)), "clear device error word");
+        if (err & ace::kErrTimeout) return fail(ACE_ERR_TIMEOUT, "a bounded device wait ran out");
+        if (err & ace::kErrNumeric) return fail(ACE_ERR_NUMERIC, "non-finite router logits were seen");
+        if (err & ace::kErrBounds) return fail(ACE_ERR_CUDA, "a device index check failed");
+    }
+    return ACE_OK;
+}
+
+ace_status check_ctl(ace_skip_ctl ctl) {
+    if (ctl.mode == ACE_SKIP_THRESHOLD) {
+        if (!(ctl.value >= 0.0f)) return fail(ACE_ERR_INVALID_ARG, "threshold tau must be >= 0 (not NaN)");
+    } else if (ctl.mode == ACE_SKIP_RATIO) {
+        if (!(ctl.value >= 0.0f && ctl.value <= 1.0f))
+            return fail(ACE_ERR_INVALID_ARG, "skip ratio q must be in [0, 1]");
+    } else {
+        return fail(ACE_ERR_INVALID_ARG, "unknown skip mode");
+    }
+    return ACE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* ace_status_string(ace_status s) {
+    switch (s) {
+        case ACE_OK: return "ACE_OK";
+        case ACE_ERR_INVALID_ARG: return "ACE_ERR_INVALID_ARG";
+        case ACE_ERR_UNSUPPORTED: return "ACE_ERR_UNSUPPORTED";
+        case ACE_ERR_OOM: return "ACE_ERR_OOM";
+        case ACE_ERR_CUDA: return "ACE_ERR_CUDA";
+        case ACE_ERR_TIMEOUT: return "ACE_ERR_TIMEOUT";
+        case ACE_ERR_NUMERIC: return "ACE_ERR_NUMERIC";
+        case ACE_ERR_STATE: return "ACE_ERR_STATE";
+    }
+    return "ACE_ERR_UNKNOWN";
+}
+
+const char* ace_last_error_message(void) { return g_last_error.c_str(); }
+
+ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w, const float* router_b,
+                            const void* w_gate, const void* w_up, const void* w_down, const void* rms_gamma,
+                            const float* a_gsp, const float* a_rcr, void* stream, ace_layer** out_layer) {
+    if (!desc_in || !out_layer) return fail(ACE_ERR_INVALID_ARG, "desc and out_layer must be non-NULL");
+    *out_layer = nullptr;
+    ace_layer_desc D = *desc_in;
+    if (D.eps <= 0.f) D.eps = 1e-6f;
+    if (D.rms_eps <= 0.f) D.rms_eps = 1e-6f;
+    if (D.router_temp <= 0.f) D.router_temp = 1.0f;
+    if (D.min_active < 1) D.min_active = 1;
+    if (D.hidden <= 0 || D.n_experts <= 0 || D.top_k <= 0 || D.ffn <= 0 || D.max_tokens <= 0)
+        return fail(ACE_ERR_INVALID_ARG, "hidden, n_experts, top_k, ffn and max_tokens must be positive");
+    if (D.top_k > D.n_experts) return fail(ACE_ERR_INVALID_ARG, "top_k > n_experts");
+    if (D.min_active > D.top_k) return fail(ACE_ERR_INVALID_ARG, "min_active > top_k");
+    if (D.dtype != ACE_BF16 && D.dtype != ACE_F32) return fail(ACE_ERR_INVALID_ARG, "unknown dtype");
+    if (D.n_experts > ace::kMaxExperts) return fail(ACE_ERR_UNSUPPORTED, "n_experts > 1024");
+    if (D.top_k > ace::kMaxTopK) return fail(ACE_ERR_UNSUPPORTED, "top_k > 16");
+    const int mult = D.dtype == ACE_BF16 ? 64 : 4;
+    if (D.hidden % mult || D.ffn % mult)
+        return fail(ACE_ERR_UNSUPPORTED, D.dtype == ACE_BF16 ? "hidden and ffn must be multiples of 64"
+                                                             : "hidden and ffn must be multiples of 4");
+    if ((long long)D.max_tokens * D.top_k > (1LL << 30)) return fail(ACE_ERR_UNSUPPORTED, "max_tokens too large");
+    if (!router_w || !w_gate || !w_up || !w_down || !rms_gamma || !a_gsp || !a_rcr)
+        return fail(ACE_ERR_INVALID_ARG, "weight, gamma and table pointers must be non-NULL");
+    if (D.has_router_bias && !router_b) return fail(ACE_ERR_INVALID_ARG, "has_router_bias set but router_b is NULL");
+    if (!tables_ok(a_gsp, D.n_experts) || !tables_ok(a_rcr, D.n_experts))
+        return fail(ACE_ERR_INVALID_ARG, "GSP/RCR tables must be finite and >= 0");
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    ace_layer* L = new ace_layer();
+    L->desc = D;
+    L->elem = D.dtype == ACE_BF16 ? 2 : 4;
+    cudaGetDevice(&L->device);
+    cudaDeviceGetAttribute(&L->num_sms, cudaDevAttrMultiProcessorCount, L->device);
+    if (L->num_sms <= 0) L->num_sms = 1;
+
+    const size_t d = D.hidden, n = D.n_experts, k = D.top_k, m = D.ffn, T = D.max_tokens, E = L->elem;
+    const size_t slots = T * k;
+    const int n_chunks = (int)((T + ace::kChunk - 1) / ace::kChunk);
+    ace::Workspace& W = L->ws;
+    cudaError_t e = cudaSuccess;
+#define ALLOC(ptr, bytes)                                                   \
+    do {                                                                    \
+        e = dalloc(&(ptr), (bytes));                                        \
+        if (e != cudaSuccess) {                                             \
+            free_layer(L);                                                  \
+            cudaGetLastError();                                             \
+            return fail(ACE_ERR_OOM, std::string("cudaMalloc failed for ") + #ptr); \
+        }                                                                   \
+    } while (0)
+    ALLOC(L->router_w, n * d * E);
+    ALLOC(L->router_b, n * sizeof(float));
+    ALLOC(L->w_gate, n * m * d * E);
+    ALLOC(L->w_up, n * m * d * E);
+    ALLOC(L->w_down, n * d * m * E);
+    ALLOC(L->gamma, d * E);
+    ALLOC(L->a_gsp, n * sizeof(float));
+    ALLOC(L->a_rcr, n * sizeof(float));
+    ALLOC(W.h, T * d * E);
+    ALLOC(W.logits, T * n * sizeof(float));
+    ALLOC(W.ids, slots * sizeof(int32_t));
+    ALLOC(W.gates, slots * sizeof(float));
+    ALLOC(W.cval, slots * sizeof(float));
+    ALLOC(W.keys, slots * sizeof(uint32_t));
+    ALLOC(W.skip, slots);
+    ALLOC(W.ghat, slots * sizeof(float));
+    ALLOC(W.tau, sizeof(float));
+    ALLOC(W.chunk_counts, (size_t)n_chunks * n * sizeof(int32_t));
+    ALLOC(W.offsets, (n + 1) * sizeof(int32_t));
+    ALLOC(W.dlist, n * sizeof(int32_t));
+    ALLOC(W.perm, slots * sizeof(int32_t));
+    ALLOC(W.slot_pos, slots * sizeof(int32_t));
+    ALLOC(W.meta, ace::kMetaCount * sizeof(int32_t));
+    ALLOC(W.act, slots * m * sizeof(float));
+    ALLOC(W.yslot, slots * d * sizeof(float));
+    ALLOC(W.err, sizeof(int));
+    ALLOC(W.x_stage, T * d * E);
+    ALLOC(W.out_stage, T * d * E);
+#undef ALLOC
+#define CK(call, where)                       \
+    do {                                      \
+        e = (call);                           \
+        if (e != cudaSuccess) {               \
+            free_layer(L);                    \
+            return cuda_fail(e, where);       \
+        }                                     \
+    } while (0)
+    CK(cudaMemcpyAsync(L->router_w, router_w, n * d * E, cudaMemcpyDeviceToDevice, s), "copy router_w");
+    if (D.has_router_bias)
+        CK(cudaMemcpyAsync(L->router_b, router_b, n * sizeof(float), cudaMemcpyDeviceToDevice, s), "copy router_b");
+    else
+        CK(cudaMemsetAsync(L->router_b, 0, n * sizeof(float), s), "zero router_b");
+    CK(cudaMemcpyAsync(L->w_gate, w_gate, n * m * d * E, cudaMemcpyDeviceToDevice, s), "copy w_gate");
+    CK(cudaMemcpyAsync(L->w_up, w_up, n * m * d * E, cudaMemcpyDeviceToDevice, s), "copy w_up");
+    CK(cudaMemcpyAsync(L->w_down, w_down, n * d * m * E, cudaMemcpyDeviceToDevice, s), "copy w_down");
+    CK(cudaMemcpyAsync(L->gamma, rms_gamma, d * E, cudaMemcpyDeviceToDevice, s), "copy gamma");
+    CK(cudaMemcpyAsync(L->a_gsp, a_gsp, n * sizeof(float), cudaMemcpyHostToDevice, s), "copy a_gsp");
+    CK(cudaMemcpyAsync(L->a_rcr, a_rcr, n * sizeof(float), cudaMemcpyHostToDevice, s), "copy a_rcr");
+    CK(cudaMemsetAsync(W.meta, 0, ace::kMetaCount * sizeof(int32_t), s), "zero meta");
+    CK(cudaMemsetAsync(W.err, 0, sizeof(int), s), "zero error word");
+    CK(cudaMemsetAsync(W.offsets, 0, (n + 1) * sizeof(int32_t), s), "zero offsets");
+    CK(ace::route_init(L), "route kernel attributes");
+    CK(ace::gemv_init(L), "gemv kernel attributes");
+    CK(cudaStreamSynchronize(s), "create: synchronize");
+#undef CK
+    *out_layer = L;
+    return ACE_OK;
+}
+
+void ace_layer_destroy(ace_layer* layer) {
+    if (!layer) return;
+    cudaDeviceSynchronize();
+    free_layer(layer);
+}
+
+ace_status ace_layer_get_desc(const ace_layer* layer, ace_layer_desc* desc) {
+    if (!layer || !desc) return fail(ACE_ERR_INVALID_ARG, "NULL argument");
+    *desc = layer->desc;
+    return ACE_OK;
+}
+
+ace_status ace_route_logits(ace_layer* L, const float* logits, int T, ace_skip_ctl ctl, void* stream) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    if (T < 0 || T > L->desc.max_tokens) return fail(ACE_ERR_INVALID_ARG, "T out of range [0, max_tokens]");
+    if (T > 0 && !logits) return fail(ACE_ERR_INVALID_ARG, "logits is NULL");
+    ace_status st = check_ctl(ctl);
+    if (st != ACE_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    L->last_T = T;
+    L->last_ctl = ctl;
+    L->last_stream = s;
+    L->last_has_logits = false;
+    if (T == 0) return ACE_OK;
+    ACE_CUDA(ace::launch_route(L, logits, T, ctl, s), "route launch");
+    return ACE_OK;
+}
+
+ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_skip_ctl ctl, void* stream) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    if (T < 0 || T > L->desc.max_tokens) return fail(ACE_ERR_INVALID_ARG, "T out of range [0, max_tokens]");
+    if (T > 0 && (!x || !out)) return fail(ACE_ERR_INVALID_ARG, "x and out must be non-NULL");
+    if (T > 0 && x == out) return fail(ACE_ERR_INVALID_ARG, "out must not alias x");
+    ace_status st = check_ctl(ctl);
+    if (st != ACE_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    L->last_T = T;
+    L->last_ctl = ctl;
+    L->last_stream = s;
+    L->last_has_logits = T > 0;
+    if (T == 0) return ACE_OK;
+    cudaEvent_t* ev = L->profiling ? L->ev : nullptr;
+    if (ev) ACE_CUDA(cudaEventRecord(ev[0], s), "event record");
+    ACE_CUDA(ace::launch_rmsnorm(L, x, T, s), "rmsnorm launch");
+    if (ev) ACE_CUDA(cudaEventRecord(ev[1], s), "event record");
+    ACE_CUDA(ace::launch_router(L, T, s), "router launch");
+    if (ev) ACE_CUDA(cudaEventRecord(ev[2], s), "event record");
+    ACE_CUDA(ace::launch_route(L, L->ws.logits, T, ctl, s), "route launch");
+    ACE_CUDA(ace::launch_experts_gemv(L, out, T, s, ev ? ev + 3 : nullptr), "expert launch");
+    L->n_stages = ev ? ace::kNumStages : 0;
+    return ACE_OK;
+}
+
+ace_status ace_moe_forward_host(ace_layer* L, const void* x_host, void* out_host, int T, ace_skip_ctl ctl,
+                                void* stream) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    if (T < 0 || T > L->desc.max_tokens) return fail(ACE_ERR_INVALID_ARG, "T out of range [0, max_tokens]");
+    if (T > 0 && (!x_host || !out_host)) return fail(ACE_ERR_INVALID_ARG, "x_host and out_host must be non-NULL");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t bytes = (size_t)T * L->desc.hidden * L->elem;
+    if (T > 0) ACE_CUDA(cudaMemcpyAsync(L->ws.x_stage, x_host, bytes, cudaMemcpyHostToDevice, s), "copy x to device");
+    ace_status st = ace_moe_forward(L, L->ws.x_stage, L->ws.out_stage, T, ctl, stream);
+    if (st != ACE_OK) return st;
+    if (T > 0)
+        ACE_CUDA(cudaMemcpyAsync(out_host, L->ws.out_stage, bytes, cudaMemcpyDeviceToHost, s), "copy out to host");
+    ACE_CUDA(cudaStreamSynchronize(s), "forward_host: synchronize");
+    return check_device_word(L);
+}
+
+ace_status ace_layer_sync(ace_layer* L) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    ACE_CUDA(cudaStreamSynchronize(L->last_stream), "synchronize");
+    return check_device_word(L);
+}
+
+ace_status ace_last_skip_mask(ace_layer* L, uint8_t* skip, int32_t* ids, float* gates_hat, float* tau,
+                              int32_t* retained) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    if (L->last_T < 0) return fail(ACE_ERR_STATE, "no forward or route call yet");
+    ACE_CUDA(cudaStreamSynchronize(L->last_stream), "synchronize");
+    ace_status st = check_device_word(L);
+    if (st != ACE_OK) return st;
+    const size_t slots = (size_t)L->last_T * L->desc.top_k;
+    if (L->last_T == 0) {
+        if (tau) *tau = L->last_ctl.mode == ACE_SKIP_THRESHOLD ? L->last_ctl.value : 0.f;
+        if (retained) *retained = 0;
+        return ACE_OK;
+    }
+    if (skip) ACE_CUDA(cudaMemcpy(skip, L->ws.skip, slots, cudaMemcpyDeviceToHost), "copy skip");
+    if (ids) ACE_CUDA(cudaMemcpy(ids, L->ws.ids, slots * 4, cudaMemcpyDeviceToHost), "copy ids");
+    if (gates_hat) ACE_CUDA(cudaMemcpy(gates_hat, L->ws.ghat, slots * 4, cudaMemcpyDeviceToHost), "copy ghat");
+    if (tau) ACE_CUDA(cudaMemcpy(tau, L->ws.tau, 4, cudaMemcpyDeviceToHost), "copy tau");
+    if (retained)
+        ACE_CUDA(cudaMemcpy(retained, L->ws.meta + ace::kMetaRetained, 4, cudaMemcpyDeviceToHost), "copy R");
+    return ACE_OK;
+}
+
+ace_status ace_last_router_logits(ace_layer* L, float* logits) {
+    if (!L || !logits) return fail(ACE_ERR_INVALID_ARG, "NULL argument");
+    if (L->last_T < 0 || !L->last_has_logits) return fail(ACE_ERR_STATE, "no forward with router logits yet");
+    ACE_CUDA(cudaStreamSynchronize(L->last_stream), "synchronize");
+    ACE_CUDA(cudaMemcpy(logits, L->ws.logits, (size_t)L->last_T * L->desc.n_experts * 4, cudaMemcpyDeviceToHost),
+             "copy logits");
+    return ACE_OK;
+}
+
+ace_status ace_last_permutation(ace_layer* L, int32_t* offsets, int32_t* perm) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    if (L->last_T < 0) return fail(ACE_ERR_STATE, "no forward or route call yet");
+    ACE_CUDA(cudaStreamSynchronize(L->last_stream), "synchronize");
+    const int n = L->desc.n_experts;
+    if (L->last_T == 0) {
+        if (offsets) memset(offsets, 0, (n + 1) * sizeof(int32_t));
+        return ACE_OK;
+    }
+    std::vector<int32_t> off(n + 1);
+    ACE_CUDA(cudaMemcpy(off.data(), L->ws.offsets, (n + 1) * 4, cudaMemcpyDeviceToHost), "copy offsets");
+    if (offsets) memcpy(offsets, off.data(), (n + 1) * 4);
+    if (perm && off[n] > 0)
+        ACE_CUDA(cudaMemcpy(perm, L->ws.perm, (size_t)off[n] * 4, cudaMemcpyDeviceToHost), "copy perm");
+    return ACE_OK;
+}
+
+ace_status ace_layer_set_profiling(ace_layer* L, int enable) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    if (enable && !L->ev[0]) {
+        for (int i = 0; i <= ace::kNumStages; ++i) ACE_CUDA(cudaEventCreate(&L->ev[i]), "event create");
+    }
+    L->profiling = enable != 0;
+    L->n_stages = 0;
+    return ACE_OK;
+}
+
+ace_status ace_last_stage_times(ace_layer* L, float* ms, int n_max, int* n_out) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    if (!L->profiling || L->n_stages == 0) return fail(ACE_ERR_STATE, "no profiled forward yet");
+    ACE_CUDA(cudaStreamSynchronize(L->last_stream), "synchronize");
+    const int n = L->n_stages < n_max ? L->n_stages : n_max;
+    for (int i = 0; i < n; ++i) ACE_CUDA(cudaEventElapsedTime(&ms[i], L->ev[i], L->ev[i + 1]), "elapsed time");
+    if (n_out) *n_out = L->n_stages;
+    return ACE_OK;
+}
+
+ace_status ace_debug_exp32(const float* x, float* y, int n, void* stream) {
+    if (n < 0 || (n > 0 && (!x || !y))) return fail(ACE_ERR_INVALID_ARG, "bad arguments");
+    if (n == 0) return ACE_OK;
+    ACE_CUDA(ace::launch_debug_exp(x, y, n, static_cast<cudaStream_t>(stream)), "exp launch");
+    return ACE_OK;
+}
+
+}  // extern "C"

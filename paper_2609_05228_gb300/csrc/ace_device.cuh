@@ -1,0 +1,101 @@
+// ace_device.cuh — device helpers shared by the library's kernels.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace ace {
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+__device__ __forceinline__ int warp_sum_int(int v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+__device__ __forceinline__ unsigned lanemask_lt() {
+    unsigned m;
+    asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+    return m;
+}
+
+// 16-byte vectors of the storage type, widened to float.
+template <typename T> struct Vec16;
+
+template <> struct Vec16<float> {
+    static constexpr int N = 4;
+    __device__ __forceinline__ static void to_float(const uint4& v, float* f) {
+        f[0] = __uint_as_float(v.x); f[1] = __uint_as_float(v.y);
+        f[2] = __uint_as_float(v.z); f[3] = __uint_as_float(v.w);
+    }
+};
+
+template <> struct Vec16<__nv_bfloat16> {
+    static constexpr int N = 8;
+    __device__ __forceinline__ static void to_float(const uint4& v, float* f) {
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            f[2 * i] = __uint_as_float(w[i] << 16);
+            f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+        }
+    }
+};
+
+__device__ __forceinline__ float to_f32(float v) { return v; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 v) { return __bfloat162float(v); }
+template <typename T> __device__ __forceinline__ T from_f32(float v);
+template <> __device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) {
+    return __float2bfloat16_rn(v);
+}
+
+// Streaming 16-byte load that does not allocate in L1 (weights are read once).
+__device__ __forceinline__ uint4 ld_stream(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+    return v;
+}
+
+// exp(x) for float32 x <= 0 in a fixed operation sequence (each multiply and
+// add rounded to nearest even, none fused), so that the gates are
+// reproducible bit for bit by any implementation following the same steps:
+//   n = rint(x * log2(e));  r = (x - n*ln2_hi) - n*ln2_lo   (Cody & Waite 1980,
+//   ln2_hi = 355/512 has 9 significant bits so n*ln2_hi is exact);
+//   p = sum_{j=0..7} r^j / j!  in Horner form;  result = p * 2^n.
+// Inputs below -87 return 0 (there 2^n would leave the normal range).
+__device__ __forceinline__ float ace_exp32(float x) {
+    const float kLog2e = 0x1.715476p+0f;     // float32(1 / ln 2)
+    const float kLn2Hi = 0x1.63p-1f;          // 355 / 512
+    const float kLn2Lo = -0x1.bd0106p-13f;    // float32(ln 2 - 355/512)
+    const float c7 = 0x1.a01a02p-13f;         // float32(1/5040)
+    const float c6 = 0x1.6c16c2p-10f;         // float32(1/720)
+    const float c5 = 0x1.111112p-7f;          // float32(1/120)
+    const float c4 = 0x1.555556p-5f;          // float32(1/24)
+    const float c3 = 0x1.555556p-3f;          // float32(1/6)
+    const float n = rintf(__fmul_rn(x, kLog2e));
+    float r = __fsub_rn(x, __fmul_rn(n, kLn2Hi));
+    r = __fsub_rn(r, __fmul_rn(n, kLn2Lo));
+    float p = c7;
+    p = __fadd_rn(__fmul_rn(p, r), c6);
+    p = __fadd_rn(__fmul_rn(p, r), c5);
+    p = __fadd_rn(__fmul_rn(p, r), c4);
+    p = __fadd_rn(__fmul_rn(p, r), c3);
+    p = __fadd_rn(__fmul_rn(p, r), 0.5f);
+    p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+    p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+    int ni = (int)n;
+    ni = ni < -126 ? -126 : (ni > 127 ? 127 : ni);
+    const float scale = __int_as_float((ni + 127) << 23);
+    const float out = __fmul_rn(p, scale);
+    return x < -87.0f ? 0.0f : out;
+}
+
+}  // namespace ace

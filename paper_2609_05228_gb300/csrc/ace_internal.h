@@ -1,0 +1,108 @@
+// ace_internal.h — layer object, workspace layout and kernel launchers of
+// libace.so. Host and device code of the library share it; nothing outside
+// csrc/ includes it.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "ace.h"
+
+namespace ace {
+
+// Device error word bits (ace_layer::ws.err).
+enum : int {
+    kErrNumeric = 1,   // a router logit was NaN / the gate sum was not finite
+    kErrTimeout = 2,   // a bounded device wait ran out
+    kErrBounds = 4,    // an index check failed (debug-style guard, access skipped)
+};
+
+// meta[] slots (int32, device): written by the compaction's last block.
+enum : int {
+    kMetaRetained = 0,     // R
+    kMetaTicket = 1,       // last-block ticket (reset by the last block)
+    kMetaDistinct = 2,     // D, experts with >= 1 retained slot
+    kMetaSlice1 = 3,       // gate/up GEMV: rows of m per work item
+    kMetaSlice2 = 4,       // down GEMV: rows of d per work item
+    kMetaTiles1 = 5,       // tensor-core GEMM 1 tiles
+    kMetaTiles2 = 6,       // tensor-core GEMM 2 tiles
+    kMetaTicket2 = 7,      // second ticket (expert kernels)
+    kMetaCount = 16,
+};
+
+constexpr int kChunk = 256;          // tokens per compaction block
+constexpr int kMaxExperts = 1024;
+constexpr int kMaxTopK = 16;
+constexpr int kGemvTokenChunk = 8;   // tokens processed per weight pass in the GEMVs
+
+struct Workspace {
+    void* h = nullptr;           // [Tmax, d] dtype: RMSNorm output
+    float* logits = nullptr;     // [Tmax, N]
+    int32_t* ids = nullptr;      // [Tmax, k] rank order
+    float* gates = nullptr;      // [Tmax, k] g
+    float* cval = nullptr;       // [Tmax, k] c = max(p_gsp, p_rcr)
+    uint32_t* keys = nullptr;    // [Tmax, k] ratio-mode candidate keys
+    uint8_t* skip = nullptr;     // [Tmax, k]
+    float* ghat = nullptr;       // [Tmax, k]
+    float* tau = nullptr;        // [1]
+    int32_t* chunk_counts = nullptr;  // [n_chunks, N] counts, then per-chunk bases
+    int32_t* offsets = nullptr;  // [N+1]
+    int32_t* dlist = nullptr;    // [N] distinct retained experts, increasing
+    int32_t* perm = nullptr;     // [Tmax*k]
+    int32_t* slot_pos = nullptr; // [Tmax*k] row of slot t*k+i in perm order, -1 if skipped
+    int32_t* meta = nullptr;     // [kMetaCount]
+    float* act = nullptr;        // [Tmax*k, m] fp32 (GEMV path)
+    float* yslot = nullptr;      // [Tmax*k, d] fp32 (GEMV path)
+    int* err = nullptr;          // device error word
+    void* x_stage = nullptr;     // [Tmax, d] dtype: host-API staging
+    void* out_stage = nullptr;   // [Tmax, d]
+};
+
+}  // namespace ace
+
+struct ace_layer {
+    ace_layer_desc desc;
+    int device = 0;
+    int num_sms = 0;
+    size_t elem = 2;             // bytes per element of dtype
+    // layer-owned weights
+    void* router_w = nullptr;    // [N, d]
+    float* router_b = nullptr;   // [N] (zeros when there is no bias)
+    void* w_gate = nullptr;      // [N, m, d]
+    void* w_up = nullptr;        // [N, m, d]
+    void* w_down = nullptr;      // [N, d, m]
+    void* gamma = nullptr;       // [d]
+    float* a_gsp = nullptr;      // [N]
+    float* a_rcr = nullptr;      // [N]
+    ace::Workspace ws;
+    // last call
+    int last_T = -1;
+    ace_skip_ctl last_ctl{0, 0.f};
+    cudaStream_t last_stream = nullptr;
+    bool last_has_logits = false;
+    // stage timing (ace_layer_set_profiling)
+    bool profiling = false;
+    cudaEvent_t ev[8] = {};
+    int n_stages = 0;
+};
+
+namespace ace {
+
+// ---- launchers (ace_route.cu) ----
+cudaError_t route_init(const ace_layer* L);   // per-layer kernel attributes
+cudaError_t launch_rmsnorm(const ace_layer* L, const void* x, int T, cudaStream_t s);
+cudaError_t launch_router(const ace_layer* L, int T, cudaStream_t s);
+// Runs top-k / gates / decision / threshold / compaction from ws.logits or `logits`.
+cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_skip_ctl ctl,
+                         cudaStream_t s);
+cudaError_t launch_debug_exp(const float* x, float* y, int n, cudaStream_t s);
+
+// ---- launchers (ace_expert_gemv.cu) ----
+// ev (nullable): events recorded before gate/up, before down, before combine, after combine.
+cudaError_t gemv_init(const ace_layer* L);
+cudaError_t launch_experts_gemv(const ace_layer* L, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
+
+constexpr int kNumStages = 6;
+
+}  // namespace ace

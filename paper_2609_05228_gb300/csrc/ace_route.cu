@@ -1,0 +1,542 @@
+// ace_route.cu — RMSNorm, router logits, top-k + gates, the Algorithm 4 skip
+// decision, the App. B.1 per-batch threshold and the compaction of retained
+// slots into per-expert groups.
+#include <math.h>
+
+#include "ace_device.cuh"
+#include "ace_internal.h"
+
+namespace ace {
+namespace {
+
+// --------------------------------------------------------------------------
+// RMSNorm (§3.1: expert and router input x = x_bar Gamma). One warp per token.
+// h = x / sqrt(mean(x^2) + rms_eps) * gamma, computed in float, stored as T.
+// --------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) k_rmsnorm(const T* __restrict__ x, const T* __restrict__ gamma,
+                                                 T* __restrict__ h, int n_tokens, int d, float rms_eps) {
+    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (warp >= n_tokens) return;
+    constexpr int V = Vec16<T>::N;
+    const T* xr = x + (size_t)warp * d;
+    float ss = 0.f;
+    for (int j = lane * V; j < d; j += 32 * V) {
+        float f[V];
+        Vec16<T>::to_float(*reinterpret_cast<const uint4*>(xr + j), f);
+#pragma unroll
+        for (int i = 0; i < V; ++i) ss = fmaf(f[i], f[i], ss);
+    }
+    ss = warp_sum(ss);
+    const float inv = 1.0f / sqrtf(ss / (float)d + rms_eps);
+    T* hr = h + (size_t)warp * d;
+    for (int j = lane * V; j < d; j += 32 * V) {
+        float f[V], gm[V];
+        Vec16<T>::to_float(*reinterpret_cast<const uint4*>(xr + j), f);
+        Vec16<T>::to_float(*reinterpret_cast<const uint4*>(gamma + j), gm);
+        T o[V];
+#pragma unroll
+        for (int i = 0; i < V; ++i) o[i] = from_f32<T>(f[i] * inv * gm[i]);
+        *reinterpret_cast<uint4*>(hr + j) = *reinterpret_cast<const uint4*>(o);
+    }
+}
+
+// --------------------------------------------------------------------------
+// Router logits z[t,e] = (h_t . w_e + b_e) / temp  (§3.2 logit). A block holds
+// kRouterTok token rows of h in shared memory; each warp takes experts
+// e = warp, warp + 8, ... and streams w_e once for all of them.
+// --------------------------------------------------------------------------
+constexpr int kRouterTok = 8;
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_router(const T* __restrict__ h, const T* __restrict__ w,
+                                                const float* __restrict__ b, float* __restrict__ z,
+                                                int n_tokens, int d, int n_exp, float inv_temp,
+                                                int use_temp) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    T* hs = reinterpret_cast<T*>(smem_raw);
+    const int t0 = blockIdx.x * kRouterTok;
+    const int nt = min(kRouterTok, n_tokens - t0);
+    constexpr int V = Vec16<T>::N;
+    const int nvec = d / V;
+    for (int i = threadIdx.x; i < kRouterTok * nvec; i += blockDim.x) {
+        const int r = i / nvec, c = i % nvec;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (r < nt) v = *reinterpret_cast<const uint4*>(h + (size_t)(t0 + r) * d + c * V);
+        reinterpret_cast<uint4*>(hs)[i] = v;
+    }
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int e = warp; e < n_exp; e += blockDim.x >> 5) {
+        float acc[kRouterTok];
+#pragma unroll
+        for (int r = 0; r < kRouterTok; ++r) acc[r] = 0.f;
+        const T* we = w + (size_t)e * d;
+        for (int c = lane; c < nvec; c += 32) {
+            float wf[V];
+            Vec16<T>::to_float(*reinterpret_cast<const uint4*>(we + c * V), wf);
+#pragma unroll
+            for (int r = 0; r < kRouterTok; ++r) {
+                float hf[V];
+                Vec16<T>::to_float(reinterpret_cast<const uint4*>(hs)[r * nvec + c], hf);
+#pragma unroll
+                for (int i = 0; i < V; ++i) acc[r] = fmaf(hf[i], wf[i], acc[r]);
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < kRouterTok; ++r) acc[r] = warp_sum(acc[r]);
+        if (lane < nt) {
+            float v = acc[0];
+#pragma unroll
+            for (int r = 1; r < kRouterTok; ++r) if (lane == r) v = acc[r];
+            v = v + b[e];
+            if (use_temp) v = v * inv_temp;
+            z[(size_t)(t0 + lane) * n_exp + e] = v;
+        }
+    }
+}
+
+// --------------------------------------------------------------------------
+// Per-token decision, float32 in a fixed operation order (Algorithm 4).
+// Lane i < k holds slot i (rank i). Every sum is taken sequentially in rank
+// order through shuffles, so all lanes hold identical totals.
+// --------------------------------------------------------------------------
+struct SlotScore {
+    float g;   // gate
+    float c;   // max(p_gsp, p_rcr)
+};
+
+// Gates and c for the slot held by this lane (lanes >= k return zeros).
+__device__ __forceinline__ SlotScore score_slot(int lane, int k, float z_i, float z_0, int id,
+                                                const float* __restrict__ a_gsp,
+                                                const float* __restrict__ a_rcr, float eps) {
+    const bool on = lane < k;
+    const float e_i = on ? ace_exp32(__fsub_rn(z_i, z_0)) : 0.f;
+    float s = __shfl_sync(0xffffffffu, e_i, 0);
+    for (int j = 1; j < k; ++j) s = __fadd_rn(s, __shfl_sync(0xffffffffu, e_i, j));
+    const float g = on ? __fdiv_rn(e_i, s) : 0.f;
+    const float sg = on ? __fmul_rn(g, a_gsp[id]) : 0.f;       // Eq. gsp_contribution
+    const float sr = on ? __fmul_rn(g, a_rcr[id]) : 0.f;       // Eq. rcr_contribution
+    float zg = __shfl_sync(0xffffffffu, sg, 0);
+    float zr = __shfl_sync(0xffffffffu, sr, 0);
+    for (int j = 1; j < k; ++j) {
+        zg = __fadd_rn(zg, __shfl_sync(0xffffffffu, sg, j));
+        zr = __fadd_rn(zr, __shfl_sync(0xffffffffu, sr, j));
+    }
+    zg = __fadd_rn(zg, eps);
+    zr = __fadd_rn(zr, eps);
+    const float pg = on ? __fdiv_rn(sg, zg) : 0.f;              // Eq. gsp_probability
+    const float pr = on ? __fdiv_rn(sr, zr) : 0.f;              // Eq. rcr_probability
+    return SlotScore{g, fmaxf(pg, pr)};                         // Eq. ace_contribution
+}
+
+// Skip flag and g_hat for the slot of this lane, given tau.
+__device__ __forceinline__ void decide_slot(int lane, int k, float g, float c, float tau, int m_min,
+                                            float eps, bool& skip_out, float& ghat_out) {
+    const bool on = lane < k;
+    // Eq. ace_candidate_intersection via max; slot 0 is the top-1 and is kept.
+    bool skip = on && lane != 0 && (c < tau);
+    const unsigned sk = __ballot_sync(0xffffffffu, skip);
+    const int active = k - __popc(sk);
+    if (active < m_min) {
+        // restore skipped slots in c-descending order, lower rank first on ties
+        int need = m_min - active;
+        unsigned rem = sk;
+        while (need > 0 && rem) {
+            float best = -1.f;
+            int bi = -1;
+            for (unsigned m = rem; m; m &= m - 1) {
+                const int j = __ffs(m) - 1;
+                const float cj = __shfl_sync(0xffffffffu, c, j);
+                if (bi < 0 || cj > best) { best = cj; bi = j; }
+            }
+            rem &= ~(1u << bi);
+            if (lane == bi) skip = false;
+            --need;
+        }
+    }
+    const unsigned keep = __ballot_sync(0xffffffffu, on && !skip);
+    float zs = 0.f;
+    for (int j = 0; j < k; ++j) {
+        const float gj = __shfl_sync(0xffffffffu, g, j);
+        if ((keep >> j) & 1u) zs = __fadd_rn(zs, gj);
+    }
+    zs = __fadd_rn(zs, eps);
+    skip_out = skip;
+    ghat_out = (on && !skip) ? __fdiv_rn(g, zs) : 0.f;
+}
+
+// Top-k over one token's logits (one warp). Lane l owns experts l, l+32, ...
+// Order: larger logit first; ties to the lower expert index. NaN ranks last.
+// On return lane i < k holds (id, z) of rank i.
+__device__ __forceinline__ void warp_topk(const float* __restrict__ zrow, int n_exp, int k, int lane,
+                                          int& my_id, float& my_z, bool& saw_nan) {
+    unsigned taken = 0u;   // bit j: expert lane + 32*j already chosen
+    my_id = -1;
+    my_z = 0.f;
+    saw_nan = false;
+    for (int r = 0; r < k; ++r) {
+        float bv = -INFINITY;
+        int bi = 0x7fffffff;
+        for (int j = 0, e = lane; e < n_exp; ++j, e += 32) {
+            if ((taken >> j) & 1u) continue;
+            float v = zrow[e];
+            if (v != v) { saw_nan = true; v = -INFINITY; }
+            if (v > bv || (v == bv && e < bi)) { bv = v; bi = e; }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+            if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
+        }
+        if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+        if (lane == r) { my_id = bi; my_z = bv; }
+    }
+}
+
+// Pass 1: top-k, gates, c. THRESHOLD mode also decides; RATIO mode writes
+// candidate keys (float bits of c, or 0xffffffff for protected slots).
+__global__ void __launch_bounds__(256) k_topk_score(const float* __restrict__ logits, int n_tokens,
+                                                    int n_exp, int k, const float* __restrict__ a_gsp,
+                                                    const float* __restrict__ a_rcr, float eps,
+                                                    int m_min, int mode, float tau,
+                                                    int32_t* __restrict__ ids, float* __restrict__ gates,
+                                                    float* __restrict__ cval, uint32_t* __restrict__ keys,
+                                                    uint8_t* __restrict__ skip, float* __restrict__ ghat,
+                                                    float* __restrict__ tau_out, int* __restrict__ err) {
+    if (mode == ACE_SKIP_THRESHOLD && blockIdx.x == 0 && threadIdx.x == 0) *tau_out = tau;
+    const int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (t >= n_tokens) return;
+    int id;
+    float zv;
+    bool nan;
+    warp_topk(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
+    const float z0 = __shfl_sync(0xffffffffu, zv, 0);
+    if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(err, kErrNumeric);
+    const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a_gsp, a_rcr, eps);
+    const size_t base = (size_t)t * k;
+    if (lane < k) {
+        ids[base + lane] = id;
+        gates[base + lane] = sc.g;
+        cval[base + lane] = sc.c;
+    }
+    if (mode == ACE_SKIP_THRESHOLD) {
+        bool sk;
+        float gh;
+        decide_slot(lane, k, sc.g, sc.c, tau, m_min, eps, sk, gh);
+        if (lane < k) {
+            skip[base + lane] = sk ? 1 : 0;
+            ghat[base + lane] = gh;
+        }
+    } else {
+        // protected: rank 0 and the (m_min-1) highest-c other slots
+        bool prot = lane == 0;
+        const int extra = min(m_min, k) - 1;
+        if (extra > 0) {
+            // other non-top-1 slots ahead of this one in (c desc, rank asc)
+            int better = 0;
+            for (int j = 1; j < k; ++j) {
+                const float cj = __shfl_sync(0xffffffffu, sc.c, j);
+                if (j != lane && (cj > sc.c || (cj == sc.c && j < lane))) ++better;
+            }
+            if (lane != 0 && better < extra) prot = true;
+        }
+        if (lane < k) keys[base + lane] = prot ? 0xffffffffu : __float_as_uint(sc.c);
+    }
+}
+
+// Pass 2 (ratio mode): decide from stored g, c and the device tau.
+__global__ void __launch_bounds__(256) k_decide(int n_tokens, int k, const float* __restrict__ gates,
+                                                const float* __restrict__ cval,
+                                                const float* __restrict__ tau_dev, int m_min, float eps,
+                                                uint8_t* __restrict__ skip, float* __restrict__ ghat) {
+    const int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (t >= n_tokens) return;
+    const size_t base = (size_t)t * k;
+    const float g = lane < k ? gates[base + lane] : 0.f;
+    const float c = lane < k ? cval[base + lane] : 0.f;
+    bool sk;
+    float gh;
+    decide_slot(lane, k, g, c, *tau_dev, m_min, eps, sk, gh);
+    if (lane < k) {
+        skip[base + lane] = sk ? 1 : 0;
+        ghat[base + lane] = gh;
+    }
+}
+
+// --------------------------------------------------------------------------
+// App. B.1 threshold for m candidates to skip: the (m+1)-th smallest
+// candidate key v (radix select over the non-negative float bits, 8 bits per
+// pass), lo = #{c < v}, hi = #{c <= v}; tau = v when lo == m or when lo is at
+// least as close to m as hi, else the next float above v. One block.
+// --------------------------------------------------------------------------
+constexpr int kSelThreads = 1024;
+
+__global__ void __launch_bounds__(kSelThreads) k_tau_select(const uint32_t* __restrict__ keys, int n,
+                                                            int m, float* __restrict__ tau_out) {
+    __shared__ int hist[32][256];
+    __shared__ int tot[256];
+    __shared__ uint32_t s_prefix;
+    __shared__ int s_want, s_below, s_last_cnt;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    uint32_t prefix = 0u, mask = 0u;
+    if (tid == 0) { s_want = m; s_below = 0; }
+    for (int pass = 0; pass < 4; ++pass) {
+        const int shift = 24 - 8 * pass;
+        for (int i = tid; i < 32 * 256; i += kSelThreads) (&hist[0][0])[i] = 0;
+        __syncthreads();
+        for (int i0 = 0; i0 < n; i0 += kSelThreads) {
+            const int i = i0 + tid;
+            const uint32_t key = i < n ? keys[i] : 0xffffffffu;
+            const bool in = key != 0xffffffffu && (key & mask) == prefix;
+            const int dg = (key >> shift) & 255;
+            const unsigned grp = __match_any_sync(0xffffffffu, in ? dg : -1);
+            if (in && (__ffs(grp) - 1) == (tid & 31)) atomicAdd(&hist[warp][dg], __popc(grp));
+        }
+        __syncthreads();
+        if (tid < 256) {
+            int s = 0;
+            for (int w = 0; w < 32; ++w) s += hist[w][tid];
+            tot[tid] = s;
+        }
+        __syncthreads();
+        if (tid == 0) {
+            int want = s_want, cum = 0, dg = 0;
+            for (; dg < 256; ++dg) {
+                if (cum + tot[dg] > want) break;
+                cum += tot[dg];
+            }
+            if (dg > 255) dg = 255;   // unreachable when m < #candidates
+            s_want = want - cum;
+            s_below += cum;
+            s_last_cnt = tot[dg];
+            s_prefix = prefix | ((uint32_t)dg << shift);
+        }
+        __syncthreads();
+        prefix = s_prefix;
+        mask |= 255u << shift;
+        __syncthreads();
+    }
+    if (tid == 0) {
+        const int lo = s_below, hi = s_below + s_last_cnt;
+        const uint32_t v = prefix;
+        float tau = __uint_as_float(v);
+        if (!(lo == m || (m - lo) <= (hi - m))) tau = __uint_as_float(v + 1u);
+        *tau_out = tau;
+    }
+}
+
+// --------------------------------------------------------------------------
+// Compaction (Algorithm 1 "evaluate only the experts indexed by I"): retained
+// slots grouped by expert, tokens increasing inside a group.
+// Pass A: per-chunk per-expert counts; the last block scans them into
+// offsets[N+1], per-chunk bases and the distinct-expert list.
+// Pass B: each chunk places its slots: rank within (chunk, expert) from a
+// per-expert token bitmap, so the order is deterministic.
+// --------------------------------------------------------------------------
+__global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, int n_exp, int n_chunks,
+                                                          const int32_t* __restrict__ ids,
+                                                          const uint8_t* __restrict__ skip,
+                                                          int32_t* __restrict__ chunk_counts,
+                                                          int32_t* __restrict__ offsets,
+                                                          int32_t* __restrict__ dlist,
+                                                          int32_t* __restrict__ meta, int d, int m,
+                                                          int target_items) {
+    __shared__ int cnt[kMaxExperts];
+    __shared__ bool is_last;
+    for (int e = threadIdx.x; e < n_exp; e += blockDim.x) cnt[e] = 0;
+    __syncthreads();
+    const int t = blockIdx.x * kChunk + threadIdx.x;
+    if (t < n_tokens) {
+        for (int i = 0; i < k; ++i)
+            if (!skip[(size_t)t * k + i]) atomicAdd(&cnt[ids[(size_t)t * k + i]], 1);
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < n_exp; e += blockDim.x)
+        chunk_counts[(size_t)blockIdx.x * n_exp + e] = cnt[e];
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) is_last = atomicAdd(&meta[kMetaTicket], 1) == n_chunks - 1;
+    __syncthreads();
+    if (!is_last) return;
+    __threadfence();
+    // last block: per-expert running bases over chunks, totals in cnt[]
+    for (int e = threadIdx.x; e < n_exp; e += blockDim.x) {
+        int run = 0;
+        for (int c = 0; c < n_chunks; ++c) {
+            volatile int32_t* p = chunk_counts + (size_t)c * n_exp + e;
+            const int v = *p;
+            *p = run;
+            run += v;
+        }
+        cnt[e] = run;
+    }
+    __syncthreads();
+    // exclusive scan of totals and of the distinct flags (warp 0)
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        const int per = (n_exp + 31) / 32;
+        const int e0 = min(lane * per, n_exp), e1 = min(e0 + per, n_exp);
+        int s = 0, dcount = 0;
+        for (int e = e0; e < e1; ++e) { s += cnt[e]; dcount += cnt[e] > 0; }
+        int xs = s, xd = dcount;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int ys = __shfl_up_sync(0xffffffffu, xs, o);
+            const int yd = __shfl_up_sync(0xffffffffu, xd, o);
+            if (lane >= o) { xs += ys; xd += yd; }
+        }
+        int run = xs - s, drun = xd - dcount;
+        for (int e = e0; e < e1; ++e) {
+            offsets[e] = run;
+            run += cnt[e];
+            if (cnt[e] > 0) dlist[drun++] = e;
+        }
+        const int total = __shfl_sync(0xffffffffu, xs, 31);
+        const int dtotal = __shfl_sync(0xffffffffu, xd, 31);
+        if (lane == 31) {
+            offsets[n_exp] = total;
+            meta[kMetaRetained] = total;
+            meta[kMetaDistinct] = dtotal;
+            // GEMV work-item sizes: rows per item, a power of two in [8, 128]
+            // dividing m (resp. d), so that D * rows/slice reaches the target.
+            int s1 = 128, s2 = 128;
+            while (s1 > 8 && (long long)dtotal * (m / s1) < target_items) s1 >>= 1;
+            while (s2 > 8 && (long long)dtotal * (d / s2) < target_items) s2 >>= 1;
+            while (m % s1) s1 >>= 1;
+            while (d % s2) s2 >>= 1;
+            meta[kMetaSlice1] = s1 < 1 ? 1 : s1;
+            meta[kMetaSlice2] = s2 < 1 ? 1 : s2;
+            meta[kMetaTicket] = 0;
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, int n_exp,
+                                                          const int32_t* __restrict__ ids,
+                                                          const uint8_t* __restrict__ skip,
+                                                          const int32_t* __restrict__ chunk_base,
+                                                          const int32_t* __restrict__ offsets,
+                                                          int32_t* __restrict__ perm,
+                                                          int32_t* __restrict__ slot_pos) {
+    constexpr int W = kChunk / 32;
+    __shared__ uint32_t bm[kMaxExperts * W];
+    for (int i = threadIdx.x; i < n_exp * W; i += blockDim.x) bm[i] = 0u;
+    __syncthreads();
+    const int t = blockIdx.x * kChunk + threadIdx.x;
+    const int w = threadIdx.x >> 5;
+    const unsigned bit = 1u << (threadIdx.x & 31);
+    if (t < n_tokens) {
+        for (int i = 0; i < k; ++i)
+            if (!skip[(size_t)t * k + i]) atomicOr(&bm[ids[(size_t)t * k + i] * W + w], bit);
+    }
+    __syncthreads();
+    if (t < n_tokens) {
+        const unsigned lt = lanemask_lt();
+        for (int i = 0; i < k; ++i) {
+            const size_t s = (size_t)t * k + i;
+            if (skip[s]) { slot_pos[s] = -1; continue; }
+            const int e = ids[s];
+            int rank = __popc(bm[e * W + w] & lt);
+            for (int ww = 0; ww < w; ++ww) rank += __popc(bm[e * W + ww]);
+            const int r = offsets[e] + chunk_base[(size_t)blockIdx.x * n_exp + e] + rank;
+            perm[r] = (int32_t)s;
+            slot_pos[s] = r;
+        }
+    }
+}
+
+__global__ void k_debug_exp(const float* __restrict__ x, float* __restrict__ y, int n) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) y[i] = ace_exp32(x[i]);
+}
+
+inline int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }
+
+}  // namespace
+
+cudaError_t launch_rmsnorm(const ace_layer* L, const void* x, int T, cudaStream_t s) {
+    const int d = L->desc.hidden;
+    const int blocks = cdiv(T, 8);
+    if (L->desc.dtype == ACE_BF16)
+        k_rmsnorm<__nv_bfloat16><<<blocks, 256, 0, s>>>(
+            (const __nv_bfloat16*)x, (const __nv_bfloat16*)L->gamma, (__nv_bfloat16*)L->ws.h, T, d,
+            L->desc.rms_eps);
+    else
+        k_rmsnorm<float><<<blocks, 256, 0, s>>>((const float*)x, (const float*)L->gamma,
+                                                (float*)L->ws.h, T, d, L->desc.rms_eps);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_router(const ace_layer* L, int T, cudaStream_t s) {
+    const int d = L->desc.hidden, n = L->desc.n_experts;
+    const size_t smem = (size_t)kRouterTok * d * L->elem;
+    const float temp = L->desc.router_temp;
+    const int use_temp = temp != 1.0f;
+    const int blocks = cdiv(T, kRouterTok);
+    if (L->desc.dtype == ACE_BF16) {
+        k_router<__nv_bfloat16><<<blocks, 256, smem, s>>>((const __nv_bfloat16*)L->ws.h, (const __nv_bfloat16*)L->router_w,
+                                      L->router_b, L->ws.logits, T, d, n, 1.0f / temp, use_temp);
+    } else {
+        k_router<float><<<blocks, 256, smem, s>>>((const float*)L->ws.h, (const float*)L->router_w, L->router_b,
+                                      L->ws.logits, T, d, n, 1.0f / temp, use_temp);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_skip_ctl ctl,
+                         cudaStream_t s) {
+    const ace_layer_desc& D = L->desc;
+    const Workspace& W = L->ws;
+    const int k = D.top_k, n = D.n_experts;
+    const int blocks = cdiv(T, 8);
+    float tau = ctl.value;
+    bool need_select = false;
+    int m_q = 0;
+    if (ctl.mode == ACE_SKIP_RATIO) {
+        const long long n_all = (long long)T * k;
+        const int prot = D.min_active < 1 ? 1 : (D.min_active > k ? k : D.min_active);
+        const long long n_cand = (long long)T * (k - prot);
+        long long mq = llround((double)ctl.value * (double)n_all);
+        if (mq < 0) mq = 0;
+        if (mq > n_cand) mq = n_cand;
+        m_q = (int)mq;
+        if (m_q == 0) tau = 0.0f;
+        else if (m_q == n_cand) tau = INFINITY;
+        else need_select = true;
+    }
+    const int mode = (ctl.mode == ACE_SKIP_RATIO && need_select) ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
+    k_topk_score<<<blocks, 256, 0, s>>>(logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode,
+                                        tau, W.ids, W.gates, W.cval, W.keys, W.skip, W.ghat, W.tau, W.err);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    if (mode == ACE_SKIP_RATIO) {
+        k_tau_select<<<1, kSelThreads, 0, s>>>(W.keys, T * k, m_q, W.tau);
+        k_decide<<<blocks, 256, 0, s>>>(T, k, W.gates, W.cval, W.tau, D.min_active, D.eps, W.skip, W.ghat);
+    }
+    const int n_chunks = cdiv(T, kChunk);
+    const int target = 4 * L->num_sms;
+    k_compact_count<<<n_chunks, kChunk, 0, s>>>(T, k, n, n_chunks, W.ids, W.skip, W.chunk_counts,
+                                                W.offsets, W.dlist, W.meta, D.hidden, D.ffn, target);
+    k_compact_place<<<n_chunks, kChunk, 0, s>>>(T, k, n, W.ids, W.skip, W.chunk_counts, W.offsets,
+                                                W.perm, W.slot_pos);
+    return cudaGetLastError();
+}
+
+cudaError_t route_init(const ace_layer* L) {
+    const size_t smem = (size_t)kRouterTok * L->desc.hidden * L->elem;
+    cudaError_t e = cudaFuncSetAttribute(k_router<__nv_bfloat16>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(k_router<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+}
+
+cudaError_t launch_debug_exp(const float* x, float* y, int n, cudaStream_t s) {
+    k_debug_exp<<<cdiv(n, 256), 256, 0, s>>>(x, y, n);
+    return cudaGetLastError();
+}
+
+}  // namespace ace

@@ -1,0 +1,56 @@
+"""The C-ABI library loads without a GPU and exports every symbol that
+include/ace.h declares; argument checks that need no device run too."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_05228_gb300 import ace, build
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "ace.h")
+
+
+@pytest.fixture(scope="module")
+def libace():
+    if not os.path.exists(ace.LIBPATH):
+        build.build()
+    return ctypes.CDLL(ace.LIBPATH)
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(ace_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ["ace_layer_create", "ace_moe_forward", "ace_last_skip_mask", "ace_layer_destroy",
+                     "ace_route_logits", "ace_moe_forward_host", "ace_last_permutation",
+                     "ace_last_router_logits", "ace_status_string", "ace_last_error_message"]:
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(libace):
+    missing = [n for n in declared_functions() if not hasattr(libace, n)]
+    assert not missing, missing
+
+
+def test_host_side_argument_checks(libace):
+    ace._lib = None
+    L = ace.lib()
+    assert L.ace_status_string(0) == b"ACE_OK"
+    assert L.ace_status_string(5) == b"ACE_ERR_TIMEOUT"
+    # NULL descriptor / bad sizes are rejected before any device call
+    out = ctypes.c_void_p()
+    st = L.ace_layer_create(None, None, None, None, None, None, None, None, None, None, ctypes.byref(out))
+    assert st == 1
+    d = ace.ace_layer_desc(64, 8, 9, 64, 16, ace.ACE_BF16, 1e-6, 1e-6, 1.0, 1, 0)   # k > N
+    st = L.ace_layer_create(ctypes.byref(d), 1, None, 1, 1, 1, 1, 1, 1, None, ctypes.byref(out))
+    assert st == 1 and b"top_k" in L.ace_last_error_message()
+    d = ace.ace_layer_desc(100, 8, 2, 64, 16, ace.ACE_BF16, 1e-6, 1e-6, 1.0, 1, 0)  # d % 64
+    st = L.ace_layer_create(ctypes.byref(d), 1, None, 1, 1, 1, 1, 1, 1, None, ctypes.byref(out))
+    assert st == 2
+    assert L.ace_moe_forward(None, None, None, 1, ace.ace_skip_ctl(0, 0.1), None) == 1
+    assert L.ace_last_skip_mask(None, None, None, None, None, None) == 1

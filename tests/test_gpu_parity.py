@@ -1,0 +1,276 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle on
+the same seeded inputs.
+
+* exp32 and the whole decision (top-k ids, skip mask, g_hat, tau, retained
+  count, offsets, permutation) are bit-exact against the oracle's float32
+  decision spec, given the same float32 logits from the input generator.
+* The full layer is compared with the fp64 oracle: rel-L2 <= 5e-3 and
+  max-abs <= 3e-2 * max|ref| (bf16), on every token whose routing is not
+  within rounding distance of a decision boundary (top-k logit gap and
+  |c - tau|); those boundary tokens are counted and must stay a minority.
+"""
+import math
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import oracle as O
+from paper_2609_05228_gb300 import ace, offline, synth
+
+pytestmark = pytest.mark.gpu
+
+RTOL_L2 = 5e-3
+RTOL_MAX = 3e-2
+RTOL_L2_F32 = 1e-5
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    ace.lib()
+    yield
+
+
+def _dev(a):
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint16:
+        return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).cuda()
+    return torch.from_numpy(a).cuda()
+
+
+def _host(t):
+    if t.dtype == torch.bfloat16:
+        return (t.view(torch.int16).cpu().numpy().view(np.uint16).astype(np.uint32) << 16).view(np.float32)
+    return t.cpu().numpy()
+
+
+# ------------------------------------------------------------------ exp32
+
+
+def test_exp32_bitexact():
+    x = np.concatenate([np.linspace(-90.0, 0.0, 1 << 20).astype(np.float32),
+                        -np.abs(synth.make_logits(512, 512, seed=5).ravel()),
+                        np.array([0.0, -0.0, -1e-30, -87.0, -86.99999], np.float32)])
+    xd = torch.from_numpy(x).cuda()
+    yd = torch.empty_like(xd)
+    ace.ace_debug_exp32(xd, yd, x.size)
+    torch.cuda.synchronize()
+    want = O.exp32(x)
+    got = yd.cpu().numpy()
+    bad = np.nonzero(got.view(np.uint32) != want.view(np.uint32))[0]
+    assert bad.size == 0, (x[bad[:5]], got[bad[:5]], want[bad[:5]])
+
+
+# ------------------------------------------------------------------ decision bits
+
+
+def _route_layer(N, k, max_tokens, m_min, tables):
+    d = m = 64
+    z16 = np.zeros(1, np.uint16)
+    w = synth.LayerWeights(synth.LayerSpec(d, N, k, m, dtype="bf16", min_active=m_min),
+                           np.zeros((N, d), np.uint16), np.zeros(N, np.float32),
+                           np.zeros((N, m, d), np.uint16), np.zeros((N, m, d), np.uint16),
+                           np.zeros((N, d, m), np.uint16), np.full(d, 0x3f80, np.uint16))
+    del z16
+    return ace.AceLayer(w, tables[0], tables[1], max_tokens)
+
+
+ROUTE_CASES = [
+    # T, N, k, m_min
+    (1, 16, 4, 1),
+    (3, 128, 8, 1),
+    (64, 128, 8, 1),
+    (257, 100, 6, 2),
+    (4096, 128, 8, 1),
+    (2048, 256, 8, 3),
+    (1000, 1024, 16, 1),
+    (16384, 128, 8, 1),
+]
+CTLS = [("threshold", 0.0), ("threshold", 0.09), ("threshold", 0.12), ("threshold", math.inf),
+        ("ratio", 0.0), ("ratio", 0.25), ("ratio", 0.5), ("ratio", 0.625), ("ratio", 1.0)]
+
+
+@pytest.mark.parametrize("T,N,k,m_min", ROUTE_CASES)
+def test_decision_bitexact(T, N, k, m_min):
+    z = synth.make_logits(T, N, seed=100 + T + N, tie_fraction=0.05)
+    tables = synth.make_tables(N, seed=7 + N, spread=0.2)
+    layer = _route_layer(N, k, T, m_min, tables)
+    zd = torch.from_numpy(z).cuda()
+    ids_ref, g_ref = O.route_fp32(z, k)
+    for mode, val in CTLS:
+        ace.ace_route_logits(layer.handle, zd, T, mode, val)
+        skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, k)
+        ref = O.decide_fp32(ids_ref, g_ref, tables[0], tables[1], mode, val, m_min, 1e-6)
+        assert (ids == ids_ref).all(), (mode, val)
+        assert (skip.astype(bool) == ref["skip"]).all(), (mode, val, int(skip.sum()), int(ref["skip"].sum()))
+        assert (gh.view(np.uint32) == ref["g_hat"].view(np.uint32)).all(), (mode, val)
+        assert np.float32(tau).view(np.uint32) == np.float32(ref["tau"]).view(np.uint32), (mode, val, tau, ref["tau"])
+        assert R == int((~ref["skip"]).sum())
+        if mode == "ratio":
+            assert T * k - R == ref["count"]
+        off, perm = ace.ace_last_permutation(layer.handle, N, R)
+        off_ref, perm_ref = O.permutation(ids_ref, ref["skip"], N)
+        assert (off == off_ref).all() and (perm == perm_ref).all(), (mode, val)
+    layer.close()
+
+
+def test_decision_repeatable():
+    T, N, k = 4096, 128, 8
+    z = synth.make_logits(T, N, seed=3)
+    tables = synth.make_tables(N, seed=1, spread=0.2)
+    layer = _route_layer(N, k, T, 1, tables)
+    zd = torch.from_numpy(z).cuda()
+    first = None
+    for _ in range(20):
+        ace.ace_route_logits(layer.handle, zd, T, "ratio", 0.5)
+        skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, k)
+        off, perm = ace.ace_last_permutation(layer.handle, N, R)
+        cur = (skip.tobytes(), gh.tobytes(), perm.tobytes())
+        if first is None:
+            first = cur
+        assert cur == first
+    layer.close()
+
+
+# ------------------------------------------------------------------ full layer
+
+_LAYERS = {}
+
+
+def _layer(kind):
+    if kind not in _LAYERS:
+        if kind == "tiny":
+            spec, seed = synth.spec_tiny(), 0
+        elif kind == "qwen":
+            spec, seed = synth.spec_qwen(), 0
+        elif kind == "qwen_zipf":
+            spec, seed = synth.spec_qwen(zipf=True), 0
+        else:
+            raise KeyError(kind)
+        w = synth.make_layer(spec, seed)
+        a_gsp, a_rcr = offline.tables(w)
+        w.extra["a_gsp"], w.extra["a_rcr"] = a_gsp, a_rcr
+        _LAYERS[kind] = (w, ace.AceLayer(w, a_gsp, a_rcr, max_tokens=4096))
+    return _LAYERS[kind]
+
+
+def _clear_tokens(dec, z_ref, k, dz, dc):
+    """Tokens whose top-k set, top-1 and every skip decision sit farther from
+    a boundary than the GPU's rounding can move them. bf16 h rounding moves a
+    logit by about 1e-3 (std) and c by about 1.5e-3 relative, so the bf16
+    margins are dz = 6e-3 and dc = 8e-3; fp32 uses 1e-4."""
+    zs = np.sort(z_ref, axis=1)[:, ::-1]
+    gap_k = zs[:, k - 1] - zs[:, k] if z_ref.shape[1] > k else np.full(z_ref.shape[0], np.inf)
+    gap_1 = zs[:, 0] - zs[:, 1]
+    tau = dec["tau"]
+    if math.isinf(tau) or tau == 0:
+        c_ok = np.ones(z_ref.shape[0], bool)
+    else:
+        c_ok = (np.abs(dec["c"] - tau) > dc * tau).all(axis=1)
+    return (gap_k > dz) & (gap_1 > dz) & c_ok
+
+
+def _run_layer(kind, T, mode, val, x_seed=1):
+    w, layer = _layer(kind)
+    spec = w.spec
+    x = synth.make_tokens(spec, T, seed=x_seed)
+    xd = _dev(x)
+    out = torch.empty_like(xd)
+    layer.forward(xd, out, T, mode, val)
+    torch.cuda.synchronize()
+    skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, spec.top_k)
+    y_gpu = _host(out).astype(np.float64)
+    y_ref, dec = O.moe_forward(x, w, mode, val, return_decision=True)
+    h = O.rmsnorm(x, w.gamma, spec.rms_eps)
+    z_ref = O.router_logits(h, w.router_w, w.router_b, spec.router_temp)
+    return w, spec, x, y_gpu, y_ref, dec, z_ref, (skip, ids, gh, tau, R)
+
+
+FORWARD_CASES = [
+    ("tiny", 64, "ratio", 0.0), ("tiny", 64, "ratio", 0.25), ("tiny", 64, "ratio", 0.5),
+    ("tiny", 64, "threshold", 0.2), ("tiny", 5, "ratio", 0.5),
+    ("qwen", 1, "ratio", 0.5), ("qwen", 8, "ratio", 0.25), ("qwen", 32, "ratio", 0.5),
+    ("qwen", 64, "ratio", 0.0), ("qwen", 64, "ratio", 0.25), ("qwen", 64, "ratio", 0.5),
+    ("qwen", 17, "threshold", 0.11), ("qwen", 129, "ratio", 0.5), ("qwen", 1000, "ratio", 0.625),
+    ("qwen_zipf", 4096, "ratio", 0.0), ("qwen_zipf", 4096, "ratio", 0.5),
+]
+
+
+@pytest.mark.parametrize("kind,T,mode,val", FORWARD_CASES)
+def test_forward_parity(kind, T, mode, val):
+    w, spec, x, y_gpu, y_ref, dec, z_ref, (skip, ids, gh, tau, R) = _run_layer(kind, T, mode, val)
+    k = spec.top_k
+    margin = 1e-4 if spec.dtype == "f32" else None
+    clear = _clear_tokens(dec, z_ref, k, margin or 6e-3, margin or 8e-3)
+    assert clear.mean() >= 0.6 or clear.sum() >= T - 1, clear.mean()
+    # decisions agree on every clear token (compared per expert id)
+    for t in np.nonzero(clear)[0]:
+        gpu = {int(ids[t, i]): bool(skip[t, i]) for i in range(k)}
+        ref = {int(dec["ids"][t, i]): bool(dec["skip"][t, i]) for i in range(k)}
+        assert gpu == ref, t
+    if mode == "ratio":
+        n_all = T * k
+        m_q = min(O.llround_pos(float(np.float32(val)) * n_all), T * (k - 1))
+        assert n_all - R == m_q
+    yr, yg = y_ref[clear], y_gpu[clear]
+    rel = np.linalg.norm(yg - yr) / max(np.linalg.norm(yr), 1e-30)
+    mx = np.abs(yg - yr).max() / max(np.abs(yr).max(), 1e-30)
+    if spec.dtype == "f32":
+        assert rel <= RTOL_L2_F32, rel
+    else:
+        assert rel <= RTOL_L2, rel
+        assert mx <= RTOL_MAX, mx
+
+
+def test_forward_q0_matches_threshold0():
+    w, layer = _layer("qwen")
+    T = 64
+    x = _dev(synth.make_tokens(w.spec, T, seed=3))
+    o1 = torch.empty_like(x)
+    o2 = torch.empty_like(x)
+    layer.forward(x, o1, T, "ratio", 0.0)
+    layer.forward(x, o2, T, "threshold", 0.0)
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2)
+
+
+def test_forward_deterministic_and_host_api():
+    w, layer = _layer("qwen")
+    T = 64
+    xh = synth.make_tokens(w.spec, T, seed=4)
+    x = _dev(xh)
+    outs = []
+    for _ in range(3):
+        o = torch.empty_like(x)
+        layer.forward(x, o, T, "ratio", 0.5)
+        outs.append(o)
+    torch.cuda.synchronize()
+    assert all(torch.equal(outs[0], o) for o in outs[1:])
+    host_out = np.zeros_like(xh)
+    ace.ace_moe_forward_host(layer.handle, xh, host_out, T, "ratio", 0.5)
+    dev_out = outs[0].view(torch.int16).cpu().numpy().view(np.uint16)
+    assert (host_out == dev_out).all()
+
+
+def test_forward_edge_cases():
+    w, layer = _layer("qwen")
+    x = _dev(synth.make_tokens(w.spec, 4, seed=5))
+    out = torch.empty_like(x)
+    layer.forward(x, out, 0, "ratio", 0.5)          # T = 0 is a no-op
+    with pytest.raises(ace.AceError) as e:
+        layer.forward(x, out, 5000, "ratio", 0.5)   # beyond max_tokens
+    assert e.value.status == 1
+    with pytest.raises(ace.AceError):
+        layer.forward(x, out, 4, "ratio", 1.5)
+    with pytest.raises(ace.AceError):
+        layer.forward(x, out, 4, "threshold", float("nan"))
+    with pytest.raises(ace.AceError):
+        layer.forward(x, x, 4, "ratio", 0.5)        # aliasing
+    # tau = +inf keeps only the top-1 expert of every token
+    layer.forward(x, out, 4, "threshold", math.inf)
+    skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, 4, w.spec.top_k)
+    assert R == 4 and (skip[:, 0] == 0).all() and (skip[:, 1:] == 1).all()
+    ace.ace_layer_sync(layer.handle)
