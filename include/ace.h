@@ -189,6 +189,9 @@ ace_status ace_debug_exp32(const float* x, float* y, int n, void* stream);
 ace_status ace_layer_set_profiling(ace_layer* layer, int enable);
 ace_status ace_last_stage_times(ace_layer* layer, float* ms, int n_max, int* n_out);
 
+/* Number of kernels the last forward / route call launched (instrumentation). */
+ace_status ace_last_launch_count(const ace_layer* layer, int* n_kernels);
+
 /* Fills *desc with the layer's descriptor (after defaults were applied). */
 ace_status ace_layer_get_desc(const ace_layer* layer, ace_layer_desc* desc);
 

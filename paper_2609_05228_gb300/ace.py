@@ -67,6 +67,7 @@ def lib() -> ctypes.CDLL:
             "ace_layer_get_desc": (_S, [_P, ctypes.POINTER(ace_layer_desc)]),
             "ace_layer_set_profiling": (_S, [_P, _I]),
             "ace_last_stage_times": (_S, [_P, _P, _I, _P]),
+            "ace_last_launch_count": (_S, [_P, _P]),
             "ace_status_string": (ctypes.c_char_p, [_S]),
             "ace_last_error_message": (ctypes.c_char_p, []),
         }
@@ -183,6 +184,12 @@ def ace_last_stage_times(layer: int) -> dict:
     n = np.zeros(1, np.int32)
     _check(lib().ace_last_stage_times(layer, ms.ctypes.data, 16, n.ctypes.data))
     return {STAGES[i] if i < len(STAGES) else f"stage{i}": float(ms[i]) for i in range(int(n[0]))}
+
+
+def ace_last_launch_count(layer: int) -> int:
+    n = np.zeros(1, np.int32)
+    _check(lib().ace_last_launch_count(layer, n.ctypes.data))
+    return int(n[0])
 
 
 def ace_layer_get_desc(layer: int) -> ace_layer_desc:

@@ -233,8 +233,10 @@ ace_status ace_route_logits(ace_layer* L, const float* logits, int T, ace_skip_c
     L->last_ctl = ctl;
     L->last_stream = s;
     L->last_has_logits = false;
+    L->last_launches = 0;
     if (T == 0) return ACE_OK;
     ACE_CUDA(ace::launch_route(L, logits, T, ctl, s), "route launch");
+    L->last_launches = ace::route_launch_count(L, T, ctl);
     return ACE_OK;
 }
 
@@ -250,16 +252,19 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
     L->last_ctl = ctl;
     L->last_stream = s;
     L->last_has_logits = T > 0;
+    L->last_launches = 0;
     if (T == 0) return ACE_OK;
     cudaEvent_t* ev = L->profiling ? L->ev : nullptr;
+    const bool small = ace::small_path(T);
     if (ev) ACE_CUDA(cudaEventRecord(ev[0], s), "event record");
-    ACE_CUDA(ace::launch_rmsnorm(L, x, T, s), "rmsnorm launch");
+    if (!small) ACE_CUDA(ace::launch_rmsnorm(L, x, T, s), "rmsnorm launch");
     if (ev) ACE_CUDA(cudaEventRecord(ev[1], s), "event record");
-    ACE_CUDA(ace::launch_router(L, T, s), "router launch");
+    ACE_CUDA(ace::launch_router(L, x, T, small, s), "router launch");
     if (ev) ACE_CUDA(cudaEventRecord(ev[2], s), "event record");
     ACE_CUDA(ace::launch_route(L, L->ws.logits, T, ctl, s), "route launch");
     ACE_CUDA(ace::launch_experts_gemv(L, out, T, s, ev ? ev + 3 : nullptr), "expert launch");
     L->n_stages = ev ? ace::kNumStages : 0;
+    L->last_launches = (small ? 1 : 2) + ace::route_launch_count(L, T, ctl) + 3;
     return ACE_OK;
 }
 
@@ -350,6 +355,12 @@ ace_status ace_last_stage_times(ace_layer* L, float* ms, int n_max, int* n_out) 
     const int n = L->n_stages < n_max ? L->n_stages : n_max;
     for (int i = 0; i < n; ++i) ACE_CUDA(cudaEventElapsedTime(&ms[i], L->ev[i], L->ev[i + 1]), "elapsed time");
     if (n_out) *n_out = L->n_stages;
+    return ACE_OK;
+}
+
+ace_status ace_last_launch_count(const ace_layer* L, int* n_kernels) {
+    if (!L || !n_kernels) return fail(ACE_ERR_INVALID_ARG, "NULL argument");
+    *n_kernels = L->last_launches;
     return ACE_OK;
 }
 

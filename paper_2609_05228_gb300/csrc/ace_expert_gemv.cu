@@ -22,6 +22,15 @@ constexpr int kTC = kGemvTokenChunk;
 
 __device__ __forceinline__ float silu(float u) { return u / (1.0f + expf(-u)); }
 
+// Rows [lo, hi) of the flattened (distinct expert, weight row) space owned by
+// this block: every block streams the same number of weight rows.
+__device__ __forceinline__ void block_range(long long total, long long& lo, long long& hi) {
+    lo = total * blockIdx.x / gridDim.x;
+    hi = total * (blockIdx.x + 1) / gridDim.x;
+}
+
+// gate/up: one warp per row pair (W_gate[e, j], W_up[e, j]); each lane issues
+// up to kCh 16-byte loads of each row before the dot products.
 template <typename T>
 __global__ void __launch_bounds__(256) k_gemv_gateup(const T* __restrict__ h, const T* __restrict__ w_gate,
                                                      const T* __restrict__ w_up,
@@ -30,52 +39,61 @@ __global__ void __launch_bounds__(256) k_gemv_gateup(const T* __restrict__ h, co
                                                      const int32_t* __restrict__ perm,
                                                      const int32_t* __restrict__ meta,
                                                      float* __restrict__ act, int d, int m, int k) {
+    constexpr int kCh = 8;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     uint4* hs = reinterpret_cast<uint4*>(smem_raw);     // [kTC][d / V] vectors
     constexpr int V = Vec16<T>::N;
     const int nvec = d / V;
     const int D = meta[kMetaDistinct];
-    const int S = meta[kMetaSlice1];
-    const int nsl = m / S;
-    const int items = D * nsl;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
-    for (int item = blockIdx.x; item < items; item += gridDim.x) {
-        const int e = dlist[item / nsl];
-        const int sl = item % nsl;
+    long long lo, hi;
+    block_range((long long)D * m, lo, hi);
+    while (lo < hi) {
+        const int e = dlist[lo / m];
+        const int rb = (int)(lo % m);
+        const int re = (int)min((long long)m, rb + (hi - lo));
         const int r0 = offsets[e], ne = offsets[e + 1] - r0;
         for (int tc0 = 0; tc0 < ne; tc0 += kTC) {
             const int ntc = min(kTC, ne - tc0);
             __syncthreads();
-            for (int i = threadIdx.x; i < kTC * nvec; i += blockDim.x) {
+            for (int i = threadIdx.x; i < ntc * nvec; i += blockDim.x) {
                 const int q = i / nvec, c = i % nvec;
-                uint4 v = make_uint4(0, 0, 0, 0);
-                if (q < ntc) {
-                    const int tok = perm[r0 + tc0 + q] / k;
-                    v = reinterpret_cast<const uint4*>(h + (size_t)tok * d)[c];
-                }
-                hs[i] = v;
+                const int tok = perm[r0 + tc0 + q] / k;
+                hs[i] = reinterpret_cast<const uint4*>(h + (size_t)tok * d)[c];
             }
             __syncthreads();
-            for (int row = warp; row < S; row += nwarps) {
-                const int j = sl * S + row;
+            for (int j = rb + warp; j < re; j += nwarps) {
                 const uint4* wg = reinterpret_cast<const uint4*>(w_gate + ((size_t)e * m + j) * d);
                 const uint4* wu = reinterpret_cast<const uint4*>(w_up + ((size_t)e * m + j) * d);
                 float ag[kTC], au[kTC];
 #pragma unroll
                 for (int q = 0; q < kTC; ++q) { ag[q] = 0.f; au[q] = 0.f; }
-                for (int c = lane; c < nvec; c += 32) {
-                    float fg[V], fu[V];
-                    Vec16<T>::to_float(ld_stream(wg + c), fg);
-                    Vec16<T>::to_float(ld_stream(wu + c), fu);
+                for (int c0 = 0; c0 < nvec; c0 += 32 * kCh) {
+                    uint4 vg[kCh], vu[kCh];
 #pragma unroll
-                    for (int q = 0; q < kTC; ++q) {
-                        if (q < ntc) {
-                            float fh[V];
-                            Vec16<T>::to_float(hs[q * nvec + c], fh);
+                    for (int i = 0; i < kCh; ++i) {
+                        const int c = c0 + lane + 32 * i;
+                        const bool ok = c < nvec;
+                        vg[i] = ok ? ld_stream(wg + c) : make_uint4(0, 0, 0, 0);
+                        vu[i] = ok ? ld_stream(wu + c) : make_uint4(0, 0, 0, 0);
+                    }
 #pragma unroll
-                            for (int i = 0; i < V; ++i) {
-                                ag[q] = fmaf(fh[i], fg[i], ag[q]);
-                                au[q] = fmaf(fh[i], fu[i], au[q]);
+                    for (int i = 0; i < kCh; ++i) {
+                        const int c = c0 + lane + 32 * i;
+                        if (c >= nvec) break;
+                        float fg[V], fu[V];
+                        Vec16<T>::to_float(vg[i], fg);
+                        Vec16<T>::to_float(vu[i], fu);
+#pragma unroll
+                        for (int q = 0; q < kTC; ++q) {
+                            if (q < ntc) {
+                                float fh[V];
+                                Vec16<T>::to_float(hs[q * nvec + c], fh);
+#pragma unroll
+                                for (int t = 0; t < V; ++t) {
+                                    ag[q] = fmaf(fh[t], fg[t], ag[q]);
+                                    au[q] = fmaf(fh[t], fu[t], au[q]);
+                                }
                             }
                         }
                     }
@@ -90,9 +108,12 @@ __global__ void __launch_bounds__(256) k_gemv_gateup(const T* __restrict__ h, co
                 }
             }
         }
+        lo += re - rb;
     }
 }
 
+// down: one warp per 4 rows W_down[e, c..c+3] (each m long); up to kCh
+// 16-byte loads per row and lane are in flight before the dot products.
 template <typename T>
 __global__ void __launch_bounds__(256) k_gemv_down(const float* __restrict__ act, const T* __restrict__ w_down,
                                                    const float* __restrict__ ghat,
@@ -101,58 +122,86 @@ __global__ void __launch_bounds__(256) k_gemv_down(const float* __restrict__ act
                                                    const int32_t* __restrict__ perm,
                                                    const int32_t* __restrict__ meta,
                                                    float* __restrict__ yslot, int d, int m) {
+    constexpr int kCh = 4;
+    constexpr int kRows = 4;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     float* as = reinterpret_cast<float*>(smem_raw);      // [kTC][m]
     __shared__ float gs[kTC];
     constexpr int V = Vec16<T>::N;
     const int nvec = m / V;
     const int D = meta[kMetaDistinct];
-    const int S = meta[kMetaSlice2];
-    const int nsl = d / S;
-    const int items = D * nsl;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
-    for (int item = blockIdx.x; item < items; item += gridDim.x) {
-        const int e = dlist[item / nsl];
-        const int sl = item % nsl;
+    long long lo, hi;
+    block_range((long long)D * d, lo, hi);
+    while (lo < hi) {
+        const int e = dlist[lo / d];
+        const int rb = (int)(lo % d);
+        const int re = (int)min((long long)d, rb + (hi - lo));
         const int r0 = offsets[e], ne = offsets[e + 1] - r0;
         for (int tc0 = 0; tc0 < ne; tc0 += kTC) {
             const int ntc = min(kTC, ne - tc0);
             __syncthreads();
-            for (int i = threadIdx.x; i < kTC * (m / 4); i += blockDim.x) {
+            for (int i = threadIdx.x; i < ntc * (m / 4); i += blockDim.x) {
                 const int q = i / (m / 4), c = i % (m / 4);
-                float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (q < ntc) v = reinterpret_cast<const float4*>(act + (size_t)(r0 + tc0 + q) * m)[c];
-                reinterpret_cast<float4*>(as)[i] = v;
+                reinterpret_cast<float4*>(as)[i] = reinterpret_cast<const float4*>(act + (size_t)(r0 + tc0 + q) * m)[c];
             }
             if (threadIdx.x < kTC) gs[threadIdx.x] = threadIdx.x < ntc ? ghat[perm[r0 + tc0 + threadIdx.x]] : 0.f;
             __syncthreads();
-            for (int row = warp; row < S; row += nwarps) {
-                const int c = sl * S + row;
-                const uint4* wd = reinterpret_cast<const uint4*>(w_down + ((size_t)e * d + c) * m);
-                float acc[kTC];
+            for (int c = rb + warp * kRows; c < re; c += nwarps * kRows) {
+                float acc[kRows][kTC];
 #pragma unroll
-                for (int q = 0; q < kTC; ++q) acc[q] = 0.f;
-                for (int v = lane; v < nvec; v += 32) {
-                    float fw[V];
-                    Vec16<T>::to_float(ld_stream(wd + v), fw);
+                for (int r = 0; r < kRows; ++r)
 #pragma unroll
-                    for (int q = 0; q < kTC; ++q) {
-                        if (q < ntc) {
-                            const float* ar = as + q * m + v * V;
+                    for (int q = 0; q < kTC; ++q) acc[r][q] = 0.f;
+                for (int v0 = 0; v0 < nvec; v0 += 32 * kCh) {
+                    uint4 wv[kRows][kCh];
 #pragma unroll
-                            for (int i = 0; i < V; ++i) acc[q] = fmaf(ar[i], fw[i], acc[q]);
+                    for (int r = 0; r < kRows; ++r) {
+                        const uint4* wd = reinterpret_cast<const uint4*>(w_down + ((size_t)e * d + c + r) * m);
+#pragma unroll
+                        for (int i = 0; i < kCh; ++i) {
+                            const int v = v0 + lane + 32 * i;
+                            wv[r][i] = (c + r < re && v < nvec) ? ld_stream(wd + v) : make_uint4(0, 0, 0, 0);
+                        }
+                    }
+#pragma unroll
+                    for (int i = 0; i < kCh; ++i) {
+                        const int v = v0 + lane + 32 * i;
+                        if (v >= nvec) break;
+#pragma unroll
+                        for (int q = 0; q < kTC; ++q) {
+                            if (q < ntc) {
+                                float a[V];
+                                const float4* ap = reinterpret_cast<const float4*>(as + q * m + v * V);
+#pragma unroll
+                                for (int t = 0; t < V / 4; ++t) {
+                                    const float4 f = ap[t];
+                                    a[4 * t] = f.x; a[4 * t + 1] = f.y; a[4 * t + 2] = f.z; a[4 * t + 3] = f.w;
+                                }
+#pragma unroll
+                                for (int r = 0; r < kRows; ++r) {
+                                    float fw[V];
+                                    Vec16<T>::to_float(wv[r][i], fw);
+#pragma unroll
+                                    for (int t = 0; t < V; ++t) acc[r][q] = fmaf(a[t], fw[t], acc[r][q]);
+                                }
+                            }
                         }
                     }
                 }
 #pragma unroll
-                for (int q = 0; q < kTC; ++q) {
-                    if (q < ntc) {
-                        const float y = warp_sum(acc[q]);
-                        if (lane == 0) yslot[(size_t)(r0 + tc0 + q) * d + c] = gs[q] * y;
+                for (int r = 0; r < kRows; ++r) {
+#pragma unroll
+                    for (int q = 0; q < kTC; ++q) {
+                        if (q < ntc) {
+                            const float y = warp_sum(acc[r][q]);
+                            if (lane == 0 && c + r < re) yslot[(size_t)(r0 + tc0 + q) * d + c + r] = gs[q] * y;
+                        }
                     }
                 }
             }
         }
+        lo += re - rb;
     }
 }
 
@@ -184,7 +233,7 @@ cudaError_t run(const ace_layer* L, void* out, int T_, cudaStream_t s, cudaEvent
     const ace_layer_desc& D = L->desc;
     const Workspace& W = L->ws;
     const int d = D.hidden, m = D.ffn, k = D.top_k;
-    const int grid = L->num_sms * 4;
+    const int grid = L->num_sms * 2;
     const size_t smem1 = (size_t)kTC * d * sizeof(T);
     const size_t smem2 = (size_t)kTC * m * sizeof(float);
     if (ev) cudaEventRecord(ev[0], s);

@@ -85,17 +85,22 @@ struct ace_layer {
     bool profiling = false;
     cudaEvent_t ev[8] = {};
     int n_stages = 0;
+    int last_launches = 0;       // kernels launched by the last forward / route call
 };
 
 namespace ace {
 
 // ---- launchers (ace_route.cu) ----
 cudaError_t route_init(const ace_layer* L);   // per-layer kernel attributes
+// Small batches (T <= 256) fuse RMSNorm into the router and run the whole
+// decision + compaction in one block.
+bool small_path(int T);
 cudaError_t launch_rmsnorm(const ace_layer* L, const void* x, int T, cudaStream_t s);
-cudaError_t launch_router(const ace_layer* L, int T, cudaStream_t s);
-// Runs top-k / gates / decision / threshold / compaction from ws.logits or `logits`.
+cudaError_t launch_router(const ace_layer* L, const void* x, int T, bool fuse_norm, cudaStream_t s);
+// Runs top-k / gates / decision / threshold / compaction from `logits`.
 cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_skip_ctl ctl,
                          cudaStream_t s);
+int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl);
 cudaError_t launch_debug_exp(const float* x, float* y, int n, cudaStream_t s);
 
 // ---- launchers (ace_expert_gemv.cu) ----

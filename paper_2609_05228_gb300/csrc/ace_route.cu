@@ -1,6 +1,12 @@
 // ace_route.cu — RMSNorm, router logits, top-k + gates, the Algorithm 4 skip
 // decision, the App. B.1 per-batch threshold and the compaction of retained
 // slots into per-expert groups.
+//
+// Two launch shapes share the same device functions (and so the same bits):
+//   T <= kSmallT: k_router (with RMSNorm fused) + k_route_small, one block
+//                 doing top-k, decision, threshold and compaction;
+//   larger T:     k_rmsnorm, k_router, k_topk_score, [k_tau_select, k_decide],
+//                 k_compact_count, k_compact_place.
 #include <math.h>
 
 #include "ace_device.cuh"
@@ -9,18 +15,16 @@
 namespace ace {
 namespace {
 
+constexpr int kSmallT = 256;
+
 // --------------------------------------------------------------------------
 // RMSNorm (§3.1: expert and router input x = x_bar Gamma). One warp per token.
 // h = x / sqrt(mean(x^2) + rms_eps) * gamma, computed in float, stored as T.
 // --------------------------------------------------------------------------
 template <typename T>
-__global__ void __launch_bounds__(256) k_rmsnorm(const T* __restrict__ x, const T* __restrict__ gamma,
-                                                 T* __restrict__ h, int n_tokens, int d, float rms_eps) {
-    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    if (warp >= n_tokens) return;
+__device__ __forceinline__ void rmsnorm_row(const T* __restrict__ xr, const T* __restrict__ gamma, T* hr, int d,
+                                            float rms_eps, int lane) {
     constexpr int V = Vec16<T>::N;
-    const T* xr = x + (size_t)warp * d;
     float ss = 0.f;
     for (int j = lane * V; j < d; j += 32 * V) {
         float f[V];
@@ -30,7 +34,6 @@ __global__ void __launch_bounds__(256) k_rmsnorm(const T* __restrict__ x, const 
     }
     ss = warp_sum(ss);
     const float inv = 1.0f / sqrtf(ss / (float)d + rms_eps);
-    T* hr = h + (size_t)warp * d;
     for (int j = lane * V; j < d; j += 32 * V) {
         float f[V], gm[V];
         Vec16<T>::to_float(*reinterpret_cast<const uint4*>(xr + j), f);
@@ -42,58 +45,104 @@ __global__ void __launch_bounds__(256) k_rmsnorm(const T* __restrict__ x, const 
     }
 }
 
-// --------------------------------------------------------------------------
-// Router logits z[t,e] = (h_t . w_e + b_e) / temp  (§3.2 logit). A block holds
-// kRouterTok token rows of h in shared memory; each warp takes experts
-// e = warp, warp + 8, ... and streams w_e once for all of them.
-// --------------------------------------------------------------------------
-constexpr int kRouterTok = 8;
-
 template <typename T>
-__global__ void __launch_bounds__(256) k_router(const T* __restrict__ h, const T* __restrict__ w,
+__global__ void __launch_bounds__(256) k_rmsnorm(const T* __restrict__ x, const T* __restrict__ gamma,
+                                                 T* __restrict__ h, int n_tokens, int d, float rms_eps) {
+    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (warp >= n_tokens) return;
+    rmsnorm_row(x + (size_t)warp * d, gamma, h + (size_t)warp * d, d, rms_eps, threadIdx.x & 31);
+}
+
+// --------------------------------------------------------------------------
+// Router logits z[t,e] = (h_t . w_e + b_e) / temp  (§3.2 logit). A block
+// covers kRouterTok tokens x 8 experts (one expert row per warp): the token
+// rows of h sit in shared memory and every lane issues its share of the
+// expert row (up to 8 x 16 bytes) before the dot products. With FUSE_NORM
+// the block computes the RMSNorm of its tokens from x itself, and blocks
+// with blockIdx.y == 0 also store h for the experts.
+// --------------------------------------------------------------------------
+constexpr int kRouterTok = 16;
+constexpr int kRouterExp = 8;
+
+template <typename T, bool FUSE_NORM>
+__global__ void __launch_bounds__(256) k_router(const T* __restrict__ src, const T* __restrict__ gamma,
+                                                T* __restrict__ h_out, const T* __restrict__ w,
                                                 const float* __restrict__ b, float* __restrict__ z,
                                                 int n_tokens, int d, int n_exp, float inv_temp,
-                                                int use_temp) {
+                                                int use_temp, float rms_eps) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    T* hs = reinterpret_cast<T*>(smem_raw);
+    uint4* hs = reinterpret_cast<uint4*>(smem_raw);
     const int t0 = blockIdx.x * kRouterTok;
     const int nt = min(kRouterTok, n_tokens - t0);
     constexpr int V = Vec16<T>::N;
     const int nvec = d / V;
-    for (int i = threadIdx.x; i < kRouterTok * nvec; i += blockDim.x) {
-        const int r = i / nvec, c = i % nvec;
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (r < nt) v = *reinterpret_cast<const uint4*>(h + (size_t)(t0 + r) * d + c * V);
-        reinterpret_cast<uint4*>(hs)[i] = v;
-    }
-    __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int e = warp; e < n_exp; e += blockDim.x >> 5) {
-        float acc[kRouterTok];
-#pragma unroll
-        for (int r = 0; r < kRouterTok; ++r) acc[r] = 0.f;
-        const T* we = w + (size_t)e * d;
-        for (int c = lane; c < nvec; c += 32) {
-            float wf[V];
-            Vec16<T>::to_float(*reinterpret_cast<const uint4*>(we + c * V), wf);
-#pragma unroll
-            for (int r = 0; r < kRouterTok; ++r) {
-                float hf[V];
-                Vec16<T>::to_float(reinterpret_cast<const uint4*>(hs)[r * nvec + c], hf);
-#pragma unroll
-                for (int i = 0; i < V; ++i) acc[r] = fmaf(hf[i], wf[i], acc[r]);
+    if (FUSE_NORM) {
+        T* hsr = reinterpret_cast<T*>(smem_raw);
+        for (int r = warp; r < kRouterTok; r += blockDim.x >> 5) {
+            if (r < nt) {
+                rmsnorm_row(src + (size_t)(t0 + r) * d, gamma, hsr + (size_t)r * d, d, rms_eps, lane);
+            } else {
+                for (int c = lane; c < nvec; c += 32) hs[r * nvec + c] = make_uint4(0, 0, 0, 0);
             }
         }
-#pragma unroll
-        for (int r = 0; r < kRouterTok; ++r) acc[r] = warp_sum(acc[r]);
-        if (lane < nt) {
-            float v = acc[0];
-#pragma unroll
-            for (int r = 1; r < kRouterTok; ++r) if (lane == r) v = acc[r];
-            v = v + b[e];
-            if (use_temp) v = v * inv_temp;
-            z[(size_t)(t0 + lane) * n_exp + e] = v;
+        __syncthreads();
+        if (blockIdx.y == 0) {
+            for (int i = threadIdx.x; i < nt * nvec; i += blockDim.x) {
+                const int r = i / nvec, c = i % nvec;
+                reinterpret_cast<uint4*>(h_out + (size_t)(t0 + r) * d)[c] = hs[i];
+            }
         }
+    } else {
+        for (int i = threadIdx.x; i < kRouterTok * nvec; i += blockDim.x) {
+            const int r = i / nvec, c = i % nvec;
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (r < nt) v = reinterpret_cast<const uint4*>(src + (size_t)(t0 + r) * d)[c];
+            hs[i] = v;
+        }
+        __syncthreads();
+    }
+    const int e = blockIdx.y * kRouterExp + warp;
+    if (e >= n_exp) return;
+    const uint4* we = reinterpret_cast<const uint4*>(w + (size_t)e * d);
+    float acc[kRouterTok];
+#pragma unroll
+    for (int r = 0; r < kRouterTok; ++r) acc[r] = 0.f;
+    constexpr int CH = 8;
+    for (int c0 = 0; c0 < nvec; c0 += 32 * CH) {
+        uint4 wv[CH];
+#pragma unroll
+        for (int i = 0; i < CH; ++i) {
+            const int c = c0 + lane + 32 * i;
+            wv[i] = c < nvec ? we[c] : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int i = 0; i < CH; ++i) {
+            const int c = c0 + lane + 32 * i;
+            if (c >= nvec) break;
+            float wf[V];
+            Vec16<T>::to_float(wv[i], wf);
+#pragma unroll
+            for (int r = 0; r < kRouterTok; ++r) {
+                if (r < nt) {
+                    float hf[V];
+                    Vec16<T>::to_float(hs[r * nvec + c], hf);
+#pragma unroll
+                    for (int j = 0; j < V; ++j) acc[r] = fmaf(hf[j], wf[j], acc[r]);
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < kRouterTok; ++r)
+        if (r < nt) acc[r] = warp_sum(acc[r]);
+    if (lane < nt) {
+        float v = acc[0];
+#pragma unroll
+        for (int r = 1; r < kRouterTok; ++r) if (lane == r) v = acc[r];
+        v = v + b[e];
+        if (use_temp) v = v * inv_temp;
+        z[(size_t)(t0 + lane) * n_exp + e] = v;
     }
 }
 
@@ -106,66 +155,6 @@ struct SlotScore {
     float g;   // gate
     float c;   // max(p_gsp, p_rcr)
 };
-
-// Gates and c for the slot held by this lane (lanes >= k return zeros).
-__device__ __forceinline__ SlotScore score_slot(int lane, int k, float z_i, float z_0, int id,
-                                                const float* __restrict__ a_gsp,
-                                                const float* __restrict__ a_rcr, float eps) {
-    const bool on = lane < k;
-    const float e_i = on ? ace_exp32(__fsub_rn(z_i, z_0)) : 0.f;
-    float s = __shfl_sync(0xffffffffu, e_i, 0);
-    for (int j = 1; j < k; ++j) s = __fadd_rn(s, __shfl_sync(0xffffffffu, e_i, j));
-    const float g = on ? __fdiv_rn(e_i, s) : 0.f;
-    const float sg = on ? __fmul_rn(g, a_gsp[id]) : 0.f;       // Eq. gsp_contribution
-    const float sr = on ? __fmul_rn(g, a_rcr[id]) : 0.f;       // Eq. rcr_contribution
-    float zg = __shfl_sync(0xffffffffu, sg, 0);
-    float zr = __shfl_sync(0xffffffffu, sr, 0);
-    for (int j = 1; j < k; ++j) {
-        zg = __fadd_rn(zg, __shfl_sync(0xffffffffu, sg, j));
-        zr = __fadd_rn(zr, __shfl_sync(0xffffffffu, sr, j));
-    }
-    zg = __fadd_rn(zg, eps);
-    zr = __fadd_rn(zr, eps);
-    const float pg = on ? __fdiv_rn(sg, zg) : 0.f;              // Eq. gsp_probability
-    const float pr = on ? __fdiv_rn(sr, zr) : 0.f;              // Eq. rcr_probability
-    return SlotScore{g, fmaxf(pg, pr)};                         // Eq. ace_contribution
-}
-
-// Skip flag and g_hat for the slot of this lane, given tau.
-__device__ __forceinline__ void decide_slot(int lane, int k, float g, float c, float tau, int m_min,
-                                            float eps, bool& skip_out, float& ghat_out) {
-    const bool on = lane < k;
-    // Eq. ace_candidate_intersection via max; slot 0 is the top-1 and is kept.
-    bool skip = on && lane != 0 && (c < tau);
-    const unsigned sk = __ballot_sync(0xffffffffu, skip);
-    const int active = k - __popc(sk);
-    if (active < m_min) {
-        // restore skipped slots in c-descending order, lower rank first on ties
-        int need = m_min - active;
-        unsigned rem = sk;
-        while (need > 0 && rem) {
-            float best = -1.f;
-            int bi = -1;
-            for (unsigned m = rem; m; m &= m - 1) {
-                const int j = __ffs(m) - 1;
-                const float cj = __shfl_sync(0xffffffffu, c, j);
-                if (bi < 0 || cj > best) { best = cj; bi = j; }
-            }
-            rem &= ~(1u << bi);
-            if (lane == bi) skip = false;
-            --need;
-        }
-    }
-    const unsigned keep = __ballot_sync(0xffffffffu, on && !skip);
-    float zs = 0.f;
-    for (int j = 0; j < k; ++j) {
-        const float gj = __shfl_sync(0xffffffffu, g, j);
-        if ((keep >> j) & 1u) zs = __fadd_rn(zs, gj);
-    }
-    zs = __fadd_rn(zs, eps);
-    skip_out = skip;
-    ghat_out = (on && !skip) ? __fdiv_rn(g, zs) : 0.f;
-}
 
 // Top-k over one token's logits (one warp). Lane l owns experts l, l+32, ...
 // Order: larger logit first; ties to the lower expert index. NaN ranks last.
@@ -195,6 +184,175 @@ __device__ __forceinline__ void warp_topk(const float* __restrict__ zrow, int n_
         if (lane == r) { my_id = bi; my_z = bv; }
     }
 }
+
+// Gates and c for the slot held by this lane (lanes >= k return zeros).
+__device__ __forceinline__ SlotScore score_slot(int lane, int k, float z_i, float z_0, int id,
+                                                const float* __restrict__ a_gsp,
+                                                const float* __restrict__ a_rcr, float eps) {
+    const bool on = lane < k;
+    const float e_i = on ? ace_exp32(__fsub_rn(z_i, z_0)) : 0.f;
+    float s = __shfl_sync(0xffffffffu, e_i, 0);
+    for (int j = 1; j < k; ++j) s = __fadd_rn(s, __shfl_sync(0xffffffffu, e_i, j));
+    const float g = on ? __fdiv_rn(e_i, s) : 0.f;
+    const float sg = on ? __fmul_rn(g, a_gsp[id]) : 0.f;       // Eq. gsp_contribution
+    const float sr = on ? __fmul_rn(g, a_rcr[id]) : 0.f;       // Eq. rcr_contribution
+    float zg = __shfl_sync(0xffffffffu, sg, 0);
+    float zr = __shfl_sync(0xffffffffu, sr, 0);
+    for (int j = 1; j < k; ++j) {
+        zg = __fadd_rn(zg, __shfl_sync(0xffffffffu, sg, j));
+        zr = __fadd_rn(zr, __shfl_sync(0xffffffffu, sr, j));
+    }
+    zg = __fadd_rn(zg, eps);
+    zr = __fadd_rn(zr, eps);
+    const float pg = on ? __fdiv_rn(sg, zg) : 0.f;              // Eq. gsp_probability
+    const float pr = on ? __fdiv_rn(sr, zr) : 0.f;              // Eq. rcr_probability
+    return SlotScore{g, fmaxf(pg, pr)};                         // Eq. ace_contribution
+}
+
+// Slots excluded from the threshold search (App. B.1): rank 0 (the top-1)
+// and the m_min-1 highest-c other slots, the ones Algorithm 4 restores first.
+__device__ __forceinline__ bool slot_protected(int lane, int k, float c, int m_min) {
+    bool prot = lane == 0;
+    const int extra = min(m_min, k) - 1;
+    if (extra > 0) {
+        int better = 0;   // non-top-1 slots ahead of this one in (c desc, rank asc)
+        for (int j = 1; j < k; ++j) {
+            const float cj = __shfl_sync(0xffffffffu, c, j);
+            if (j != lane && (cj > c || (cj == c && j < lane))) ++better;
+        }
+        if (lane != 0 && better < extra) prot = true;
+    }
+    return prot;
+}
+
+// Skip flag and g_hat for the slot of this lane, given tau.
+__device__ __forceinline__ void decide_slot(int lane, int k, float g, float c, float tau, int m_min,
+                                            float eps, bool& skip_out, float& ghat_out) {
+    const bool on = lane < k;
+    // Eq. ace_candidate_intersection via max; slot 0 is the top-1 and is kept.
+    bool skip = on && lane != 0 && (c < tau);
+    const unsigned sk = __ballot_sync(0xffffffffu, skip);
+    const int active = k - __popc(sk);
+    if (active < m_min) {
+        // restore skipped slots in c-descending order, lower rank first on ties
+        int need = m_min - active;
+        unsigned rem = sk;
+        while (need > 0 && rem) {
+            float best = -1.f;
+            int bi = -1;
+            for (unsigned mm = rem; mm; mm &= mm - 1) {
+                const int j = __ffs(mm) - 1;
+                const float cj = __shfl_sync(0xffffffffu, c, j);
+                if (bi < 0 || cj > best) { best = cj; bi = j; }
+            }
+            rem &= ~(1u << bi);
+            if (lane == bi) skip = false;
+            --need;
+        }
+    }
+    const unsigned keep = __ballot_sync(0xffffffffu, on && !skip);
+    float zs = 0.f;
+    for (int j = 0; j < k; ++j) {
+        const float gj = __shfl_sync(0xffffffffu, g, j);
+        if ((keep >> j) & 1u) zs = __fadd_rn(zs, gj);
+    }
+    zs = __fadd_rn(zs, eps);
+    skip_out = skip;
+    ghat_out = (on && !skip) ? __fdiv_rn(g, zs) : 0.f;
+}
+
+// --------------------------------------------------------------------------
+// App. B.1 threshold for m candidates to skip: the (m+1)-th smallest
+// candidate key v (radix select over the non-negative float bits, 8 bits per
+// pass), lo = #{c < v}, hi = #{c <= v}; tau = v when lo == m or when lo is at
+// least as close to m as hi, else the next float above v. Whole block;
+// requires 0 < m < #candidates. Keys 0xffffffff are protected slots.
+// --------------------------------------------------------------------------
+struct SelectSmem {
+    int hist[256];
+    uint32_t prefix;
+    int want, below, last_cnt;
+    float tau;
+};
+
+__device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem& S) {
+    const int tid = threadIdx.x;
+    uint32_t prefix = 0u, mask = 0u;
+    if (tid == 0) { S.want = m; S.below = 0; }
+    for (int pass = 0; pass < 4; ++pass) {
+        const int shift = 24 - 8 * pass;
+        for (int i = tid; i < 256; i += blockDim.x) S.hist[i] = 0;
+        __syncthreads();
+        for (int i0 = 0; i0 < n; i0 += blockDim.x) {
+            const int i = i0 + tid;
+            const uint32_t key = i < n ? keys[i] : 0xffffffffu;
+            const bool in = key != 0xffffffffu && (key & mask) == prefix;
+            const int dg = (key >> shift) & 255;
+            const unsigned grp = __match_any_sync(0xffffffffu, in ? dg : -1);
+            if (in && (__ffs(grp) - 1) == (tid & 31)) atomicAdd(&S.hist[dg], __popc(grp));
+        }
+        __syncthreads();
+        if (tid == 0) {
+            int want = S.want, cum = 0, dg = 0;
+            for (; dg < 255; ++dg) {
+                if (cum + S.hist[dg] > want) break;
+                cum += S.hist[dg];
+            }
+            S.want = want - cum;
+            S.below += cum;
+            S.last_cnt = S.hist[dg];
+            S.prefix = prefix | ((uint32_t)dg << shift);
+        }
+        __syncthreads();
+        prefix = S.prefix;
+        mask |= 255u << shift;
+    }
+    if (tid == 0) {
+        const int lo = S.below, hi = S.below + S.last_cnt;
+        float tau = __uint_as_float(prefix);
+        if (!(lo == m || (m - lo) <= (hi - m))) tau = __uint_as_float(prefix + 1u);
+        S.tau = tau;
+    }
+    __syncthreads();
+    return S.tau;
+}
+
+// Exclusive scan of cnt[0..n_exp) by warp 0 of the block: offsets[e],
+// offsets[n_exp] = total, the distinct-expert list and the meta totals.
+// Also fills off_s (shared) when given.
+__device__ void scan_counts_warp0(const int* cnt, int n_exp, int32_t* __restrict__ offsets,
+                                  int32_t* __restrict__ dlist, int32_t* __restrict__ meta, int* off_s) {
+    const int lane = threadIdx.x;
+    const int per = (n_exp + 31) / 32;
+    const int e0 = min(lane * per, n_exp), e1 = min(e0 + per, n_exp);
+    int s = 0, dcount = 0;
+    for (int e = e0; e < e1; ++e) { s += cnt[e]; dcount += cnt[e] > 0; }
+    int xs = s, xd = dcount;
+    for (int o = 1; o < 32; o <<= 1) {
+        const int ys = __shfl_up_sync(0xffffffffu, xs, o);
+        const int yd = __shfl_up_sync(0xffffffffu, xd, o);
+        if (lane >= o) { xs += ys; xd += yd; }
+    }
+    int run = xs - s, drun = xd - dcount;
+    for (int e = e0; e < e1; ++e) {
+        offsets[e] = run;
+        if (off_s) off_s[e] = run;
+        run += cnt[e];
+        if (cnt[e] > 0) dlist[drun++] = e;
+    }
+    const int total = __shfl_sync(0xffffffffu, xs, 31);
+    const int dtotal = __shfl_sync(0xffffffffu, xd, 31);
+    if (lane == 31) {
+        offsets[n_exp] = total;
+        if (off_s) off_s[n_exp] = total;
+        meta[kMetaRetained] = total;
+        meta[kMetaDistinct] = dtotal;
+    }
+}
+
+// --------------------------------------------------------------------------
+// Large-T kernels
+// --------------------------------------------------------------------------
 
 // Pass 1: top-k, gates, c. THRESHOLD mode also decides; RATIO mode writes
 // candidate keys (float bits of c, or 0xffffffff for protected slots).
@@ -232,18 +390,7 @@ __global__ void __launch_bounds__(256) k_topk_score(const float* __restrict__ lo
             ghat[base + lane] = gh;
         }
     } else {
-        // protected: rank 0 and the (m_min-1) highest-c other slots
-        bool prot = lane == 0;
-        const int extra = min(m_min, k) - 1;
-        if (extra > 0) {
-            // other non-top-1 slots ahead of this one in (c desc, rank asc)
-            int better = 0;
-            for (int j = 1; j < k; ++j) {
-                const float cj = __shfl_sync(0xffffffffu, sc.c, j);
-                if (j != lane && (cj > sc.c || (cj == sc.c && j < lane))) ++better;
-            }
-            if (lane != 0 && better < extra) prot = true;
-        }
+        const bool prot = slot_protected(lane, k, sc.c, m_min);
         if (lane < k) keys[base + lane] = prot ? 0xffffffffu : __float_as_uint(sc.c);
     }
 }
@@ -268,84 +415,28 @@ __global__ void __launch_bounds__(256) k_decide(int n_tokens, int k, const float
     }
 }
 
-// --------------------------------------------------------------------------
-// App. B.1 threshold for m candidates to skip: the (m+1)-th smallest
-// candidate key v (radix select over the non-negative float bits, 8 bits per
-// pass), lo = #{c < v}, hi = #{c <= v}; tau = v when lo == m or when lo is at
-// least as close to m as hi, else the next float above v. One block.
-// --------------------------------------------------------------------------
 constexpr int kSelThreads = 1024;
 
 __global__ void __launch_bounds__(kSelThreads) k_tau_select(const uint32_t* __restrict__ keys, int n,
                                                             int m, float* __restrict__ tau_out) {
-    __shared__ int hist[32][256];
-    __shared__ int tot[256];
-    __shared__ uint32_t s_prefix;
-    __shared__ int s_want, s_below, s_last_cnt;
-    const int tid = threadIdx.x, warp = tid >> 5;
-    uint32_t prefix = 0u, mask = 0u;
-    if (tid == 0) { s_want = m; s_below = 0; }
-    for (int pass = 0; pass < 4; ++pass) {
-        const int shift = 24 - 8 * pass;
-        for (int i = tid; i < 32 * 256; i += kSelThreads) (&hist[0][0])[i] = 0;
-        __syncthreads();
-        for (int i0 = 0; i0 < n; i0 += kSelThreads) {
-            const int i = i0 + tid;
-            const uint32_t key = i < n ? keys[i] : 0xffffffffu;
-            const bool in = key != 0xffffffffu && (key & mask) == prefix;
-            const int dg = (key >> shift) & 255;
-            const unsigned grp = __match_any_sync(0xffffffffu, in ? dg : -1);
-            if (in && (__ffs(grp) - 1) == (tid & 31)) atomicAdd(&hist[warp][dg], __popc(grp));
-        }
-        __syncthreads();
-        if (tid < 256) {
-            int s = 0;
-            for (int w = 0; w < 32; ++w) s += hist[w][tid];
-            tot[tid] = s;
-        }
-        __syncthreads();
-        if (tid == 0) {
-            int want = s_want, cum = 0, dg = 0;
-            for (; dg < 256; ++dg) {
-                if (cum + tot[dg] > want) break;
-                cum += tot[dg];
-            }
-            if (dg > 255) dg = 255;   // unreachable when m < #candidates
-            s_want = want - cum;
-            s_below += cum;
-            s_last_cnt = tot[dg];
-            s_prefix = prefix | ((uint32_t)dg << shift);
-        }
-        __syncthreads();
-        prefix = s_prefix;
-        mask |= 255u << shift;
-        __syncthreads();
-    }
-    if (tid == 0) {
-        const int lo = s_below, hi = s_below + s_last_cnt;
-        const uint32_t v = prefix;
-        float tau = __uint_as_float(v);
-        if (!(lo == m || (m - lo) <= (hi - m))) tau = __uint_as_float(v + 1u);
-        *tau_out = tau;
-    }
+    __shared__ SelectSmem S;
+    const float tau = block_select_tau(keys, n, m, S);
+    if (threadIdx.x == 0) *tau_out = tau;
 }
 
-// --------------------------------------------------------------------------
 // Compaction (Algorithm 1 "evaluate only the experts indexed by I"): retained
 // slots grouped by expert, tokens increasing inside a group.
 // Pass A: per-chunk per-expert counts; the last block scans them into
 // offsets[N+1], per-chunk bases and the distinct-expert list.
 // Pass B: each chunk places its slots: rank within (chunk, expert) from a
 // per-expert token bitmap, so the order is deterministic.
-// --------------------------------------------------------------------------
 __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, int n_exp, int n_chunks,
                                                           const int32_t* __restrict__ ids,
                                                           const uint8_t* __restrict__ skip,
                                                           int32_t* __restrict__ chunk_counts,
                                                           int32_t* __restrict__ offsets,
                                                           int32_t* __restrict__ dlist,
-                                                          int32_t* __restrict__ meta, int d, int m,
-                                                          int target_items) {
+                                                          int32_t* __restrict__ meta) {
     __shared__ int cnt[kMaxExperts];
     __shared__ bool is_last;
     for (int e = threadIdx.x; e < n_exp; e += blockDim.x) cnt[e] = 0;
@@ -376,42 +467,9 @@ __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, i
         cnt[e] = run;
     }
     __syncthreads();
-    // exclusive scan of totals and of the distinct flags (warp 0)
     if (threadIdx.x < 32) {
-        const int lane = threadIdx.x;
-        const int per = (n_exp + 31) / 32;
-        const int e0 = min(lane * per, n_exp), e1 = min(e0 + per, n_exp);
-        int s = 0, dcount = 0;
-        for (int e = e0; e < e1; ++e) { s += cnt[e]; dcount += cnt[e] > 0; }
-        int xs = s, xd = dcount;
-        for (int o = 1; o < 32; o <<= 1) {
-            const int ys = __shfl_up_sync(0xffffffffu, xs, o);
-            const int yd = __shfl_up_sync(0xffffffffu, xd, o);
-            if (lane >= o) { xs += ys; xd += yd; }
-        }
-        int run = xs - s, drun = xd - dcount;
-        for (int e = e0; e < e1; ++e) {
-            offsets[e] = run;
-            run += cnt[e];
-            if (cnt[e] > 0) dlist[drun++] = e;
-        }
-        const int total = __shfl_sync(0xffffffffu, xs, 31);
-        const int dtotal = __shfl_sync(0xffffffffu, xd, 31);
-        if (lane == 31) {
-            offsets[n_exp] = total;
-            meta[kMetaRetained] = total;
-            meta[kMetaDistinct] = dtotal;
-            // GEMV work-item sizes: rows per item, a power of two in [8, 128]
-            // dividing m (resp. d), so that D * rows/slice reaches the target.
-            int s1 = 128, s2 = 128;
-            while (s1 > 8 && (long long)dtotal * (m / s1) < target_items) s1 >>= 1;
-            while (s2 > 8 && (long long)dtotal * (d / s2) < target_items) s2 >>= 1;
-            while (m % s1) s1 >>= 1;
-            while (d % s2) s2 >>= 1;
-            meta[kMetaSlice1] = s1 < 1 ? 1 : s1;
-            meta[kMetaSlice2] = s2 < 1 ? 1 : s2;
-            meta[kMetaTicket] = 0;
-        }
+        scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, nullptr);
+        if (threadIdx.x == 0) meta[kMetaTicket] = 0;
     }
 }
 
@@ -449,6 +507,113 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
     }
 }
 
+// --------------------------------------------------------------------------
+// Small-T kernel: the whole decision and compaction in one block.
+// --------------------------------------------------------------------------
+constexpr int kSmallThreads = 1024;
+
+__global__ void __launch_bounds__(kSmallThreads) k_route_small(
+    const float* __restrict__ logits, int n_tokens, int n_exp, int k, const float* __restrict__ a_gsp,
+    const float* __restrict__ a_rcr, float eps, int m_min, int mode, float tau_in, int m_q,
+    int32_t* __restrict__ ids, float* __restrict__ gates, float* __restrict__ cval, uint8_t* __restrict__ skip,
+    float* __restrict__ ghat, float* __restrict__ tau_out, int32_t* __restrict__ offsets,
+    int32_t* __restrict__ dlist, int32_t* __restrict__ perm, int32_t* __restrict__ slot_pos,
+    int32_t* __restrict__ meta, int* __restrict__ err) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int ns = n_tokens * k;
+    float* g_s = reinterpret_cast<float*>(smem_raw);
+    float* c_s = g_s + ns;
+    uint32_t* key_s = reinterpret_cast<uint32_t*>(c_s + ns);
+    int* id_s = reinterpret_cast<int*>(key_s + ns);
+    int* cnt = id_s + ns;                                            // [n_exp]
+    int* off_s = cnt + n_exp;                                        // [n_exp + 1]
+    uint32_t* bm = reinterpret_cast<uint32_t*>(off_s + n_exp + 1);   // [n_exp * 8]
+    uint8_t* skip_s = reinterpret_cast<uint8_t*>(bm + n_exp * 8);    // [ns]
+    __shared__ SelectSmem S;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
+    const bool ratio = mode == ACE_SKIP_RATIO;
+    for (int i = threadIdx.x; i < n_exp; i += blockDim.x) cnt[i] = 0;
+    for (int i = threadIdx.x; i < n_exp * 8; i += blockDim.x) bm[i] = 0u;
+    // phase 1: top-k, gates, c (and the decision in threshold mode)
+    for (int t = warp; t < n_tokens; t += nwarps) {
+        int id;
+        float zv;
+        bool nan;
+        warp_topk(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
+        const float z0 = __shfl_sync(0xffffffffu, zv, 0);
+        if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(err, kErrNumeric);
+        const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a_gsp, a_rcr, eps);
+        const int base = t * k;
+        if (lane < k) {
+            ids[base + lane] = id;
+            gates[base + lane] = sc.g;
+            cval[base + lane] = sc.c;
+            id_s[base + lane] = id;
+            g_s[base + lane] = sc.g;
+            c_s[base + lane] = sc.c;
+        }
+        if (!ratio) {
+            bool sk;
+            float gh;
+            decide_slot(lane, k, sc.g, sc.c, tau_in, m_min, eps, sk, gh);
+            if (lane < k) {
+                skip[base + lane] = sk ? 1 : 0;
+                skip_s[base + lane] = sk ? 1 : 0;
+                ghat[base + lane] = gh;
+            }
+        } else {
+            const bool prot = slot_protected(lane, k, sc.c, m_min);
+            if (lane < k) key_s[base + lane] = prot ? 0xffffffffu : __float_as_uint(sc.c);
+        }
+    }
+    __syncthreads();
+    // phase 2: threshold and decision (ratio mode)
+    if (ratio) {
+        const float tau = block_select_tau(key_s, ns, m_q, S);
+        if (threadIdx.x == 0) *tau_out = tau;
+        for (int t = warp; t < n_tokens; t += nwarps) {
+            const int base = t * k;
+            const float g = lane < k ? g_s[base + lane] : 0.f;
+            const float c = lane < k ? c_s[base + lane] : 0.f;
+            bool sk;
+            float gh;
+            decide_slot(lane, k, g, c, tau, m_min, eps, sk, gh);
+            if (lane < k) {
+                skip[base + lane] = sk ? 1 : 0;
+                skip_s[base + lane] = sk ? 1 : 0;
+                ghat[base + lane] = gh;
+            }
+        }
+        __syncthreads();
+    } else if (threadIdx.x == 0) {
+        *tau_out = tau_in;
+    }
+    // phase 3: compaction of retained slots (one chunk of <= 256 tokens)
+    for (int s = threadIdx.x; s < ns; s += blockDim.x) {
+        if (skip_s[s]) continue;
+        const int e = id_s[s], t = s / k;
+        atomicAdd(&cnt[e], 1);
+        atomicOr(&bm[e * 8 + (t >> 5)], 1u << (t & 31));
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, off_s);
+    __syncthreads();
+    for (int s = threadIdx.x; s < ns; s += blockDim.x) {
+        if (skip_s[s]) { slot_pos[s] = -1; continue; }
+        const int e = id_s[s], t = s / k, w = t >> 5;
+        int rank = __popc(bm[e * 8 + w] & ((1u << (t & 31)) - 1u));
+        for (int ww = 0; ww < w; ++ww) rank += __popc(bm[e * 8 + ww]);
+        const int r = off_s[e] + rank;
+        perm[r] = s;
+        slot_pos[s] = r;
+    }
+}
+
+size_t small_smem_bytes(int T, int k, int n_exp) {
+    const size_t ns = (size_t)T * k;
+    return ns * 16 + (size_t)n_exp * 4 + (size_t)(n_exp + 1) * 4 + (size_t)n_exp * 32 + ns + 16;
+}
+
 __global__ void k_debug_exp(const float* __restrict__ x, float* __restrict__ y, int n) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i < n) y[i] = ace_exp32(x[i]);
@@ -456,7 +621,46 @@ __global__ void k_debug_exp(const float* __restrict__ x, float* __restrict__ y, 
 
 inline int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }
 
+size_t router_smem(const ace_layer* L) { return (size_t)kRouterTok * L->desc.hidden * L->elem; }
+
+template <typename T, bool FUSE>
+cudaError_t router_launch(const ace_layer* L, const void* src, int T_, cudaStream_t s) {
+    const int d = L->desc.hidden, n = L->desc.n_experts;
+    const float temp = L->desc.router_temp;
+    const dim3 blocks(cdiv(T_, kRouterTok), cdiv(n, kRouterExp));
+    k_router<T, FUSE><<<blocks, 256, router_smem(L), s>>>((const T*)src, (const T*)L->gamma, (T*)L->ws.h,
+                                                          (const T*)L->router_w, L->router_b, L->ws.logits, T_, d,
+                                                          n, 1.0f / temp, temp != 1.0f, L->desc.rms_eps);
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t set_router_attrs(size_t smem) {
+    cudaError_t e = cudaFuncSetAttribute(k_router<T, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(k_router<T, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+}
+
+int select_mq(const ace_layer* L, int T, ace_skip_ctl ctl, float* tau, bool* need_select) {
+    const int k = L->desc.top_k;
+    *tau = ctl.value;
+    *need_select = false;
+    if (ctl.mode != ACE_SKIP_RATIO) return 0;
+    const long long n_all = (long long)T * k;
+    const int prot = L->desc.min_active < 1 ? 1 : (L->desc.min_active > k ? k : L->desc.min_active);
+    const long long n_cand = (long long)T * (k - prot);
+    long long mq = llround((double)ctl.value * (double)n_all);
+    if (mq < 0) mq = 0;
+    if (mq > n_cand) mq = n_cand;
+    if (mq == 0) *tau = 0.0f;
+    else if (mq == n_cand) *tau = INFINITY;
+    else *need_select = true;
+    return (int)mq;
+}
+
 }  // namespace
+
+bool small_path(int T) { return T <= kSmallT; }
 
 cudaError_t launch_rmsnorm(const ace_layer* L, const void* x, int T, cudaStream_t s) {
     const int d = L->desc.hidden;
@@ -471,20 +675,12 @@ cudaError_t launch_rmsnorm(const ace_layer* L, const void* x, int T, cudaStream_
     return cudaGetLastError();
 }
 
-cudaError_t launch_router(const ace_layer* L, int T, cudaStream_t s) {
-    const int d = L->desc.hidden, n = L->desc.n_experts;
-    const size_t smem = (size_t)kRouterTok * d * L->elem;
-    const float temp = L->desc.router_temp;
-    const int use_temp = temp != 1.0f;
-    const int blocks = cdiv(T, kRouterTok);
-    if (L->desc.dtype == ACE_BF16) {
-        k_router<__nv_bfloat16><<<blocks, 256, smem, s>>>((const __nv_bfloat16*)L->ws.h, (const __nv_bfloat16*)L->router_w,
-                                      L->router_b, L->ws.logits, T, d, n, 1.0f / temp, use_temp);
-    } else {
-        k_router<float><<<blocks, 256, smem, s>>>((const float*)L->ws.h, (const float*)L->router_w, L->router_b,
-                                      L->ws.logits, T, d, n, 1.0f / temp, use_temp);
-    }
-    return cudaGetLastError();
+cudaError_t launch_router(const ace_layer* L, const void* x, int T, bool fuse_norm, cudaStream_t s) {
+    const void* src = fuse_norm ? x : L->ws.h;
+    if (L->desc.dtype == ACE_BF16)
+        return fuse_norm ? router_launch<__nv_bfloat16, true>(L, src, T, s)
+                         : router_launch<__nv_bfloat16, false>(L, src, T, s);
+    return fuse_norm ? router_launch<float, true>(L, src, T, s) : router_launch<float, false>(L, src, T, s);
 }
 
 cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_skip_ctl ctl,
@@ -492,46 +688,46 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     const ace_layer_desc& D = L->desc;
     const Workspace& W = L->ws;
     const int k = D.top_k, n = D.n_experts;
-    const int blocks = cdiv(T, 8);
-    float tau = ctl.value;
-    bool need_select = false;
-    int m_q = 0;
-    if (ctl.mode == ACE_SKIP_RATIO) {
-        const long long n_all = (long long)T * k;
-        const int prot = D.min_active < 1 ? 1 : (D.min_active > k ? k : D.min_active);
-        const long long n_cand = (long long)T * (k - prot);
-        long long mq = llround((double)ctl.value * (double)n_all);
-        if (mq < 0) mq = 0;
-        if (mq > n_cand) mq = n_cand;
-        m_q = (int)mq;
-        if (m_q == 0) tau = 0.0f;
-        else if (m_q == n_cand) tau = INFINITY;
-        else need_select = true;
+    float tau;
+    bool need_select;
+    const int m_q = select_mq(L, T, ctl, &tau, &need_select);
+    const int mode = need_select ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
+    if (T <= kSmallT) {
+        k_route_small<<<1, kSmallThreads, small_smem_bytes(T, k, n), s>>>(
+            logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode, tau, m_q, W.ids, W.gates, W.cval,
+            W.skip, W.ghat, W.tau, W.offsets, W.dlist, W.perm, W.slot_pos, W.meta, W.err);
+        return cudaGetLastError();
     }
-    const int mode = (ctl.mode == ACE_SKIP_RATIO && need_select) ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
+    const int blocks = cdiv(T, 8);
     k_topk_score<<<blocks, 256, 0, s>>>(logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode,
                                         tau, W.ids, W.gates, W.cval, W.keys, W.skip, W.ghat, W.tau, W.err);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
     if (mode == ACE_SKIP_RATIO) {
         k_tau_select<<<1, kSelThreads, 0, s>>>(W.keys, T * k, m_q, W.tau);
         k_decide<<<blocks, 256, 0, s>>>(T, k, W.gates, W.cval, W.tau, D.min_active, D.eps, W.skip, W.ghat);
     }
     const int n_chunks = cdiv(T, kChunk);
-    const int target = 4 * L->num_sms;
     k_compact_count<<<n_chunks, kChunk, 0, s>>>(T, k, n, n_chunks, W.ids, W.skip, W.chunk_counts,
-                                                W.offsets, W.dlist, W.meta, D.hidden, D.ffn, target);
+                                                W.offsets, W.dlist, W.meta);
     k_compact_place<<<n_chunks, kChunk, 0, s>>>(T, k, n, W.ids, W.skip, W.chunk_counts, W.offsets,
                                                 W.perm, W.slot_pos);
     return cudaGetLastError();
 }
 
+int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl) {
+    if (T <= kSmallT) return 1;
+    float tau;
+    bool sel;
+    select_mq(L, T, ctl, &tau, &sel);
+    return sel ? 5 : 3;
+}
+
 cudaError_t route_init(const ace_layer* L) {
-    const size_t smem = (size_t)kRouterTok * L->desc.hidden * L->elem;
-    cudaError_t e = cudaFuncSetAttribute(k_router<__nv_bfloat16>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = set_router_attrs<__nv_bfloat16>(router_smem(L));
     if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(k_router<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    e = set_router_attrs<float>(router_smem(L));
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(k_route_small, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)small_smem_bytes(kSmallT, L->desc.top_k, L->desc.n_experts));
 }
 
 cudaError_t launch_debug_exp(const float* x, float* y, int n, cudaStream_t s) {
