@@ -172,7 +172,7 @@ def ace_debug_exp32(x, y, n: int, stream=None) -> None:
     _check(lib().ace_debug_exp32(_ptr(x), _ptr(y), int(n), _stream(stream)))
 
 
-STAGES = ["rmsnorm", "router", "route", "gate_up", "down", "combine"]
+STAGES = ["rmsnorm", "router", "route", "gather", "gate_up", "down", "combine"]
 
 
 def ace_layer_set_profiling(layer: int, enable: bool) -> None:

@@ -39,11 +39,11 @@ cudaError_t dalloc(P** p, size_t bytes) {
 
 void free_layer(ace_layer* L) {
     if (!L) return;
-    void* ptrs[] = {L->router_w, L->router_b, L->w_gate, L->w_up, L->w_down, L->gamma, L->a_gsp, L->a_rcr,
-                    L->ws.h, L->ws.logits, L->ws.ids, L->ws.gates, L->ws.cval, L->ws.keys, L->ws.skip,
+    void* ptrs[] = {L->router_w, L->router_b, L->w_gate, L->w_up, L->w_gu, L->w_down, L->gamma, L->a_gsp,
+                    L->a_rcr, L->ws.h, L->ws.logits, L->ws.ids, L->ws.gates, L->ws.cval, L->ws.keys, L->ws.skip,
                     L->ws.ghat, L->ws.tau, L->ws.chunk_counts, L->ws.offsets, L->ws.dlist, L->ws.perm,
-                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.err, L->ws.x_stage,
-                    L->ws.out_stage};
+                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.g_perm,
+                    L->ws.act_bf16, L->ws.tt_off, L->ws.err, L->ws.x_stage, L->ws.out_stage};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     for (cudaEvent_t e : L->ev)
@@ -151,10 +151,15 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
             return fail(ACE_ERR_OOM, std::string("cudaMalloc failed for ") + #ptr); \
         }                                                                   \
     } while (0)
+    L->tc = ace::tc_supported(L);
     ALLOC(L->router_w, n * d * E);
     ALLOC(L->router_b, n * sizeof(float));
-    ALLOC(L->w_gate, n * m * d * E);
-    ALLOC(L->w_up, n * m * d * E);
+    if (L->tc) {
+        ALLOC(L->w_gu, n * 2 * m * d * E);
+    } else {
+        ALLOC(L->w_gate, n * m * d * E);
+        ALLOC(L->w_up, n * m * d * E);
+    }
     ALLOC(L->w_down, n * d * m * E);
     ALLOC(L->gamma, d * E);
     ALLOC(L->a_gsp, n * sizeof(float));
@@ -174,7 +179,14 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     ALLOC(W.perm, slots * sizeof(int32_t));
     ALLOC(W.slot_pos, slots * sizeof(int32_t));
     ALLOC(W.meta, ace::kMetaCount * sizeof(int32_t));
-    ALLOC(W.act, slots * m * sizeof(float));
+    if (L->tc) {
+        ALLOC(W.h_perm, slots * d * E);
+        ALLOC(W.g_perm, slots * sizeof(float));
+        ALLOC(W.act_bf16, slots * m * E);
+        ALLOC(W.tt_off, (n + 1) * sizeof(int32_t));
+    } else {
+        ALLOC(W.act, slots * m * sizeof(float));
+    }
     ALLOC(W.yslot, slots * d * sizeof(float));
     ALLOC(W.err, sizeof(int));
     ALLOC(W.x_stage, T * d * E);
@@ -193,8 +205,12 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
         CK(cudaMemcpyAsync(L->router_b, router_b, n * sizeof(float), cudaMemcpyDeviceToDevice, s), "copy router_b");
     else
         CK(cudaMemsetAsync(L->router_b, 0, n * sizeof(float), s), "zero router_b");
-    CK(cudaMemcpyAsync(L->w_gate, w_gate, n * m * d * E, cudaMemcpyDeviceToDevice, s), "copy w_gate");
-    CK(cudaMemcpyAsync(L->w_up, w_up, n * m * d * E, cudaMemcpyDeviceToDevice, s), "copy w_up");
+    if (L->tc) {
+        CK(ace::tc_pack_gate_up(L, w_gate, w_up, s), "pack gate/up weights");
+    } else {
+        CK(cudaMemcpyAsync(L->w_gate, w_gate, n * m * d * E, cudaMemcpyDeviceToDevice, s), "copy w_gate");
+        CK(cudaMemcpyAsync(L->w_up, w_up, n * m * d * E, cudaMemcpyDeviceToDevice, s), "copy w_up");
+    }
     CK(cudaMemcpyAsync(L->w_down, w_down, n * d * m * E, cudaMemcpyDeviceToDevice, s), "copy w_down");
     CK(cudaMemcpyAsync(L->gamma, rms_gamma, d * E, cudaMemcpyDeviceToDevice, s), "copy gamma");
     CK(cudaMemcpyAsync(L->a_gsp, a_gsp, n * sizeof(float), cudaMemcpyHostToDevice, s), "copy a_gsp");
@@ -204,6 +220,7 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     CK(cudaMemsetAsync(W.offsets, 0, (n + 1) * sizeof(int32_t), s), "zero offsets");
     CK(ace::route_init(L), "route kernel attributes");
     CK(ace::gemv_init(L), "gemv kernel attributes");
+    if (L->tc) CK(ace::tc_init(L), "tensor-core expert setup");
     CK(cudaStreamSynchronize(s), "create: synchronize");
 #undef CK
     *out_layer = L;
@@ -262,9 +279,15 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
     ACE_CUDA(ace::launch_router(L, x, T, small, s), "router launch");
     if (ev) ACE_CUDA(cudaEventRecord(ev[2], s), "event record");
     ACE_CUDA(ace::launch_route(L, L->ws.logits, T, ctl, s), "route launch");
-    ACE_CUDA(ace::launch_experts_gemv(L, out, T, s, ev ? ev + 3 : nullptr), "expert launch");
+    if (ev) ACE_CUDA(cudaEventRecord(ev[3], s), "event record");
+    if (L->tc) {
+        ACE_CUDA(ace::launch_experts_tc(L, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
+    } else {
+        if (ev) ACE_CUDA(cudaEventRecord(ev[4], s), "event record");   // no gather stage
+        ACE_CUDA(ace::launch_experts_gemv(L, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
+    }
     L->n_stages = ev ? ace::kNumStages : 0;
-    L->last_launches = (small ? 1 : 2) + ace::route_launch_count(L, T, ctl) + 3;
+    L->last_launches = (small ? 1 : 2) + ace::route_launch_count(L, T, ctl) + (L->tc ? 4 : 3);
     return ACE_OK;
 }
 

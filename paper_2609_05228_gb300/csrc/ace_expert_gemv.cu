@@ -236,7 +236,6 @@ cudaError_t run(const ace_layer* L, void* out, int T_, cudaStream_t s, cudaEvent
     const int grid = L->num_sms * 2;
     const size_t smem1 = (size_t)kTC * d * sizeof(T);
     const size_t smem2 = (size_t)kTC * m * sizeof(float);
-    if (ev) cudaEventRecord(ev[0], s);
     k_gemv_gateup<T><<<grid, 256, smem1, s>>>((const T*)W.h, (const T*)L->w_gate, (const T*)L->w_up,
                                               W.offsets, W.dlist, W.perm, W.meta, W.act, d, m, k);
     if (ev) cudaEventRecord(ev[1], s);

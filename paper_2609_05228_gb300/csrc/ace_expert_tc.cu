@@ -1,0 +1,604 @@
+// ace_expert_tc.cu — the SwiGLU experts (Eq. swiglu_expert) over retained
+// slots only, as a persistent grouped GEMM on the 5th-generation tensor cores
+// (tcgen05.mma, accumulators in TMEM, operands staged by TMA).
+//
+// One kernel template serves both projections and both batch regimes:
+//   GEMM 1 (gate/up, K = d): act[r, j] = SiLU(h_r . W_gate[e, j]) * (h_r . W_up[e, j])
+//   GEMM 2 (down,    K = m): y[r, c]   = g_hat(r) * (act[r] . W_down[e, c])
+// where rows r are retained slots in expert-grouped order (the compaction's
+// permutation) and e is the slot's expert.
+//   * decode (SWAP): the 128-row MMA operand is a tile of weight rows and the
+//     N = 16 operand is up to 16 token rows of one expert, so each weight tile
+//     is streamed once and the MMA does the reduction the GEMV would do on
+//     the CUDA cores;
+//   * prefill: the 128-row operand is a tile of token rows, N = 256 weight rows.
+// Gate and up rows are interleaved in blocks of 16 (W_gu packed at create
+// time), so one accumulator tile holds matching gate and up outputs and the
+// SiLU-and-product runs in the epilogue.
+//
+// Warp roles (192 threads): warp 0 issues TMA loads into a STAGES-deep ring,
+// warp 1 owns TMEM and issues the MMAs (one thread), warps 2..5 run the
+// epilogue from TMEM (each warp reads its 32-lane quadrant). Two accumulator
+// buffers let the epilogue of one tile overlap the MMAs of the next. Every
+// mbarrier wait is bounded; on expiry the kernel sets kErrTimeout, stops
+// issuing work and releases TMEM before returning.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <math.h>
+
+#include "ace_device.cuh"
+#include "ace_internal.h"
+
+namespace ace {
+namespace {
+
+constexpr int kBK = 64;                 // K elements per stage (128 bytes of bf16)
+constexpr int kUmmaK = 16;              // K per tcgen05.mma (kind::f16)
+constexpr int kThreads = 192;
+constexpr long long kSpinCycles = 4000000000LL;   // ~2 s at 2 GHz
+
+struct TcParams {
+    CUtensorMap tm_tok;                 // token rows [rows, K] bf16
+    CUtensorMap tm_w;                   // weight rows [N * w_rows, K] bf16
+    const int32_t* offsets;             // [N+1]
+    const int32_t* dlist;               // [N]
+    const int32_t* tt_off;              // [N+1] token-tile prefix over distinct experts
+    const int32_t* meta;
+    const float* ghat_perm;             // [R] g_hat of row r (GEMM 2)
+    void* out;                          // act bf16 [rows, m] or y fp32 [rows, d]
+    int K;                              // reduction length
+    int w_rows;                         // weight rows per expert (2m or d)
+    int w_tiles;                        // w_rows / weight tile
+    int out_ld;                         // row length of out
+    int* err;
+};
+
+// ---------------------------------------------------------------- PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait: false (and kErrTimeout set) if the phase did not complete.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const long long t0 = clock64();
+    while (!mbar_try_wait(bar, parity)) {
+        if (clock64() - t0 > kSpinCycles) {
+            atomicOr(err, kErrTimeout);
+            return false;
+        }
+    }
+    return true;
+}
+
+__device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];"
+        ::"r"(smem_u32(smem_dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor: K-major tile whose rows are 128 bytes,
+// stored in the 128-byte swizzle pattern (8-row atoms of 1024 bytes).
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((addr >> 4) & 0x3FFF);          // start address
+    d |= (uint64_t)1 << 16;                         // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(1024 >> 4) << 32;               // stride byte offset: 8 rows x 128 B
+    d |= (uint64_t)1 << 46;                         // descriptor version
+    d |= (uint64_t)2 << 61;                         // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor, kind::f16: bf16 A and B, f32 accumulator, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+    return (1u << 4)                        // D format f32
+           | (1u << 7)                      // A format bf16
+           | (1u << 10)                     // B format bf16
+           | ((uint32_t)(N >> 3) << 17)     // N / 8
+           | ((uint32_t)(M >> 4) << 24);    // M / 16
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+
+// 32 lanes x 32 bits x 16 columns: thread i gets columns [col, col+16) of lane (quadrant base + i).
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+__device__ __forceinline__ float silu(float u) { return u / (1.0f + __expf(-u)); }
+
+// ---------------------------------------------------------------- tile schedule
+
+struct Tile {
+    int e;        // expert
+    int row0;     // first token row (perm order)
+    int nrows;    // valid token rows
+    int wrow0;    // first weight row in the [N * w_rows] map
+    int wt;       // weight tile index within the expert
+};
+
+template <int TOKTILE, int WTILE>
+__device__ __forceinline__ Tile tile_at(const TcParams& p, int D, int tile) {
+    const int tt = tile / p.w_tiles;
+    const int wt = tile - tt * p.w_tiles;
+    int lo = 0, hi = D;                       // largest j with tt_off[j] <= tt
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (p.tt_off[mid] <= tt) lo = mid; else hi = mid;
+    }
+    Tile t;
+    t.e = p.dlist[lo];
+    const int blk = tt - p.tt_off[lo];
+    const int beg = p.offsets[t.e];
+    t.row0 = beg + blk * TOKTILE;
+    t.nrows = min(TOKTILE, p.offsets[t.e + 1] - t.row0);
+    t.wrow0 = t.e * p.w_rows + wt * WTILE;
+    t.wt = wt;
+    return t;
+}
+
+// ---------------------------------------------------------------- kernel
+
+// SWAP: A (M = 128) = weight rows, B (N = TOKTILE) = token rows.
+// !SWAP: A (M = 128) = token rows, B (N = WTILE) = weight rows.
+// EPI 0: SwiGLU into act (bf16); EPI 1: g_hat-scaled rows into y (fp32).
+template <bool SWAP, int EPI, int STAGES>
+struct TcCfg {
+    static constexpr int TOKTILE = SWAP ? 16 : 128;
+    static constexpr int WTILE = SWAP ? 128 : 256;
+    static constexpr int BM = 128;
+    static constexpr int BN = SWAP ? TOKTILE : WTILE;
+    static constexpr int A_ROWS = BM;
+    static constexpr int B_ROWS = BN;
+    static constexpr int A_BYTES = A_ROWS * kBK * 2;
+    static constexpr int B_BYTES = B_ROWS * kBK * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int ACC_COLS = BN;                       // fp32 columns per accumulator
+    static constexpr int TMEM_COLS = (2 * ACC_COLS) < 32 ? 32 : 2 * ACC_COLS;
+    static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+};
+
+template <bool SWAP, int EPI, int STAGES>
+__global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant__ TcParams p) {
+    using C = TcCfg<SWAP, EPI, STAGES>;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+    uint64_t* empty = full + STAGES;
+    uint64_t* acc_full = empty + STAGES;
+    uint64_t* acc_empty = acc_full + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int D = p.meta[kMetaDistinct];
+    const int n_tiles = p.tt_off[D] * p.w_tiles;
+    const int kblocks = p.K / kBK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&acc_full[a], 1);
+            mbar_init(&acc_empty[a], 4);          // one arrival per epilogue warp
+        }
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"((uint32_t)C::TMEM_COLS));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            long long issued = 0;
+            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+                const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, D, tile);
+                for (int kb = 0; kb < kblocks; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                    unsigned char* sa = smem + stage * C::STAGE_BYTES;
+                    unsigned char* sb = sa + C::A_BYTES;
+                    mbar_expect_tx(&full[stage], C::STAGE_BYTES);
+                    if (SWAP) {
+                        tma_load_2d(sa, &p.tm_w, &full[stage], kb * kBK, t.wrow0);
+                        tma_load_2d(sb, &p.tm_tok, &full[stage], kb * kBK, t.row0);
+                    } else {
+                        tma_load_2d(sa, &p.tm_tok, &full[stage], kb * kBK, t.row0);
+                        tma_load_2d(sb, &p.tm_w, &full[stage], kb * kBK, t.wrow0);
+                    }
+                    ++issued;
+                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                }
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                // our own copies must land before the block exits: wait (bounded)
+                // on the full barrier of each of the last STAGES fills
+                for (long long f = issued - 1; f >= 0 && f >= issued - STAGES; --f) {
+                    if (!mbar_wait(&full[f % STAGES], (uint32_t)((f / STAGES) & 1), p.err)) break;
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16(C::BM, C::BN);
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+                if (!mbar_wait(&acc_empty[acc], acc_phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * C::ACC_COLS);
+                for (int kb = 0; kb < kblocks; ++kb) {
+                    if (!mbar_wait(&full[stage], phase, p.err) || *abort_flag) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t a_addr = smem_u32(smem + stage * C::STAGE_BYTES);
+                    const uint32_t b_addr = a_addr + C::A_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
+                        const uint64_t ad = smem_desc_sw128(a_addr + kk * kUmmaK * 2);
+                        const uint64_t bd = smem_desc_sw128(b_addr + kk * kUmmaK * 2);
+                        mma_bf16(d_tmem, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    mma_commit(&empty[stage]);           // frees the stage when these MMAs finish
+                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                }
+                if (!ok) break;
+                mma_commit(&acc_full[acc]);              // accumulator ready for the epilogue
+                if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+            }
+            if (!ok) *abort_flag = 1;
+        }
+    } else {
+        // ------------------------------------------------ epilogue (warps 2..5)
+        const int quad = warp & 3;                       // TMEM lane quadrant of this warp
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+            bool ok = true;
+            if (lane == 0) ok = mbar_wait(&acc_full[acc], acc_phase, p.err) && !*abort_flag;
+            ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+            if (!ok) break;
+            tc_fence_after();
+            const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, D, tile);
+            const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * C::ACC_COLS);
+            if (SWAP) {
+                // lane = weight row (32 per warp), columns = TOKTILE (16) tokens
+                uint32_t r[16];
+                tmem_ld16(tbase, r);
+                tmem_ld_wait();
+                if (EPI == 0) {
+                    // rows: 16 gate then 16 up of FFN block (4 * wt + quad)
+                    const int j = (t.wt * 4 + quad) * 16 + (lane & 15);
+                    __nv_bfloat16* act = static_cast<__nv_bfloat16*>(p.out);
+#pragma unroll
+                    for (int c = 0; c < 16; ++c) {
+                        const float v = __uint_as_float(r[c]);
+                        const float u = __shfl_xor_sync(0xffffffffu, v, 16);
+                        if (lane < 16 && c < t.nrows)
+                            act[(size_t)(t.row0 + c) * p.out_ld + j] = __float2bfloat16_rn(silu(v) * u);
+                    }
+                } else {
+                    const int col = t.wt * C::WTILE + quad * 32 + lane;
+                    float* y = static_cast<float*>(p.out);
+#pragma unroll
+                    for (int c = 0; c < 16; ++c) {
+                        if (c < t.nrows)
+                            y[(size_t)(t.row0 + c) * p.out_ld + col] = p.ghat_perm[t.row0 + c] * __uint_as_float(r[c]);
+                    }
+                }
+            } else {
+                // lane = token row, columns = WTILE weight rows
+                const int row = quad * 32 + lane;
+                const bool valid = row < t.nrows;
+                const size_t orow = (size_t)(t.row0 + row);
+                if (EPI == 0) {
+                    __nv_bfloat16* act = static_cast<__nv_bfloat16*>(p.out);
+#pragma unroll 1
+                    for (int blk = 0; blk < C::WTILE / 32; ++blk) {
+                        uint32_t g[16], u[16];
+                        tmem_ld16(tbase + blk * 32, g);
+                        tmem_ld16(tbase + blk * 32 + 16, u);
+                        tmem_ld_wait();
+                        if (valid) {
+                            __align__(16) __nv_bfloat16 o[16];
+#pragma unroll
+                            for (int i = 0; i < 16; ++i)
+                                o[i] = __float2bfloat16_rn(silu(__uint_as_float(g[i])) * __uint_as_float(u[i]));
+                            const int j0 = (t.wt * (C::WTILE / 32) + blk) * 16;
+                            uint4* dst = reinterpret_cast<uint4*>(act + orow * p.out_ld + j0);
+                            dst[0] = reinterpret_cast<const uint4*>(o)[0];
+                            dst[1] = reinterpret_cast<const uint4*>(o)[1];
+                        }
+                    }
+                } else {
+                    float* y = static_cast<float*>(p.out);
+                    const float gh = valid ? p.ghat_perm[orow] : 0.f;
+#pragma unroll 1
+                    for (int c0 = 0; c0 < C::WTILE; c0 += 16) {
+                        uint32_t r[16];
+                        tmem_ld16(tbase + c0, r);
+                        tmem_ld_wait();
+                        if (valid) {
+                            float4* dst = reinterpret_cast<float4*>(y + orow * p.out_ld + t.wt * C::WTILE + c0);
+#pragma unroll
+                            for (int i = 0; i < 4; ++i)
+                                dst[i] = make_float4(gh * __uint_as_float(r[4 * i]), gh * __uint_as_float(r[4 * i + 1]),
+                                                     gh * __uint_as_float(r[4 * i + 2]), gh * __uint_as_float(r[4 * i + 3]));
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acc_empty[acc]);
+            if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) {
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                     "r"((uint32_t)C::TMEM_COLS));
+    }
+}
+
+// ---------------------------------------------------------------- helper kernels
+
+// h_perm[r] = h[perm[r] / k], g_perm[r] = g_hat[perm[r]]: token rows in
+// expert-grouped order for the TMA loads of GEMM 1.
+__global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __restrict__ h,
+                                                     const int32_t* __restrict__ perm,
+                                                     const float* __restrict__ ghat,
+                                                     const int32_t* __restrict__ meta,
+                                                     __nv_bfloat16* __restrict__ h_perm, float* __restrict__ g_perm,
+                                                     int d, int k) {
+    const int R = meta[kMetaRetained];
+    const int nvec = d / 8;
+    const long long total = (long long)R * nvec;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int r = (int)(i / nvec), c = (int)(i % nvec);
+        const int s = perm[r];
+        reinterpret_cast<uint4*>(h_perm + (size_t)r * d)[c] = reinterpret_cast<const uint4*>(h + (size_t)(s / k) * d)[c];
+        if (c == 0) g_perm[r] = ghat[s];
+    }
+}
+
+// out[t, c] = sum_{i kept, rank order} y[slot_pos[t*k+i], c]  (Eq. ace_sparse_output)
+__global__ void __launch_bounds__(256) k_combine_bf16(const float* __restrict__ y, const int32_t* __restrict__ slot_pos,
+                                                      __nv_bfloat16* __restrict__ out, int n_tokens, int d, int k) {
+    const int nq = d / 8;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)n_tokens * nq) return;
+    const int t = (int)(idx / nq), c8 = (int)(idx % nq);
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int i = 0; i < k; ++i) {
+        const int r = slot_pos[(size_t)t * k + i];
+        if (r < 0) continue;
+        const float4* src = reinterpret_cast<const float4*>(y + (size_t)r * d) + 2 * c8;
+        const float4 a = src[0], b = src[1];
+        acc[0] += a.x; acc[1] += a.y; acc[2] += a.z; acc[3] += a.w;
+        acc[4] += b.x; acc[5] += b.y; acc[6] += b.z; acc[7] += b.w;
+    }
+    __align__(16) __nv_bfloat16 o[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) o[i] = __float2bfloat16_rn(acc[i]);
+    reinterpret_cast<uint4*>(out + (size_t)t * d)[c8] = *reinterpret_cast<const uint4*>(o);
+}
+
+// ---------------------------------------------------------------- host side
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+cudaError_t get_encoder() {
+    if (g_encode) return cudaSuccess;
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess) return e;
+    if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    return cudaSuccess;
+}
+
+// 2-D bf16 map over [rows, cols] (row-major), box [box_rows, 64], 128-byte swizzle.
+cudaError_t make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+    cudaError_t e = get_encoder();
+    if (e != cudaSuccess) return e;
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {cols * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)kBK, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+constexpr int kStagesSwap = 10;
+constexpr int kStagesWide = 4;
+
+template <bool SWAP, int EPI>
+constexpr int stages_for() { return SWAP ? kStagesSwap : kStagesWide; }
+
+template <bool SWAP, int EPI>
+cudaError_t set_attr() {
+    constexpr int S = stages_for<SWAP, EPI>();
+    return cudaFuncSetAttribute(k_expert_tc<SWAP, EPI, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                TcCfg<SWAP, EPI, S>::SMEM);
+}
+
+template <bool SWAP, int EPI>
+cudaError_t launch_gemm(const ace_layer* L, const TcParams& p, cudaStream_t s) {
+    constexpr int S = stages_for<SWAP, EPI>();
+    k_expert_tc<SWAP, EPI, S><<<L->num_sms, kThreads, TcCfg<SWAP, EPI, S>::SMEM, s>>>(p);
+    return cudaGetLastError();
+}
+
+// W_gu[e, 32b + i] = W_gate[e, 16b + i] (i < 16), W_up[e, 16b + i - 16] (i >= 16).
+__global__ void __launch_bounds__(256) k_pack_gate_up(const uint4* __restrict__ wg, const uint4* __restrict__ wu,
+                                                      uint4* __restrict__ wgu, int n_exp, int m, int d) {
+    const int nvec = d / 8;
+    const long long total = (long long)n_exp * 2 * m * nvec;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const long long row = i / nvec;
+        const int c = (int)(i % nvec);
+        const int e = (int)(row / (2 * m));
+        const int pr = (int)(row % (2 * m));
+        const int b = pr >> 5, li = pr & 31;
+        const int j = b * 16 + (li & 15);
+        const uint4* src = li < 16 ? wg : wu;
+        wgu[i] = src[((long long)e * m + j) * nvec + c];
+    }
+}
+
+}  // namespace
+
+cudaError_t tc_pack_gate_up(ace_layer* L, const void* w_gate, const void* w_up, cudaStream_t s) {
+    const ace_layer_desc& D = L->desc;
+    k_pack_gate_up<<<L->num_sms * 8, 256, 0, s>>>((const uint4*)w_gate, (const uint4*)w_up, (uint4*)L->w_gu,
+                                                  D.n_experts, D.ffn, D.hidden);
+    return cudaGetLastError();
+}
+
+int tc_token_tile(int T) { return T <= kTcSmallT ? 16 : 128; }
+
+bool tc_supported(const ace_layer* L) {
+    const ace_layer_desc& D = L->desc;
+    return D.dtype == ACE_BF16 && D.ffn % 128 == 0 && D.hidden % 256 == 0;
+}
+
+cudaError_t tc_init(ace_layer* L) {
+    if (!tc_supported(L)) return cudaSuccess;
+    const ace_layer_desc& D = L->desc;
+    cudaError_t e;
+    if ((e = set_attr<true, 0>()) != cudaSuccess) return e;
+    if ((e = set_attr<true, 1>()) != cudaSuccess) return e;
+    if ((e = set_attr<false, 0>()) != cudaSuccess) return e;
+    if ((e = set_attr<false, 1>()) != cudaSuccess) return e;
+    const uint64_t rows = (uint64_t)D.max_tokens * D.top_k;
+    const uint64_t n = D.n_experts, d = D.hidden, m = D.ffn;
+    // token maps: decode tiles of 16 rows and prefill tiles of 128 rows
+    if ((e = make_map(&L->tcm.tok1_small, L->ws.h_perm, rows, d, 16)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.tok1_big, L->ws.h_perm, rows, d, 128)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.tok2_small, L->ws.act_bf16, rows, m, 16)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.tok2_big, L->ws.act_bf16, rows, m, 128)) != cudaSuccess) return e;
+    // weight maps: W_gu [N * 2m, d] and W_down [N * d, m]
+    if ((e = make_map(&L->tcm.wgu_small, L->w_gu, n * 2 * m, d, 128)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.wgu_big, L->w_gu, n * 2 * m, d, 256)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.wd_small, L->w_down, n * d, m, 128)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.wd_big, L->w_down, n * d, m, 256)) != cudaSuccess) return e;
+    return cudaSuccess;
+}
+
+cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t s, cudaEvent_t* ev) {
+    const ace_layer_desc& D = L->desc;
+    const Workspace& W = L->ws;
+    const int d = D.hidden, m = D.ffn, k = D.top_k;
+    const bool small = T <= kTcSmallT;
+    const int rows_total = T * k;
+    (void)rows_total;
+    k_gather_rows<<<L->num_sms * 4, 256, 0, s>>>((const __nv_bfloat16*)W.h, W.perm, W.ghat, W.meta,
+                                                 (__nv_bfloat16*)W.h_perm, W.g_perm, d, k);
+    if (ev) cudaEventRecord(ev[0], s);
+    TcParams p1{};
+    p1.tm_tok = small ? L->tcm.tok1_small : L->tcm.tok1_big;
+    p1.tm_w = small ? L->tcm.wgu_small : L->tcm.wgu_big;
+    p1.offsets = W.offsets;
+    p1.dlist = W.dlist;
+    p1.tt_off = W.tt_off;
+    p1.meta = W.meta;
+    p1.ghat_perm = W.g_perm;
+    p1.out = W.act_bf16;
+    p1.K = d;
+    p1.w_rows = 2 * m;
+    p1.w_tiles = 2 * m / (small ? 128 : 256);
+    p1.out_ld = m;
+    p1.err = W.err;
+    cudaError_t e = small ? launch_gemm<true, 0>(L, p1, s) : launch_gemm<false, 0>(L, p1, s);
+    if (e != cudaSuccess) return e;
+    if (ev) cudaEventRecord(ev[1], s);
+    TcParams p2 = p1;
+    p2.tm_tok = small ? L->tcm.tok2_small : L->tcm.tok2_big;
+    p2.tm_w = small ? L->tcm.wd_small : L->tcm.wd_big;
+    p2.out = W.yslot;
+    p2.K = m;
+    p2.w_rows = d;
+    p2.w_tiles = d / (small ? 128 : 256);
+    p2.out_ld = d;
+    e = small ? launch_gemm<true, 1>(L, p2, s) : launch_gemm<false, 1>(L, p2, s);
+    if (e != cudaSuccess) return e;
+    if (ev) cudaEventRecord(ev[2], s);
+    const long long nthreads = (long long)T * (d / 8);
+    k_combine_bf16<<<(int)((nthreads + 255) / 256), 256, 0, s>>>(W.yslot, W.slot_pos, (__nv_bfloat16*)out, T, d, k);
+    if (ev) cudaEventRecord(ev[3], s);
+    return cudaGetLastError();
+}
+
+}  // namespace ace

@@ -3,8 +3,9 @@
 // csrc/ includes it.
 #pragma once
 
-#include <cuda_runtime.h>
+#include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_runtime.h>
 #include <stdint.h>
 
 #include "ace.h"
@@ -32,6 +33,7 @@ enum : int {
 };
 
 constexpr int kChunk = 256;          // tokens per compaction block
+constexpr int kTcSmallT = 256;       // tensor-core experts: decode tiling up to this many tokens
 constexpr int kMaxExperts = 1024;
 constexpr int kMaxTopK = 16;
 constexpr int kGemvTokenChunk = 8;   // tokens processed per weight pass in the GEMVs
@@ -52,11 +54,23 @@ struct Workspace {
     int32_t* perm = nullptr;     // [Tmax*k]
     int32_t* slot_pos = nullptr; // [Tmax*k] row of slot t*k+i in perm order, -1 if skipped
     int32_t* meta = nullptr;     // [kMetaCount]
-    float* act = nullptr;        // [Tmax*k, m] fp32 (GEMV path)
-    float* yslot = nullptr;      // [Tmax*k, d] fp32 (GEMV path)
+    float* act = nullptr;        // [Tmax*k, m] fp32 (CUDA-core path)
+    float* yslot = nullptr;      // [Tmax*k, d] fp32: g_hat-scaled expert outputs per retained slot
+    void* h_perm = nullptr;      // [Tmax*k, d] bf16: h rows in expert-grouped order (tensor path)
+    float* g_perm = nullptr;     // [Tmax*k] g_hat in expert-grouped order
+    void* act_bf16 = nullptr;    // [Tmax*k, m] bf16 (tensor path)
+    int32_t* tt_off = nullptr;   // [N+1] token-tile prefix over distinct experts
     int* err = nullptr;          // device error word
     void* x_stage = nullptr;     // [Tmax, d] dtype: host-API staging
     void* out_stage = nullptr;   // [Tmax, d]
+};
+
+// Tensor maps of the tensor-core expert path (built once at create time).
+struct TcMaps {
+    CUtensorMap tok1_small, tok1_big;   // h_perm, boxes of 16 / 128 rows
+    CUtensorMap tok2_small, tok2_big;   // act_bf16
+    CUtensorMap wgu_small, wgu_big;     // W_gu, boxes of 128 / 256 rows
+    CUtensorMap wd_small, wd_big;       // W_down
 };
 
 }  // namespace ace
@@ -69,8 +83,11 @@ struct ace_layer {
     // layer-owned weights
     void* router_w = nullptr;    // [N, d]
     float* router_b = nullptr;   // [N] (zeros when there is no bias)
-    void* w_gate = nullptr;      // [N, m, d]
-    void* w_up = nullptr;        // [N, m, d]
+    void* w_gate = nullptr;      // [N, m, d] (CUDA-core path only)
+    void* w_up = nullptr;        // [N, m, d] (CUDA-core path only)
+    void* w_gu = nullptr;        // [N, 2m, d] gate/up rows interleaved in blocks of 16 (tensor path)
+    bool tc = false;             // tensor-core expert path in use
+    ace::TcMaps tcm;
     void* w_down = nullptr;      // [N, d, m]
     void* gamma = nullptr;       // [d]
     float* a_gsp = nullptr;      // [N]
@@ -83,7 +100,7 @@ struct ace_layer {
     bool last_has_logits = false;
     // stage timing (ace_layer_set_profiling)
     bool profiling = false;
-    cudaEvent_t ev[8] = {};
+    cudaEvent_t ev[10] = {};
     int n_stages = 0;
     int last_launches = 0;       // kernels launched by the last forward / route call
 };
@@ -108,6 +125,14 @@ cudaError_t launch_debug_exp(const float* x, float* y, int n, cudaStream_t s);
 cudaError_t gemv_init(const ace_layer* L);
 cudaError_t launch_experts_gemv(const ace_layer* L, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
 
-constexpr int kNumStages = 6;
+constexpr int kNumStages = 7;
+
+// ---- tensor-core expert path (ace_expert_tc.cu) ----
+bool tc_supported(const ace_layer* L);
+int tc_token_tile(int T);
+cudaError_t tc_init(ace_layer* L);
+cudaError_t tc_pack_gate_up(ace_layer* L, const void* w_gate, const void* w_up, cudaStream_t s);
+// ev (nullable): recorded after gather, after gate/up, after down, after combine.
+cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
 
 }  // namespace ace

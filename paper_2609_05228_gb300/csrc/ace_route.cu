@@ -292,16 +292,34 @@ __device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem
             if (in && (__ffs(grp) - 1) == (tid & 31)) atomicAdd(&S.hist[dg], __popc(grp));
         }
         __syncthreads();
-        if (tid == 0) {
-            int want = S.want, cum = 0, dg = 0;
-            for (; dg < 255; ++dg) {
-                if (cum + S.hist[dg] > want) break;
-                cum += S.hist[dg];
+        if (tid < 32) {
+            // warp 0: lane l owns bins 8l..8l+7; find the bin where the running
+            // count first exceeds `want`
+            const int want = S.want;
+            int h8[8], loc = 0;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) { h8[j] = S.hist[tid * 8 + j]; loc += h8[j]; }
+            int inc = loc;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xffffffffu, inc, o);
+                if (tid >= o) inc += y;
             }
-            S.want = want - cum;
-            S.below += cum;
-            S.last_cnt = S.hist[dg];
-            S.prefix = prefix | ((uint32_t)dg << shift);
+            const int exc = inc - loc;
+            const bool mine = exc <= want && want < inc;
+            const unsigned who = __ballot_sync(0xffffffffu, mine);
+            const int owner = who ? __ffs(who) - 1 : 31;
+            if (tid == owner) {
+                int cum = exc, dg = tid * 8;
+                for (int j = 0; j < 7; ++j, ++dg) {
+                    if (cum + h8[j] > want) break;
+                    cum += h8[j];
+                }
+                S.want = want - cum;
+                S.below += cum;
+                S.last_cnt = S.hist[dg];
+                S.prefix = prefix | ((uint32_t)dg << shift);
+            }
         }
         __syncthreads();
         prefix = S.prefix;
@@ -320,31 +338,47 @@ __device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem
 // Exclusive scan of cnt[0..n_exp) by warp 0 of the block: offsets[e],
 // offsets[n_exp] = total, the distinct-expert list and the meta totals.
 // Also fills off_s (shared) when given.
+// With tok_tile > 0 it also writes tt_off[j] = sum over distinct experts
+// before j of ceil(count / tok_tile) (the token-tile schedule of the
+// tensor-core experts) and tt_off[D].
 __device__ void scan_counts_warp0(const int* cnt, int n_exp, int32_t* __restrict__ offsets,
-                                  int32_t* __restrict__ dlist, int32_t* __restrict__ meta, int* off_s) {
+                                  int32_t* __restrict__ dlist, int32_t* __restrict__ meta, int* off_s,
+                                  int tok_tile, int32_t* __restrict__ tt_off) {
     const int lane = threadIdx.x;
     const int per = (n_exp + 31) / 32;
     const int e0 = min(lane * per, n_exp), e1 = min(e0 + per, n_exp);
-    int s = 0, dcount = 0;
-    for (int e = e0; e < e1; ++e) { s += cnt[e]; dcount += cnt[e] > 0; }
-    int xs = s, xd = dcount;
+    const int tt = tok_tile > 0 ? tok_tile : 1;
+    int s = 0, dcount = 0, tiles = 0;
+    for (int e = e0; e < e1; ++e) {
+        s += cnt[e];
+        dcount += cnt[e] > 0;
+        tiles += (cnt[e] + tt - 1) / tt;
+    }
+    int xs = s, xd = dcount, xt = tiles;
     for (int o = 1; o < 32; o <<= 1) {
         const int ys = __shfl_up_sync(0xffffffffu, xs, o);
         const int yd = __shfl_up_sync(0xffffffffu, xd, o);
-        if (lane >= o) { xs += ys; xd += yd; }
+        const int yt = __shfl_up_sync(0xffffffffu, xt, o);
+        if (lane >= o) { xs += ys; xd += yd; xt += yt; }
     }
-    int run = xs - s, drun = xd - dcount;
+    int run = xs - s, drun = xd - dcount, trun = xt - tiles;
     for (int e = e0; e < e1; ++e) {
         offsets[e] = run;
         if (off_s) off_s[e] = run;
         run += cnt[e];
-        if (cnt[e] > 0) dlist[drun++] = e;
+        if (cnt[e] > 0) {
+            if (tok_tile > 0) tt_off[drun] = trun;
+            trun += (cnt[e] + tt - 1) / tt;
+            dlist[drun++] = e;
+        }
     }
     const int total = __shfl_sync(0xffffffffu, xs, 31);
     const int dtotal = __shfl_sync(0xffffffffu, xd, 31);
+    const int ttotal = __shfl_sync(0xffffffffu, xt, 31);
     if (lane == 31) {
         offsets[n_exp] = total;
         if (off_s) off_s[n_exp] = total;
+        if (tok_tile > 0) tt_off[dtotal] = ttotal;
         meta[kMetaRetained] = total;
         meta[kMetaDistinct] = dtotal;
     }
@@ -436,7 +470,8 @@ __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, i
                                                           int32_t* __restrict__ chunk_counts,
                                                           int32_t* __restrict__ offsets,
                                                           int32_t* __restrict__ dlist,
-                                                          int32_t* __restrict__ meta) {
+                                                          int32_t* __restrict__ meta, int tok_tile,
+                                                          int32_t* __restrict__ tt_off) {
     __shared__ int cnt[kMaxExperts];
     __shared__ bool is_last;
     for (int e = threadIdx.x; e < n_exp; e += blockDim.x) cnt[e] = 0;
@@ -468,7 +503,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, i
     }
     __syncthreads();
     if (threadIdx.x < 32) {
-        scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, nullptr);
+        scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, nullptr, tok_tile, tt_off);
         if (threadIdx.x == 0) meta[kMetaTicket] = 0;
     }
 }
@@ -518,7 +553,7 @@ __global__ void __launch_bounds__(kSmallThreads) k_route_small(
     int32_t* __restrict__ ids, float* __restrict__ gates, float* __restrict__ cval, uint8_t* __restrict__ skip,
     float* __restrict__ ghat, float* __restrict__ tau_out, int32_t* __restrict__ offsets,
     int32_t* __restrict__ dlist, int32_t* __restrict__ perm, int32_t* __restrict__ slot_pos,
-    int32_t* __restrict__ meta, int* __restrict__ err) {
+    int32_t* __restrict__ meta, int* __restrict__ err, int tok_tile, int32_t* __restrict__ tt_off) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int ns = n_tokens * k;
     float* g_s = reinterpret_cast<float*>(smem_raw);
@@ -596,7 +631,7 @@ __global__ void __launch_bounds__(kSmallThreads) k_route_small(
         atomicOr(&bm[e * 8 + (t >> 5)], 1u << (t & 31));
     }
     __syncthreads();
-    if (threadIdx.x < 32) scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, off_s);
+    if (threadIdx.x < 32) scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, off_s, tok_tile, tt_off);
     __syncthreads();
     for (int s = threadIdx.x; s < ns; s += blockDim.x) {
         if (skip_s[s]) { slot_pos[s] = -1; continue; }
@@ -692,10 +727,11 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     bool need_select;
     const int m_q = select_mq(L, T, ctl, &tau, &need_select);
     const int mode = need_select ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
+    const int tok_tile = L->tc ? tc_token_tile(T) : 0;
     if (T <= kSmallT) {
         k_route_small<<<1, kSmallThreads, small_smem_bytes(T, k, n), s>>>(
             logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode, tau, m_q, W.ids, W.gates, W.cval,
-            W.skip, W.ghat, W.tau, W.offsets, W.dlist, W.perm, W.slot_pos, W.meta, W.err);
+            W.skip, W.ghat, W.tau, W.offsets, W.dlist, W.perm, W.slot_pos, W.meta, W.err, tok_tile, W.tt_off);
         return cudaGetLastError();
     }
     const int blocks = cdiv(T, 8);
@@ -707,7 +743,7 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     }
     const int n_chunks = cdiv(T, kChunk);
     k_compact_count<<<n_chunks, kChunk, 0, s>>>(T, k, n, n_chunks, W.ids, W.skip, W.chunk_counts,
-                                                W.offsets, W.dlist, W.meta);
+                                                W.offsets, W.dlist, W.meta, tok_tile, W.tt_off);
     k_compact_place<<<n_chunks, kChunk, 0, s>>>(T, k, n, W.ids, W.skip, W.chunk_counts, W.offsets,
                                                 W.perm, W.slot_pos);
     return cudaGetLastError();
