@@ -137,8 +137,12 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     cudaDeviceGetAttribute(&L->num_sms, cudaDevAttrMultiProcessorCount, L->device);
     if (L->num_sms <= 0) L->num_sms = 1;
 
-    const size_t d = D.hidden, n = D.n_experts, k = D.top_k, m = D.ffn, T = D.max_tokens, E = L->elem;
-    const size_t slots = T * k;
+    const size_t d = D.hidden, n = D.n_experts, k = D.top_k, m = D.ffn, E = L->elem;
+    // Buffers read by tensor maps are padded so that every TMA box (up to
+    // 256 rows) lies inside the tensor.
+    const size_t T = D.max_tokens < 256 ? 256 : D.max_tokens;
+    const size_t slots = (size_t)D.max_tokens * k < 256 ? 256 : (size_t)D.max_tokens * k;
+    const size_t n_pad = (n + 255) / 256 * 256;
     const int n_chunks = (int)((T + ace::kChunk - 1) / ace::kChunk);
     ace::Workspace& W = L->ws;
     cudaError_t e = cudaSuccess;
@@ -152,7 +156,7 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
         }                                                                   \
     } while (0)
     L->tc = ace::tc_supported(L);
-    ALLOC(L->router_w, n * d * E);
+    ALLOC(L->router_w, n_pad * d * E);
     ALLOC(L->router_b, n * sizeof(float));
     if (L->tc) {
         ALLOC(L->w_gu, n * 2 * m * d * E);
@@ -200,6 +204,7 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
             return cuda_fail(e, where);       \
         }                                     \
     } while (0)
+    CK(cudaMemsetAsync(L->router_w, 0, n_pad * d * E, s), "zero router_w padding");
     CK(cudaMemcpyAsync(L->router_w, router_w, n * d * E, cudaMemcpyDeviceToDevice, s), "copy router_w");
     if (D.has_router_bias)
         CK(cudaMemcpyAsync(L->router_b, router_b, n * sizeof(float), cudaMemcpyDeviceToDevice, s), "copy router_b");
@@ -276,7 +281,10 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
     if (ev) ACE_CUDA(cudaEventRecord(ev[0], s), "event record");
     if (!small) ACE_CUDA(ace::launch_rmsnorm(L, x, T, s), "rmsnorm launch");
     if (ev) ACE_CUDA(cudaEventRecord(ev[1], s), "event record");
-    ACE_CUDA(ace::launch_router(L, x, T, small, s), "router launch");
+    if (L->tc && !small)
+        ACE_CUDA(ace::launch_router_tc(L, T, s), "router launch");
+    else
+        ACE_CUDA(ace::launch_router(L, x, T, small, s), "router launch");
     if (ev) ACE_CUDA(cudaEventRecord(ev[2], s), "event record");
     ACE_CUDA(ace::launch_route(L, L->ws.logits, T, ctl, s), "route launch");
     if (ev) ACE_CUDA(cudaEventRecord(ev[3], s), "event record");

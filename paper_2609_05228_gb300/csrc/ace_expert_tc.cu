@@ -51,6 +51,12 @@ struct TcParams {
     int w_tiles;                        // w_rows / weight tile
     int out_ld;                         // row length of out
     int* err;
+    // single-group schedule (router logits): rows > 0 replaces the expert groups
+    int single_rows;
+    const float* bias;                  // [n_valid_cols] (EPI 2)
+    float inv_temp;
+    int use_temp;
+    int n_valid_cols;                   // columns of out that exist (EPI 2)
 };
 
 // ---------------------------------------------------------------- PTX wrappers
@@ -169,6 +175,15 @@ template <int TOKTILE, int WTILE>
 __device__ __forceinline__ Tile tile_at(const TcParams& p, int D, int tile) {
     const int tt = tile / p.w_tiles;
     const int wt = tile - tt * p.w_tiles;
+    if (p.single_rows > 0) {
+        Tile t;
+        t.e = 0;
+        t.row0 = tt * TOKTILE;
+        t.nrows = min(TOKTILE, p.single_rows - t.row0);
+        t.wrow0 = wt * WTILE;
+        t.wt = wt;
+        return t;
+    }
     int lo = 0, hi = D;                       // largest j with tt_off[j] <= tt
     while (hi - lo > 1) {
         const int mid = (lo + hi) >> 1;
@@ -189,7 +204,8 @@ __device__ __forceinline__ Tile tile_at(const TcParams& p, int D, int tile) {
 
 // SWAP: A (M = 128) = weight rows, B (N = TOKTILE) = token rows.
 // !SWAP: A (M = 128) = token rows, B (N = WTILE) = weight rows.
-// EPI 0: SwiGLU into act (bf16); EPI 1: g_hat-scaled rows into y (fp32).
+// EPI 0: SwiGLU into act (bf16); EPI 1: g_hat-scaled rows into y (fp32);
+// EPI 2: router logits (fp32, + bias, / temperature), !SWAP only.
 template <bool SWAP, int EPI, int STAGES>
 struct TcCfg {
     static constexpr int TOKTILE = SWAP ? 16 : 128;
@@ -219,8 +235,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int D = p.meta[kMetaDistinct];
-    const int n_tiles = p.tt_off[D] * p.w_tiles;
+    const int D = p.single_rows > 0 ? 1 : p.meta[kMetaDistinct];
+    const int n_tiles = (p.single_rows > 0 ? (p.single_rows + C::TOKTILE - 1) / C::TOKTILE : p.tt_off[D]) * p.w_tiles;
     const int kblocks = p.K / kBK;
 
     if (threadIdx.x == 0) {
@@ -372,6 +388,27 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                             uint4* dst = reinterpret_cast<uint4*>(act + orow * p.out_ld + j0);
                             dst[0] = reinterpret_cast<const uint4*>(o)[0];
                             dst[1] = reinterpret_cast<const uint4*>(o)[1];
+                        }
+                    }
+                } else if (EPI == 2) {
+                    float* z = static_cast<float*>(p.out);
+#pragma unroll 1
+                    for (int c0 = 0; c0 < C::WTILE; c0 += 16) {
+                        const int col0 = t.wt * C::WTILE + c0;
+                        if (col0 >= p.n_valid_cols) break;
+                        uint32_t r[16];
+                        tmem_ld16(tbase + c0, r);
+                        tmem_ld_wait();
+                        if (valid) {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                const int col = col0 + i;
+                                if (col < p.n_valid_cols) {
+                                    float v = __uint_as_float(r[i]) + p.bias[col];
+                                    if (p.use_temp) v = v * p.inv_temp;
+                                    z[orow * p.out_ld + col] = v;
+                                }
+                            }
                         }
                     }
                 } else {
@@ -542,7 +579,11 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = set_attr<true, 1>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 0>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 1>()) != cudaSuccess) return e;
-    const uint64_t rows = (uint64_t)D.max_tokens * D.top_k;
+    if ((e = set_attr<false, 2>()) != cudaSuccess) return e;
+    // row counts as allocated at create time (padded to at least 256 rows)
+    const uint64_t rows = (uint64_t)D.max_tokens * D.top_k < 256 ? 256 : (uint64_t)D.max_tokens * D.top_k;
+    const uint64_t h_rows = D.max_tokens < 256 ? 256 : (uint64_t)D.max_tokens;
+    const uint64_t n_pad = ((uint64_t)D.n_experts + 255) / 256 * 256;
     const uint64_t n = D.n_experts, d = D.hidden, m = D.ffn;
     // token maps: decode tiles of 16 rows and prefill tiles of 128 rows
     if ((e = make_map(&L->tcm.tok1_small, L->ws.h_perm, rows, d, 16)) != cudaSuccess) return e;
@@ -554,7 +595,29 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = make_map(&L->tcm.wgu_big, L->w_gu, n * 2 * m, d, 256)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.wd_small, L->w_down, n * d, m, 128)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.wd_big, L->w_down, n * d, m, 256)) != cudaSuccess) return e;
+    // router: h [Tmax, d] in 128-row boxes, W_r [N, d] in 256-row boxes
+    if ((e = make_map(&L->tcm.h_rows, L->ws.h, h_rows, d, 128)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.w_router, L->router_w, n_pad, d, 256)) != cudaSuccess) return e;
     return cudaSuccess;
+}
+
+cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s) {
+    const ace_layer_desc& D = L->desc;
+    TcParams p{};
+    p.tm_tok = L->tcm.h_rows;
+    p.tm_w = L->tcm.w_router;
+    p.out = L->ws.logits;
+    p.K = D.hidden;
+    p.w_rows = D.n_experts;
+    p.w_tiles = (D.n_experts + 255) / 256;
+    p.out_ld = D.n_experts;
+    p.err = L->ws.err;
+    p.single_rows = T;
+    p.bias = L->router_b;
+    p.inv_temp = 1.0f / D.router_temp;
+    p.use_temp = D.router_temp != 1.0f;
+    p.n_valid_cols = D.n_experts;
+    return launch_gemm<false, 2>(L, p, s);
 }
 
 cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t s, cudaEvent_t* ev) {

@@ -71,6 +71,7 @@ struct TcMaps {
     CUtensorMap tok2_small, tok2_big;   // act_bf16
     CUtensorMap wgu_small, wgu_big;     // W_gu, boxes of 128 / 256 rows
     CUtensorMap wd_small, wd_big;       // W_down
+    CUtensorMap h_rows, w_router;       // router GEMM: h and W_r
 };
 
 }  // namespace ace
@@ -134,5 +135,7 @@ cudaError_t tc_init(ace_layer* L);
 cudaError_t tc_pack_gate_up(ace_layer* L, const void* w_gate, const void* w_up, cudaStream_t s);
 // ev (nullable): recorded after gather, after gate/up, after down, after combine.
 cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
+// Router logits on the tensor cores (T > kTcSmallT): z = (h W_r^T + b) / temp.
+cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s);
 
 }  // namespace ace

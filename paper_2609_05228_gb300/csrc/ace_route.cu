@@ -21,27 +21,45 @@ constexpr int kSmallT = 256;
 // RMSNorm (§3.1: expert and router input x = x_bar Gamma). One warp per token.
 // h = x / sqrt(mean(x^2) + rms_eps) * gamma, computed in float, stored as T.
 // --------------------------------------------------------------------------
+// The row is read once into registers (all 16-byte loads issued before any
+// arithmetic), then normalised from registers; supports d <= 32 * 16 * V.
+constexpr int kNormVec = 16;
+
 template <typename T>
 __device__ __forceinline__ void rmsnorm_row(const T* __restrict__ xr, const T* __restrict__ gamma, T* hr, int d,
                                             float rms_eps, int lane) {
     constexpr int V = Vec16<T>::N;
-    float ss = 0.f;
-    for (int j = lane * V; j < d; j += 32 * V) {
-        float f[V];
-        Vec16<T>::to_float(*reinterpret_cast<const uint4*>(xr + j), f);
+    const int nvec = d / V;
+    const uint4* xv = reinterpret_cast<const uint4*>(xr);
+    const uint4* gv = reinterpret_cast<const uint4*>(gamma);
+    uint4 xs[kNormVec];
 #pragma unroll
-        for (int i = 0; i < V; ++i) ss = fmaf(f[i], f[i], ss);
+    for (int i = 0; i < kNormVec; ++i) {
+        const int c = lane + 32 * i;
+        xs[i] = c < nvec ? xv[c] : make_uint4(0, 0, 0, 0);
+    }
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < kNormVec; ++i) {
+        float f[V];
+        Vec16<T>::to_float(xs[i], f);
+#pragma unroll
+        for (int j = 0; j < V; ++j) ss = fmaf(f[j], f[j], ss);
     }
     ss = warp_sum(ss);
     const float inv = 1.0f / sqrtf(ss / (float)d + rms_eps);
-    for (int j = lane * V; j < d; j += 32 * V) {
-        float f[V], gm[V];
-        Vec16<T>::to_float(*reinterpret_cast<const uint4*>(xr + j), f);
-        Vec16<T>::to_float(*reinterpret_cast<const uint4*>(gamma + j), gm);
-        T o[V];
 #pragma unroll
-        for (int i = 0; i < V; ++i) o[i] = from_f32<T>(f[i] * inv * gm[i]);
-        *reinterpret_cast<uint4*>(hr + j) = *reinterpret_cast<const uint4*>(o);
+    for (int i = 0; i < kNormVec; ++i) {
+        const int c = lane + 32 * i;
+        if (c < nvec) {
+            float f[V], gm[V];
+            Vec16<T>::to_float(xs[i], f);
+            Vec16<T>::to_float(gv[c], gm);
+            T o[V];
+#pragma unroll
+            for (int j = 0; j < V; ++j) o[j] = from_f32<T>(f[j] * inv * gm[j]);
+            reinterpret_cast<uint4*>(hr)[c] = *reinterpret_cast<const uint4*>(o);
+        }
     }
 }
 
@@ -156,23 +174,36 @@ struct SlotScore {
     float c;   // max(p_gsp, p_rcr)
 };
 
-// Top-k over one token's logits (one warp). Lane l owns experts l, l+32, ...
-// Order: larger logit first; ties to the lower expert index. NaN ranks last.
-// On return lane i < k holds (id, z) of rank i.
+// Top-k over one token's logits (one warp). Lane l owns experts l + 32 j,
+// j < NPL, held in registers. Order: larger logit first; ties to the lower
+// expert index. NaN ranks last. On return lane i < k holds (id, z) of rank i.
+template <int NPL>
 __device__ __forceinline__ void warp_topk(const float* __restrict__ zrow, int n_exp, int k, int lane,
                                           int& my_id, float& my_z, bool& saw_nan) {
-    unsigned taken = 0u;   // bit j: expert lane + 32*j already chosen
+    float v[NPL];
+    unsigned taken = 0u;   // bit j: expert lane + 32*j chosen already (or absent)
+    saw_nan = false;
+#pragma unroll
+    for (int j = 0; j < NPL; ++j) {
+        const int e = lane + 32 * j;
+        if (e < n_exp) {
+            float z = zrow[e];
+            if (z != z) { saw_nan = true; z = -INFINITY; }
+            v[j] = z;
+        } else {
+            v[j] = -INFINITY;
+            taken |= 1u << j;
+        }
+    }
     my_id = -1;
     my_z = 0.f;
-    saw_nan = false;
     for (int r = 0; r < k; ++r) {
         float bv = -INFINITY;
         int bi = 0x7fffffff;
-        for (int j = 0, e = lane; e < n_exp; ++j, e += 32) {
-            if ((taken >> j) & 1u) continue;
-            float v = zrow[e];
-            if (v != v) { saw_nan = true; v = -INFINITY; }
-            if (v > bv || (v == bv && e < bi)) { bv = v; bi = e; }
+#pragma unroll
+        for (int j = 0; j < NPL; ++j) {
+            const int e = lane + 32 * j;
+            if (!((taken >> j) & 1u) && (v[j] > bv || (v[j] == bv && e < bi))) { bv = v[j]; bi = e; }
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
@@ -269,27 +300,31 @@ __device__ __forceinline__ void decide_slot(int lane, int k, float g, float c, f
 // requires 0 < m < #candidates. Keys 0xffffffff are protected slots.
 // --------------------------------------------------------------------------
 struct SelectSmem {
-    int hist[256];
+    int hist[32][256];     // one histogram per warp (blockDim <= 1024)
+    int tot[256];
     uint32_t prefix;
     int want, below, last_cnt;
     float tau;
 };
 
 __device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem& S) {
-    const int tid = threadIdx.x;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int nwarps = blockDim.x >> 5;
     uint32_t prefix = 0u, mask = 0u;
     if (tid == 0) { S.want = m; S.below = 0; }
     for (int pass = 0; pass < 4; ++pass) {
         const int shift = 24 - 8 * pass;
-        for (int i = tid; i < 256; i += blockDim.x) S.hist[i] = 0;
+        for (int i = tid; i < nwarps * 256; i += blockDim.x) (&S.hist[0][0])[i] = 0;
         __syncthreads();
-        for (int i0 = 0; i0 < n; i0 += blockDim.x) {
-            const int i = i0 + tid;
-            const uint32_t key = i < n ? keys[i] : 0xffffffffu;
-            const bool in = key != 0xffffffffu && (key & mask) == prefix;
-            const int dg = (key >> shift) & 255;
-            const unsigned grp = __match_any_sync(0xffffffffu, in ? dg : -1);
-            if (in && (__ffs(grp) - 1) == (tid & 31)) atomicAdd(&S.hist[dg], __popc(grp));
+        for (int i = tid; i < n; i += blockDim.x) {
+            const uint32_t key = keys[i];
+            if (key != 0xffffffffu && (key & mask) == prefix) atomicAdd(&S.hist[warp][(key >> shift) & 255], 1);
+        }
+        __syncthreads();
+        for (int b = tid; b < 256; b += blockDim.x) {
+            int t = 0;
+            for (int w = 0; w < nwarps; ++w) t += S.hist[w][b];
+            S.tot[b] = t;
         }
         __syncthreads();
         if (tid < 32) {
@@ -298,7 +333,7 @@ __device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem
             const int want = S.want;
             int h8[8], loc = 0;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) { h8[j] = S.hist[tid * 8 + j]; loc += h8[j]; }
+            for (int j = 0; j < 8; ++j) { h8[j] = S.tot[tid * 8 + j]; loc += h8[j]; }
             int inc = loc;
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
@@ -317,7 +352,7 @@ __device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem
                 }
                 S.want = want - cum;
                 S.below += cum;
-                S.last_cnt = S.hist[dg];
+                S.last_cnt = S.tot[dg];
                 S.prefix = prefix | ((uint32_t)dg << shift);
             }
         }
@@ -390,6 +425,7 @@ __device__ void scan_counts_warp0(const int* cnt, int n_exp, int32_t* __restrict
 
 // Pass 1: top-k, gates, c. THRESHOLD mode also decides; RATIO mode writes
 // candidate keys (float bits of c, or 0xffffffff for protected slots).
+template <int NPL>
 __global__ void __launch_bounds__(256) k_topk_score(const float* __restrict__ logits, int n_tokens,
                                                     int n_exp, int k, const float* __restrict__ a_gsp,
                                                     const float* __restrict__ a_rcr, float eps,
@@ -405,7 +441,7 @@ __global__ void __launch_bounds__(256) k_topk_score(const float* __restrict__ lo
     int id;
     float zv;
     bool nan;
-    warp_topk(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
+    warp_topk<NPL>(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
     const float z0 = __shfl_sync(0xffffffffu, zv, 0);
     if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(err, kErrNumeric);
     const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a_gsp, a_rcr, eps);
@@ -547,6 +583,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
 // --------------------------------------------------------------------------
 constexpr int kSmallThreads = 1024;
 
+template <int NPL>
 __global__ void __launch_bounds__(kSmallThreads) k_route_small(
     const float* __restrict__ logits, int n_tokens, int n_exp, int k, const float* __restrict__ a_gsp,
     const float* __restrict__ a_rcr, float eps, int m_min, int mode, float tau_in, int m_q,
@@ -574,7 +611,7 @@ __global__ void __launch_bounds__(kSmallThreads) k_route_small(
         int id;
         float zv;
         bool nan;
-        warp_topk(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
+        warp_topk<NPL>(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
         const float z0 = __shfl_sync(0xffffffffu, zv, 0);
         if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(err, kErrNumeric);
         const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a_gsp, a_rcr, eps);
@@ -729,14 +766,24 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     const int mode = need_select ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
     const int tok_tile = L->tc ? tc_token_tile(T) : 0;
     if (T <= kSmallT) {
-        k_route_small<<<1, kSmallThreads, small_smem_bytes(T, k, n), s>>>(
-            logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode, tau, m_q, W.ids, W.gates, W.cval,
-            W.skip, W.ghat, W.tau, W.offsets, W.dlist, W.perm, W.slot_pos, W.meta, W.err, tok_tile, W.tt_off);
+#define ACE_ROUTE_SMALL(NPL)                                                                                   \
+    k_route_small<NPL><<<1, kSmallThreads, small_smem_bytes(T, k, n), s>>>(                                   \
+        logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode, tau, m_q, W.ids, W.gates, W.cval,      \
+        W.skip, W.ghat, W.tau, W.offsets, W.dlist, W.perm, W.slot_pos, W.meta, W.err, tok_tile, W.tt_off)
+        if (n <= 128) ACE_ROUTE_SMALL(4);
+        else if (n <= 256) ACE_ROUTE_SMALL(8);
+        else ACE_ROUTE_SMALL(32);
+#undef ACE_ROUTE_SMALL
         return cudaGetLastError();
     }
     const int blocks = cdiv(T, 8);
-    k_topk_score<<<blocks, 256, 0, s>>>(logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode,
-                                        tau, W.ids, W.gates, W.cval, W.keys, W.skip, W.ghat, W.tau, W.err);
+#define ACE_TOPK(NPL)                                                                                          \
+    k_topk_score<NPL><<<blocks, 256, 0, s>>>(logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode,   \
+                                             tau, W.ids, W.gates, W.cval, W.keys, W.skip, W.ghat, W.tau, W.err)
+    if (n <= 128) ACE_TOPK(4);
+    else if (n <= 256) ACE_TOPK(8);
+    else ACE_TOPK(32);
+#undef ACE_TOPK
     if (mode == ACE_SKIP_RATIO) {
         k_tau_select<<<1, kSelThreads, 0, s>>>(W.keys, T * k, m_q, W.tau);
         k_decide<<<blocks, 256, 0, s>>>(T, k, W.gates, W.cval, W.tau, D.min_active, D.eps, W.skip, W.ghat);
@@ -762,8 +809,12 @@ cudaError_t route_init(const ace_layer* L) {
     if (e != cudaSuccess) return e;
     e = set_router_attrs<float>(router_smem(L));
     if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(k_route_small, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)small_smem_bytes(kSmallT, L->desc.top_k, L->desc.n_experts));
+    const int sm = (int)small_smem_bytes(kSmallT, L->desc.top_k, L->desc.n_experts);
+    if ((e = cudaFuncSetAttribute(k_route_small<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm)) != cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(k_route_small<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm)) != cudaSuccess)
+        return e;
+    return cudaFuncSetAttribute(k_route_small<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
 }
 
 cudaError_t launch_debug_exp(const float* x, float* y, int n, cudaStream_t s) {
