@@ -42,8 +42,7 @@ void free_layer(ace_layer* L) {
     void* ptrs[] = {L->router_w, L->router_b, L->w_gate, L->w_up, L->w_gu, L->w_down, L->gamma, L->a_gsp,
                     L->a_rcr, L->ws.h, L->ws.logits, L->ws.ids, L->ws.gates, L->ws.cval, L->ws.keys, L->ws.skip,
                     L->ws.ghat, L->ws.tau, L->ws.chunk_counts, L->ws.offsets, L->ws.dlist, L->ws.perm,
-                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.g_perm,
-                    L->ws.act_bf16, L->ws.tt_off, L->ws.err, L->ws.x_stage, L->ws.out_stage};
+                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.act_bf16, L->ws.tt_off, L->ws.tt_tab, L->ws.tile_cnt, L->ws.err, L->ws.x_stage, L->ws.out_stage};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     for (cudaEvent_t e : L->ev)
@@ -183,11 +182,12 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     ALLOC(W.perm, slots * sizeof(int32_t));
     ALLOC(W.slot_pos, slots * sizeof(int32_t));
     ALLOC(W.meta, ace::kMetaCount * sizeof(int32_t));
+    ALLOC(W.tile_cnt, (T / 8 + 1) * sizeof(int32_t));
     if (L->tc) {
         ALLOC(W.h_perm, slots * d * E);
-        ALLOC(W.g_perm, slots * sizeof(float));
         ALLOC(W.act_bf16, slots * m * E);
         ALLOC(W.tt_off, (n + 1) * sizeof(int32_t));
+        ALLOC(W.tt_tab, (n + slots / 16 + 1) * sizeof(int4));
     } else {
         ALLOC(W.act, slots * m * sizeof(float));
     }
@@ -221,6 +221,7 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     CK(cudaMemcpyAsync(L->a_gsp, a_gsp, n * sizeof(float), cudaMemcpyHostToDevice, s), "copy a_gsp");
     CK(cudaMemcpyAsync(L->a_rcr, a_rcr, n * sizeof(float), cudaMemcpyHostToDevice, s), "copy a_rcr");
     CK(cudaMemsetAsync(W.meta, 0, ace::kMetaCount * sizeof(int32_t), s), "zero meta");
+    CK(cudaMemsetAsync(W.tile_cnt, 0, (T / 8 + 1) * sizeof(int32_t), s), "zero tickets");
     CK(cudaMemsetAsync(W.err, 0, sizeof(int), s), "zero error word");
     CK(cudaMemsetAsync(W.offsets, 0, (n + 1) * sizeof(int32_t), s), "zero offsets");
     CK(ace::route_init(L), "route kernel attributes");
@@ -281,12 +282,18 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
     if (ev) ACE_CUDA(cudaEventRecord(ev[0], s), "event record");
     if (!small) ACE_CUDA(ace::launch_rmsnorm(L, x, T, s), "rmsnorm launch");
     if (ev) ACE_CUDA(cudaEventRecord(ev[1], s), "event record");
-    if (L->tc && !small)
-        ACE_CUDA(ace::launch_router_tc(L, T, s), "router launch");
-    else
-        ACE_CUDA(ace::launch_router(L, x, T, small, s), "router launch");
-    if (ev) ACE_CUDA(cudaEventRecord(ev[2], s), "event record");
-    ACE_CUDA(ace::launch_route(L, L->ws.logits, T, ctl, s), "route launch");
+    if (small) {
+        // router and routing in one launch (stage "router" holds both)
+        ACE_CUDA(ace::launch_route_fused(L, x, L->ws.logits, T, ctl, s), "route launch");
+        if (ev) ACE_CUDA(cudaEventRecord(ev[2], s), "event record");
+    } else {
+        if (L->tc)
+            ACE_CUDA(ace::launch_router_tc(L, T, s), "router launch");
+        else
+            ACE_CUDA(ace::launch_router(L, x, T, false, s), "router launch");
+        if (ev) ACE_CUDA(cudaEventRecord(ev[2], s), "event record");
+        ACE_CUDA(ace::launch_route(L, L->ws.logits, T, ctl, s), "route launch");
+    }
     if (ev) ACE_CUDA(cudaEventRecord(ev[3], s), "event record");
     if (L->tc) {
         ACE_CUDA(ace::launch_experts_tc(L, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
@@ -295,7 +302,7 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
         ACE_CUDA(ace::launch_experts_gemv(L, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
     }
     L->n_stages = ev ? ace::kNumStages : 0;
-    L->last_launches = (small ? 1 : 2) + ace::route_launch_count(L, T, ctl) + (L->tc ? 4 : 3);
+    L->last_launches = (small ? 1 : 2 + ace::route_launch_count(L, T, ctl)) + (L->tc ? 4 : 3);
     return ACE_OK;
 }
 

@@ -42,9 +42,8 @@ struct TcParams {
     CUtensorMap tm_w;                   // weight rows [N * w_rows, K] bf16
     const int32_t* offsets;             // [N+1]
     const int32_t* dlist;               // [N]
-    const int32_t* tt_off;              // [N+1] token-tile prefix over distinct experts
+    const int4* tt_tab;                 // token tiles (expert, first row, rows, 0)
     const int32_t* meta;
-    const float* ghat_perm;             // [R] g_hat of row r (GEMM 2)
     void* out;                          // act bf16 [rows, m] or y fp32 [rows, d]
     int K;                              // reduction length
     int w_rows;                         // weight rows per expert (2m or d)
@@ -57,6 +56,9 @@ struct TcParams {
     float inv_temp;
     int use_temp;
     int n_valid_cols;                   // columns of out that exist (EPI 2)
+    const int32_t* perm;                // [R] slot of row r (GEMM 2 epilogue)
+    const float* ghat;                  // [T*k] g_hat by slot (GEMM 2 reads ghat[perm[r]])
+    int k;
 };
 
 // ---------------------------------------------------------------- PTX wrappers
@@ -172,29 +174,20 @@ struct Tile {
 };
 
 template <int TOKTILE, int WTILE>
-__device__ __forceinline__ Tile tile_at(const TcParams& p, int D, int tile) {
+__device__ __forceinline__ Tile tile_at(const TcParams& p, int tile) {
     const int tt = tile / p.w_tiles;
     const int wt = tile - tt * p.w_tiles;
+    Tile t;
     if (p.single_rows > 0) {
-        Tile t;
         t.e = 0;
         t.row0 = tt * TOKTILE;
         t.nrows = min(TOKTILE, p.single_rows - t.row0);
-        t.wrow0 = wt * WTILE;
-        t.wt = wt;
-        return t;
+    } else {
+        const int4 v = p.tt_tab[tt];
+        t.e = v.x;
+        t.row0 = v.y;
+        t.nrows = v.z;
     }
-    int lo = 0, hi = D;                       // largest j with tt_off[j] <= tt
-    while (hi - lo > 1) {
-        const int mid = (lo + hi) >> 1;
-        if (p.tt_off[mid] <= tt) lo = mid; else hi = mid;
-    }
-    Tile t;
-    t.e = p.dlist[lo];
-    const int blk = tt - p.tt_off[lo];
-    const int beg = p.offsets[t.e];
-    t.row0 = beg + blk * TOKTILE;
-    t.nrows = min(TOKTILE, p.offsets[t.e + 1] - t.row0);
     t.wrow0 = t.e * p.w_rows + wt * WTILE;
     t.wt = wt;
     return t;
@@ -235,8 +228,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int D = p.single_rows > 0 ? 1 : p.meta[kMetaDistinct];
-    const int n_tiles = (p.single_rows > 0 ? (p.single_rows + C::TOKTILE - 1) / C::TOKTILE : p.tt_off[D]) * p.w_tiles;
     const int kblocks = p.K / kBK;
 
     if (threadIdx.x == 0) {
@@ -260,6 +251,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    // everything above overlaps the predecessor kernel (PDL); its results are read below
+    pdl_wait();
+    const int n_tiles = (p.single_rows > 0 ? (p.single_rows + C::TOKTILE - 1) / C::TOKTILE : p.meta[kMetaTokTiles]) *
+                        p.w_tiles;
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
@@ -269,7 +264,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
             bool ok = true;
             long long issued = 0;
             for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-                const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, D, tile);
+                const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile);
                 for (int kb = 0; kb < kblocks; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
                     unsigned char* sa = smem + stage * C::STAGE_BYTES;
@@ -339,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
             ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
             if (!ok) break;
             tc_fence_after();
-            const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, D, tile);
+            const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile);
             const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * C::ACC_COLS);
             if (SWAP) {
                 // lane = weight row (32 per warp), columns = TOKTILE (16) tokens
@@ -363,7 +358,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
 #pragma unroll
                     for (int c = 0; c < 16; ++c) {
                         if (c < t.nrows)
-                            y[(size_t)(t.row0 + c) * p.out_ld + col] = p.ghat_perm[t.row0 + c] * __uint_as_float(r[c]);
+                            y[(size_t)(t.row0 + c) * p.out_ld + col] = p.ghat[p.perm[t.row0 + c]] * __uint_as_float(r[c]);
                     }
                 }
             } else {
@@ -413,7 +408,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                     }
                 } else {
                     float* y = static_cast<float*>(p.out);
-                    const float gh = valid ? p.ghat_perm[orow] : 0.f;
+                    const float gh = valid ? p.ghat[p.perm[orow]] : 0.f;
 #pragma unroll 1
                     for (int c0 = 0; c0 < C::WTILE; c0 += 16) {
                         uint32_t r[16];
@@ -437,6 +432,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
     }
     tc_fence_before();
     __syncthreads();
+    pdl_trigger();
     tc_fence_after();
     if (warp == 1) {
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
@@ -446,14 +442,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
 
 // ---------------------------------------------------------------- helper kernels
 
-// h_perm[r] = h[perm[r] / k], g_perm[r] = g_hat[perm[r]]: token rows in
-// expert-grouped order for the TMA loads of GEMM 1.
+// h_perm[r] = h[perm[r] / k]: token rows in expert-grouped order for the
+// TMA tile loads of GEMM 1.
 __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __restrict__ h,
                                                      const int32_t* __restrict__ perm,
-                                                     const float* __restrict__ ghat,
                                                      const int32_t* __restrict__ meta,
-                                                     __nv_bfloat16* __restrict__ h_perm, float* __restrict__ g_perm,
+                                                     __nv_bfloat16* __restrict__ h_perm,
                                                      int d, int k) {
+    pdl_wait();
     const int R = meta[kMetaRetained];
     const int nvec = d / 8;
     const long long total = (long long)R * nvec;
@@ -462,13 +458,13 @@ __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __rest
         const int r = (int)(i / nvec), c = (int)(i % nvec);
         const int s = perm[r];
         reinterpret_cast<uint4*>(h_perm + (size_t)r * d)[c] = reinterpret_cast<const uint4*>(h + (size_t)(s / k) * d)[c];
-        if (c == 0) g_perm[r] = ghat[s];
     }
 }
 
 // out[t, c] = sum_{i kept, rank order} y[slot_pos[t*k+i], c]  (Eq. ace_sparse_output)
 __global__ void __launch_bounds__(256) k_combine_bf16(const float* __restrict__ y, const int32_t* __restrict__ slot_pos,
                                                       __nv_bfloat16* __restrict__ out, int n_tokens, int d, int k) {
+    pdl_wait();
     const int nq = d / 8;
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= (long long)n_tokens * nq) return;
@@ -526,15 +522,16 @@ constexpr int stages_for() { return SWAP ? kStagesSwap : kStagesWide; }
 template <bool SWAP, int EPI>
 cudaError_t set_attr() {
     constexpr int S = stages_for<SWAP, EPI>();
-    return cudaFuncSetAttribute(k_expert_tc<SWAP, EPI, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                TcCfg<SWAP, EPI, S>::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(k_expert_tc<SWAP, EPI, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         TcCfg<SWAP, EPI, S>::SMEM);
+    if (e != cudaSuccess) return e;
+    return prefer_shared(k_expert_tc<SWAP, EPI, S>);
 }
 
 template <bool SWAP, int EPI>
 cudaError_t launch_gemm(const ace_layer* L, const TcParams& p, cudaStream_t s) {
     constexpr int S = stages_for<SWAP, EPI>();
-    k_expert_tc<SWAP, EPI, S><<<L->num_sms, kThreads, TcCfg<SWAP, EPI, S>::SMEM, s>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(k_expert_tc<SWAP, EPI, S>, dim3(L->num_sms), dim3(kThreads), TcCfg<SWAP, EPI, S>::SMEM, s, p);
 }
 
 // W_gu[e, 32b + i] = W_gate[e, 16b + i] (i < 16), W_up[e, 16b + i - 16] (i >= 16).
@@ -580,12 +577,14 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = set_attr<false, 0>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 1>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 2>()) != cudaSuccess) return e;
+    if ((e = prefer_shared(k_gather_rows)) != cudaSuccess) return e;
+    if ((e = prefer_shared(k_combine_bf16)) != cudaSuccess) return e;
     // row counts as allocated at create time (padded to at least 256 rows)
     const uint64_t rows = (uint64_t)D.max_tokens * D.top_k < 256 ? 256 : (uint64_t)D.max_tokens * D.top_k;
     const uint64_t h_rows = D.max_tokens < 256 ? 256 : (uint64_t)D.max_tokens;
     const uint64_t n_pad = ((uint64_t)D.n_experts + 255) / 256 * 256;
     const uint64_t n = D.n_experts, d = D.hidden, m = D.ffn;
-    // token maps: decode tiles of 16 rows and prefill tiles of 128 rows
+    // token maps: h_perm (GEMM 1) and act (GEMM 2), tiles of 16 / 128 rows
     if ((e = make_map(&L->tcm.tok1_small, L->ws.h_perm, rows, d, 16)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.tok1_big, L->ws.h_perm, rows, d, 128)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.tok2_small, L->ws.act_bf16, rows, m, 16)) != cudaSuccess) return e;
@@ -625,26 +624,27 @@ cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t
     const Workspace& W = L->ws;
     const int d = D.hidden, m = D.ffn, k = D.top_k;
     const bool small = T <= kTcSmallT;
-    const int rows_total = T * k;
-    (void)rows_total;
-    k_gather_rows<<<L->num_sms * 4, 256, 0, s>>>((const __nv_bfloat16*)W.h, W.perm, W.ghat, W.meta,
-                                                 (__nv_bfloat16*)W.h_perm, W.g_perm, d, k);
+    cudaError_t e = launch_pdl(k_gather_rows, dim3(L->num_sms * 4), dim3(256), 0, s, (const __nv_bfloat16*)W.h,
+                               (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k);
+    if (e != cudaSuccess) return e;
     if (ev) cudaEventRecord(ev[0], s);
     TcParams p1{};
     p1.tm_tok = small ? L->tcm.tok1_small : L->tcm.tok1_big;
     p1.tm_w = small ? L->tcm.wgu_small : L->tcm.wgu_big;
     p1.offsets = W.offsets;
     p1.dlist = W.dlist;
-    p1.tt_off = W.tt_off;
+    p1.tt_tab = W.tt_tab;
     p1.meta = W.meta;
-    p1.ghat_perm = W.g_perm;
+    p1.perm = W.perm;
+    p1.ghat = W.ghat;
+    p1.k = k;
     p1.out = W.act_bf16;
     p1.K = d;
     p1.w_rows = 2 * m;
     p1.w_tiles = 2 * m / (small ? 128 : 256);
     p1.out_ld = m;
     p1.err = W.err;
-    cudaError_t e = small ? launch_gemm<true, 0>(L, p1, s) : launch_gemm<false, 0>(L, p1, s);
+    e = small ? launch_gemm<true, 0>(L, p1, s) : launch_gemm<false, 0>(L, p1, s);
     if (e != cudaSuccess) return e;
     if (ev) cudaEventRecord(ev[1], s);
     TcParams p2 = p1;
@@ -659,9 +659,10 @@ cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t
     if (e != cudaSuccess) return e;
     if (ev) cudaEventRecord(ev[2], s);
     const long long nthreads = (long long)T * (d / 8);
-    k_combine_bf16<<<(int)((nthreads + 255) / 256), 256, 0, s>>>(W.yslot, W.slot_pos, (__nv_bfloat16*)out, T, d, k);
+    e = launch_pdl(k_combine_bf16, dim3((unsigned)((nthreads + 255) / 256)), dim3(256), 0, s, (const float*)W.yslot,
+                   (const int32_t*)W.slot_pos, (__nv_bfloat16*)out, T, d, k);
     if (ev) cudaEventRecord(ev[3], s);
-    return cudaGetLastError();
+    return e;
 }
 
 }  // namespace ace

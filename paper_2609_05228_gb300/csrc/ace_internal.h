@@ -8,6 +8,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "ace.h"
 
 namespace ace {
@@ -28,7 +30,8 @@ enum : int {
     kMetaSlice2 = 4,       // down GEMV: rows of d per work item
     kMetaTiles1 = 5,       // tensor-core GEMM 1 tiles
     kMetaTiles2 = 6,       // tensor-core GEMM 2 tiles
-    kMetaTicket2 = 7,      // second ticket (expert kernels)
+    kMetaTicket2 = 7,      // second ticket (fused small-T routing)
+    kMetaTokTiles = 8,     // token tiles of the tensor-core expert schedule
     kMetaCount = 16,
 };
 
@@ -57,9 +60,10 @@ struct Workspace {
     float* act = nullptr;        // [Tmax*k, m] fp32 (CUDA-core path)
     float* yslot = nullptr;      // [Tmax*k, d] fp32: g_hat-scaled expert outputs per retained slot
     void* h_perm = nullptr;      // [Tmax*k, d] bf16: h rows in expert-grouped order (tensor path)
-    float* g_perm = nullptr;     // [Tmax*k] g_hat in expert-grouped order
     void* act_bf16 = nullptr;    // [Tmax*k, m] bf16 (tensor path)
     int32_t* tt_off = nullptr;   // [N+1] token-tile prefix over distinct experts
+    int4* tt_tab = nullptr;      // [N + Tmax*k/16 + 1] token tiles: (expert, first row, rows, 0)
+    int32_t* tile_cnt = nullptr; // [Tmax/8 + 1] per-token-tile tickets of the fused small-T kernel
     int* err = nullptr;          // device error word
     void* x_stage = nullptr;     // [Tmax, d] dtype: host-API staging
     void* out_stage = nullptr;   // [Tmax, d]
@@ -68,7 +72,7 @@ struct Workspace {
 // Tensor maps of the tensor-core expert path (built once at create time).
 struct TcMaps {
     CUtensorMap tok1_small, tok1_big;   // h_perm, boxes of 16 / 128 rows
-    CUtensorMap tok2_small, tok2_big;   // act_bf16
+    CUtensorMap tok2_small, tok2_big;   // act_bf16, boxes of 16 / 128 rows
     CUtensorMap wgu_small, wgu_big;     // W_gu, boxes of 128 / 256 rows
     CUtensorMap wd_small, wd_big;       // W_down
     CUtensorMap h_rows, w_router;       // router GEMM: h and W_r
@@ -119,7 +123,37 @@ cudaError_t launch_router(const ace_layer* L, const void* x, int T, bool fuse_no
 cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_skip_ctl ctl,
                          cudaStream_t s);
 int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl);
+// T <= 256: RMSNorm + router + decision + compaction in one launch; with
+// x == nullptr the logits are taken from `logits` instead.
+cudaError_t launch_route_fused(const ace_layer* L, const void* x, const float* logits, int T, ace_skip_ctl ctl,
+                               cudaStream_t s);
 cudaError_t launch_debug_exp(const float* x, float* y, int n, cudaStream_t s);
+
+// Launch with programmatic stream serialization (PDL): the kernel may start
+// while its predecessor on the stream finishes and must execute
+// griddepcontrol.wait before reading the predecessor's results.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// Prefer the largest shared-memory carveout (all kernels share one L1/shared split).
+template <typename K>
+inline cudaError_t prefer_shared(K kernel) {
+    return cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                (int)cudaSharedmemCarveoutMaxShared);
+}
 
 // ---- launchers (ace_expert_gemv.cu) ----
 // ev (nullable): events recorded before gate/up, before down, before combine, after combine.

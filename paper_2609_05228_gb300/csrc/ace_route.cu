@@ -3,8 +3,8 @@
 // slots into per-expert groups.
 //
 // Two launch shapes share the same device functions (and so the same bits):
-//   T <= kSmallT: k_router (with RMSNorm fused) + k_route_small, one block
-//                 doing top-k, decision, threshold and compaction;
+//   T <= kSmallT: k_route_fused, one launch for RMSNorm, router, top-k,
+//                 decision, threshold and compaction;
 //   larger T:     k_rmsnorm, k_router, k_topk_score, [k_tau_select, k_decide],
 //                 k_compact_count, k_compact_place.
 #include <math.h>
@@ -187,7 +187,7 @@ __device__ __forceinline__ void warp_topk(const float* __restrict__ zrow, int n_
     for (int j = 0; j < NPL; ++j) {
         const int e = lane + 32 * j;
         if (e < n_exp) {
-            float z = zrow[e];
+            float z = __ldcg(zrow + e);
             if (z != z) { saw_nan = true; z = -INFINITY; }
             v[j] = z;
         } else {
@@ -299,17 +299,19 @@ __device__ __forceinline__ void decide_slot(int lane, int k, float g, float c, f
 // least as close to m as hi, else the next float above v. Whole block;
 // requires 0 < m < #candidates. Keys 0xffffffff are protected slots.
 // --------------------------------------------------------------------------
+template <int NW>
 struct SelectSmem {
-    int hist[32][256];     // one histogram per warp (blockDim <= 1024)
+    int hist[NW][256];     // one histogram per warp
     int tot[256];
     uint32_t prefix;
     int want, below, last_cnt;
     float tau;
 };
 
-__device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem& S) {
+template <int NW>
+__device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem<NW>& S) {
     const int tid = threadIdx.x, warp = tid >> 5;
-    const int nwarps = blockDim.x >> 5;
+    constexpr int nwarps = NW;
     uint32_t prefix = 0u, mask = 0u;
     if (tid == 0) { S.want = m; S.below = 0; }
     for (int pass = 0; pass < 4; ++pass) {
@@ -416,6 +418,21 @@ __device__ void scan_counts_warp0(const int* cnt, int n_exp, int32_t* __restrict
         if (tok_tile > 0) tt_off[dtotal] = ttotal;
         meta[kMetaRetained] = total;
         meta[kMetaDistinct] = dtotal;
+        meta[kMetaTokTiles] = tok_tile > 0 ? ttotal : 0;
+    }
+}
+
+// After scan_counts_warp0 and a block barrier: the flat token-tile table of
+// the tensor-core experts, tt_tab[tt] = (expert, first row, rows, 0).
+__device__ void fill_tile_table(const int32_t* offsets, const int32_t* dlist, const int32_t* tt_off,
+                                const int32_t* meta, int tok_tile, int4* tt_tab) {
+    if (tok_tile <= 0) return;
+    const int D = meta[kMetaDistinct];
+    for (int j = threadIdx.x; j < D; j += blockDim.x) {
+        const int e = dlist[j];
+        const int beg = offsets[e], cnt = offsets[e + 1] - beg, base = tt_off[j];
+        for (int b = 0; b * tok_tile < cnt; ++b)
+            tt_tab[base + b] = make_int4(e, beg + b * tok_tile, min(tok_tile, cnt - b * tok_tile), 0);
     }
 }
 
@@ -489,7 +506,7 @@ constexpr int kSelThreads = 1024;
 
 __global__ void __launch_bounds__(kSelThreads) k_tau_select(const uint32_t* __restrict__ keys, int n,
                                                             int m, float* __restrict__ tau_out) {
-    __shared__ SelectSmem S;
+    __shared__ SelectSmem<kSelThreads / 32> S;
     const float tau = block_select_tau(keys, n, m, S);
     if (threadIdx.x == 0) *tau_out = tau;
 }
@@ -507,7 +524,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, i
                                                           int32_t* __restrict__ offsets,
                                                           int32_t* __restrict__ dlist,
                                                           int32_t* __restrict__ meta, int tok_tile,
-                                                          int32_t* __restrict__ tt_off) {
+                                                          int32_t* __restrict__ tt_off, int4* __restrict__ tt_tab) {
     __shared__ int cnt[kMaxExperts];
     __shared__ bool is_last;
     for (int e = threadIdx.x; e < n_exp; e += blockDim.x) cnt[e] = 0;
@@ -542,6 +559,8 @@ __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, i
         scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, nullptr, tok_tile, tt_off);
         if (threadIdx.x == 0) meta[kMetaTicket] = 0;
     }
+    __syncthreads();
+    fill_tile_table(offsets, dlist, tt_off, meta, tok_tile, tt_tab);
 }
 
 __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, int n_exp,
@@ -579,19 +598,231 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
 }
 
 // --------------------------------------------------------------------------
-// Small-T kernel: the whole decision and compaction in one block.
+// Small-T fused kernel (T <= kSmallT): RMSNorm + router logits + top-k +
+// decision + threshold + compaction in one launch.
+//   phase A (every block, LOGITS only): block (bx, by) normalises tokens
+//     [8 bx, 8 bx + 8) into fp32 shared memory (blocks with by == 0 also
+//     store h for the experts) and computes their logits for experts
+//     [8 by, 8 by + 8), one expert row per warp;
+//   phase B (last block of each token tile, by an atomic ticket): top-k,
+//     gates and c for the tile's tokens (and the decision in threshold mode);
+//   phase C (the globally last block): the App. B.1 threshold in ratio mode,
+//     the decision, and the compaction of retained slots.
+// Tickets are reset by the block that consumed them. No block waits on another.
 // --------------------------------------------------------------------------
-constexpr int kSmallThreads = 1024;
+constexpr int kFuseTok = 8;
+constexpr int kFuseWarps = 8;
 
-template <int NPL>
-__global__ void __launch_bounds__(kSmallThreads) k_route_small(
-    const float* __restrict__ logits, int n_tokens, int n_exp, int k, const float* __restrict__ a_gsp,
-    const float* __restrict__ a_rcr, float eps, int m_min, int mode, float tau_in, int m_q,
-    int32_t* __restrict__ ids, float* __restrict__ gates, float* __restrict__ cval, uint8_t* __restrict__ skip,
-    float* __restrict__ ghat, float* __restrict__ tau_out, int32_t* __restrict__ offsets,
-    int32_t* __restrict__ dlist, int32_t* __restrict__ perm, int32_t* __restrict__ slot_pos,
-    int32_t* __restrict__ meta, int* __restrict__ err, int tok_tile, int32_t* __restrict__ tt_off) {
+struct FusedArgs {
+    const void* x;
+    const void* gamma;
+    void* h_out;
+    const void* w_r;
+    const float* b_r;
+    float inv_temp;
+    int use_temp;
+    float rms_eps;
+    int d;
+    float* logits;
+    int n_tokens, n_exp, k;
+    const float* a_gsp;
+    const float* a_rcr;
+    float eps;
+    int m_min, mode;
+    float tau_in;
+    int m_q;
+    int32_t* ids;
+    float* gates;
+    float* cval;
+    uint32_t* keys;
+    uint8_t* skip;
+    float* ghat;
+    float* tau_out;
+    int32_t* offsets;
+    int32_t* dlist;
+    int32_t* perm;
+    int32_t* slot_pos;
+    int32_t* meta;
+    int* err;
+    int tok_tile;
+    int32_t* tt_off;
+    int4* tt_tab;
+    int32_t* tile_cnt;
+};
+
+// RMSNorm of one row into fp32 shared memory; optionally also the row in T.
+template <typename T>
+__device__ __forceinline__ void rmsnorm_row_f32(const T* __restrict__ xr, const T* __restrict__ gamma, float* hs,
+                                                T* __restrict__ h_out, int d, float rms_eps, int lane) {
+    constexpr int V = Vec16<T>::N;
+    const int nvec = d / V;
+    const uint4* xv = reinterpret_cast<const uint4*>(xr);
+    const uint4* gv = reinterpret_cast<const uint4*>(gamma);
+    uint4 xs[kNormVec];
+#pragma unroll
+    for (int i = 0; i < kNormVec; ++i) {
+        const int c = lane + 32 * i;
+        xs[i] = c < nvec ? xv[c] : make_uint4(0, 0, 0, 0);
+    }
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < kNormVec; ++i) {
+        float f[V];
+        Vec16<T>::to_float(xs[i], f);
+#pragma unroll
+        for (int j = 0; j < V; ++j) ss = fmaf(f[j], f[j], ss);
+    }
+    ss = warp_sum(ss);
+    const float inv = 1.0f / sqrtf(ss / (float)d + rms_eps);
+#pragma unroll
+    for (int i = 0; i < kNormVec; ++i) {
+        const int c = lane + 32 * i;
+        if (c < nvec) {
+            float f[V], gm[V];
+            Vec16<T>::to_float(xs[i], f);
+            Vec16<T>::to_float(gv[c], gm);
+            T o[V];
+#pragma unroll
+            for (int j = 0; j < V; ++j) {
+                o[j] = from_f32<T>(f[j] * inv * gm[j]);
+                f[j] = to_f32(o[j]);                       // the stored (rounded) value feeds the router
+            }
+#pragma unroll
+            for (int j = 0; j < V; j += 4)
+                *reinterpret_cast<float4*>(hs + c * V + j) = make_float4(f[j], f[j + 1], f[j + 2], f[j + 3]);
+            if (h_out) reinterpret_cast<uint4*>(h_out)[c] = *reinterpret_cast<const uint4*>(o);
+        }
+    }
+}
+
+__host__ __device__ inline size_t fused_phase_c_bytes(int T, int k, int n_exp) {
+    const size_t ns = (size_t)T * k;
+    return ns * 16 + (size_t)n_exp * 4 + (size_t)(n_exp + 1) * 4 + (size_t)n_exp * 32 + ns + 16;
+}
+
+template <typename T, int NPL, bool LOGITS>
+__global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_constant__ FusedArgs a) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
+    __shared__ SelectSmem<kFuseWarps> S;
+    __shared__ int s_last;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int t0 = blockIdx.x * kFuseTok;
+    const int nt = min(kFuseTok, a.n_tokens - t0);
+    const int n_exp = a.n_exp, k = a.k;
+    if (LOGITS) {
+        // ---------------- phase A: RMSNorm + logits for 8 tokens x 8 experts
+        float* hs = reinterpret_cast<float*>(smem_raw);          // [kFuseTok][d]
+        const int d = a.d;
+        constexpr int V = Vec16<T>::N;
+        const int nvec = d / V;
+        {
+            const int r = warp;                                   // one token row per warp
+            if (r < nt) {
+                const size_t off = (size_t)(t0 + r) * d;
+                rmsnorm_row_f32<T>(static_cast<const T*>(a.x) + off, static_cast<const T*>(a.gamma), hs + (size_t)r * d,
+                                   blockIdx.y == 0 ? static_cast<T*>(a.h_out) + off : nullptr, d, a.rms_eps, lane);
+            } else {
+                for (int c = lane; c < d / 4; c += 32)
+                    reinterpret_cast<float4*>(hs + (size_t)r * d)[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+        }
+        __syncthreads();
+        const int e = blockIdx.y * kFuseWarps + warp;
+        if (e < n_exp) {
+            const uint4* we = reinterpret_cast<const uint4*>(static_cast<const T*>(a.w_r) + (size_t)e * d);
+            float acc[kFuseTok];
+#pragma unroll
+            for (int r = 0; r < kFuseTok; ++r) acc[r] = 0.f;
+            constexpr int CH = 8;
+            for (int c0 = 0; c0 < nvec; c0 += 32 * CH) {
+                uint4 wv[CH];
+#pragma unroll
+                for (int i = 0; i < CH; ++i) {
+                    const int c = c0 + lane + 32 * i;
+                    wv[i] = c < nvec ? we[c] : make_uint4(0, 0, 0, 0);
+                }
+#pragma unroll
+                for (int i = 0; i < CH; ++i) {
+                    const int c = c0 + lane + 32 * i;
+                    if (c >= nvec) break;
+                    float wf[V];
+                    Vec16<T>::to_float(wv[i], wf);
+#pragma unroll
+                    for (int r = 0; r < kFuseTok; ++r) {
+                        const float4* hp = reinterpret_cast<const float4*>(hs + (size_t)r * d + c * V);
+#pragma unroll
+                        for (int j = 0; j < V / 4; ++j) {
+                            const float4 hv = hp[j];
+                            acc[r] = fmaf(hv.x, wf[4 * j], acc[r]);
+                            acc[r] = fmaf(hv.y, wf[4 * j + 1], acc[r]);
+                            acc[r] = fmaf(hv.z, wf[4 * j + 2], acc[r]);
+                            acc[r] = fmaf(hv.w, wf[4 * j + 3], acc[r]);
+                        }
+                    }
+                }
+            }
+#pragma unroll
+            for (int r = 0; r < kFuseTok; ++r) acc[r] = warp_sum(acc[r]);
+            if (lane < nt) {
+                float v = acc[0];
+#pragma unroll
+                for (int r = 1; r < kFuseTok; ++r) if (lane == r) v = acc[r];
+                v = v + a.b_r[e];
+                if (a.use_temp) v = v * a.inv_temp;
+                a.logits[(size_t)(t0 + lane) * n_exp + e] = v;
+            }
+        }
+        __threadfence();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            s_last = atomicAdd(&a.tile_cnt[blockIdx.x], 1) == (int)gridDim.y - 1;
+            if (s_last) a.tile_cnt[blockIdx.x] = 0;
+        }
+        __syncthreads();
+        if (!s_last) return;
+        __threadfence();
+    }
+    // ---------------- phase B: top-k, gates, c for this token tile
+    const bool ratio = a.mode == ACE_SKIP_RATIO;
+    for (int r = warp; r < nt; r += kFuseWarps) {
+        const int t = t0 + r;
+        int id;
+        float zv;
+        bool nan;
+        warp_topk<NPL>(a.logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
+        const float z0 = __shfl_sync(0xffffffffu, zv, 0);
+        if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(a.err, kErrNumeric);
+        const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a.a_gsp, a.a_rcr, a.eps);
+        const size_t base = (size_t)t * k;
+        if (lane < k) {
+            a.ids[base + lane] = id;
+            a.gates[base + lane] = sc.g;
+            a.cval[base + lane] = sc.c;
+        }
+        if (!ratio) {
+            bool sk;
+            float gh;
+            decide_slot(lane, k, sc.g, sc.c, a.tau_in, a.m_min, a.eps, sk, gh);
+            if (lane < k) {
+                a.skip[base + lane] = sk ? 1 : 0;
+                a.ghat[base + lane] = gh;
+            }
+        } else {
+            const bool prot = slot_protected(lane, k, sc.c, a.m_min);
+            if (lane < k) a.keys[base + lane] = prot ? 0xffffffffu : __float_as_uint(sc.c);
+        }
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        s_last = atomicAdd(&a.meta[kMetaTicket2], 1) == (int)gridDim.x - 1;
+        if (s_last) a.meta[kMetaTicket2] = 0;
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    // ---------------- phase C: threshold, decision, compaction (all tokens)
+    const int n_tokens = a.n_tokens;
     const int ns = n_tokens * k;
     float* g_s = reinterpret_cast<float*>(smem_raw);
     float* c_s = g_s + ns;
@@ -601,66 +832,39 @@ __global__ void __launch_bounds__(kSmallThreads) k_route_small(
     int* off_s = cnt + n_exp;                                        // [n_exp + 1]
     uint32_t* bm = reinterpret_cast<uint32_t*>(off_s + n_exp + 1);   // [n_exp * 8]
     uint8_t* skip_s = reinterpret_cast<uint8_t*>(bm + n_exp * 8);    // [ns]
-    __shared__ SelectSmem S;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
-    const bool ratio = mode == ACE_SKIP_RATIO;
     for (int i = threadIdx.x; i < n_exp; i += blockDim.x) cnt[i] = 0;
     for (int i = threadIdx.x; i < n_exp * 8; i += blockDim.x) bm[i] = 0u;
-    // phase 1: top-k, gates, c (and the decision in threshold mode)
-    for (int t = warp; t < n_tokens; t += nwarps) {
-        int id;
-        float zv;
-        bool nan;
-        warp_topk<NPL>(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
-        const float z0 = __shfl_sync(0xffffffffu, zv, 0);
-        if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(err, kErrNumeric);
-        const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a_gsp, a_rcr, eps);
-        const int base = t * k;
-        if (lane < k) {
-            ids[base + lane] = id;
-            gates[base + lane] = sc.g;
-            cval[base + lane] = sc.c;
-            id_s[base + lane] = id;
-            g_s[base + lane] = sc.g;
-            c_s[base + lane] = sc.c;
-        }
-        if (!ratio) {
-            bool sk;
-            float gh;
-            decide_slot(lane, k, sc.g, sc.c, tau_in, m_min, eps, sk, gh);
-            if (lane < k) {
-                skip[base + lane] = sk ? 1 : 0;
-                skip_s[base + lane] = sk ? 1 : 0;
-                ghat[base + lane] = gh;
-            }
+    for (int i = threadIdx.x; i < ns; i += blockDim.x) {
+        id_s[i] = __ldcg(a.ids + i);
+        if (ratio) {
+            g_s[i] = __ldcg(a.gates + i);
+            c_s[i] = __ldcg(a.cval + i);
+            key_s[i] = __ldcg(a.keys + i);
         } else {
-            const bool prot = slot_protected(lane, k, sc.c, m_min);
-            if (lane < k) key_s[base + lane] = prot ? 0xffffffffu : __float_as_uint(sc.c);
+            skip_s[i] = __ldcg(a.skip + i);
         }
     }
     __syncthreads();
-    // phase 2: threshold and decision (ratio mode)
     if (ratio) {
-        const float tau = block_select_tau(key_s, ns, m_q, S);
-        if (threadIdx.x == 0) *tau_out = tau;
-        for (int t = warp; t < n_tokens; t += nwarps) {
+        const float tau = block_select_tau(key_s, ns, a.m_q, S);
+        if (threadIdx.x == 0) *a.tau_out = tau;
+        for (int t = warp; t < n_tokens; t += kFuseWarps) {
             const int base = t * k;
             const float g = lane < k ? g_s[base + lane] : 0.f;
             const float c = lane < k ? c_s[base + lane] : 0.f;
             bool sk;
             float gh;
-            decide_slot(lane, k, g, c, tau, m_min, eps, sk, gh);
+            decide_slot(lane, k, g, c, tau, a.m_min, a.eps, sk, gh);
             if (lane < k) {
-                skip[base + lane] = sk ? 1 : 0;
+                a.skip[base + lane] = sk ? 1 : 0;
                 skip_s[base + lane] = sk ? 1 : 0;
-                ghat[base + lane] = gh;
+                a.ghat[base + lane] = gh;
             }
         }
         __syncthreads();
     } else if (threadIdx.x == 0) {
-        *tau_out = tau_in;
+        *a.tau_out = a.tau_in;
     }
-    // phase 3: compaction of retained slots (one chunk of <= 256 tokens)
     for (int s = threadIdx.x; s < ns; s += blockDim.x) {
         if (skip_s[s]) continue;
         const int e = id_s[s], t = s / k;
@@ -668,22 +872,24 @@ __global__ void __launch_bounds__(kSmallThreads) k_route_small(
         atomicOr(&bm[e * 8 + (t >> 5)], 1u << (t & 31));
     }
     __syncthreads();
-    if (threadIdx.x < 32) scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, off_s, tok_tile, tt_off);
+    if (threadIdx.x < 32) scan_counts_warp0(cnt, n_exp, a.offsets, a.dlist, a.meta, off_s, a.tok_tile, a.tt_off);
     __syncthreads();
+    fill_tile_table(a.offsets, a.dlist, a.tt_off, a.meta, a.tok_tile, a.tt_tab);
     for (int s = threadIdx.x; s < ns; s += blockDim.x) {
-        if (skip_s[s]) { slot_pos[s] = -1; continue; }
+        if (skip_s[s]) { a.slot_pos[s] = -1; continue; }
         const int e = id_s[s], t = s / k, w = t >> 5;
         int rank = __popc(bm[e * 8 + w] & ((1u << (t & 31)) - 1u));
         for (int ww = 0; ww < w; ++ww) rank += __popc(bm[e * 8 + ww]);
         const int r = off_s[e] + rank;
-        perm[r] = s;
-        slot_pos[s] = r;
+        a.perm[r] = s;
+        a.slot_pos[s] = r;
     }
 }
 
-size_t small_smem_bytes(int T, int k, int n_exp) {
-    const size_t ns = (size_t)T * k;
-    return ns * 16 + (size_t)n_exp * 4 + (size_t)(n_exp + 1) * 4 + (size_t)n_exp * 32 + ns + 16;
+size_t fused_smem_bytes(const ace_layer* L, int T) {
+    const size_t a = (size_t)kFuseTok * L->desc.hidden * sizeof(float);
+    const size_t c = fused_phase_c_bytes(T, L->desc.top_k, L->desc.n_experts);
+    return a > c ? a : c;
 }
 
 __global__ void k_debug_exp(const float* __restrict__ x, float* __restrict__ y, int n) {
@@ -734,6 +940,89 @@ int select_mq(const ace_layer* L, int T, ace_skip_ctl ctl, float* tau, bool* nee
 
 bool small_path(int T) { return T <= kSmallT; }
 
+namespace {
+template <typename T, int NPL, bool LOGITS>
+cudaError_t fused_launch(const ace_layer* L, const FusedArgs& a, int n_tok, cudaStream_t s) {
+    const dim3 grid(cdiv(n_tok, kFuseTok), LOGITS ? cdiv(L->desc.n_experts, kFuseWarps) : 1);
+    k_route_fused<T, NPL, LOGITS><<<grid, kFuseWarps * 32, fused_smem_bytes(L, kSmallT), s>>>(a);
+    return cudaGetLastError();
+}
+
+template <typename T, bool LOGITS>
+cudaError_t fused_dispatch(const ace_layer* L, const FusedArgs& a, int n_tok, cudaStream_t s) {
+    const int n = L->desc.n_experts;
+    if (n <= 128) return fused_launch<T, 4, LOGITS>(L, a, n_tok, s);
+    if (n <= 256) return fused_launch<T, 8, LOGITS>(L, a, n_tok, s);
+    return fused_launch<T, 32, LOGITS>(L, a, n_tok, s);
+}
+
+template <typename T, int NPL, bool LOGITS>
+cudaError_t fused_attr(int smem) {
+    return cudaFuncSetAttribute(k_route_fused<T, NPL, LOGITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+}
+
+template <typename T>
+cudaError_t fused_attrs(int smem) {
+    cudaError_t e;
+    if ((e = fused_attr<T, 4, true>(smem)) != cudaSuccess) return e;
+    if ((e = fused_attr<T, 8, true>(smem)) != cudaSuccess) return e;
+    if ((e = fused_attr<T, 32, true>(smem)) != cudaSuccess) return e;
+    if ((e = fused_attr<T, 4, false>(smem)) != cudaSuccess) return e;
+    if ((e = fused_attr<T, 8, false>(smem)) != cudaSuccess) return e;
+    return fused_attr<T, 32, false>(smem);
+}
+}  // namespace
+
+// T <= kSmallT: the whole routing in one launch. x == nullptr: logits are given.
+cudaError_t launch_route_fused(const ace_layer* L, const void* x, const float* logits, int T, ace_skip_ctl ctl,
+                               cudaStream_t s) {
+    const ace_layer_desc& D = L->desc;
+    const Workspace& W = L->ws;
+    FusedArgs a{};
+    float tau;
+    bool need_select;
+    a.m_q = select_mq(L, T, ctl, &tau, &need_select);
+    a.mode = need_select ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
+    a.tau_in = tau;
+    a.x = x;
+    a.gamma = L->gamma;
+    a.h_out = W.h;
+    a.w_r = L->router_w;
+    a.b_r = L->router_b;
+    a.inv_temp = 1.0f / D.router_temp;
+    a.use_temp = D.router_temp != 1.0f;
+    a.rms_eps = D.rms_eps;
+    a.d = D.hidden;
+    a.logits = const_cast<float*>(logits);
+    a.n_tokens = T;
+    a.n_exp = D.n_experts;
+    a.k = D.top_k;
+    a.a_gsp = L->a_gsp;
+    a.a_rcr = L->a_rcr;
+    a.eps = D.eps;
+    a.m_min = D.min_active;
+    a.ids = W.ids;
+    a.gates = W.gates;
+    a.cval = W.cval;
+    a.keys = W.keys;
+    a.skip = W.skip;
+    a.ghat = W.ghat;
+    a.tau_out = W.tau;
+    a.offsets = W.offsets;
+    a.dlist = W.dlist;
+    a.perm = W.perm;
+    a.slot_pos = W.slot_pos;
+    a.meta = W.meta;
+    a.err = W.err;
+    a.tok_tile = L->tc ? tc_token_tile(T) : 0;
+    a.tt_off = W.tt_off;
+    a.tt_tab = W.tt_tab;
+    a.tile_cnt = W.tile_cnt;
+    const bool bf = D.dtype == ACE_BF16;
+    if (x) return bf ? fused_dispatch<__nv_bfloat16, true>(L, a, T, s) : fused_dispatch<float, true>(L, a, T, s);
+    return bf ? fused_dispatch<__nv_bfloat16, false>(L, a, T, s) : fused_dispatch<float, false>(L, a, T, s);
+}
+
 cudaError_t launch_rmsnorm(const ace_layer* L, const void* x, int T, cudaStream_t s) {
     const int d = L->desc.hidden;
     const int blocks = cdiv(T, 8);
@@ -765,17 +1054,7 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     const int m_q = select_mq(L, T, ctl, &tau, &need_select);
     const int mode = need_select ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
     const int tok_tile = L->tc ? tc_token_tile(T) : 0;
-    if (T <= kSmallT) {
-#define ACE_ROUTE_SMALL(NPL)                                                                                   \
-    k_route_small<NPL><<<1, kSmallThreads, small_smem_bytes(T, k, n), s>>>(                                   \
-        logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode, tau, m_q, W.ids, W.gates, W.cval,      \
-        W.skip, W.ghat, W.tau, W.offsets, W.dlist, W.perm, W.slot_pos, W.meta, W.err, tok_tile, W.tt_off)
-        if (n <= 128) ACE_ROUTE_SMALL(4);
-        else if (n <= 256) ACE_ROUTE_SMALL(8);
-        else ACE_ROUTE_SMALL(32);
-#undef ACE_ROUTE_SMALL
-        return cudaGetLastError();
-    }
+    if (T <= kSmallT) return launch_route_fused(L, nullptr, logits, T, ctl, s);
     const int blocks = cdiv(T, 8);
 #define ACE_TOPK(NPL)                                                                                          \
     k_topk_score<NPL><<<blocks, 256, 0, s>>>(logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode,   \
@@ -790,14 +1069,14 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     }
     const int n_chunks = cdiv(T, kChunk);
     k_compact_count<<<n_chunks, kChunk, 0, s>>>(T, k, n, n_chunks, W.ids, W.skip, W.chunk_counts,
-                                                W.offsets, W.dlist, W.meta, tok_tile, W.tt_off);
+                                                W.offsets, W.dlist, W.meta, tok_tile, W.tt_off, W.tt_tab);
     k_compact_place<<<n_chunks, kChunk, 0, s>>>(T, k, n, W.ids, W.skip, W.chunk_counts, W.offsets,
                                                 W.perm, W.slot_pos);
     return cudaGetLastError();
 }
 
 int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl) {
-    if (T <= kSmallT) return 1;
+    if (T <= kSmallT) return 1;   // fused with the router in the forward
     float tau;
     bool sel;
     select_mq(L, T, ctl, &tau, &sel);
@@ -809,12 +1088,18 @@ cudaError_t route_init(const ace_layer* L) {
     if (e != cudaSuccess) return e;
     e = set_router_attrs<float>(router_smem(L));
     if (e != cudaSuccess) return e;
-    const int sm = (int)small_smem_bytes(kSmallT, L->desc.top_k, L->desc.n_experts);
-    if ((e = cudaFuncSetAttribute(k_route_small<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm)) != cudaSuccess)
-        return e;
-    if ((e = cudaFuncSetAttribute(k_route_small<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm)) != cudaSuccess)
-        return e;
-    return cudaFuncSetAttribute(k_route_small<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+    const int sm = (int)fused_smem_bytes(L, kSmallT);
+    if ((e = fused_attrs<__nv_bfloat16>(sm)) != cudaSuccess) return e;
+    if ((e = fused_attrs<float>(sm)) != cudaSuccess) return e;
+    const void* ks[] = {(const void*)k_route_fused<__nv_bfloat16, 4, true>, (const void*)k_route_fused<__nv_bfloat16, 8, true>,
+                        (const void*)k_route_fused<__nv_bfloat16, 32, true>, (const void*)k_route_fused<float, 4, true>,
+                        (const void*)k_route_fused<float, 8, true>, (const void*)k_route_fused<float, 32, true>,
+                        (const void*)k_rmsnorm<__nv_bfloat16>, (const void*)k_topk_score<4>, (const void*)k_topk_score<8>,
+                        (const void*)k_topk_score<32>, (const void*)k_tau_select, (const void*)k_decide,
+                        (const void*)k_compact_count, (const void*)k_compact_place};
+    for (const void* kf : ks)
+        if ((e = prefer_shared(kf)) != cudaSuccess) return e;
+    return cudaSuccess;
 }
 
 cudaError_t launch_debug_exp(const float* x, float* y, int n, cudaStream_t s) {
