@@ -153,6 +153,18 @@ def stage_times(torch, layer, x, out, T, q, steps, flush):
     return out_stages
 
 
+def aggregate(step_ms: float, tokens_per_rank: int, world: int, dist=None, device=None):
+    """Whole-job throughput: every rank's tokens over the slowest rank's step
+    time (max over ranks). Returns (tokens/s, max step ms)."""
+    t = float(step_ms)
+    if world > 1:
+        import torch
+        x = torch.tensor([t], dtype=torch.float64, device=device)
+        dist.all_reduce(x, op=dist.ReduceOp.MAX)
+        t = float(x.item())
+    return world * tokens_per_rank / (t * 1e-3), t
+
+
 def algorithmic(w, T, R, D):
     """Algorithmic bytes and flops of one forward (retained work only) and of
     the gate/up expert kernel. D = distinct experts with >= 1 retained slot."""
@@ -199,10 +211,7 @@ def run_ours(args, rank, world, torch, dist):
     if world > 1:
         dist.barrier()
     step_ms = float(np.mean(ms))
-    tmax = torch.tensor([step_ms], device=dev)
-    if world > 1:
-        dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
-    step_ms_max = float(tmax.item())
+    value, step_ms_max = aggregate(step_ms, T, world, dist, dev)
 
     # the dominant kernel's duration, from events on its own stream
     stages = stage_times(torch, layer, x, out, T, q, args.steps, flush)
@@ -229,7 +238,7 @@ def run_ours(args, rank, world, torch, dist):
 
     result = {
         "metric": METRIC,
-        "value": round(world * T / (step_ms_max * 1e-3), 1),
+        "value": round(value, 1),
         "unit": "tokens/s",
         "n_gpus": world,
         "steps": args.steps,
