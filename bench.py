@@ -41,6 +41,26 @@ METRIC = "ACE MoE-layer tokens/s (prefill, decode) + speedup vs skip=0; % of roo
 L2_FLUSH_BYTES = 512 << 20
 
 
+def _recorded_traffic(path="profiles/decode_T64_q0.5_expert_tc_full.md"):
+    """DRAM bytes per launch of the gate/up kernel from the committed ncu
+    summary, or None when the kernel source has changed since the capture."""
+    import hashlib
+    try:
+        rec = {}
+        with open(os.path.join(ROOT, path)) as f:
+            for line in f:
+                line = line.strip()
+                if "=" in line and " " not in line.split("=", 1)[0]:
+                    k, v = line.split("=", 1)
+                    rec[k] = v
+        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
+                return None
+        return int(rec["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -51,7 +71,7 @@ def _peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+    """nvidia-smi clocks and throttle reasons sampled every 100 ms."""
 
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -62,7 +82,7 @@ class ClockSampler:
         self.gpu = gpu_index
         try:
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={gpu_index}", f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except Exception:
             self.proc = None
@@ -174,7 +194,7 @@ def algorithmic(w, T, R, D):
     w_bytes = 3 * d * m * e * D
     total_bytes = w_bytes + N * d * e + 2 * T * d * e
     flops = 6 * d * m * R + 2 * d * N * T
-    gate_up_bytes = 2 * d * m * e * D + R * d * e + R * m * 4
+    gate_up_bytes = 2 * d * m * e * D + R * d * e + R * m * e
     return total_bytes, flops, gate_up_bytes
 
 
@@ -259,9 +279,10 @@ def run_ours(args, rank, world, torch, dist):
         "q0_ms_per_step": round(t0, 5),
         "stage_us": stage_avg,
         "wall_s": round(wall, 3),
-        "roofline": {"bound": "hbm", "kernel": "k_gemv_gateup", "achieved": round(achieved, 1),
+        "roofline": {"bound": "hbm", "kernel": "k_expert_tc gate/up (tcgen05, SWAP)", "achieved": round(achieved, 1),
                      "peak": hbm, "unit": "GB/s", "frac": round(achieved / hbm, 4),
-                     "peak_source": peak_kind, "traffic": None,
+                     "peak_source": peak_kind,
+                     "traffic": _recorded_traffic() if args.workload == "decode" else None,
                      "algorithmic_bytes": gu_bytes, "kernel_us": round(gu_ms * 1e3, 2)},
         "layer_roofline": {"bytes": total_bytes, "flops": flops,
                            "hbm_frac": round(total_bytes / (step_ms * 1e-3) / 1e9 / hbm, 4),
@@ -356,7 +377,7 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="decode", choices=sorted(WORKLOADS))
