@@ -192,6 +192,44 @@ ace_status ace_last_stage_times(ace_layer* layer, float* ms, int n_max, int* n_o
 /* Number of kernels the last forward / route call launched (instrumentation). */
 ace_status ace_last_launch_count(const ace_layer* layer, int* n_kernels);
 
+/*
+ * ace_route_decide_noalloc — the routing decision of ace_route_logits
+ * (top-k, gates, Algorithm 4 skip decision, per-batch threshold in ratio
+ * mode) without a layer and without allocating any device memory. The paper
+ * has no counterpart; this is a deployment variant.
+ *
+ * For callers that cannot allocate device memory: a serving runtime that owns
+ * every byte of the GPU through its own pool and forbids cudaMalloc after
+ * start-up, code that runs while another component holds the allocator, or a
+ * plugin host that hands in pre-allocated buffers only. The caller supplies
+ * inputs and outputs; the intermediate values (gates, scores, candidate
+ * keys, the compaction and the kernel's tickets) live in one fixed device
+ * array inside this library (about 100 KB, 256-byte aligned). Every GPU that
+ * loads the library holds that array until the process exits.
+ *   logits    [T, N] device float32     router logits
+ *   a_gsp     [N]    device float32     GSP table (finite, >= 0)
+ *   a_rcr     [N]    device float32     RCR table (finite, >= 0)
+ *   eps       the paper's epsilon (1e-6 if <= 0); min_active = m_min (>= 1)
+ *   ids       [T, k] device int32 out   routed expert of slot i (rank order)
+ *   skip      [T, k] device uint8 out   1 = skipped
+ *   gates_hat [T, k] device float32 out renormalised gate, 0 where skipped
+ *   tau       [1]    device float32 out threshold used
+ * Limits: 1 <= T <= 256, 1 <= N <= 1024, 1 <= k <= min(16, N), T*k <= 4096;
+ * larger sizes return ACE_ERR_INVALID_ARG with a message and launch nothing.
+ * The results are bit-identical to ace_route_logits on the same inputs.
+ * The first call on a device (with that device current) looks up the array's
+ * device address; make that first call before any stream capture. All calls
+ * share the one array and it keeps the last call's contents (the kernel's
+ * counters are cleared at the start of every call): calls that overlap on
+ * the GPU, on different streams or devices sharing the library state per
+ * device, race. Asynchronous on `stream`; errors found by the kernel (NaN
+ * logits) are not reported by this entry point.
+ */
+ace_status ace_route_decide_noalloc(const float* logits, int T, int n_experts, int top_k,
+                                    const float* a_gsp, const float* a_rcr, float eps, int min_active,
+                                    ace_skip_ctl ctl, int32_t* ids, uint8_t* skip, float* gates_hat,
+                                    float* tau, void* stream);
+
 /* Fills *desc with the layer's descriptor (after defaults were applied). */
 ace_status ace_layer_get_desc(const ace_layer* layer, ace_layer_desc* desc);
 

@@ -68,6 +68,8 @@ def lib() -> ctypes.CDLL:
             "ace_layer_set_profiling": (_S, [_P, _I]),
             "ace_last_stage_times": (_S, [_P, _P, _I, _P]),
             "ace_last_launch_count": (_S, [_P, _P]),
+            "ace_route_decide_noalloc": (_S, [_P, _I, _I, _I, _P, _P, ctypes.c_float, _I, ace_skip_ctl, _P, _P, _P,
+                                              _P, _P]),
             "ace_status_string": (ctypes.c_char_p, [_S]),
             "ace_last_error_message": (ctypes.c_char_p, []),
         }
@@ -184,6 +186,14 @@ def ace_last_stage_times(layer: int) -> dict:
     n = np.zeros(1, np.int32)
     _check(lib().ace_last_stage_times(layer, ms.ctypes.data, 16, n.ctypes.data))
     return {STAGES[i] if i < len(STAGES) else f"stage{i}": float(ms[i]) for i in range(int(n[0]))}
+
+
+def ace_route_decide_noalloc(logits, T: int, n_experts: int, top_k: int, a_gsp, a_rcr, eps: float,
+                             min_active: int, mode, value: float, ids, skip, gates_hat, tau, stream=None) -> None:
+    """Routing decision without a layer or any device allocation (all pointers are device buffers)."""
+    _check(lib().ace_route_decide_noalloc(_ptr(logits), int(T), int(n_experts), int(top_k), _ptr(a_gsp), _ptr(a_rcr),
+                                          float(eps), int(min_active), _ctl(mode, value), _ptr(ids), _ptr(skip),
+                                          _ptr(gates_hat), _ptr(tau), _stream(stream)))
 
 
 def ace_last_launch_count(layer: int) -> int:

@@ -82,6 +82,10 @@ ace_status check_ctl(ace_skip_ctl ctl) {
 
 }  // namespace
 
+namespace ace {
+void set_last_error(const char* msg) { g_last_error = msg; }
+}  // namespace ace
+
 extern "C" {
 
 const char* ace_status_string(ace_status s) {

@@ -129,6 +129,28 @@ cudaError_t launch_route_fused(const ace_layer* L, const void* x, const float* l
                                cudaStream_t s);
 cudaError_t launch_debug_exp(const float* x, float* y, int n, cudaStream_t s);
 
+// Caller-provided scratch for the decision-only launch of the fused small-T
+// kernel (used by the entry point that allocates nothing).
+struct DecideScratch {
+    float* gates;        // [T*k]
+    float* cval;         // [T*k]
+    uint32_t* keys;      // [T*k]
+    int32_t* offsets;    // [N+1]
+    int32_t* dlist;      // [N]
+    int32_t* perm;       // [T*k]
+    int32_t* slot_pos;   // [T*k]
+    int32_t* meta;       // [kMetaCount], tickets must start at zero
+    int32_t* tile_cnt;   // [T/8 + 1], must start at zero
+    int* err;            // [1]
+};
+void set_last_error(const char* msg);   // the thread-local text of ace_last_error_message()
+size_t route_decide_smem(int T, int k, int n_exp);
+cudaError_t route_decide_attr(int smem_bytes);
+cudaError_t launch_route_decide_scratch(const float* logits, int T, int n_exp, int k, const float* a_gsp,
+                                        const float* a_rcr, float eps, int m_min, ace_skip_ctl ctl, int32_t* ids,
+                                        uint8_t* skip, float* ghat, float* tau_out, const DecideScratch& sc,
+                                        cudaStream_t s);
+
 // Launch with programmatic stream serialization (PDL): the kernel may start
 // while its predecessor on the stream finishes and must execute
 // griddepcontrol.wait before reading the predecessor's results.

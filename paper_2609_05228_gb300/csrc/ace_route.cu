@@ -1102,6 +1102,74 @@ cudaError_t route_init(const ace_layer* L) {
     return cudaSuccess;
 }
 
+// Decision-only launch of k_route_fused on scratch the caller owns (no layer).
+size_t route_decide_smem(int T, int k, int n_exp) { return fused_phase_c_bytes(T, k, n_exp); }
+
+cudaError_t route_decide_attr(int smem_bytes) {
+    cudaError_t e;
+    if ((e = cudaFuncSetAttribute(k_route_fused<__nv_bfloat16, 4, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  smem_bytes)) != cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(k_route_fused<__nv_bfloat16, 8, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  smem_bytes)) != cudaSuccess)
+        return e;
+    return cudaFuncSetAttribute(k_route_fused<__nv_bfloat16, 32, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                smem_bytes);
+}
+
+cudaError_t launch_route_decide_scratch(const float* logits, int T, int n_exp, int k, const float* a_gsp,
+                                        const float* a_rcr, float eps, int m_min, ace_skip_ctl ctl, int32_t* ids,
+                                        uint8_t* skip, float* ghat, float* tau_out, const DecideScratch& sc,
+                                        cudaStream_t s) {
+    FusedArgs a{};
+    float tau = ctl.value;
+    bool need_select = false;
+    int m_q = 0;
+    if (ctl.mode == ACE_SKIP_RATIO) {
+        const long long n_all = (long long)T * k;
+        const int prot = m_min < 1 ? 1 : (m_min > k ? k : m_min);
+        const long long n_cand = (long long)T * (k - prot);
+        long long mq = llround((double)ctl.value * (double)n_all);
+        mq = mq < 0 ? 0 : (mq > n_cand ? n_cand : mq);
+        m_q = (int)mq;
+        if (mq == 0) tau = 0.0f;
+        else if (mq == n_cand) tau = INFINITY;
+        else need_select = true;
+    }
+    a.mode = need_select ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
+    a.tau_in = tau;
+    a.m_q = m_q;
+    a.logits = const_cast<float*>(logits);
+    a.n_tokens = T;
+    a.n_exp = n_exp;
+    a.k = k;
+    a.a_gsp = a_gsp;
+    a.a_rcr = a_rcr;
+    a.eps = eps;
+    a.m_min = m_min;
+    a.ids = ids;
+    a.gates = sc.gates;
+    a.cval = sc.cval;
+    a.keys = sc.keys;
+    a.skip = skip;
+    a.ghat = ghat;
+    a.tau_out = tau_out;
+    a.offsets = sc.offsets;
+    a.dlist = sc.dlist;
+    a.perm = sc.perm;
+    a.slot_pos = sc.slot_pos;
+    a.meta = sc.meta;
+    a.err = sc.err;
+    a.tok_tile = 0;
+    a.tile_cnt = sc.tile_cnt;
+    const size_t smem = route_decide_smem(T, k, n_exp);
+    const dim3 grid(cdiv(T, kFuseTok), 1);
+    if (n_exp <= 128) k_route_fused<__nv_bfloat16, 4, false><<<grid, kFuseWarps * 32, smem, s>>>(a);
+    else if (n_exp <= 256) k_route_fused<__nv_bfloat16, 8, false><<<grid, kFuseWarps * 32, smem, s>>>(a);
+    else k_route_fused<__nv_bfloat16, 32, false><<<grid, kFuseWarps * 32, smem, s>>>(a);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_debug_exp(const float* x, float* y, int n, cudaStream_t s) {
     k_debug_exp<<<cdiv(n, 256), 256, 0, s>>>(x, y, n);
     return cudaGetLastError();
