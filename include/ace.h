@@ -92,7 +92,8 @@ typedef struct ace_layer ace_layer;   /* opaque */
  * allocates nothing.
  * Errors: INVALID_ARG for NULL pointers, non-positive sizes, k > N, tables
  * that are negative or non-finite; UNSUPPORTED for d or m not a multiple of
- * 64 (bf16) or 4 (f32), N > 1024, k > 16; OOM; CUDA.
+ * 64 (bf16) or 4 (f32), hidden above 4096 (bf16) or 2048 (f32), N > 1024,
+ * k > 16; OOM; CUDA.
  */
 ace_status ace_layer_create(const ace_layer_desc* desc,
                             const void* router_w, const float* router_b,

@@ -126,6 +126,9 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
         return fail(ACE_ERR_UNSUPPORTED, D.dtype == ACE_BF16 ? "hidden and ffn must be multiples of 64"
                                                              : "hidden and ffn must be multiples of 4");
     if ((long long)D.max_tokens * D.top_k > (1LL << 30)) return fail(ACE_ERR_UNSUPPORTED, "max_tokens too large");
+    // RMSNorm keeps a token row in registers: 16 x 16-byte vectors per lane
+    if (D.hidden > (D.dtype == ACE_BF16 ? 4096 : 2048))
+        return fail(ACE_ERR_UNSUPPORTED, "hidden must be <= 4096 (bf16) or <= 2048 (f32)");
     if (!router_w || !w_gate || !w_up || !w_down || !rms_gamma || !a_gsp || !a_rcr)
         return fail(ACE_ERR_INVALID_ARG, "weight, gamma and table pointers must be non-NULL");
     if (D.has_router_bias && !router_b) return fail(ACE_ERR_INVALID_ARG, "has_router_bias set but router_b is NULL");
