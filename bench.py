@@ -8,8 +8,9 @@ skip ratio 0.5 (per-batch threshold, App. B.1). A step is one full layer
 forward: RMSNorm, router, top-k, skip decision, threshold, compaction,
 experts and combine. Inputs are synthetic (seeded N(0,1) tokens, N(0, 0.02^2)
 weights) and resident in HBM; the forward is replayed from a CUDA graph and
-each step is timed with CUDA events; L2 is flushed (a 512 MB write) between
-steps, outside the timed events.
+each step is timed with CUDA events; L2 is flushed between steps (a 512 MB
+write, then a 256 MB read so dirty lines are written back), outside the
+timed events.
 
 Prints one JSON line (rank 0). `--impl reference` times the CPU oracle
 instead, on a bounded sample of the same workload.
@@ -39,6 +40,21 @@ WORKLOADS = {
 }
 METRIC = "ACE MoE-layer tokens/s (prefill, decode) + speedup vs skip=0; % of roofline"
 L2_FLUSH_BYTES = 512 << 20
+
+
+class L2Flush:
+    """Between timed steps: write a 512 MB buffer (evicts L2), then read a
+    256 MB buffer so that the dirty lines are written back before the next
+    step starts. Both run outside the timed events."""
+
+    def __init__(self, torch, device):
+        self.w = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=device)
+        self.r = torch.ones(L2_FLUSH_BYTES // 8, dtype=torch.float32, device=device)
+        self.sink = torch.empty(1, dtype=torch.float32, device=device)
+
+    def zero_(self):
+        self.w.zero_()
+        self.sink.copy_(self.r.sum().reshape(1))
 
 
 def _recorded_traffic(path="profiles/decode_T64_q0.5_expert_tc_full.md"):
@@ -157,19 +173,28 @@ def time_point(torch, layer, x, out, T, q, steps, warmup, flush):
 
 def stage_times(torch, layer, x, out, T, q, steps, flush):
     """Per-kernel-stage device times (ms) from the library's own CUDA events,
-    recorded on the forward's stream; eager launches, L2 flushed per step."""
+    recorded on the forward's stream inside a replayed CUDA graph (the events
+    are external event-record nodes); L2 flushed before every replay."""
     from paper_2609_05228_gb300 import ace
     s = torch.cuda.Stream()
     ace.ace_layer_set_profiling(layer.handle, True)
-    out_stages = []
-    with torch.cuda.stream(s):
-        for i in range(steps + 2):
-            flush.zero_()
+    try:
+        with torch.cuda.stream(s):
             ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q, s)
-            st = ace.ace_last_stage_times(layer.handle)
-            if i >= 2:
-                out_stages.append(st)
-    ace.ace_layer_set_profiling(layer.handle, False)
+        s.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q, torch.cuda.current_stream())
+        out_stages = []
+        with torch.cuda.stream(s):
+            for i in range(steps + 2):
+                flush.zero_()
+                g.replay()
+                st = ace.ace_last_stage_times(layer.handle)
+                if i >= 2:
+                    out_stages.append(st)
+    finally:
+        ace.ace_layer_set_profiling(layer.handle, False)
     return out_stages
 
 
@@ -209,7 +234,7 @@ def run_ours(args, rank, world, torch, dist):
     xh = synth.make_tokens(spec, T, seed=1 + rank)
     x = torch.from_numpy(xh.view(np.int16)).view(torch.bfloat16).to(dev)
     out = torch.empty_like(x)
-    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush = L2Flush(torch, dev)
 
     # decision statistics of this batch (R, distinct experts) and launches per step
     ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q)
@@ -234,7 +259,7 @@ def run_ours(args, rank, world, torch, dist):
     value, step_ms_max = aggregate(step_ms, T, world, dist, dev)
 
     # the dominant kernel's duration, from events on its own stream
-    stages = stage_times(torch, layer, x, out, T, q, args.steps, flush)
+    stages = stage_times(torch, layer, x, out, T, q, min(args.steps, 200), flush)
     # skip ratio 0 with the same kernels, for the speedup
     ms0 = time_point(torch, layer, x, out, T, 0.0, max(10, args.steps // 2), 3, flush)
     t0 = float(np.mean(ms0))
@@ -271,7 +296,7 @@ def run_ours(args, rank, world, torch, dist):
         "data": "synthetic (seeded N(0,1) tokens, N(0,0.02^2) weights, offline GSP/RCR tables)",
         "config": {"workload": wl["name"], "tokens_per_step": T, "skip_ratio": q,
                    "parallelism": f"replicas{world}" if world > 1 else "single GPU",
-                   "l2": "flushed (512 MB write) between timed steps", "graph": "CUDA graph replay"},
+                   "l2": "flushed between timed steps (512 MB write, then a 256 MB read)", "graph": "CUDA graph replay"},
         "realised_skip_ratio": round((T * spec.top_k - R) / (T * spec.top_k), 6),
         "retained_slots": R,
         "distinct_experts": D,
@@ -308,7 +333,7 @@ def sweep(torch, args):
                            ("prefill", [4096], [0.0, 0.25, 0.5, 0.625])]:
         wl = WORKLOADS[wlname]
         w, layer = build_layer(wl, max_tokens=max(Ts))
-        flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+        flush = L2Flush(torch, "cuda")
         for T in Ts:
             xh = synth.make_tokens(w.spec, T, seed=1)
             x = torch.from_numpy(xh.view(np.int16)).view(torch.bfloat16).cuda()

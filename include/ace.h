@@ -180,12 +180,14 @@ ace_status ace_debug_exp32(const float* x, float* y, int n, void* stream);
 /*
  * Stage timing (instrumentation; the paper has no counterpart). When enabled,
  * each ace_moe_forward records CUDA events on its stream around its stages:
- *   0 RMSNorm, 1 router logits, 2 top-k + decision + threshold + compaction,
- *   3 expert gate/up, 4 expert down, 5 combine.
+ *   0 RMSNorm (T > 256), 1 router logits (T <= 256: the whole fused
+ *   routing), 2 top-k + decision + threshold + compaction (T > 256),
+ *   3 token-row gather, 4 expert gate/up, 5 expert down, 6 combine.
  * ace_last_stage_times synchronises the last stream and writes up to n_max
  * stage durations in milliseconds (host float32) of the last forward; it
- * returns the stage count in *n_out. Enabling it is not allowed while the
- * stream is being captured.
+ * returns the stage count in *n_out. A forward captured into a CUDA graph
+ * with timing enabled records external event nodes, so every replay of the
+ * graph updates the times. Stage 3 (gather) is empty for the fp32 layer.
  */
 ace_status ace_layer_set_profiling(ace_layer* layer, int enable);
 ace_status ace_last_stage_times(ace_layer* layer, float* ms, int n_max, int* n_out);

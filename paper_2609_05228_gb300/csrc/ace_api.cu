@@ -42,7 +42,7 @@ void free_layer(ace_layer* L) {
     void* ptrs[] = {L->router_w, L->router_b, L->w_gate, L->w_up, L->w_gu, L->w_down, L->gamma, L->a_gsp,
                     L->a_rcr, L->ws.h, L->ws.logits, L->ws.ids, L->ws.gates, L->ws.cval, L->ws.keys, L->ws.skip,
                     L->ws.ghat, L->ws.tau, L->ws.chunk_counts, L->ws.offsets, L->ws.dlist, L->ws.perm,
-                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.act_bf16, L->ws.tt_off, L->ws.tt_tab, L->ws.tile_cnt, L->ws.err, L->ws.x_stage, L->ws.out_stage};
+                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.act_bf16, L->ws.tt_off, L->ws.tt_tab, L->ws.tile_cnt, L->ws.sel_hist, L->ws.sel_state, L->ws.err, L->ws.x_stage, L->ws.out_stage};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     for (cudaEvent_t e : L->ev)
@@ -190,6 +190,8 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     ALLOC(W.slot_pos, slots * sizeof(int32_t));
     ALLOC(W.meta, ace::kMetaCount * sizeof(int32_t));
     ALLOC(W.tile_cnt, (T / 8 + 1) * sizeof(int32_t));
+    ALLOC(W.sel_hist, 2048 * sizeof(int32_t));
+    ALLOC(W.sel_state, 8 * sizeof(int32_t));
     if (L->tc) {
         ALLOC(W.h_perm, slots * d * E);
         ALLOC(W.act_bf16, slots * m * E);
@@ -229,6 +231,8 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     CK(cudaMemcpyAsync(L->a_rcr, a_rcr, n * sizeof(float), cudaMemcpyHostToDevice, s), "copy a_rcr");
     CK(cudaMemsetAsync(W.meta, 0, ace::kMetaCount * sizeof(int32_t), s), "zero meta");
     CK(cudaMemsetAsync(W.tile_cnt, 0, (T / 8 + 1) * sizeof(int32_t), s), "zero tickets");
+    CK(cudaMemsetAsync(W.sel_hist, 0, 2048 * sizeof(int32_t), s), "zero select histogram");
+    CK(cudaMemsetAsync(W.sel_state, 0, 8 * sizeof(int32_t), s), "zero select state");
     CK(cudaMemsetAsync(W.err, 0, sizeof(int), s), "zero error word");
     CK(cudaMemsetAsync(W.offsets, 0, (n + 1) * sizeof(int32_t), s), "zero offsets");
     CK(ace::route_init(L), "route kernel attributes");
@@ -286,26 +290,26 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
     if (T == 0) return ACE_OK;
     cudaEvent_t* ev = L->profiling ? L->ev : nullptr;
     const bool small = ace::small_path(T);
-    if (ev) ACE_CUDA(cudaEventRecord(ev[0], s), "event record");
+    if (ev) ACE_CUDA(ace::record_stage(ev[0], s), "event record");
     if (!small) ACE_CUDA(ace::launch_rmsnorm(L, x, T, s), "rmsnorm launch");
-    if (ev) ACE_CUDA(cudaEventRecord(ev[1], s), "event record");
+    if (ev) ACE_CUDA(ace::record_stage(ev[1], s), "event record");
     if (small) {
         // router and routing in one launch (stage "router" holds both)
         ACE_CUDA(ace::launch_route_fused(L, x, L->ws.logits, T, ctl, s), "route launch");
-        if (ev) ACE_CUDA(cudaEventRecord(ev[2], s), "event record");
+        if (ev) ACE_CUDA(ace::record_stage(ev[2], s), "event record");
     } else {
         if (L->tc)
             ACE_CUDA(ace::launch_router_tc(L, T, s), "router launch");
         else
             ACE_CUDA(ace::launch_router(L, x, T, false, s), "router launch");
-        if (ev) ACE_CUDA(cudaEventRecord(ev[2], s), "event record");
+        if (ev) ACE_CUDA(ace::record_stage(ev[2], s), "event record");
         ACE_CUDA(ace::launch_route(L, L->ws.logits, T, ctl, s), "route launch");
     }
-    if (ev) ACE_CUDA(cudaEventRecord(ev[3], s), "event record");
+    if (ev) ACE_CUDA(ace::record_stage(ev[3], s), "event record");
     if (L->tc) {
         ACE_CUDA(ace::launch_experts_tc(L, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
     } else {
-        if (ev) ACE_CUDA(cudaEventRecord(ev[4], s), "event record");   // no gather stage
+        if (ev) ACE_CUDA(ace::record_stage(ev[4], s), "event record");   // no gather stage
         ACE_CUDA(ace::launch_experts_gemv(L, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
     }
     L->n_stages = ev ? ace::kNumStages : 0;

@@ -238,13 +238,13 @@ cudaError_t run(const ace_layer* L, void* out, int T_, cudaStream_t s, cudaEvent
     const size_t smem2 = (size_t)kTC * m * sizeof(float);
     k_gemv_gateup<T><<<grid, 256, smem1, s>>>((const T*)W.h, (const T*)L->w_gate, (const T*)L->w_up,
                                               W.offsets, W.dlist, W.perm, W.meta, W.act, d, m, k);
-    if (ev) cudaEventRecord(ev[1], s);
+    if (ev) ace::record_stage(ev[1], s);
     k_gemv_down<T><<<grid, 256, smem2, s>>>(W.act, (const T*)L->w_down, W.ghat, W.offsets, W.dlist, W.perm,
                                             W.meta, W.yslot, d, m);
     const long long n = (long long)T_ * (d / 4);
-    if (ev) cudaEventRecord(ev[2], s);
+    if (ev) ace::record_stage(ev[2], s);
     k_combine<T><<<(int)((n + 255) / 256), 256, 0, s>>>(W.yslot, W.slot_pos, (T*)out, T_, d, k);
-    if (ev) cudaEventRecord(ev[3], s);
+    if (ev) ace::record_stage(ev[3], s);
     return cudaGetLastError();
 }
 

@@ -229,6 +229,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int kblocks = p.K / kBK;
+    if (threadIdx.x == 0) {
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_tok)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_w)) : "memory");
+    }
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -443,7 +447,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
 // ---------------------------------------------------------------- helper kernels
 
 // h_perm[r] = h[perm[r] / k]: token rows in expert-grouped order for the
-// TMA tile loads of GEMM 1.
+// TMA tile loads of GEMM 1. One warp per row; d <= 4096 (16 vectors per lane).
 __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __restrict__ h,
                                                      const int32_t* __restrict__ perm,
                                                      const int32_t* __restrict__ meta,
@@ -452,12 +456,23 @@ __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __rest
     pdl_wait();
     const int R = meta[kMetaRetained];
     const int nvec = d / 8;
-    const long long total = (long long)R * nvec;
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const int r = (int)(i / nvec), c = (int)(i % nvec);
-        const int s = perm[r];
-        reinterpret_cast<uint4*>(h_perm + (size_t)r * d)[c] = reinterpret_cast<const uint4*>(h + (size_t)(s / k) * d)[c];
+    const int lane = threadIdx.x & 31;
+    const int wpb = blockDim.x >> 5;
+    for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < R; r += gridDim.x * wpb) {
+        const int tok = perm[r] / k;
+        const uint4* src = reinterpret_cast<const uint4*>(h + (size_t)tok * d);
+        uint4* dst = reinterpret_cast<uint4*>(h_perm + (size_t)r * d);
+        uint4 v[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int c = lane + 32 * i;
+            if (c < nvec) v[i] = src[c];
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int c = lane + 32 * i;
+            if (c < nvec) dst[c] = v[i];
+        }
     }
 }
 
@@ -627,7 +642,7 @@ cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t
     cudaError_t e = launch_pdl(k_gather_rows, dim3(L->num_sms * 4), dim3(256), 0, s, (const __nv_bfloat16*)W.h,
                                (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k);
     if (e != cudaSuccess) return e;
-    if (ev) cudaEventRecord(ev[0], s);
+    if (ev) ace::record_stage(ev[0], s);
     TcParams p1{};
     p1.tm_tok = small ? L->tcm.tok1_small : L->tcm.tok1_big;
     p1.tm_w = small ? L->tcm.wgu_small : L->tcm.wgu_big;
@@ -646,7 +661,7 @@ cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t
     p1.err = W.err;
     e = small ? launch_gemm<true, 0>(L, p1, s) : launch_gemm<false, 0>(L, p1, s);
     if (e != cudaSuccess) return e;
-    if (ev) cudaEventRecord(ev[1], s);
+    if (ev) ace::record_stage(ev[1], s);
     TcParams p2 = p1;
     p2.tm_tok = small ? L->tcm.tok2_small : L->tcm.tok2_big;
     p2.tm_w = small ? L->tcm.wd_small : L->tcm.wd_big;
@@ -657,11 +672,11 @@ cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t
     p2.out_ld = d;
     e = small ? launch_gemm<true, 1>(L, p2, s) : launch_gemm<false, 1>(L, p2, s);
     if (e != cudaSuccess) return e;
-    if (ev) cudaEventRecord(ev[2], s);
+    if (ev) ace::record_stage(ev[2], s);
     const long long nthreads = (long long)T * (d / 8);
     e = launch_pdl(k_combine_bf16, dim3((unsigned)((nthreads + 255) / 256)), dim3(256), 0, s, (const float*)W.yslot,
                    (const int32_t*)W.slot_pos, (__nv_bfloat16*)out, T, d, k);
-    if (ev) cudaEventRecord(ev[3], s);
+    if (ev) ace::record_stage(ev[3], s);
     return e;
 }
 

@@ -64,6 +64,8 @@ struct Workspace {
     int32_t* tt_off = nullptr;   // [N+1] token-tile prefix over distinct experts
     int4* tt_tab = nullptr;      // [N + Tmax*k/16 + 1] token tiles: (expert, first row, rows, 0)
     int32_t* tile_cnt = nullptr; // [Tmax/8 + 1] per-token-tile tickets of the fused small-T kernel
+    int32_t* sel_hist = nullptr; // [2048] global histogram of the multi-block threshold select (kept zero)
+    int32_t* sel_state = nullptr;// [8] prefix / want / below / ticket of the multi-block select
     int* err = nullptr;          // device error word
     void* x_stage = nullptr;     // [Tmax, d] dtype: host-API staging
     void* out_stage = nullptr;   // [Tmax, d]
@@ -168,6 +170,16 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// Stage-timing event: an external event-record node while the stream is
+// being captured (so graph replays record it), a plain record otherwise.
+inline cudaError_t record_stage(cudaEvent_t ev, cudaStream_t s) {
+    cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+    cudaError_t e = cudaStreamIsCapturing(s, &st);
+    if (e != cudaSuccess) return e;
+    return st == cudaStreamCaptureStatusActive ? cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal)
+                                               : cudaEventRecord(ev, s);
 }
 
 // Prefer the largest shared-memory carveout (all kernels share one L1/shared split).

@@ -5,7 +5,7 @@
 // Two launch shapes share the same device functions (and so the same bits):
 //   T <= kSmallT: k_route_fused, one launch for RMSNorm, router, top-k,
 //                 decision, threshold and compaction;
-//   larger T:     k_rmsnorm, k_router, k_topk_score, [k_tau_select, k_decide],
+//   larger T:     k_rmsnorm, router GEMM, k_topk_score, [3 x k_select_pass, k_decide],
 //                 k_compact_count, k_compact_place.
 #include <math.h>
 
@@ -502,13 +502,84 @@ __global__ void __launch_bounds__(256) k_decide(int n_tokens, int k, const float
     }
 }
 
-constexpr int kSelThreads = 1024;
+// Multi-block App. B.1 threshold for large T: three passes over the
+// candidate keys with 11/11/10-bit digits (bits [31:21], [20:10], [9:0]).
+// Each block histograms its chunk in shared memory and adds the non-empty
+// bins to one global histogram; the last block of the pass (ticket) finds
+// the digit holding the (m+1)-th smallest key, records it in `state`, and
+// clears the histogram for the next pass. The last pass writes tau with the
+// same tie rule as block_select_tau.
+// state: [0] prefix, [1] want, [2] below, [3] ticket, [4] last bin count
+constexpr int kMsBins = 2048;
+constexpr int kMsKeysPerBlock = 4096;
 
-__global__ void __launch_bounds__(kSelThreads) k_tau_select(const uint32_t* __restrict__ keys, int n,
-                                                            int m, float* __restrict__ tau_out) {
-    __shared__ SelectSmem<kSelThreads / 32> S;
-    const float tau = block_select_tau(keys, n, m, S);
-    if (threadIdx.x == 0) *tau_out = tau;
+__global__ void __launch_bounds__(1024) k_select_pass(const uint32_t* __restrict__ keys, int n, int m, int pass,
+                                                      int32_t* __restrict__ ghist, int32_t* __restrict__ state,
+                                                      float* __restrict__ tau_out) {
+    __shared__ int hist[kMsBins];
+    __shared__ bool is_last;
+    pdl_wait();
+    const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
+    const int bits = pass == 2 ? 10 : 11;
+    const uint32_t dmask = (1u << bits) - 1u;
+    const uint32_t pmask = pass == 0 ? 0u : (pass == 1 ? 0xFFE00000u : 0xFFFFFC00u);
+    const uint32_t prefix = pass == 0 ? 0u : (uint32_t)__ldcg(state + 0);
+    for (int i = threadIdx.x; i < kMsBins; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    const int lo = blockIdx.x * kMsKeysPerBlock, hi = min(n, lo + kMsKeysPerBlock);
+    for (int i = lo + threadIdx.x; i < hi; i += blockDim.x) {
+        const uint32_t key = keys[i];
+        if (key != 0xffffffffu && (key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & dmask], 1);
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < kMsBins; i += blockDim.x)
+        if (hist[i]) atomicAdd(&ghist[i], hist[i]);
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) is_last = atomicAdd(&state[3], 1) == (int)gridDim.x - 1;
+    __syncthreads();
+    if (!is_last) return;
+    __threadfence();
+    for (int i = threadIdx.x; i < kMsBins; i += blockDim.x) {
+        hist[i] = __ldcg(ghist + i);
+        ghist[i] = 0;
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        const int want = pass == 0 ? m : __ldcg(state + 1);
+        const int below0 = pass == 0 ? 0 : __ldcg(state + 2);
+        int loc = 0;
+        for (int j = 0; j < kMsBins / 32; ++j) loc += hist[lane * (kMsBins / 32) + j];
+        int inc = loc;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, inc, o);
+            if (lane >= o) inc += y;
+        }
+        const int exc = inc - loc;
+        const unsigned who = __ballot_sync(0xffffffffu, exc <= want && want < inc);
+        const int owner = who ? __ffs(who) - 1 : 31;
+        if (lane == owner) {
+            int cum = exc, dg = lane * (kMsBins / 32);
+            for (int j = 0; j < kMsBins / 32 - 1; ++j, ++dg) {
+                if (cum + hist[dg] > want) break;
+                cum += hist[dg];
+            }
+            const uint32_t pre = prefix | ((uint32_t)dg << shift);
+            const int below = below0 + cum;
+            state[0] = (int32_t)pre;
+            state[1] = want - cum;
+            state[2] = below;
+            state[4] = hist[dg];
+            state[3] = 0;
+            if (pass == 2) {
+                const int lo_c = below, hi_c = below + hist[dg];
+                float tau = __uint_as_float(pre);
+                if (!(lo_c == m || (m - lo_c) <= (hi_c - m))) tau = __uint_as_float(pre + 1u);
+                *tau_out = tau;
+            }
+        }
+    }
 }
 
 // Compaction (Algorithm 1 "evaluate only the experts indexed by I"): retained
@@ -1064,7 +1135,13 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     else ACE_TOPK(32);
 #undef ACE_TOPK
     if (mode == ACE_SKIP_RATIO) {
-        k_tau_select<<<1, kSelThreads, 0, s>>>(W.keys, T * k, m_q, W.tau);
+        const int nk = T * k;
+        const int sb = cdiv(nk, kMsKeysPerBlock);
+        for (int pass = 0; pass < 3; ++pass) {
+            cudaError_t e = launch_pdl(k_select_pass, dim3(sb), dim3(1024), 0, s, (const uint32_t*)W.keys, nk, m_q,
+                                       pass, W.sel_hist, W.sel_state, W.tau);
+            if (e != cudaSuccess) return e;
+        }
         k_decide<<<blocks, 256, 0, s>>>(T, k, W.gates, W.cval, W.tau, D.min_active, D.eps, W.skip, W.ghat);
     }
     const int n_chunks = cdiv(T, kChunk);
@@ -1080,7 +1157,7 @@ int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl) {
     float tau;
     bool sel;
     select_mq(L, T, ctl, &tau, &sel);
-    return sel ? 5 : 3;
+    return sel ? 7 : 3;
 }
 
 cudaError_t route_init(const ace_layer* L) {
@@ -1095,8 +1172,8 @@ cudaError_t route_init(const ace_layer* L) {
                         (const void*)k_route_fused<__nv_bfloat16, 32, true>, (const void*)k_route_fused<float, 4, true>,
                         (const void*)k_route_fused<float, 8, true>, (const void*)k_route_fused<float, 32, true>,
                         (const void*)k_rmsnorm<__nv_bfloat16>, (const void*)k_topk_score<4>, (const void*)k_topk_score<8>,
-                        (const void*)k_topk_score<32>, (const void*)k_tau_select, (const void*)k_decide,
-                        (const void*)k_compact_count, (const void*)k_compact_place};
+                        (const void*)k_topk_score<32>, (const void*)k_decide,
+                        (const void*)k_compact_count, (const void*)k_compact_place, (const void*)k_select_pass};
     for (const void* kf : ks)
         if ((e = prefer_shared(kf)) != cudaSuccess) return e;
     return cudaSuccess;
