@@ -67,6 +67,8 @@ typedef struct ace_layer_desc {
     float router_temp;   /* logits are divided by it; 1 if <= 0 */
     int min_active;      /* m_min of Algorithm 4 (1 = only the top-1 safeguard) */
     int has_router_bias; /* router_b is read when non-zero */
+    int add_residual;    /* non-zero: out = x + y (the decoder-block residual around
+                            the MoE layer), added in fp32 before rounding to dtype */
 } ace_layer_desc;
 
 typedef struct ace_skip_ctl {
@@ -109,7 +111,10 @@ void ace_layer_destroy(ace_layer* layer);
  * ace_moe_forward — y_t = sum_{i in I_t} g^_i f_{e_i}(x_t) for t < T
  * (Eq. ace_sparse_output), with RMSNorm, router, top-k, the skip decision of
  * Algorithm 4, compaction of the retained slots and the SwiGLU experts all on
- * the GPU. No residual is added.
+ * the GPU. out = y, or x + y when the layer was created with add_residual.
+ * Batches of T <= 256 sum a token's slot outputs in rank order (bitwise
+ * reproducible); larger batches accumulate them with fp32 atomics (results
+ * may differ between runs in the last bit).
  *   x    [T, d]  device, dtype     layer input (pre-RMSNorm hidden states)
  *   out  [T, d]  device, dtype     layer output; must not alias x
  *   T    0..max_tokens             T = 0 is a no-op

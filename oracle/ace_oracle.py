@@ -231,13 +231,17 @@ def ace_decide(z: np.ndarray, k: int, a_gsp, a_rcr, mode: str, value: float,
 
 
 def moe_forward(x: np.ndarray, w, mode: str = "threshold", value: float = 0.0,
-                decision: dict | None = None, return_decision: bool = False):
+                decision: dict | None = None, return_decision: bool = False,
+                tokens: np.ndarray | None = None):
     """ACE MoE layer output y_t = sum_{i in I_t} g_hat_i f_{e_i}(x_t)
     (Eq. ace_sparse_output; Algorithm 1 online loop for one layer), fp64.
 
     `w` is a synth.LayerWeights-like object (router_w, router_b, w_gate, w_up,
     w_down, gamma, spec). `a_gsp`/`a_rcr` tables are read from w.extra.
-    No residual connection is inside the layer.
+    No residual connection is inside the layer. With `tokens` (indices), the
+    decision is still taken over the whole batch (the per-batch threshold
+    needs every token) but the experts are evaluated for those tokens only;
+    the returned y then has one row per listed token.
     """
     spec = w.spec
     h = rmsnorm(x, w.gamma, spec.rms_eps)
@@ -246,14 +250,16 @@ def moe_forward(x: np.ndarray, w, mode: str = "threshold", value: float = 0.0,
         decision = ace_decide(z, spec.top_k, w.extra["a_gsp"], w.extra["a_rcr"], mode,
                               value, spec.min_active, spec.eps)
     ids, skip, g_hat = decision["ids"], decision["skip"], decision["g_hat"]
-    y = np.zeros_like(h)
+    rows = np.arange(h.shape[0]) if tokens is None else np.asarray(tokens)
+    hs, ids_s, skip_s, gh_s = h[rows], ids[rows], skip[rows], g_hat[rows]
+    y = np.zeros_like(hs)
     for e in range(spec.n_experts):
-        sel = (ids == e) & ~skip
+        sel = (ids_s == e) & ~skip_s
         tok, slot = np.nonzero(sel)
         if tok.size == 0:
             continue
-        f = swiglu_expert(h[tok], w.w_gate[e], w.w_up[e], w.w_down[e])
-        y[tok] += g_hat[tok, slot][:, None] * f
+        f = swiglu_expert(hs[tok], w.w_gate[e], w.w_up[e], w.w_down[e])
+        y[tok] += gh_s[tok, slot][:, None] * f
     if return_decision:
         return y, decision
     return y

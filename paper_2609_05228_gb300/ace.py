@@ -31,7 +31,7 @@ class ace_layer_desc(ctypes.Structure):
     _fields_ = [("hidden", ctypes.c_int), ("n_experts", ctypes.c_int), ("top_k", ctypes.c_int),
                 ("ffn", ctypes.c_int), ("max_tokens", ctypes.c_int), ("dtype", ctypes.c_int),
                 ("eps", ctypes.c_float), ("rms_eps", ctypes.c_float), ("router_temp", ctypes.c_float),
-                ("min_active", ctypes.c_int), ("has_router_bias", ctypes.c_int)]
+                ("min_active", ctypes.c_int), ("has_router_bias", ctypes.c_int), ("add_residual", ctypes.c_int)]
 
 
 class ace_skip_ctl(ctypes.Structure):
@@ -217,7 +217,7 @@ class AceLayer:
     """Owns one ace_layer. `w` holds nn.Linear-shaped host arrays (bf16 as
     uint16 bits or float32); a_gsp / a_rcr are the offline tables."""
 
-    def __init__(self, w, a_gsp, a_rcr, max_tokens: int, device: int = 0):
+    def __init__(self, w, a_gsp, a_rcr, max_tokens: int, device: int = 0, residual: bool = False):
         import torch
 
         spec = w.spec
@@ -234,7 +234,7 @@ class AceLayer:
         has_bias = bool(np.any(w.router_b != 0))
         self.desc = ace_layer_desc(spec.hidden, spec.n_experts, spec.top_k, spec.ffn, int(max_tokens),
                                    ACE_BF16 if bf else ACE_F32, spec.eps, spec.rms_eps, spec.router_temp,
-                                   spec.min_active, int(has_bias))
+                                   spec.min_active, int(has_bias), int(residual))
         tensors = [up(w.router_w), torch.from_numpy(np.ascontiguousarray(w.router_b, np.float32)).to(dev),
                    up(w.w_gate), up(w.w_up), up(w.w_down), up(w.gamma)]
         torch.cuda.synchronize(dev)

@@ -208,8 +208,8 @@ __global__ void __launch_bounds__(256) k_gemv_down(const float* __restrict__ act
 // out[t, c] = sum_{i kept, rank order} y[slot_pos[t*k+i], c]
 template <typename T>
 __global__ void __launch_bounds__(256) k_combine(const float* __restrict__ yslot,
-                                                 const int32_t* __restrict__ slot_pos, T* __restrict__ out,
-                                                 int n_tokens, int d, int k) {
+                                                 const int32_t* __restrict__ slot_pos, const T* __restrict__ resid,
+                                                 T* __restrict__ out, int n_tokens, int d, int k) {
     const int nq = d / 4;
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= (long long)n_tokens * nq) return;
@@ -221,6 +221,13 @@ __global__ void __launch_bounds__(256) k_combine(const float* __restrict__ yslot
         const float4 y = reinterpret_cast<const float4*>(yslot + (size_t)r * d)[c4];
         acc.x += y.x; acc.y += y.y; acc.z += y.z; acc.w += y.w;
     }
+    if (resid) {
+        const T* xr = resid + (size_t)t * d + c4 * 4;
+        acc.x = to_f32(xr[0]) + acc.x;
+        acc.y = to_f32(xr[1]) + acc.y;
+        acc.z = to_f32(xr[2]) + acc.z;
+        acc.w = to_f32(xr[3]) + acc.w;
+    }
     T* o = out + (size_t)t * d + c4 * 4;
     o[0] = from_f32<T>(acc.x);
     o[1] = from_f32<T>(acc.y);
@@ -229,7 +236,8 @@ __global__ void __launch_bounds__(256) k_combine(const float* __restrict__ yslot
 }
 
 template <typename T>
-cudaError_t run(const ace_layer* L, void* out, int T_, cudaStream_t s, cudaEvent_t* ev) {
+cudaError_t run(const ace_layer* L, const void* x, void* out, int T_, cudaStream_t s, cudaEvent_t* ev) {
+    const T* resid = L->desc.add_residual ? static_cast<const T*>(x) : nullptr;
     const ace_layer_desc& D = L->desc;
     const Workspace& W = L->ws;
     const int d = D.hidden, m = D.ffn, k = D.top_k;
@@ -243,7 +251,7 @@ cudaError_t run(const ace_layer* L, void* out, int T_, cudaStream_t s, cudaEvent
                                             W.meta, W.yslot, d, m);
     const long long n = (long long)T_ * (d / 4);
     if (ev) ace::record_stage(ev[2], s);
-    k_combine<T><<<(int)((n + 255) / 256), 256, 0, s>>>(W.yslot, W.slot_pos, (T*)out, T_, d, k);
+    k_combine<T><<<(int)((n + 255) / 256), 256, 0, s>>>(W.yslot, W.slot_pos, resid, (T*)out, T_, d, k);
     if (ev) ace::record_stage(ev[3], s);
     return cudaGetLastError();
 }
@@ -269,9 +277,9 @@ cudaError_t gemv_init(const ace_layer* L) {
     return e;
 }
 
-cudaError_t launch_experts_gemv(const ace_layer* L, void* out, int T, cudaStream_t s, cudaEvent_t* ev) {
-    if (L->desc.dtype == ACE_BF16) return run<__nv_bfloat16>(L, out, T, s, ev);
-    return run<float>(L, out, T, s, ev);
+cudaError_t launch_experts_gemv(const ace_layer* L, const void* x, void* out, int T, cudaStream_t s, cudaEvent_t* ev) {
+    if (L->desc.dtype == ACE_BF16) return run<__nv_bfloat16>(L, x, out, T, s, ev);
+    return run<float>(L, x, out, T, s, ev);
 }
 
 }  // namespace ace

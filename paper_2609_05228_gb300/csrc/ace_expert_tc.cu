@@ -163,6 +163,12 @@ __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.
 
 __device__ __forceinline__ float silu(float u) { return u / (1.0f + __expf(-u)); }
 
+// Vector atomic add of four floats (16-byte aligned address) at L2.
+__device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d) {
+    asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
+                 : "memory");
+}
+
 // ---------------------------------------------------------------- tile schedule
 
 struct Tile {
@@ -197,8 +203,9 @@ __device__ __forceinline__ Tile tile_at(const TcParams& p, int tile) {
 
 // SWAP: A (M = 128) = weight rows, B (N = TOKTILE) = token rows.
 // !SWAP: A (M = 128) = token rows, B (N = WTILE) = weight rows.
-// EPI 0: SwiGLU into act (bf16); EPI 1: g_hat-scaled rows into y (fp32);
-// EPI 2: router logits (fp32, + bias, / temperature), !SWAP only.
+// EPI 0: SwiGLU into act (bf16); EPI 1: g_hat-scaled down-projection rows,
+// per slot into y (SWAP, fp32) or added into the token's fp32 row of out_acc
+// (!SWAP); EPI 2: router logits (fp32, + bias, / temperature), SWAP only.
 template <bool SWAP, int EPI, int STAGES>
 struct TcCfg {
     static constexpr int TOKTILE = SWAP ? 16 : 128;
@@ -356,13 +363,28 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                         if (lane < 16 && c < t.nrows)
                             act[(size_t)(t.row0 + c) * p.out_ld + j] = __float2bfloat16_rn(silu(v) * u);
                     }
-                } else {
+                } else if (EPI == 1) {
                     const int col = t.wt * C::WTILE + quad * 32 + lane;
                     float* y = static_cast<float*>(p.out);
 #pragma unroll
                     for (int c = 0; c < 16; ++c) {
                         if (c < t.nrows)
                             y[(size_t)(t.row0 + c) * p.out_ld + col] = p.ghat[p.perm[t.row0 + c]] * __uint_as_float(r[c]);
+                    }
+                } else {
+                    // router logits: lane = expert, columns = tokens
+                    const int e = t.wt * C::WTILE + quad * 32 + lane;
+                    if (e < p.n_valid_cols) {
+                        float* z = static_cast<float*>(p.out);
+                        const float b = p.bias[e];
+#pragma unroll
+                        for (int c = 0; c < 16; ++c) {
+                            if (c < t.nrows) {
+                                float v = __uint_as_float(r[c]) + b;
+                                if (p.use_temp) v = v * p.inv_temp;
+                                z[(size_t)(t.row0 + c) * p.out_ld + e] = v;
+                            }
+                        }
                     }
                 }
             } else {
@@ -411,19 +433,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                         }
                     }
                 } else {
-                    float* y = static_cast<float*>(p.out);
-                    const float gh = valid ? p.ghat[p.perm[orow]] : 0.f;
+                    // g_hat-scaled output of this slot added into its token's fp32 row
+                    float* acc_out = static_cast<float*>(p.out);
+                    const int slot = valid ? p.perm[orow] : 0;
+                    const float gh = valid ? p.ghat[slot] : 0.f;
+                    float* dst_row = acc_out + (size_t)(slot / p.k) * p.out_ld + t.wt * C::WTILE;
 #pragma unroll 1
                     for (int c0 = 0; c0 < C::WTILE; c0 += 16) {
                         uint32_t r[16];
                         tmem_ld16(tbase + c0, r);
                         tmem_ld_wait();
                         if (valid) {
-                            float4* dst = reinterpret_cast<float4*>(y + orow * p.out_ld + t.wt * C::WTILE + c0);
 #pragma unroll
                             for (int i = 0; i < 4; ++i)
-                                dst[i] = make_float4(gh * __uint_as_float(r[4 * i]), gh * __uint_as_float(r[4 * i + 1]),
-                                                     gh * __uint_as_float(r[4 * i + 2]), gh * __uint_as_float(r[4 * i + 3]));
+                                red_add_v4(dst_row + c0 + 4 * i, gh * __uint_as_float(r[4 * i]), gh * __uint_as_float(r[4 * i + 1]),
+                                           gh * __uint_as_float(r[4 * i + 2]), gh * __uint_as_float(r[4 * i + 3]));
                         }
                     }
                 }
@@ -478,6 +502,7 @@ __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __rest
 
 // out[t, c] = sum_{i kept, rank order} y[slot_pos[t*k+i], c]  (Eq. ace_sparse_output)
 __global__ void __launch_bounds__(256) k_combine_bf16(const float* __restrict__ y, const int32_t* __restrict__ slot_pos,
+                                                      const __nv_bfloat16* __restrict__ resid,
                                                       __nv_bfloat16* __restrict__ out, int n_tokens, int d, int k) {
     pdl_wait();
     const int nq = d / 8;
@@ -493,10 +518,38 @@ __global__ void __launch_bounds__(256) k_combine_bf16(const float* __restrict__ 
         acc[0] += a.x; acc[1] += a.y; acc[2] += a.z; acc[3] += a.w;
         acc[4] += b.x; acc[5] += b.y; acc[6] += b.z; acc[7] += b.w;
     }
+    if (resid) {
+        float xr[8];
+        Vec16<__nv_bfloat16>::to_float(reinterpret_cast<const uint4*>(resid + (size_t)t * d)[c8], xr);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] = xr[i] + acc[i];
+    }
     __align__(16) __nv_bfloat16 o[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) o[i] = __float2bfloat16_rn(acc[i]);
     reinterpret_cast<uint4*>(out + (size_t)t * d)[c8] = *reinterpret_cast<const uint4*>(o);
+}
+
+// out[t, :] = bf16(acc[t, :]); acc[t, :] = 0 (ready for the next forward).
+__global__ void __launch_bounds__(256) k_finalize_bf16(float* __restrict__ acc, const __nv_bfloat16* __restrict__ resid,
+                                                       __nv_bfloat16* __restrict__ out, long long n8) {
+    pdl_wait();
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n8; i += (long long)gridDim.x * blockDim.x) {
+        float4* a = reinterpret_cast<float4*>(acc) + 2 * i;
+        float4 u = a[0], v = a[1];
+        if (resid) {
+            float xr[8];
+            Vec16<__nv_bfloat16>::to_float(reinterpret_cast<const uint4*>(resid)[i], xr);
+            u = make_float4(xr[0] + u.x, xr[1] + u.y, xr[2] + u.z, xr[3] + u.w);
+            v = make_float4(xr[4] + v.x, xr[5] + v.y, xr[6] + v.z, xr[7] + v.w);
+        }
+        __align__(16) __nv_bfloat16 o[8] = {__float2bfloat16_rn(u.x), __float2bfloat16_rn(u.y), __float2bfloat16_rn(u.z),
+                                            __float2bfloat16_rn(u.w), __float2bfloat16_rn(v.x), __float2bfloat16_rn(v.y),
+                                            __float2bfloat16_rn(v.z), __float2bfloat16_rn(v.w)};
+        reinterpret_cast<uint4*>(out)[i] = *reinterpret_cast<const uint4*>(o);
+        a[0] = make_float4(0.f, 0.f, 0.f, 0.f);
+        a[1] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
 }
 
 // ---------------------------------------------------------------- host side
@@ -591,7 +644,8 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = set_attr<true, 1>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 0>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 1>()) != cudaSuccess) return e;
-    if ((e = set_attr<false, 2>()) != cudaSuccess) return e;
+    if ((e = set_attr<true, 2>()) != cudaSuccess) return e;
+    if ((e = prefer_shared(k_finalize_bf16)) != cudaSuccess) return e;
     if ((e = prefer_shared(k_gather_rows)) != cudaSuccess) return e;
     if ((e = prefer_shared(k_combine_bf16)) != cudaSuccess) return e;
     // row counts as allocated at create time (padded to at least 256 rows)
@@ -610,8 +664,8 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = make_map(&L->tcm.wd_small, L->w_down, n * d, m, 128)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.wd_big, L->w_down, n * d, m, 256)) != cudaSuccess) return e;
     // router: h [Tmax, d] in 128-row boxes, W_r [N, d] in 256-row boxes
-    if ((e = make_map(&L->tcm.h_rows, L->ws.h, h_rows, d, 128)) != cudaSuccess) return e;
-    if ((e = make_map(&L->tcm.w_router, L->router_w, n_pad, d, 256)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.h_rows, L->ws.h, h_rows, d, 16)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.w_router, L->router_w, n_pad, d, 128)) != cudaSuccess) return e;
     return cudaSuccess;
 }
 
@@ -623,7 +677,7 @@ cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s) {
     p.out = L->ws.logits;
     p.K = D.hidden;
     p.w_rows = D.n_experts;
-    p.w_tiles = (D.n_experts + 255) / 256;
+    p.w_tiles = (D.n_experts + 127) / 128;
     p.out_ld = D.n_experts;
     p.err = L->ws.err;
     p.single_rows = T;
@@ -631,10 +685,11 @@ cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s) {
     p.inv_temp = 1.0f / D.router_temp;
     p.use_temp = D.router_temp != 1.0f;
     p.n_valid_cols = D.n_experts;
-    return launch_gemm<false, 2>(L, p, s);
+    return launch_gemm<true, 2>(L, p, s);
 }
 
-cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t s, cudaEvent_t* ev) {
+cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, cudaStream_t s, cudaEvent_t* ev) {
+    const __nv_bfloat16* resid = L->desc.add_residual ? static_cast<const __nv_bfloat16*>(x) : nullptr;
     const ace_layer_desc& D = L->desc;
     const Workspace& W = L->ws;
     const int d = D.hidden, m = D.ffn, k = D.top_k;
@@ -665,7 +720,7 @@ cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t
     TcParams p2 = p1;
     p2.tm_tok = small ? L->tcm.tok2_small : L->tcm.tok2_big;
     p2.tm_w = small ? L->tcm.wd_small : L->tcm.wd_big;
-    p2.out = W.yslot;
+    p2.out = small ? (void*)W.yslot : (void*)W.out_acc;
     p2.K = m;
     p2.w_rows = d;
     p2.w_tiles = d / (small ? 128 : 256);
@@ -674,8 +729,12 @@ cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t
     if (e != cudaSuccess) return e;
     if (ev) ace::record_stage(ev[2], s);
     const long long nthreads = (long long)T * (d / 8);
-    e = launch_pdl(k_combine_bf16, dim3((unsigned)((nthreads + 255) / 256)), dim3(256), 0, s, (const float*)W.yslot,
-                   (const int32_t*)W.slot_pos, (__nv_bfloat16*)out, T, d, k);
+    if (small)
+        e = launch_pdl(k_combine_bf16, dim3((unsigned)((nthreads + 255) / 256)), dim3(256), 0, s, (const float*)W.yslot,
+                       (const int32_t*)W.slot_pos, resid, (__nv_bfloat16*)out, T, d, k);
+    else
+        e = launch_pdl(k_finalize_bf16, dim3((unsigned)(L->num_sms * 8)), dim3(256), 0, s, W.out_acc, resid,
+                       (__nv_bfloat16*)out, nthreads);
     if (ev) ace::record_stage(ev[3], s);
     return e;
 }

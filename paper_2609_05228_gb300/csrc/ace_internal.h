@@ -60,6 +60,7 @@ struct Workspace {
     float* act = nullptr;        // [Tmax*k, m] fp32 (CUDA-core path)
     float* yslot = nullptr;      // [Tmax*k, d] fp32: g_hat-scaled expert outputs per retained slot
     void* h_perm = nullptr;      // [Tmax*k, d] bf16: h rows in expert-grouped order (tensor path)
+    float* out_acc = nullptr;    // [Tmax, d] fp32: large-batch output accumulator (kept zero between calls)
     void* act_bf16 = nullptr;    // [Tmax*k, m] bf16 (tensor path)
     int32_t* tt_off = nullptr;   // [N+1] token-tile prefix over distinct experts
     int4* tt_tab = nullptr;      // [N + Tmax*k/16 + 1] token tiles: (expert, first row, rows, 0)
@@ -192,7 +193,7 @@ inline cudaError_t prefer_shared(K kernel) {
 // ---- launchers (ace_expert_gemv.cu) ----
 // ev (nullable): events recorded before gate/up, before down, before combine, after combine.
 cudaError_t gemv_init(const ace_layer* L);
-cudaError_t launch_experts_gemv(const ace_layer* L, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
+cudaError_t launch_experts_gemv(const ace_layer* L, const void* x, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
 
 constexpr int kNumStages = 7;
 
@@ -202,7 +203,7 @@ int tc_token_tile(int T);
 cudaError_t tc_init(ace_layer* L);
 cudaError_t tc_pack_gate_up(ace_layer* L, const void* w_gate, const void* w_up, cudaStream_t s);
 // ev (nullable): recorded after gather, after gate/up, after down, after combine.
-cudaError_t launch_experts_tc(const ace_layer* L, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
+cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
 // Router logits on the tensor cores (T > kTcSmallT): z = (h W_r^T + b) / temp.
 cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s);
 
