@@ -32,11 +32,22 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 WORKLOADS = {
-    "decode": dict(zipf=False, T=64, q=0.5,
+    "decode": dict(spec="qwen", zipf=False, T=64, q=0.5, layers=1, tables="offline",
                    name="ACE MoE layer decode: d=2048 N=128 top-8 m=768 bf16, batch 64 tokens, skip ratio 0.5"),
-    "prefill": dict(zipf=True, T=4096, q=0.5,
+    "prefill": dict(spec="qwen", zipf=True, T=4096, q=0.5, layers=1, tables="offline",
                     name="ACE MoE layer prefill: d=2048 N=128 top-8 m=768 bf16, 4096 tokens Zipf(1.1) routing, "
                          "skip ratio 0.5"),
+    "stack_prefill": dict(spec="qwen", zipf=False, T=16384, q=0.5, layers=4, tables="offline",
+                          name="4-layer stack of the d=2048 N=128 top-8 m=768 layer (residual), prefill 16384 tokens, "
+                               "skip ratio 0.5"),
+    "stack_decode": dict(spec="qwen", zipf=False, T=32, q=0.5, layers=4, tables="offline",
+                         name="4-layer stack of the d=2048 N=128 top-8 m=768 layer (residual), decode 32 tokens, "
+                              "skip ratio 0.5"),
+    "large_prefill": dict(spec="large", zipf=True, T=8192, q=0.5, layers=1, tables="random",
+                          name="large MoE layer d=4096 N=256 top-8 m=2048 bf16, prefill 8192 tokens Zipf routing, "
+                               "skip ratio 0.5"),
+    "large_decode": dict(spec="large", zipf=True, T=128, q=0.5, layers=1, tables="random",
+                         name="large MoE layer d=4096 N=256 top-8 m=2048 bf16, decode 128 tokens, skip ratio 0.5"),
 }
 METRIC = "ACE MoE-layer tokens/s (prefill, decode) + speedup vs skip=0; % of roofline"
 L2_FLUSH_BYTES = 512 << 20
@@ -75,6 +86,14 @@ def _recorded_traffic(path="profiles/decode_T64_q0.5_expert_tc_full.md"):
         return int(rec["dram_bytes_per_launch"])
     except Exception:
         return None
+
+
+def _peak_sustained():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops_sustained"])
+    except Exception:
+        return 1700.0
 
 
 def _peaks():
@@ -133,28 +152,53 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def build_layer(wl, max_tokens):
-    from paper_2609_05228_gb300 import ace, offline, synth
-    spec = synth.spec_qwen(zipf=wl["zipf"])
-    w = synth.make_layer(spec, seed=0)
-    a_gsp, a_rcr = offline.tables(w)
-    w.extra["a_gsp"], w.extra["a_rcr"] = a_gsp, a_rcr
-    layer = ace.AceLayer(w, a_gsp, a_rcr, max_tokens=max_tokens)
-    return w, layer
+class Stack:
+    """The workload's layers on one device; a step chains their forwards.
+    In a stack every layer adds its input back (out = x + MoE(x))."""
+
+    def __init__(self, wl, max_tokens):
+        from paper_2609_05228_gb300 import ace, offline, synth
+        spec = synth.spec_qwen(zipf=wl["zipf"]) if wl["spec"] == "qwen" else synth.spec_large(zipf=wl["zipf"])
+        self.ws, self.layers = [], []
+        n = wl["layers"]
+        for l in range(n):
+            w = synth.make_layer(spec, seed=0 if n == 1 else 100 + l)
+            if wl["tables"] == "offline":
+                w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables(w)
+            else:   # the large layer: seeded positive tables stand in (the forward takes any valid tables)
+                w.extra["a_gsp"], w.extra["a_rcr"] = synth.make_tables(spec.n_experts, seed=5, spread=0.1)
+            self.ws.append(w)
+            self.layers.append(ace.AceLayer(w, w.extra["a_gsp"], w.extra["a_rcr"], max_tokens=max_tokens,
+                                            residual=n > 1))
+            del w
+        self.spec = spec
+
+    def buffers(self, torch, x):
+        return [torch.empty_like(x) for _ in self.layers]
+
+    def forward(self, x, bufs, T, q, stream=None):
+        from paper_2609_05228_gb300 import ace
+        cur = x
+        for layer, out in zip(self.layers, bufs):
+            ace.ace_moe_forward(layer.handle, cur, out, T, "ratio", q, stream)
+            cur = out
+
+    def close(self):
+        for layer in self.layers:
+            layer.close()
 
 
-def time_point(torch, layer, x, out, T, q, steps, warmup, flush):
+def time_point(torch, model, x, bufs, T, q, steps, warmup, flush):
     """Device time per step (ms) of a graph-replayed forward."""
-    from paper_2609_05228_gb300 import ace
     s = torch.cuda.Stream()
     torch.cuda.synchronize()
     # warm the path once eagerly (outside capture)
     with torch.cuda.stream(s):
-        ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q, s)
+        model.forward(x, bufs, T, q, s)
     s.synchronize()
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=s):
-        ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q, torch.cuda.current_stream())
+        model.forward(x, bufs, T, q, torch.cuda.current_stream())
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     with torch.cuda.stream(s):
@@ -171,30 +215,33 @@ def time_point(torch, layer, x, out, T, q, steps, warmup, flush):
     return [a.elapsed_time(b) for a, b in zip(starts, ends)]
 
 
-def stage_times(torch, layer, x, out, T, q, steps, flush):
-    """Per-kernel-stage device times (ms) from the library's own CUDA events,
-    recorded on the forward's stream inside a replayed CUDA graph (the events
-    are external event-record nodes); L2 flushed before every replay."""
+def stage_times(torch, model, x, bufs, T, q, steps, flush):
+    """Per-kernel-stage device times (ms, summed over the layers) from the
+    library's own CUDA events, recorded on the forward's stream inside a
+    replayed CUDA graph (external event-record nodes); L2 flushed before
+    every replay."""
     from paper_2609_05228_gb300 import ace
     s = torch.cuda.Stream()
-    ace.ace_layer_set_profiling(layer.handle, True)
+    for layer in model.layers:
+        ace.ace_layer_set_profiling(layer.handle, True)
     try:
         with torch.cuda.stream(s):
-            ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q, s)
+            model.forward(x, bufs, T, q, s)
         s.synchronize()
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=s):
-            ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q, torch.cuda.current_stream())
+            model.forward(x, bufs, T, q, torch.cuda.current_stream())
         out_stages = []
         with torch.cuda.stream(s):
             for i in range(steps + 2):
                 flush.zero_()
                 g.replay()
-                st = ace.ace_last_stage_times(layer.handle)
+                per = [ace.ace_last_stage_times(layer.handle) for layer in model.layers]
                 if i >= 2:
-                    out_stages.append(st)
+                    out_stages.append({k: sum(p[k] for p in per) for k in per[0]})
     finally:
-        ace.ace_layer_set_profiling(layer.handle, False)
+        for layer in model.layers:
+            ace.ace_layer_set_profiling(layer.handle, False)
     return out_stages
 
 
@@ -229,16 +276,16 @@ def run_ours(args, rank, world, torch, dist):
     T, q = wl["T"], wl["q"]
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
-    w, layer = build_layer(wl, max_tokens=max(T, 64))
-    spec = w.spec
+    model = Stack(wl, max_tokens=max(T, 64))
+    spec, w, layer = model.spec, model.ws[0], model.layers[0]
     xh = synth.make_tokens(spec, T, seed=1 + rank)
     x = torch.from_numpy(xh.view(np.int16)).view(torch.bfloat16).to(dev)
-    out = torch.empty_like(x)
+    bufs = model.buffers(torch, x)
     flush = L2Flush(torch, dev)
 
-    # decision statistics of this batch (R, distinct experts) and launches per step
-    ace.ace_moe_forward(layer.handle, x, out, T, "ratio", q)
-    launches = ace.ace_last_launch_count(layer.handle)
+    # decision statistics of the first layer's batch (R, distinct experts) and launches per step
+    model.forward(x, bufs, T, q)
+    launches = sum(ace.ace_last_launch_count(l.handle) for l in model.layers)
     skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, spec.top_k)
     off, _ = ace.ace_last_permutation(layer.handle, spec.n_experts, R)
     D = int((np.diff(off) > 0).sum())
@@ -249,7 +296,7 @@ def run_ours(args, rank, world, torch, dist):
     torch.cuda.synchronize()
     clocks = ClockSampler(dev.index)
     t_wall = time.perf_counter()
-    ms = time_point(torch, layer, x, out, T, q, args.steps, args.warmup, flush)
+    ms = time_point(torch, model, x, bufs, T, q, args.steps, args.warmup, flush)
     torch.cuda.synchronize()
     wall = time.perf_counter() - t_wall
     clk = clocks.stop()
@@ -259,27 +306,43 @@ def run_ours(args, rank, world, torch, dist):
     value, step_ms_max = aggregate(step_ms, T, world, dist, dev)
 
     # the dominant kernel's duration, from events on its own stream
-    stages = stage_times(torch, layer, x, out, T, q, min(args.steps, 200), flush)
+    stages = stage_times(torch, model, x, bufs, T, q, min(args.steps, 200), flush)
     # skip ratio 0 with the same kernels, for the speedup
-    ms0 = time_point(torch, layer, x, out, T, 0.0, max(10, args.steps // 2), 3, flush)
+    ms0 = time_point(torch, model, x, bufs, T, 0.0, max(10, min(args.steps // 2, 200)), 3, flush)
     t0 = float(np.mean(ms0))
 
-    # end to end through the host-buffer C call (pinned buffers, copies included)
+    # end to end through the host-buffer C call (pinned buffers, copies included; one layer)
     xp = torch.from_numpy(xh.view(np.int16)).pin_memory()
     op = torch.empty_like(xp).pin_memory()
     for _ in range(3):
         ace.ace_moe_forward_host(layer.handle, xp, op, T, "ratio", q)
-    e2e_steps = max(10, args.steps)
+    e2e_steps = max(10, min(args.steps, 300))
     t = time.perf_counter()
     for _ in range(e2e_steps):
-        ace.ace_moe_forward_host(layer.handle, xp, op, T, "ratio", q)
+        for l in model.layers:
+            ace.ace_moe_forward_host(l.handle, xp, op, T, "ratio", q)
     e2e_s = (time.perf_counter() - t) / e2e_steps
 
     hbm, bf16, peak_kind = _peaks()
+    bf16_sust = _peak_sustained()
+    n_layers = len(model.layers)
     total_bytes, flops, gu_bytes = algorithmic(w, T, R, D)
-    gu_ms = float(np.mean([st["gate_up"] for st in stages])) if stages else float("nan")
-    achieved = gu_bytes / (gu_ms * 1e-3) / 1e9
+    gu_flops = 4 * spec.hidden * spec.ffn * R
+    gu_ms = float(np.mean([st["gate_up"] for st in stages])) / n_layers if stages else float("nan")
     stage_avg = {k: round(float(np.mean([st[k] for st in stages])) * 1e3, 2) for k in stages[0]} if stages else {}
+    tensor_bound = R / max(D, 1) > 280           # tokens per expert above the ridge (FLOP/B)
+    if tensor_bound:
+        achieved = gu_flops / (gu_ms * 1e-3) / 1e12
+        roof = {"bound": "tensor", "kernel": "k_expert_tc gate/up (tcgen05)", "achieved": round(achieved, 1),
+                "peak": bf16_sust, "unit": "TFLOP/s", "frac": round(achieved / bf16_sust, 4),
+                "peak_source": peak_kind + " (sustained bf16)", "traffic": None,
+                "algorithmic_flops": gu_flops, "kernel_us": round(gu_ms * 1e3, 2)}
+    else:
+        achieved = gu_bytes / (gu_ms * 1e-3) / 1e9
+        roof = {"bound": "hbm", "kernel": "k_expert_tc gate/up (tcgen05" + (", SWAP)" if T <= 256 else ")"),
+                "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s", "frac": round(achieved / hbm, 4),
+                "peak_source": peak_kind, "traffic": _recorded_traffic() if args.workload == "decode" else None,
+                "algorithmic_bytes": gu_bytes, "kernel_us": round(gu_ms * 1e3, 2)}
 
     result = {
         "metric": METRIC,
@@ -293,8 +356,9 @@ def run_ours(args, rank, world, torch, dist):
         "scaling": "weak",
         "vs_baseline": None,
         "dtype": "bf16",
-        "data": "synthetic (seeded N(0,1) tokens, N(0,0.02^2) weights, offline GSP/RCR tables)",
-        "config": {"workload": wl["name"], "tokens_per_step": T, "skip_ratio": q,
+        "data": "synthetic (seeded N(0,1) tokens, N(0,0.02^2) weights, " +
+                ("offline GSP/RCR tables)" if wl["tables"] == "offline" else "seeded positive tables)"),
+        "config": {"workload": wl["name"], "tokens_per_step": T, "layers": n_layers, "skip_ratio": q,
                    "parallelism": f"replicas{world}" if world > 1 else "single GPU",
                    "l2": "flushed between timed steps (512 MB write, then a 256 MB read)", "graph": "CUDA graph replay"},
         "realised_skip_ratio": round((T * spec.top_k - R) / (T * spec.top_k), 6),
@@ -304,24 +368,21 @@ def run_ours(args, rank, world, torch, dist):
         "q0_ms_per_step": round(t0, 5),
         "stage_us": stage_avg,
         "wall_s": round(wall, 3),
-        "roofline": {"bound": "hbm", "kernel": "k_expert_tc gate/up (tcgen05, SWAP)", "achieved": round(achieved, 1),
-                     "peak": hbm, "unit": "GB/s", "frac": round(achieved / hbm, 4),
-                     "peak_source": peak_kind,
-                     "traffic": _recorded_traffic() if args.workload == "decode" else None,
-                     "algorithmic_bytes": gu_bytes, "kernel_us": round(gu_ms * 1e3, 2)},
-        "layer_roofline": {"bytes": total_bytes, "flops": flops,
-                           "hbm_frac": round(total_bytes / (step_ms * 1e-3) / 1e9 / hbm, 4),
-                           "tensor_frac": round(flops / (step_ms * 1e-3) / 1e12 / bf16, 5)},
+        "roofline": roof,
+        "layer_roofline": {"bytes": total_bytes * n_layers, "flops": flops * n_layers,
+                           "hbm_frac": round(total_bytes * n_layers / (step_ms * 1e-3) / 1e9 / hbm, 4),
+                           "tensor_frac": round(flops * n_layers / (step_ms * 1e-3) / 1e12 / bf16_sust, 5)},
         "e2e": {"value": round(T / e2e_s, 1), "unit": "tokens/s",
-                "h2d_bytes_per_step": int(T * spec.hidden * 2), "d2h_bytes_per_step": int(T * spec.hidden * 2)},
+                "h2d_bytes_per_step": int(n_layers * T * spec.hidden * 2),
+                "d2h_bytes_per_step": int(n_layers * T * spec.hidden * 2)},
         "gpu_launches": args.steps * launches,
         "clocks": clk,
     }
     if rank == 0 and not args.no_cpu_baseline:
-        result["cpu_baseline"] = cpu_baseline(w, wl, budget_s=args.cpu_seconds)
+        result["cpu_baseline"] = cpu_baseline(model.ws, wl, budget_s=args.cpu_seconds)
     if rank == 0 and args.sweep:
         result["sweep"] = sweep(torch, args)
-    layer.close()
+    model.close()
     return result
 
 
@@ -331,42 +392,46 @@ def sweep(torch, args):
     pts = []
     for wlname, Ts, qs in [("decode", [1, 8, 32, 64], [0.0, 0.25, 0.5]),
                            ("prefill", [4096], [0.0, 0.25, 0.5, 0.625])]:
-        wl = WORKLOADS[wlname]
-        w, layer = build_layer(wl, max_tokens=max(Ts))
+        model = Stack(WORKLOADS[wlname], max_tokens=max(Ts))
         flush = L2Flush(torch, "cuda")
         for T in Ts:
-            xh = synth.make_tokens(w.spec, T, seed=1)
+            xh = synth.make_tokens(model.spec, T, seed=1)
             x = torch.from_numpy(xh.view(np.int16)).view(torch.bfloat16).cuda()
-            out = torch.empty_like(x)
+            bufs = model.buffers(torch, x)
             base = None
             for q in qs:
-                ms = time_point(torch, layer, x, out, T, q, 20, 3, flush)
+                ms = time_point(torch, model, x, bufs, T, q, 20, 3, flush)
                 t = float(np.median(ms))
                 base = t if q == 0.0 else base
                 pts.append({"workload": wlname, "T": T, "q": q, "us": round(t * 1e3, 2),
                             "tokens_per_s": round(T / (t * 1e-3), 1),
                             "speedup_vs_q0": round(base / t, 4) if base else None})
-        layer.close()
+        model.close()
     return pts
 
 
-def cpu_baseline(w, wl, budget_s=12.0):
-    """The CPU oracle (fp64) on a bounded sample of the same workload."""
+def cpu_baseline(ws, wl, budget_s=12.0):
+    """The CPU oracle (fp64) on a bounded sample of the same workload: the
+    stacked layers over a sample of tokens (64, or 256 for prefill)."""
     import oracle as O
     from paper_2609_05228_gb300 import synth
     T = wl["T"] if wl["T"] <= 64 else 256
-    x = synth.make_tokens(w.spec, T, seed=1)
+    x = synth.make_tokens(ws[0].spec, T, seed=1)
     n = 0
     t0 = time.perf_counter()
     while True:
-        O.moe_forward(x, w, "ratio", wl["q"])
+        cur = O.to_f64(x)
+        for i, w in enumerate(ws):
+            y = O.moe_forward(cur, w, "ratio", wl["q"])
+            cur = cur + y if len(ws) > 1 else y
         n += 1
         if time.perf_counter() - t0 > budget_s:
             break
     dt = time.perf_counter() - t0
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
     return {"value": round(n * T / dt, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
-            "sample": f"{n} forwards of {T} tokens ({dt:.1f} s), numpy fp64 with its default BLAS threads"}
+            "sample": f"{n} forwards of {T} tokens through {len(ws)} layer(s) ({dt:.1f} s), numpy fp64 "
+                      "with its default BLAS threads"}
 
 
 def run_reference(args):
@@ -374,26 +439,39 @@ def run_reference(args):
     import oracle as O
     from paper_2609_05228_gb300 import offline, synth
     wl = WORKLOADS[args.workload]
-    spec = synth.spec_qwen(zipf=wl["zipf"])
-    w = synth.make_layer(spec, seed=0)
-    w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables(w)
+    spec = synth.spec_qwen(zipf=wl["zipf"]) if wl["spec"] == "qwen" else synth.spec_large(zipf=wl["zipf"])
+    ws = []
+    for l in range(wl["layers"]):
+        w = synth.make_layer(spec, seed=0 if wl["layers"] == 1 else 100 + l)
+        if wl["tables"] == "offline":
+            w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables(w)
+        else:
+            w.extra["a_gsp"], w.extra["a_rcr"] = synth.make_tables(spec.n_experts, seed=5, spread=0.1)
+        ws.append(w)
     T = wl["T"] if wl["T"] <= 64 else 256
     x = synth.make_tokens(spec, T, seed=1)
+
+    def step():
+        cur = O.to_f64(x)
+        for w in ws:
+            y = O.moe_forward(cur, w, "ratio", wl["q"])
+            cur = cur + y if len(ws) > 1 else y
+
     for _ in range(args.warmup):
-        O.moe_forward(x, w, "ratio", wl["q"])
+        step()
     times = []
     for _ in range(args.steps):
         t = time.perf_counter()
-        O.moe_forward(x, w, "ratio", wl["q"])
+        step()
         times.append(time.perf_counter() - t)
-    step = float(np.mean(times))
+    st = float(np.mean(times))
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
-    val = round(T / step, 2)
+    val = round(T / st, 2)
     return {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s", "n_gpus": 1,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step * 1e3, 3),
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(st * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": wl["name"], "tokens_per_step": T, "skip_ratio": wl["q"],
-                                            "sample": f"{T} tokens per step"},
+            "data": "synthetic", "config": {"workload": wl["name"], "tokens_per_step": T, "layers": len(ws),
+                                            "skip_ratio": wl["q"], "sample": f"{T} tokens per step"},
             "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                              "sample": f"{args.steps} steps of {T} tokens"},
             "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}

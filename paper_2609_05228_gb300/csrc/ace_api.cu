@@ -42,7 +42,7 @@ void free_layer(ace_layer* L) {
     void* ptrs[] = {L->router_w, L->router_b, L->w_gate, L->w_up, L->w_gu, L->w_down, L->gamma, L->a_gsp,
                     L->a_rcr, L->ws.h, L->ws.logits, L->ws.ids, L->ws.gates, L->ws.cval, L->ws.keys, L->ws.skip,
                     L->ws.ghat, L->ws.tau, L->ws.chunk_counts, L->ws.offsets, L->ws.dlist, L->ws.perm,
-                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.out_acc, L->ws.act_bf16, L->ws.tt_off, L->ws.tt_tab, L->ws.tile_cnt, L->ws.sel_hist, L->ws.sel_state, L->ws.err, L->ws.x_stage, L->ws.out_stage};
+                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.act_bf16, L->ws.tt_off, L->ws.tt_tab, L->ws.tile_cnt, L->ws.sel_hist, L->ws.sel_state, L->ws.err, L->ws.x_stage, L->ws.out_stage};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     for (cudaEvent_t e : L->ev)
@@ -194,15 +194,14 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     ALLOC(W.sel_state, 8 * sizeof(int32_t));
     if (L->tc) {
         ALLOC(W.h_perm, slots * d * E);
-        ALLOC(W.out_acc, T * d * sizeof(float));
         ALLOC(W.act_bf16, slots * m * E);
         ALLOC(W.tt_off, (n + 1) * sizeof(int32_t));
         ALLOC(W.tt_tab, (n + slots / 16 + 1) * sizeof(int4));
     } else {
         ALLOC(W.act, slots * m * sizeof(float));
     }
-    // per-slot expert outputs: every batch on the CUDA-core path, batches of
-    // up to 256 tokens on the tensor path (larger ones accumulate in out_acc)
+    // fp32 per-slot expert outputs: every batch on the CUDA-core path, batches
+    // of up to 256 tokens on the tensor path (larger ones write bf16 rows over h_perm)
     const size_t yslot_rows = L->tc ? (size_t)(D.max_tokens < 256 ? D.max_tokens : 256) * k : slots;
     ALLOC(W.yslot, yslot_rows * d * sizeof(float));
     ALLOC(W.err, sizeof(int));
@@ -236,7 +235,6 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     CK(cudaMemsetAsync(W.meta, 0, ace::kMetaCount * sizeof(int32_t), s), "zero meta");
     CK(cudaMemsetAsync(W.tile_cnt, 0, (T / 8 + 1) * sizeof(int32_t), s), "zero tickets");
     CK(cudaMemsetAsync(W.sel_hist, 0, 2048 * sizeof(int32_t), s), "zero select histogram");
-    if (L->tc) CK(cudaMemsetAsync(W.out_acc, 0, T * d * sizeof(float), s), "zero output accumulator");
     CK(cudaMemsetAsync(W.sel_state, 0, 8 * sizeof(int32_t), s), "zero select state");
     CK(cudaMemsetAsync(W.err, 0, sizeof(int), s), "zero error word");
     CK(cudaMemsetAsync(W.offsets, 0, (n + 1) * sizeof(int32_t), s), "zero offsets");
@@ -318,7 +316,7 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
         ACE_CUDA(ace::launch_experts_gemv(L, x, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
     }
     L->n_stages = ev ? ace::kNumStages : 0;
-    L->last_launches = (small ? 1 : 2 + ace::route_launch_count(L, T, ctl)) + (L->tc ? 4 : 3);
+    L->last_launches = (small ? 1 : 2 + ace::route_launch_count(L, T, ctl)) + (L->tc ? (small ? 3 : 4) : 3);
     return ACE_OK;
 }
 

@@ -35,7 +35,6 @@ namespace {
 constexpr int kBK = 64;                 // K elements per stage (128 bytes of bf16)
 constexpr int kUmmaK = 16;              // K per tcgen05.mma (kind::f16)
 constexpr int kThreads = 192;
-constexpr long long kSpinCycles = 4000000000LL;   // ~2 s at 2 GHz
 
 struct TcParams {
     CUtensorMap tm_tok;                 // token rows [rows, K] bf16
@@ -44,7 +43,7 @@ struct TcParams {
     const int32_t* dlist;               // [N]
     const int4* tt_tab;                 // token tiles (expert, first row, rows, 0)
     const int32_t* meta;
-    void* out;                          // act bf16 [rows, m] or y fp32 [rows, d]
+    void* out;                          // act bf16 [rows, m], y [rows, d] (fp32 SWAP / bf16) or logits
     int K;                              // reduction length
     int w_rows;                         // weight rows per expert (2m or d)
     int w_tiles;                        // w_rows / weight tile
@@ -56,54 +55,13 @@ struct TcParams {
     float inv_temp;
     int use_temp;
     int n_valid_cols;                   // columns of out that exist (EPI 2)
-    const int32_t* perm;                // [R] slot of row r (GEMM 2 epilogue)
+    const int32_t* perm;                // [R] slot of row r (GEMM 2 epilogue; direct token rows)
+    int direct_rows;                    // SWAP: token rows loaded one by one from h (tm_tok: one-row boxes)
     const float* ghat;                  // [T*k] g_hat by slot (GEMM 2 reads ghat[perm[r]])
     int k;
 };
 
 // ---------------------------------------------------------------- PTX wrappers
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-                 : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// Bounded wait: false (and kErrTimeout set) if the phase did not complete.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const long long t0 = clock64();
-    while (!mbar_try_wait(bar, parity)) {
-        if (clock64() - t0 > kSpinCycles) {
-            atomicOr(err, kErrTimeout);
-            return false;
-        }
-    }
-    return true;
-}
 
 __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
     asm volatile(
@@ -163,12 +121,6 @@ __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.
 
 __device__ __forceinline__ float silu(float u) { return u / (1.0f + __expf(-u)); }
 
-// Vector atomic add of four floats (16-byte aligned address) at L2.
-__device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d) {
-    asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
-                 : "memory");
-}
-
 // ---------------------------------------------------------------- tile schedule
 
 struct Tile {
@@ -203,9 +155,9 @@ __device__ __forceinline__ Tile tile_at(const TcParams& p, int tile) {
 
 // SWAP: A (M = 128) = weight rows, B (N = TOKTILE) = token rows.
 // !SWAP: A (M = 128) = token rows, B (N = WTILE) = weight rows.
-// EPI 0: SwiGLU into act (bf16); EPI 1: g_hat-scaled down-projection rows,
-// per slot into y (SWAP, fp32) or added into the token's fp32 row of out_acc
-// (!SWAP); EPI 2: router logits (fp32, + bias, / temperature), SWAP only.
+// EPI 0: SwiGLU into act (bf16); EPI 1: g_hat-scaled down-projection rows
+// per slot, into y (fp32 for SWAP, bf16 otherwise); EPI 2: router logits
+// (fp32, + bias, / temperature), SWAP only.
 template <bool SWAP, int EPI, int STAGES>
 struct TcCfg {
     static constexpr int TOKTILE = SWAP ? 16 : 128;
@@ -269,36 +221,49 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
-        if (lane == 0) {
-            int stage = 0;
-            uint32_t phase = 0;
-            bool ok = true;
-            long long issued = 0;
-            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-                const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile);
-                for (int kb = 0; kb < kblocks; ++kb) {
-                    if (!mbar_wait(&empty[stage], phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
-                    unsigned char* sa = smem + stage * C::STAGE_BYTES;
-                    unsigned char* sb = sa + C::A_BYTES;
-                    mbar_expect_tx(&full[stage], C::STAGE_BYTES);
+        // Lane 0 waits for free stages and loads the A tile (and the B tile);
+        // with direct token rows (SWAP, GEMM 1) lane i < rows loads token row
+        // i of the tile from h itself (a one-row box; the 128-byte swizzle
+        // follows the shared-memory address, so the rows form the same tile).
+        const bool direct = SWAP && p.direct_rows;
+        int stage = 0;
+        uint32_t phase = 0;
+        bool ok = true;
+        long long issued = 0;
+        for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+            const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile);
+            const int my_row = (direct && lane < t.nrows) ? p.perm[t.row0 + lane] / p.k : 0;
+            const uint32_t bytes = direct ? (uint32_t)(C::A_BYTES + t.nrows * kBK * 2) : (uint32_t)C::STAGE_BYTES;
+            for (int kb = 0; kb < kblocks; ++kb) {
+                int go = 1;
+                if (lane == 0) go = mbar_wait(&empty[stage], phase ^ 1u, p.err) && !*abort_flag;
+                if (!__shfl_sync(0xffffffffu, go, 0)) { ok = false; break; }
+                unsigned char* sa = smem + stage * C::STAGE_BYTES;
+                unsigned char* sb = sa + C::A_BYTES;
+                if (lane == 0) {
+                    mbar_expect_tx(&full[stage], bytes);
                     if (SWAP) {
                         tma_load_2d(sa, &p.tm_w, &full[stage], kb * kBK, t.wrow0);
-                        tma_load_2d(sb, &p.tm_tok, &full[stage], kb * kBK, t.row0);
+                        if (!direct) tma_load_2d(sb, &p.tm_tok, &full[stage], kb * kBK, t.row0);
                     } else {
                         tma_load_2d(sa, &p.tm_tok, &full[stage], kb * kBK, t.row0);
                         tma_load_2d(sb, &p.tm_w, &full[stage], kb * kBK, t.wrow0);
                     }
-                    ++issued;
-                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
+                if (direct) {
+                    __syncwarp();
+                    if (lane < t.nrows) tma_load_2d(sb + lane * (kBK * 2), &p.tm_tok, &full[stage], kb * kBK, my_row);
+                }
+                ++issued;
+                if (++stage == STAGES) { stage = 0; phase ^= 1u; }
             }
-            if (!ok) {
-                *abort_flag = 1;
-                // our own copies must land before the block exits: wait (bounded)
-                // on the full barrier of each of the last STAGES fills
-                for (long long f = issued - 1; f >= 0 && f >= issued - STAGES; --f) {
-                    if (!mbar_wait(&full[f % STAGES], (uint32_t)((f / STAGES) & 1), p.err)) break;
-                }
+        }
+        if (!ok && lane == 0) {
+            *abort_flag = 1;
+            // our own copies must land before the block exits: wait (bounded)
+            // on the full barrier of each of the last STAGES fills
+            for (long long f = issued - 1; f >= 0 && f >= issued - STAGES; --f) {
+                if (!mbar_wait(&full[f % STAGES], (uint32_t)((f / STAGES) & 1), p.err)) break;
             }
         }
     } else if (warp == 1) {
@@ -433,21 +398,30 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                         }
                     }
                 } else {
-                    // g_hat-scaled output of this slot added into its token's fp32 row
-                    float* acc_out = static_cast<float*>(p.out);
-                    const int slot = valid ? p.perm[orow] : 0;
-                    const float gh = valid ? p.ghat[slot] : 0.f;
-                    float* dst_row = acc_out + (size_t)(slot / p.k) * p.out_ld + t.wt * C::WTILE;
+                    // g_hat-scaled output row of this slot, rounded to bf16, at its
+                    // expert-grouped row (the combine sums a token's rows in rank order)
+                    __nv_bfloat16* y = static_cast<__nv_bfloat16*>(p.out);
+                    const float gh = valid ? p.ghat[p.perm[orow]] : 0.f;
+                    uint4* dst = reinterpret_cast<uint4*>(y + orow * p.out_ld + t.wt * C::WTILE);
 #pragma unroll 1
-                    for (int c0 = 0; c0 < C::WTILE; c0 += 16) {
-                        uint32_t r[16];
-                        tmem_ld16(tbase + c0, r);
+                    for (int c0 = 0; c0 < C::WTILE; c0 += 64) {
+                        uint32_t r[4][16];
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) tmem_ld16(tbase + c0 + 16 * q, r[q]);
                         tmem_ld_wait();
                         if (valid) {
 #pragma unroll
-                            for (int i = 0; i < 4; ++i)
-                                red_add_v4(dst_row + c0 + 4 * i, gh * __uint_as_float(r[4 * i]), gh * __uint_as_float(r[4 * i + 1]),
-                                           gh * __uint_as_float(r[4 * i + 2]), gh * __uint_as_float(r[4 * i + 3]));
+                            for (int q = 0; q < 4; ++q) {
+                                uint32_t w[8];
+#pragma unroll
+                                for (int i = 0; i < 8; ++i) {
+                                    const __nv_bfloat162 b2 = __floats2bfloat162_rn(gh * __uint_as_float(r[q][2 * i]),
+                                                                                    gh * __uint_as_float(r[q][2 * i + 1]));
+                                    w[i] = *reinterpret_cast<const uint32_t*>(&b2);
+                                }
+                                dst[(c0 + 16 * q) / 8] = make_uint4(w[0], w[1], w[2], w[3]);
+                                dst[(c0 + 16 * q) / 8 + 1] = make_uint4(w[4], w[5], w[6], w[7]);
+                            }
                         }
                     }
                 }
@@ -500,8 +474,39 @@ __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __rest
     }
 }
 
-// out[t, c] = sum_{i kept, rank order} y[slot_pos[t*k+i], c]  (Eq. ace_sparse_output)
-__global__ void __launch_bounds__(256) k_combine_bf16(const float* __restrict__ y, const int32_t* __restrict__ slot_pos,
+// out[t, c] = (x[t, c] +) sum_{i kept, rank order} y[slot_pos[t*k+i], c]
+// (Eq. ace_sparse_output; y rows already carry g_hat). One thread per 8
+// columns of a token, so a warp reads 256 contiguous columns of each row.
+// The token's k row indices are read first and all k row loads are issued
+// before the sum, which still runs in rank order.
+template <typename Y>
+struct Row8;
+template <>
+struct Row8<float> {
+    float4 a, b;
+    __device__ __forceinline__ void load(const float* p) {
+        a = reinterpret_cast<const float4*>(p)[0];
+        b = reinterpret_cast<const float4*>(p)[1];
+    }
+    __device__ __forceinline__ void add_to(float* acc) const {
+        acc[0] += a.x; acc[1] += a.y; acc[2] += a.z; acc[3] += a.w;
+        acc[4] += b.x; acc[5] += b.y; acc[6] += b.z; acc[7] += b.w;
+    }
+};
+template <>
+struct Row8<__nv_bfloat16> {
+    uint4 v;
+    __device__ __forceinline__ void load(const __nv_bfloat16* p) { v = *reinterpret_cast<const uint4*>(p); }
+    __device__ __forceinline__ void add_to(float* acc) const {
+        float f[8];
+        Vec16<__nv_bfloat16>::to_float(v, f);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[j] += f[j];
+    }
+};
+
+template <typename Y, int KMAX>
+__global__ void __launch_bounds__(256) k_combine_bf16(const Y* __restrict__ y, const int32_t* __restrict__ slot_pos,
                                                       const __nv_bfloat16* __restrict__ resid,
                                                       __nv_bfloat16* __restrict__ out, int n_tokens, int d, int k) {
     pdl_wait();
@@ -509,15 +514,17 @@ __global__ void __launch_bounds__(256) k_combine_bf16(const float* __restrict__ 
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= (long long)n_tokens * nq) return;
     const int t = (int)(idx / nq), c8 = (int)(idx % nq);
+    int r[KMAX];
+#pragma unroll
+    for (int i = 0; i < KMAX; ++i) r[i] = i < k ? __ldg(slot_pos + (size_t)t * k + i) : -1;
+    Row8<Y> v[KMAX];
+#pragma unroll
+    for (int i = 0; i < KMAX; ++i)
+        if (r[i] >= 0) v[i].load(y + (size_t)r[i] * d + 8 * c8);
     float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    for (int i = 0; i < k; ++i) {
-        const int r = slot_pos[(size_t)t * k + i];
-        if (r < 0) continue;
-        const float4* src = reinterpret_cast<const float4*>(y + (size_t)r * d) + 2 * c8;
-        const float4 a = src[0], b = src[1];
-        acc[0] += a.x; acc[1] += a.y; acc[2] += a.z; acc[3] += a.w;
-        acc[4] += b.x; acc[5] += b.y; acc[6] += b.z; acc[7] += b.w;
-    }
+#pragma unroll
+    for (int i = 0; i < KMAX; ++i)
+        if (r[i] >= 0) v[i].add_to(acc);
     if (resid) {
         float xr[8];
         Vec16<__nv_bfloat16>::to_float(reinterpret_cast<const uint4*>(resid + (size_t)t * d)[c8], xr);
@@ -528,28 +535,6 @@ __global__ void __launch_bounds__(256) k_combine_bf16(const float* __restrict__ 
 #pragma unroll
     for (int i = 0; i < 8; ++i) o[i] = __float2bfloat16_rn(acc[i]);
     reinterpret_cast<uint4*>(out + (size_t)t * d)[c8] = *reinterpret_cast<const uint4*>(o);
-}
-
-// out[t, :] = bf16(acc[t, :]); acc[t, :] = 0 (ready for the next forward).
-__global__ void __launch_bounds__(256) k_finalize_bf16(float* __restrict__ acc, const __nv_bfloat16* __restrict__ resid,
-                                                       __nv_bfloat16* __restrict__ out, long long n8) {
-    pdl_wait();
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n8; i += (long long)gridDim.x * blockDim.x) {
-        float4* a = reinterpret_cast<float4*>(acc) + 2 * i;
-        float4 u = a[0], v = a[1];
-        if (resid) {
-            float xr[8];
-            Vec16<__nv_bfloat16>::to_float(reinterpret_cast<const uint4*>(resid)[i], xr);
-            u = make_float4(xr[0] + u.x, xr[1] + u.y, xr[2] + u.z, xr[3] + u.w);
-            v = make_float4(xr[4] + v.x, xr[5] + v.y, xr[6] + v.z, xr[7] + v.w);
-        }
-        __align__(16) __nv_bfloat16 o[8] = {__float2bfloat16_rn(u.x), __float2bfloat16_rn(u.y), __float2bfloat16_rn(u.z),
-                                            __float2bfloat16_rn(u.w), __float2bfloat16_rn(v.x), __float2bfloat16_rn(v.y),
-                                            __float2bfloat16_rn(v.z), __float2bfloat16_rn(v.w)};
-        reinterpret_cast<uint4*>(out)[i] = *reinterpret_cast<const uint4*>(o);
-        a[0] = make_float4(0.f, 0.f, 0.f, 0.f);
-        a[1] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
 }
 
 // ---------------------------------------------------------------- host side
@@ -644,17 +629,15 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = set_attr<true, 1>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 0>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 1>()) != cudaSuccess) return e;
-    if ((e = set_attr<true, 2>()) != cudaSuccess) return e;
-    if ((e = prefer_shared(k_finalize_bf16)) != cudaSuccess) return e;
+    if ((e = set_attr<false, 2>()) != cudaSuccess) return e;
     if ((e = prefer_shared(k_gather_rows)) != cudaSuccess) return e;
-    if ((e = prefer_shared(k_combine_bf16)) != cudaSuccess) return e;
+
     // row counts as allocated at create time (padded to at least 256 rows)
     const uint64_t rows = (uint64_t)D.max_tokens * D.top_k < 256 ? 256 : (uint64_t)D.max_tokens * D.top_k;
     const uint64_t h_rows = D.max_tokens < 256 ? 256 : (uint64_t)D.max_tokens;
     const uint64_t n_pad = ((uint64_t)D.n_experts + 255) / 256 * 256;
     const uint64_t n = D.n_experts, d = D.hidden, m = D.ffn;
     // token maps: h_perm (GEMM 1) and act (GEMM 2), tiles of 16 / 128 rows
-    if ((e = make_map(&L->tcm.tok1_small, L->ws.h_perm, rows, d, 16)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.tok1_big, L->ws.h_perm, rows, d, 128)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.tok2_small, L->ws.act_bf16, rows, m, 16)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.tok2_big, L->ws.act_bf16, rows, m, 128)) != cudaSuccess) return e;
@@ -664,20 +647,24 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = make_map(&L->tcm.wd_small, L->w_down, n * d, m, 128)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.wd_big, L->w_down, n * d, m, 256)) != cudaSuccess) return e;
     // router: h [Tmax, d] in 128-row boxes, W_r [N, d] in 256-row boxes
-    if ((e = make_map(&L->tcm.h_rows, L->ws.h, h_rows, d, 16)) != cudaSuccess) return e;
-    if ((e = make_map(&L->tcm.w_router, L->router_w, n_pad, d, 128)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.h_rows_big, L->ws.h, h_rows, d, 128)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.h_row1, L->ws.h, h_rows, d, 1)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.w_router_big, L->router_w, n_pad, d, 256)) != cudaSuccess) return e;
     return cudaSuccess;
 }
 
+// Router logits on the tensor cores for batches over 256 tokens (smaller
+// ones are routed by the fused kernel): 128 tokens x 256 experts per tile,
+// so W_r (N padded to 256 rows) is re-read from L2 once per 128 tokens.
 cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s) {
     const ace_layer_desc& D = L->desc;
     TcParams p{};
-    p.tm_tok = L->tcm.h_rows;
-    p.tm_w = L->tcm.w_router;
+    p.tm_tok = L->tcm.h_rows_big;
+    p.tm_w = L->tcm.w_router_big;
     p.out = L->ws.logits;
     p.K = D.hidden;
     p.w_rows = D.n_experts;
-    p.w_tiles = (D.n_experts + 127) / 128;
+    p.w_tiles = (D.n_experts + 255) / 256;
     p.out_ld = D.n_experts;
     p.err = L->ws.err;
     p.single_rows = T;
@@ -685,7 +672,7 @@ cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s) {
     p.inv_temp = 1.0f / D.router_temp;
     p.use_temp = D.router_temp != 1.0f;
     p.n_valid_cols = D.n_experts;
-    return launch_gemm<true, 2>(L, p, s);
+    return launch_gemm<false, 2>(L, p, s);
 }
 
 cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, cudaStream_t s, cudaEvent_t* ev) {
@@ -694,12 +681,18 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     const Workspace& W = L->ws;
     const int d = D.hidden, m = D.ffn, k = D.top_k;
     const bool small = T <= kTcSmallT;
-    cudaError_t e = launch_pdl(k_gather_rows, dim3(L->num_sms * 4), dim3(256), 0, s, (const __nv_bfloat16*)W.h,
-                               (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k);
-    if (e != cudaSuccess) return e;
+    cudaError_t e = cudaSuccess;
+    // batches up to 256 tokens: GEMM 1 loads token rows straight from h; larger
+    // ones gather them into expert-grouped order first (128-row TMA tiles)
+    if (!small) {
+        e = launch_pdl(k_gather_rows, dim3(L->num_sms * 4), dim3(256), 0, s, (const __nv_bfloat16*)W.h,
+                       (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k);
+        if (e != cudaSuccess) return e;
+    }
     if (ev) ace::record_stage(ev[0], s);
     TcParams p1{};
-    p1.tm_tok = small ? L->tcm.tok1_small : L->tcm.tok1_big;
+    p1.tm_tok = small ? L->tcm.h_row1 : L->tcm.tok1_big;
+    p1.direct_rows = small ? 1 : 0;
     p1.tm_w = small ? L->tcm.wgu_small : L->tcm.wgu_big;
     p1.offsets = W.offsets;
     p1.dlist = W.dlist;
@@ -718,9 +711,12 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     if (e != cudaSuccess) return e;
     if (ev) ace::record_stage(ev[1], s);
     TcParams p2 = p1;
+    p2.direct_rows = 0;
     p2.tm_tok = small ? L->tcm.tok2_small : L->tcm.tok2_big;
     p2.tm_w = small ? L->tcm.wd_small : L->tcm.wd_big;
-    p2.out = small ? (void*)W.yslot : (void*)W.out_acc;
+    // y per slot: fp32 rows for SWAP tiles; bf16 rows otherwise, written over
+    // h_perm, which GEMM 1 (complete before GEMM 2 reads anything) no longer needs
+    p2.out = small ? (void*)W.yslot : W.h_perm;
     p2.K = m;
     p2.w_rows = d;
     p2.w_tiles = d / (small ? 128 : 256);
@@ -729,12 +725,18 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     if (e != cudaSuccess) return e;
     if (ev) ace::record_stage(ev[2], s);
     const long long nthreads = (long long)T * (d / 8);
-    if (small)
-        e = launch_pdl(k_combine_bf16, dim3((unsigned)((nthreads + 255) / 256)), dim3(256), 0, s, (const float*)W.yslot,
-                       (const int32_t*)W.slot_pos, resid, (__nv_bfloat16*)out, T, d, k);
-    else
-        e = launch_pdl(k_finalize_bf16, dim3((unsigned)(L->num_sms * 8)), dim3(256), 0, s, W.out_acc, resid,
-                       (__nv_bfloat16*)out, nthreads);
+    const dim3 grid((unsigned)((nthreads + 255) / 256));
+    const int32_t* sp = W.slot_pos;
+    __nv_bfloat16* o = static_cast<__nv_bfloat16*>(out);
+    if (small) {
+        const float* y = W.yslot;
+        e = k <= 8 ? launch_pdl(k_combine_bf16<float, 8>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k)
+                   : launch_pdl(k_combine_bf16<float, kMaxTopK>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k);
+    } else {
+        const __nv_bfloat16* y = static_cast<const __nv_bfloat16*>(W.h_perm);
+        e = k <= 8 ? launch_pdl(k_combine_bf16<__nv_bfloat16, 8>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k)
+                   : launch_pdl(k_combine_bf16<__nv_bfloat16, kMaxTopK>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k);
+    }
     if (ev) ace::record_stage(ev[3], s);
     return e;
 }

@@ -59,8 +59,8 @@ struct Workspace {
     int32_t* meta = nullptr;     // [kMetaCount]
     float* act = nullptr;        // [Tmax*k, m] fp32 (CUDA-core path)
     float* yslot = nullptr;      // [Tmax*k, d] fp32: g_hat-scaled expert outputs per retained slot
-    void* h_perm = nullptr;      // [Tmax*k, d] bf16: h rows in expert-grouped order (tensor path)
-    float* out_acc = nullptr;    // [Tmax, d] fp32: large-batch output accumulator (kept zero between calls)
+    void* h_perm = nullptr;      // [Tmax*k, d] bf16: h rows in expert-grouped order (tensor path); for
+                                 // batches over 256 tokens GEMM 2 then writes its bf16 y rows over it
     void* act_bf16 = nullptr;    // [Tmax*k, m] bf16 (tensor path)
     int32_t* tt_off = nullptr;   // [N+1] token-tile prefix over distinct experts
     int4* tt_tab = nullptr;      // [N + Tmax*k/16 + 1] token tiles: (expert, first row, rows, 0)
@@ -74,11 +74,12 @@ struct Workspace {
 
 // Tensor maps of the tensor-core expert path (built once at create time).
 struct TcMaps {
-    CUtensorMap tok1_small, tok1_big;   // h_perm, boxes of 16 / 128 rows
+    CUtensorMap tok1_big;               // h_perm, boxes of 128 rows
     CUtensorMap tok2_small, tok2_big;   // act_bf16, boxes of 16 / 128 rows
     CUtensorMap wgu_small, wgu_big;     // W_gu, boxes of 128 / 256 rows
     CUtensorMap wd_small, wd_big;       // W_down
-    CUtensorMap h_rows, w_router;       // router GEMM: h and W_r
+    CUtensorMap h_rows_big, w_router_big;   // router GEMM (batches over 256 tokens): 128-row / 256-row boxes
+    CUtensorMap h_row1;                 // h in one-row boxes: GEMM 1 token rows for batches <= 256
 };
 
 }  // namespace ace

@@ -25,22 +25,22 @@ constexpr int kSmallT = 256;
 // arithmetic), then normalised from registers; supports d <= 32 * 16 * V.
 constexpr int kNormVec = 16;
 
-template <typename T>
+template <typename T, int NV = kNormVec>
 __device__ __forceinline__ void rmsnorm_row(const T* __restrict__ xr, const T* __restrict__ gamma, T* hr, int d,
                                             float rms_eps, int lane) {
     constexpr int V = Vec16<T>::N;
     const int nvec = d / V;
     const uint4* xv = reinterpret_cast<const uint4*>(xr);
     const uint4* gv = reinterpret_cast<const uint4*>(gamma);
-    uint4 xs[kNormVec];
+    uint4 xs[NV];
 #pragma unroll
-    for (int i = 0; i < kNormVec; ++i) {
+    for (int i = 0; i < NV; ++i) {
         const int c = lane + 32 * i;
         xs[i] = c < nvec ? xv[c] : make_uint4(0, 0, 0, 0);
     }
     float ss = 0.f;
 #pragma unroll
-    for (int i = 0; i < kNormVec; ++i) {
+    for (int i = 0; i < NV; ++i) {
         float f[V];
         Vec16<T>::to_float(xs[i], f);
 #pragma unroll
@@ -49,7 +49,7 @@ __device__ __forceinline__ void rmsnorm_row(const T* __restrict__ xr, const T* _
     ss = warp_sum(ss);
     const float inv = 1.0f / sqrtf(ss / (float)d + rms_eps);
 #pragma unroll
-    for (int i = 0; i < kNormVec; ++i) {
+    for (int i = 0; i < NV; ++i) {
         const int c = lane + 32 * i;
         if (c < nvec) {
             float f[V], gm[V];
@@ -63,12 +63,15 @@ __device__ __forceinline__ void rmsnorm_row(const T* __restrict__ xr, const T* _
     }
 }
 
-template <typename T>
+// NV = 16-byte vectors per lane, sized to the row so that short rows hold
+// fewer registers and more rows (more loads in flight) fit on an SM.
+template <typename T, int NV>
 __global__ void __launch_bounds__(256) k_rmsnorm(const T* __restrict__ x, const T* __restrict__ gamma,
                                                  T* __restrict__ h, int n_tokens, int d, float rms_eps) {
+    pdl_wait();
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     if (warp >= n_tokens) return;
-    rmsnorm_row(x + (size_t)warp * d, gamma, h + (size_t)warp * d, d, rms_eps, threadIdx.x & 31);
+    rmsnorm_row<T, NV>(x + (size_t)warp * d, gamma, h + (size_t)warp * d, d, rms_eps, threadIdx.x & 31);
 }
 
 // --------------------------------------------------------------------------
@@ -176,11 +179,22 @@ struct SlotScore {
 
 // Top-k over one token's logits (one warp). Lane l owns experts l + 32 j,
 // j < NPL, held in registers. Order: larger logit first; ties to the lower
-// expert index. NaN ranks last. On return lane i < k holds (id, z) of rank i.
+// expert index. NaN ranks last (as -inf), -0 equals +0. On return lane i < k
+// holds (id, z) of rank i. Each round takes two warp reductions: the largest
+// key (the logit mapped to an order-preserving unsigned integer), then the
+// lowest expert index holding it.
+__device__ __forceinline__ uint32_t order_key(float f) {
+    const uint32_t u = __float_as_uint(__fadd_rn(f, 0.0f));     // -0 -> +0
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float key_value(uint32_t k) {
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
 template <int NPL>
 __device__ __forceinline__ void warp_topk(const float* __restrict__ zrow, int n_exp, int k, int lane,
                                           int& my_id, float& my_z, bool& saw_nan) {
-    float v[NPL];
+    uint32_t v[NPL];
     unsigned taken = 0u;   // bit j: expert lane + 32*j chosen already (or absent)
     saw_nan = false;
 #pragma unroll
@@ -189,30 +203,25 @@ __device__ __forceinline__ void warp_topk(const float* __restrict__ zrow, int n_
         if (e < n_exp) {
             float z = __ldcg(zrow + e);
             if (z != z) { saw_nan = true; z = -INFINITY; }
-            v[j] = z;
+            v[j] = order_key(z);
         } else {
-            v[j] = -INFINITY;
+            v[j] = 0u;
             taken |= 1u << j;
         }
     }
     my_id = -1;
     my_z = 0.f;
     for (int r = 0; r < k; ++r) {
-        float bv = -INFINITY;
-        int bi = 0x7fffffff;
+        uint32_t bk = 0u;
+        int bj = -1;
 #pragma unroll
-        for (int j = 0; j < NPL; ++j) {
-            const int e = lane + 32 * j;
-            if (!((taken >> j) & 1u) && (v[j] > bv || (v[j] == bv && e < bi))) { bv = v[j]; bi = e; }
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-            if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
-        }
-        if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
-        if (lane == r) { my_id = bi; my_z = bv; }
+        for (int j = 0; j < NPL; ++j)
+            if (!((taken >> j) & 1u) && (bj < 0 || v[j] > bk)) { bk = v[j]; bj = j; }
+        const uint32_t top = __reduce_max_sync(0xffffffffu, bj >= 0 ? bk : 0u);
+        const uint32_t e = __reduce_min_sync(0xffffffffu, (bj >= 0 && bk == top) ? (uint32_t)(lane + 32 * bj)
+                                                                                  : 0xffffffffu);
+        if ((int)(e & 31u) == lane) taken |= 1u << (e >> 5);
+        if (lane == r) { my_id = (int)e; my_z = key_value(top); }
     }
 }
 
@@ -292,6 +301,48 @@ __device__ __forceinline__ void decide_slot(int lane, int k, float g, float c, f
     ghat_out = (on && !skip) ? __fdiv_rn(g, zs) : 0.f;
 }
 
+// The same decision with one thread per token: the token's k gates and c
+// values sit in registers (loops fully unrolled over kMaxTopK), and every
+// step -- the skip test, the restore order, the rank-order sum and the
+// division -- is the one decide_slot takes, so the bits agree.
+__device__ __forceinline__ void decide_token(const float* g_in, const float* c_in, int k, float tau, int m_min,
+                                             float eps, uint8_t* skip_out, float* ghat_out,
+                                             uint8_t* skip_copy) {
+    float g[kMaxTopK], c[kMaxTopK];
+    unsigned sk = 0u;
+#pragma unroll
+    for (int j = 0; j < kMaxTopK; ++j) {
+        g[j] = j < k ? g_in[j] : 0.f;
+        c[j] = j < k ? c_in[j] : 0.f;
+        if (j < k && j != 0 && c[j] < tau) sk |= 1u << j;   // Eq. ace_candidate_intersection via max
+    }
+    int need = m_min - (k - __popc(sk));
+    while (need > 0 && sk) {
+        // restore the skipped slot of largest c, lower rank first on ties
+        float best = -1.f;
+        int bi = -1;
+#pragma unroll
+        for (int j = 0; j < kMaxTopK; ++j)
+            if (((sk >> j) & 1u) && (bi < 0 || c[j] > best)) { best = c[j]; bi = j; }
+        sk &= ~(1u << bi);
+        --need;
+    }
+    float zs = 0.f;
+#pragma unroll
+    for (int j = 0; j < kMaxTopK; ++j)
+        if (j < k && !((sk >> j) & 1u)) zs = __fadd_rn(zs, g[j]);
+    zs = __fadd_rn(zs, eps);
+#pragma unroll
+    for (int j = 0; j < kMaxTopK; ++j) {
+        if (j < k) {
+            const bool s = (sk >> j) & 1u;
+            skip_out[j] = s ? 1 : 0;
+            if (skip_copy) skip_copy[j] = s ? 1 : 0;
+            ghat_out[j] = s ? 0.f : __fdiv_rn(g[j], zs);
+        }
+    }
+}
+
 // --------------------------------------------------------------------------
 // App. B.1 threshold for m candidates to skip: the (m+1)-th smallest
 // candidate key v (radix select over the non-negative float bits, 8 bits per
@@ -299,10 +350,13 @@ __device__ __forceinline__ void decide_slot(int lane, int k, float g, float c, f
 // least as close to m as hi, else the next float above v. Whole block;
 // requires 0 < m < #candidates. Keys 0xffffffff are protected slots.
 // --------------------------------------------------------------------------
+// One shared 256-bin histogram per pass, filled with one atomic per distinct
+// bin of a warp (the keys cluster: c lies in [0, 1]); a block-wide scan
+// (thread b owns bin b; blockDim.x == 256) finds the digit.
 template <int NW>
 struct SelectSmem {
-    int hist[NW][256];     // one histogram per warp
-    int tot[256];
+    int hist[256];
+    int wtot[NW];
     uint32_t prefix;
     int want, below, last_cnt;
     float tau;
@@ -310,66 +364,56 @@ struct SelectSmem {
 
 template <int NW>
 __device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem<NW>& S) {
-    const int tid = threadIdx.x, warp = tid >> 5;
-    constexpr int nwarps = NW;
+    static_assert(NW * 32 == 256, "one thread per bin");
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     uint32_t prefix = 0u, mask = 0u;
-    if (tid == 0) { S.want = m; S.below = 0; }
+    int want = m, below = 0, last_cnt = 0;
     for (int pass = 0; pass < 4; ++pass) {
         const int shift = 24 - 8 * pass;
-        for (int i = tid; i < nwarps * 256; i += blockDim.x) (&S.hist[0][0])[i] = 0;
+        S.hist[tid] = 0;
         __syncthreads();
-        for (int i = tid; i < n; i += blockDim.x) {
-            const uint32_t key = keys[i];
-            if (key != 0xffffffffu && (key & mask) == prefix) atomicAdd(&S.hist[warp][(key >> shift) & 255], 1);
+        for (int i0 = 0; i0 < n; i0 += 256) {
+            const int i = i0 + tid;
+            const uint32_t key = i < n ? keys[i] : 0xffffffffu;
+            if (key != 0xffffffffu && (key & mask) == prefix) {
+                const int bin = (int)((key >> shift) & 255u);
+                const unsigned peers = __match_any_sync(__activemask(), bin);
+                if (lane == __ffs(peers) - 1) atomicAdd(&S.hist[bin], __popc(peers));
+            }
         }
         __syncthreads();
-        for (int b = tid; b < 256; b += blockDim.x) {
-            int t = 0;
-            for (int w = 0; w < nwarps; ++w) t += S.hist[w][b];
-            S.tot[b] = t;
+        const int v = S.hist[tid];
+        int inc = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, inc, o);
+            if (lane >= o) inc += y;
         }
+        if (lane == 31) S.wtot[warp] = inc;
         __syncthreads();
-        if (tid < 32) {
-            // warp 0: lane l owns bins 8l..8l+7; find the bin where the running
-            // count first exceeds `want`
-            const int want = S.want;
-            int h8[8], loc = 0;
+        int base = 0;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) { h8[j] = S.tot[tid * 8 + j]; loc += h8[j]; }
-            int inc = loc;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int y = __shfl_up_sync(0xffffffffu, inc, o);
-                if (tid >= o) inc += y;
-            }
-            const int exc = inc - loc;
-            const bool mine = exc <= want && want < inc;
-            const unsigned who = __ballot_sync(0xffffffffu, mine);
-            const int owner = who ? __ffs(who) - 1 : 31;
-            if (tid == owner) {
-                int cum = exc, dg = tid * 8;
-                for (int j = 0; j < 7; ++j, ++dg) {
-                    if (cum + h8[j] > want) break;
-                    cum += h8[j];
-                }
-                S.want = want - cum;
-                S.below += cum;
-                S.last_cnt = S.tot[dg];
-                S.prefix = prefix | ((uint32_t)dg << shift);
-            }
+        for (int w = 0; w < NW; ++w) base += w < warp ? S.wtot[w] : 0;
+        const int exc = base + inc - v;
+        // the owner of `want`; the last bin if want lies past every count
+        if ((exc <= want && want < exc + v) || (tid == 255 && want >= exc + v)) {
+            S.prefix = prefix | ((uint32_t)tid << shift);
+            S.want = want - exc;
+            S.below = below + exc;
+            S.last_cnt = v;
         }
         __syncthreads();
         prefix = S.prefix;
+        want = S.want;
+        below = S.below;
+        last_cnt = S.last_cnt;
         mask |= 255u << shift;
+        __syncthreads();                     // S is rewritten by the next pass
     }
-    if (tid == 0) {
-        const int lo = S.below, hi = S.below + S.last_cnt;
-        float tau = __uint_as_float(prefix);
-        if (!(lo == m || (m - lo) <= (hi - m))) tau = __uint_as_float(prefix + 1u);
-        S.tau = tau;
-    }
-    __syncthreads();
-    return S.tau;
+    const int lo = below, hi = below + last_cnt;
+    float tau = __uint_as_float(prefix);
+    if (!(lo == m || (m - lo) <= (hi - m))) tau = __uint_as_float(prefix + 1u);
+    return tau;
 }
 
 // Exclusive scan of cnt[0..n_exp) by warp 0 of the block: offsets[e],
@@ -451,6 +495,7 @@ __global__ void __launch_bounds__(256) k_topk_score(const float* __restrict__ lo
                                                     float* __restrict__ cval, uint32_t* __restrict__ keys,
                                                     uint8_t* __restrict__ skip, float* __restrict__ ghat,
                                                     float* __restrict__ tau_out, int* __restrict__ err) {
+    pdl_wait();
     if (mode == ACE_SKIP_THRESHOLD && blockIdx.x == 0 && threadIdx.x == 0) *tau_out = tau;
     const int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
@@ -482,24 +527,17 @@ __global__ void __launch_bounds__(256) k_topk_score(const float* __restrict__ lo
     }
 }
 
-// Pass 2 (ratio mode): decide from stored g, c and the device tau.
+// Pass 2 (ratio mode): decide from stored g, c and the device tau, one
+// thread per token.
 __global__ void __launch_bounds__(256) k_decide(int n_tokens, int k, const float* __restrict__ gates,
                                                 const float* __restrict__ cval,
                                                 const float* __restrict__ tau_dev, int m_min, float eps,
                                                 uint8_t* __restrict__ skip, float* __restrict__ ghat) {
-    const int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
+    pdl_wait();
+    const int t = blockIdx.x * blockDim.x + threadIdx.x;
     if (t >= n_tokens) return;
     const size_t base = (size_t)t * k;
-    const float g = lane < k ? gates[base + lane] : 0.f;
-    const float c = lane < k ? cval[base + lane] : 0.f;
-    bool sk;
-    float gh;
-    decide_slot(lane, k, g, c, *tau_dev, m_min, eps, sk, gh);
-    if (lane < k) {
-        skip[base + lane] = sk ? 1 : 0;
-        ghat[base + lane] = gh;
-    }
+    decide_token(gates + base, cval + base, k, __ldcg(tau_dev), m_min, eps, skip + base, ghat + base, nullptr);
 }
 
 // Multi-block App. B.1 threshold for large T: three passes over the
@@ -517,6 +555,7 @@ __global__ void __launch_bounds__(1024) k_select_pass(const uint32_t* __restrict
                                                       int32_t* __restrict__ ghist, int32_t* __restrict__ state,
                                                       float* __restrict__ tau_out) {
     __shared__ int hist[kMsBins];
+    __shared__ int wtot[32];
     __shared__ bool is_last;
     pdl_wait();
     const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
@@ -524,60 +563,74 @@ __global__ void __launch_bounds__(1024) k_select_pass(const uint32_t* __restrict
     const uint32_t dmask = (1u << bits) - 1u;
     const uint32_t pmask = pass == 0 ? 0u : (pass == 1 ? 0xFFE00000u : 0xFFFFFC00u);
     const uint32_t prefix = pass == 0 ? 0u : (uint32_t)__ldcg(state + 0);
-    for (int i = threadIdx.x; i < kMsBins; i += blockDim.x) hist[i] = 0;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int i = tid; i < kMsBins; i += blockDim.x) hist[i] = 0;
     __syncthreads();
     const int lo = blockIdx.x * kMsKeysPerBlock, hi = min(n, lo + kMsKeysPerBlock);
-    for (int i = lo + threadIdx.x; i < hi; i += blockDim.x) {
-        const uint32_t key = keys[i];
-        if (key != 0xffffffffu && (key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & dmask], 1);
+    for (int i0 = lo; i0 < hi; i0 += blockDim.x) {
+        const int i = i0 + tid;
+        const uint32_t key = i < hi ? keys[i] : 0xffffffffu;
+        if (key != 0xffffffffu && (key & pmask) == prefix) {
+            // keys cluster in few bins (c lies in [0, 1]): one atomic per distinct bin of the warp
+            const int bin = (int)((key >> shift) & dmask);
+            const unsigned peers = __match_any_sync(__activemask(), bin);
+            if (lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+        }
     }
     __syncthreads();
-    for (int i = threadIdx.x; i < kMsBins; i += blockDim.x)
+    for (int i = tid; i < kMsBins; i += blockDim.x)
         if (hist[i]) atomicAdd(&ghist[i], hist[i]);
     __threadfence();
     __syncthreads();
-    if (threadIdx.x == 0) is_last = atomicAdd(&state[3], 1) == (int)gridDim.x - 1;
+    if (tid == 0) is_last = atomicAdd(&state[3], 1) == (int)gridDim.x - 1;
     __syncthreads();
     if (!is_last) return;
     __threadfence();
-    for (int i = threadIdx.x; i < kMsBins; i += blockDim.x) {
-        hist[i] = __ldcg(ghist + i);
-        ghist[i] = 0;
+    // last block: thread i owns bins 2i, 2i+1 (blockDim.x == kMsBins / 2)
+    const int b0 = __ldcg(ghist + 2 * tid), b1 = __ldcg(ghist + 2 * tid + 1);
+    ghist[2 * tid] = 0;
+    ghist[2 * tid + 1] = 0;
+    const int want = pass == 0 ? m : __ldcg(state + 1);
+    const int below0 = pass == 0 ? 0 : __ldcg(state + 2);
+    const int loc = b0 + b1;
+    int inc = loc;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+    }
+    if (lane == 31) wtot[warp] = inc;
+    __syncthreads();
+    if (warp == 0) {
+        const int v = wtot[lane];
+        int wi = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += y;
+        }
+        wtot[lane] = wi - v;            // exclusive prefix of the warp totals
     }
     __syncthreads();
-    if (threadIdx.x < 32) {
-        const int lane = threadIdx.x;
-        const int want = pass == 0 ? m : __ldcg(state + 1);
-        const int below0 = pass == 0 ? 0 : __ldcg(state + 2);
-        int loc = 0;
-        for (int j = 0; j < kMsBins / 32; ++j) loc += hist[lane * (kMsBins / 32) + j];
-        int inc = loc;
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, inc, o);
-            if (lane >= o) inc += y;
-        }
-        const int exc = inc - loc;
-        const unsigned who = __ballot_sync(0xffffffffu, exc <= want && want < inc);
-        const int owner = who ? __ffs(who) - 1 : 31;
-        if (lane == owner) {
-            int cum = exc, dg = lane * (kMsBins / 32);
-            for (int j = 0; j < kMsBins / 32 - 1; ++j, ++dg) {
-                if (cum + hist[dg] > want) break;
-                cum += hist[dg];
-            }
-            const uint32_t pre = prefix | ((uint32_t)dg << shift);
-            const int below = below0 + cum;
-            state[0] = (int32_t)pre;
-            state[1] = want - cum;
-            state[2] = below;
-            state[4] = hist[dg];
-            state[3] = 0;
-            if (pass == 2) {
-                const int lo_c = below, hi_c = below + hist[dg];
-                float tau = __uint_as_float(pre);
-                if (!(lo_c == m || (m - lo_c) <= (hi_c - m))) tau = __uint_as_float(pre + 1u);
-                *tau_out = tau;
-            }
+    const int exc = inc - loc + wtot[warp];
+    const int total = __shfl_sync(0xffffffffu, inc, 31) + wtot[warp];   // valid in the last warp
+    // the owner of `want`; the last thread if want lies past every count
+    const bool mine = (exc <= want && want < exc + loc) || (tid == (int)blockDim.x - 1 && want >= total);
+    if (mine) {
+        int cum = exc, dg = 2 * tid, cnt = b0;
+        if (cum + b0 <= want) { cum += b0; dg += 1; cnt = b1; }
+        const uint32_t pre = prefix | ((uint32_t)dg << shift);
+        const int below = below0 + cum;
+        state[0] = (int32_t)pre;
+        state[1] = want - cum;
+        state[2] = below;
+        state[4] = cnt;
+        state[3] = 0;
+        if (pass == 2) {
+            const int lo_c = below, hi_c = below + cnt;
+            float tau = __uint_as_float(pre);
+            if (!(lo_c == m || (m - lo_c) <= (hi_c - m))) tau = __uint_as_float(pre + 1u);
+            *tau_out = tau;
         }
     }
 }
@@ -600,6 +653,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, i
     __shared__ bool is_last;
     for (int e = threadIdx.x; e < n_exp; e += blockDim.x) cnt[e] = 0;
     __syncthreads();
+    pdl_wait();
     const int t = blockIdx.x * kChunk + threadIdx.x;
     if (t < n_tokens) {
         for (int i = 0; i < k; ++i)
@@ -615,13 +669,22 @@ __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, i
     if (!is_last) return;
     __threadfence();
     // last block: per-expert running bases over chunks, totals in cnt[]
+    // (16 chunk counts in flight per thread, not one L2 round trip per chunk)
+    constexpr int kBatch = 16;
     for (int e = threadIdx.x; e < n_exp; e += blockDim.x) {
         int run = 0;
-        for (int c = 0; c < n_chunks; ++c) {
-            volatile int32_t* p = chunk_counts + (size_t)c * n_exp + e;
-            const int v = *p;
-            *p = run;
-            run += v;
+        for (int c0 = 0; c0 < n_chunks; c0 += kBatch) {
+            int v[kBatch];
+#pragma unroll
+            for (int j = 0; j < kBatch; ++j)
+                v[j] = c0 + j < n_chunks ? __ldcg(chunk_counts + (size_t)(c0 + j) * n_exp + e) : 0;
+#pragma unroll
+            for (int j = 0; j < kBatch; ++j) {
+                if (c0 + j < n_chunks) {
+                    chunk_counts[(size_t)(c0 + j) * n_exp + e] = run;
+                    run += v[j];
+                }
+            }
         }
         cnt[e] = run;
     }
@@ -645,6 +708,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
     __shared__ uint32_t bm[kMaxExperts * W];
     for (int i = threadIdx.x; i < n_exp * W; i += blockDim.x) bm[i] = 0u;
     __syncthreads();
+    pdl_wait();
     const int t = blockIdx.x * kChunk + threadIdx.x;
     const int w = threadIdx.x >> 5;
     const unsigned bit = 1u << (threadIdx.x & 31);
@@ -721,54 +785,9 @@ struct FusedArgs {
     int32_t* tile_cnt;
 };
 
-// RMSNorm of one row into fp32 shared memory; optionally also the row in T.
-template <typename T>
-__device__ __forceinline__ void rmsnorm_row_f32(const T* __restrict__ xr, const T* __restrict__ gamma, float* hs,
-                                                T* __restrict__ h_out, int d, float rms_eps, int lane) {
-    constexpr int V = Vec16<T>::N;
-    const int nvec = d / V;
-    const uint4* xv = reinterpret_cast<const uint4*>(xr);
-    const uint4* gv = reinterpret_cast<const uint4*>(gamma);
-    uint4 xs[kNormVec];
-#pragma unroll
-    for (int i = 0; i < kNormVec; ++i) {
-        const int c = lane + 32 * i;
-        xs[i] = c < nvec ? xv[c] : make_uint4(0, 0, 0, 0);
-    }
-    float ss = 0.f;
-#pragma unroll
-    for (int i = 0; i < kNormVec; ++i) {
-        float f[V];
-        Vec16<T>::to_float(xs[i], f);
-#pragma unroll
-        for (int j = 0; j < V; ++j) ss = fmaf(f[j], f[j], ss);
-    }
-    ss = warp_sum(ss);
-    const float inv = 1.0f / sqrtf(ss / (float)d + rms_eps);
-#pragma unroll
-    for (int i = 0; i < kNormVec; ++i) {
-        const int c = lane + 32 * i;
-        if (c < nvec) {
-            float f[V], gm[V];
-            Vec16<T>::to_float(xs[i], f);
-            Vec16<T>::to_float(gv[c], gm);
-            T o[V];
-#pragma unroll
-            for (int j = 0; j < V; ++j) {
-                o[j] = from_f32<T>(f[j] * inv * gm[j]);
-                f[j] = to_f32(o[j]);                       // the stored (rounded) value feeds the router
-            }
-#pragma unroll
-            for (int j = 0; j < V; j += 4)
-                *reinterpret_cast<float4*>(hs + c * V + j) = make_float4(f[j], f[j + 1], f[j + 2], f[j + 3]);
-            if (h_out) reinterpret_cast<uint4*>(h_out)[c] = *reinterpret_cast<const uint4*>(o);
-        }
-    }
-}
-
 __host__ __device__ inline size_t fused_phase_c_bytes(int T, int k, int n_exp) {
     const size_t ns = (size_t)T * k;
-    return ns * 16 + (size_t)n_exp * 4 + (size_t)(n_exp + 1) * 4 + (size_t)n_exp * 32 + ns + 16;
+    return 16 + ns * 16 + (size_t)n_exp * 4 + (size_t)(n_exp + 1) * 4 + (size_t)n_exp * 32 + ns + 16;
 }
 
 template <typename T, int NPL, bool LOGITS>
@@ -781,55 +800,82 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
     const int nt = min(kFuseTok, a.n_tokens - t0);
     const int n_exp = a.n_exp, k = a.k;
     if (LOGITS) {
-        // ---------------- phase A: RMSNorm + logits for 8 tokens x 8 experts
-        float* hs = reinterpret_cast<float*>(smem_raw);          // [kFuseTok][d]
+        // ---------------- phase A: RMSNorm + logits for 8 tokens x 8 experts.
+        // One thread bulk-copies gamma and the block's 8 router rows (layer
+        // constants, before the dependency wait) and the tile's x rows into
+        // shared memory, so the block waits for one round trip; the rows
+        // are then normalised in place and the dot products read shared memory.
         const int d = a.d;
         constexpr int V = Vec16<T>::N;
         const int nvec = d / V;
-        {
-            const int r = warp;                                   // one token row per warp
-            if (r < nt) {
-                const size_t off = (size_t)(t0 + r) * d;
-                rmsnorm_row_f32<T>(static_cast<const T*>(a.x) + off, static_cast<const T*>(a.gamma), hs + (size_t)r * d,
-                                   blockIdx.y == 0 ? static_cast<T*>(a.h_out) + off : nullptr, d, a.rms_eps, lane);
-            } else {
-                for (int c = lane; c < d / 4; c += 32)
-                    reinterpret_cast<float4*>(hs + (size_t)r * d)[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+        uint64_t* bar = reinterpret_cast<uint64_t*>(smem_raw);
+        T* xs = reinterpret_cast<T*>(smem_raw + 16);             // [kFuseTok][d] -> h in place
+        T* gs = xs + (size_t)kFuseTok * d;                        // [d]
+        T* wsm = gs + d;                                          // [kFuseWarps][d]
+        const int e0 = blockIdx.y * kFuseWarps;
+        const int ne = min(kFuseWarps, n_exp - e0);
+        const uint32_t row_bytes = (uint32_t)(d * sizeof(T));
+        if (threadIdx.x == 0) {
+            mbar_init(bar, 1);
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            mbar_expect_tx(bar, (uint32_t)(nt + 1 + ne) * row_bytes);
+            bulk_g2s(gs, a.gamma, row_bytes, bar);
+            bulk_g2s(wsm, static_cast<const T*>(a.w_r) + (size_t)e0 * d, (uint32_t)ne * row_bytes, bar);
+        }
+        pdl_wait();                                               // x is the predecessor's output
+        if (threadIdx.x == 0) bulk_g2s(xs, static_cast<const T*>(a.x) + (size_t)t0 * d, (uint32_t)nt * row_bytes, bar);
+        if (!mbar_wait(bar, 0, a.err)) return;
+        const uint4* gv = reinterpret_cast<const uint4*>(gs);
+        if (warp < nt) {
+            // h = x / sqrt(mean(x^2) + eps) * gamma, rounded to T (the stored h feeds the router)
+            uint4* xr = reinterpret_cast<uint4*>(xs) + (size_t)warp * nvec;
+            float ss = 0.f;
+#pragma unroll 1
+            for (int c = lane; c < nvec; c += 32) {
+                float f[V];
+                Vec16<T>::to_float(xr[c], f);
+#pragma unroll
+                for (int j = 0; j < V; ++j) ss = fmaf(f[j], f[j], ss);
+            }
+            ss = warp_sum(ss);
+            const float inv = 1.0f / sqrtf(ss / (float)d + a.rms_eps);
+            uint4* hg = blockIdx.y == 0 ? reinterpret_cast<uint4*>(static_cast<T*>(a.h_out) + (size_t)(t0 + warp) * d)
+                                        : nullptr;
+#pragma unroll 1
+            for (int c = lane; c < nvec; c += 32) {
+                float f[V], gm[V];
+                Vec16<T>::to_float(xr[c], f);
+                Vec16<T>::to_float(gv[c], gm);
+                T o[V];
+#pragma unroll
+                for (int j = 0; j < V; ++j) o[j] = from_f32<T>(f[j] * inv * gm[j]);
+                const uint4 ov = *reinterpret_cast<const uint4*>(o);
+                xr[c] = ov;
+                if (hg) hg[c] = ov;
             }
         }
         __syncthreads();
-        const int e = blockIdx.y * kFuseWarps + warp;
-        if (e < n_exp) {
-            const uint4* we = reinterpret_cast<const uint4*>(static_cast<const T*>(a.w_r) + (size_t)e * d);
+        if (threadIdx.x == 0) mbar_inval(bar);
+        if (warp < ne) {
+            const int e = e0 + warp;
+            const uint4* wr = reinterpret_cast<const uint4*>(wsm) + (size_t)warp * nvec;
+            const uint4* hx = reinterpret_cast<const uint4*>(xs);
             float acc[kFuseTok];
 #pragma unroll
             for (int r = 0; r < kFuseTok; ++r) acc[r] = 0.f;
-            constexpr int CH = 8;
-            for (int c0 = 0; c0 < nvec; c0 += 32 * CH) {
-                uint4 wv[CH];
+#pragma unroll 1
+            for (int c = lane; c < nvec; c += 32) {
+                float wf[V];
+                Vec16<T>::to_float(wr[c], wf);
 #pragma unroll
-                for (int i = 0; i < CH; ++i) {
-                    const int c = c0 + lane + 32 * i;
-                    wv[i] = c < nvec ? we[c] : make_uint4(0, 0, 0, 0);
-                }
+                for (int r = 0; r < kFuseTok; ++r) {
+                    float hf[V];
+                    Vec16<T>::to_float(hx[(size_t)r * nvec + c], hf);
 #pragma unroll
-                for (int i = 0; i < CH; ++i) {
-                    const int c = c0 + lane + 32 * i;
-                    if (c >= nvec) break;
-                    float wf[V];
-                    Vec16<T>::to_float(wv[i], wf);
-#pragma unroll
-                    for (int r = 0; r < kFuseTok; ++r) {
-                        const float4* hp = reinterpret_cast<const float4*>(hs + (size_t)r * d + c * V);
-#pragma unroll
-                        for (int j = 0; j < V / 4; ++j) {
-                            const float4 hv = hp[j];
-                            acc[r] = fmaf(hv.x, wf[4 * j], acc[r]);
-                            acc[r] = fmaf(hv.y, wf[4 * j + 1], acc[r]);
-                            acc[r] = fmaf(hv.z, wf[4 * j + 2], acc[r]);
-                            acc[r] = fmaf(hv.w, wf[4 * j + 3], acc[r]);
-                        }
-                    }
+                    for (int j = 0; j < V; ++j) acc[r] = fmaf(hf[j], wf[j], acc[r]);
                 }
             }
 #pragma unroll
@@ -852,6 +898,8 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         __syncthreads();
         if (!s_last) return;
         __threadfence();
+    } else {
+        pdl_wait();                                               // logits are the predecessor's output
     }
     // ---------------- phase B: top-k, gates, c for this token tile
     const bool ratio = a.mode == ACE_SKIP_RATIO;
@@ -895,7 +943,7 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
     // ---------------- phase C: threshold, decision, compaction (all tokens)
     const int n_tokens = a.n_tokens;
     const int ns = n_tokens * k;
-    float* g_s = reinterpret_cast<float*>(smem_raw);
+    float* g_s = reinterpret_cast<float*>(smem_raw + 16);
     float* c_s = g_s + ns;
     uint32_t* key_s = reinterpret_cast<uint32_t*>(c_s + ns);
     int* id_s = reinterpret_cast<int*>(key_s + ns);
@@ -919,18 +967,10 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
     if (ratio) {
         const float tau = block_select_tau(key_s, ns, a.m_q, S);
         if (threadIdx.x == 0) *a.tau_out = tau;
-        for (int t = warp; t < n_tokens; t += kFuseWarps) {
+        for (int t = threadIdx.x; t < n_tokens; t += blockDim.x) {
             const int base = t * k;
-            const float g = lane < k ? g_s[base + lane] : 0.f;
-            const float c = lane < k ? c_s[base + lane] : 0.f;
-            bool sk;
-            float gh;
-            decide_slot(lane, k, g, c, tau, a.m_min, a.eps, sk, gh);
-            if (lane < k) {
-                a.skip[base + lane] = sk ? 1 : 0;
-                skip_s[base + lane] = sk ? 1 : 0;
-                a.ghat[base + lane] = gh;
-            }
+            decide_token(g_s + base, c_s + base, k, tau, a.m_min, a.eps, a.skip + base, a.ghat + base,
+                         skip_s + base);
         }
         __syncthreads();
     } else if (threadIdx.x == 0) {
@@ -958,7 +998,7 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
 }
 
 size_t fused_smem_bytes(const ace_layer* L, int T) {
-    const size_t a = (size_t)kFuseTok * L->desc.hidden * sizeof(float);
+    const size_t a = 16 + (size_t)(kFuseTok + 1 + kFuseWarps) * L->desc.hidden * L->elem;
     const size_t c = fused_phase_c_bytes(T, L->desc.top_k, L->desc.n_experts);
     return a > c ? a : c;
 }
@@ -1015,8 +1055,7 @@ namespace {
 template <typename T, int NPL, bool LOGITS>
 cudaError_t fused_launch(const ace_layer* L, const FusedArgs& a, int n_tok, cudaStream_t s) {
     const dim3 grid(cdiv(n_tok, kFuseTok), LOGITS ? cdiv(L->desc.n_experts, kFuseWarps) : 1);
-    k_route_fused<T, NPL, LOGITS><<<grid, kFuseWarps * 32, fused_smem_bytes(L, kSmallT), s>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(k_route_fused<T, NPL, LOGITS>, grid, dim3(kFuseWarps * 32), fused_smem_bytes(L, kSmallT), s, a);
 }
 
 template <typename T, bool LOGITS>
@@ -1094,17 +1133,22 @@ cudaError_t launch_route_fused(const ace_layer* L, const void* x, const float* l
     return bf ? fused_dispatch<__nv_bfloat16, false>(L, a, T, s) : fused_dispatch<float, false>(L, a, T, s);
 }
 
-cudaError_t launch_rmsnorm(const ace_layer* L, const void* x, int T, cudaStream_t s) {
+template <typename E>
+cudaError_t launch_rmsnorm_t(const ace_layer* L, const void* x, int T, cudaStream_t s) {
     const int d = L->desc.hidden;
     const int blocks = cdiv(T, 8);
-    if (L->desc.dtype == ACE_BF16)
-        k_rmsnorm<__nv_bfloat16><<<blocks, 256, 0, s>>>(
-            (const __nv_bfloat16*)x, (const __nv_bfloat16*)L->gamma, (__nv_bfloat16*)L->ws.h, T, d,
-            L->desc.rms_eps);
-    else
-        k_rmsnorm<float><<<blocks, 256, 0, s>>>((const float*)x, (const float*)L->gamma,
-                                                (float*)L->ws.h, T, d, L->desc.rms_eps);
-    return cudaGetLastError();
+    const int nv = cdiv(d / Vec16<E>::N, 32);      // vectors per lane (<= kNormVec, checked at create)
+    const E* xt = static_cast<const E*>(x);
+    const E* g = static_cast<const E*>(L->gamma);
+    E* h = static_cast<E*>(L->ws.h);
+    const float eps = L->desc.rms_eps;
+    if (nv <= 4) return launch_pdl(k_rmsnorm<E, 4>, dim3(blocks), dim3(256), 0, s, xt, g, h, T, d, eps);
+    if (nv <= 8) return launch_pdl(k_rmsnorm<E, 8>, dim3(blocks), dim3(256), 0, s, xt, g, h, T, d, eps);
+    return launch_pdl(k_rmsnorm<E, kNormVec>, dim3(blocks), dim3(256), 0, s, xt, g, h, T, d, eps);
+}
+
+cudaError_t launch_rmsnorm(const ace_layer* L, const void* x, int T, cudaStream_t s) {
+    return L->desc.dtype == ACE_BF16 ? launch_rmsnorm_t<__nv_bfloat16>(L, x, T, s) : launch_rmsnorm_t<float>(L, x, T, s);
 }
 
 cudaError_t launch_router(const ace_layer* L, const void* x, int T, bool fuse_norm, cudaStream_t s) {
@@ -1127,29 +1171,35 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     const int tok_tile = L->tc ? tc_token_tile(T) : 0;
     if (T <= kSmallT) return launch_route_fused(L, nullptr, logits, T, ctl, s);
     const int blocks = cdiv(T, 8);
-#define ACE_TOPK(NPL)                                                                                          \
-    k_topk_score<NPL><<<blocks, 256, 0, s>>>(logits, T, n, k, L->a_gsp, L->a_rcr, D.eps, D.min_active, mode,   \
-                                             tau, W.ids, W.gates, W.cval, W.keys, W.skip, W.ghat, W.tau, W.err)
-    if (n <= 128) ACE_TOPK(4);
-    else if (n <= 256) ACE_TOPK(8);
-    else ACE_TOPK(32);
+    cudaError_t e;
+#define ACE_TOPK(NPL)                                                                                             \
+    launch_pdl(k_topk_score<NPL>, dim3(blocks), dim3(256), 0, s, logits, T, n, k, (const float*)L->a_gsp,         \
+               (const float*)L->a_rcr, D.eps, D.min_active, mode, tau, W.ids, W.gates, W.cval, W.keys, W.skip,    \
+               W.ghat, W.tau, W.err)
+    if (n <= 128) e = ACE_TOPK(4);
+    else if (n <= 256) e = ACE_TOPK(8);
+    else e = ACE_TOPK(32);
 #undef ACE_TOPK
+    if (e != cudaSuccess) return e;
     if (mode == ACE_SKIP_RATIO) {
         const int nk = T * k;
         const int sb = cdiv(nk, kMsKeysPerBlock);
         for (int pass = 0; pass < 3; ++pass) {
-            cudaError_t e = launch_pdl(k_select_pass, dim3(sb), dim3(1024), 0, s, (const uint32_t*)W.keys, nk, m_q,
-                                       pass, W.sel_hist, W.sel_state, W.tau);
+            e = launch_pdl(k_select_pass, dim3(sb), dim3(kMsBins / 2), 0, s, (const uint32_t*)W.keys, nk, m_q, pass,
+                           W.sel_hist, W.sel_state, W.tau);
             if (e != cudaSuccess) return e;
         }
-        k_decide<<<blocks, 256, 0, s>>>(T, k, W.gates, W.cval, W.tau, D.min_active, D.eps, W.skip, W.ghat);
+        e = launch_pdl(k_decide, dim3(cdiv(T, 256)), dim3(256), 0, s, T, k, (const float*)W.gates, (const float*)W.cval,
+                       (const float*)W.tau, D.min_active, D.eps, W.skip, W.ghat);
+        if (e != cudaSuccess) return e;
     }
     const int n_chunks = cdiv(T, kChunk);
-    k_compact_count<<<n_chunks, kChunk, 0, s>>>(T, k, n, n_chunks, W.ids, W.skip, W.chunk_counts,
-                                                W.offsets, W.dlist, W.meta, tok_tile, W.tt_off, W.tt_tab);
-    k_compact_place<<<n_chunks, kChunk, 0, s>>>(T, k, n, W.ids, W.skip, W.chunk_counts, W.offsets,
-                                                W.perm, W.slot_pos);
-    return cudaGetLastError();
+    e = launch_pdl(k_compact_count, dim3(n_chunks), dim3(kChunk), 0, s, T, k, n, n_chunks, (const int32_t*)W.ids,
+                   (const uint8_t*)W.skip, W.chunk_counts, W.offsets, W.dlist, W.meta, tok_tile, W.tt_off, W.tt_tab);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(k_compact_place, dim3(n_chunks), dim3(kChunk), 0, s, T, k, n, (const int32_t*)W.ids,
+                      (const uint8_t*)W.skip, (const int32_t*)W.chunk_counts, (const int32_t*)W.offsets, W.perm,
+                      W.slot_pos);
 }
 
 int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl) {
@@ -1171,7 +1221,7 @@ cudaError_t route_init(const ace_layer* L) {
     const void* ks[] = {(const void*)k_route_fused<__nv_bfloat16, 4, true>, (const void*)k_route_fused<__nv_bfloat16, 8, true>,
                         (const void*)k_route_fused<__nv_bfloat16, 32, true>, (const void*)k_route_fused<float, 4, true>,
                         (const void*)k_route_fused<float, 8, true>, (const void*)k_route_fused<float, 32, true>,
-                        (const void*)k_rmsnorm<__nv_bfloat16>, (const void*)k_topk_score<4>, (const void*)k_topk_score<8>,
+                        (const void*)k_topk_score<4>, (const void*)k_topk_score<8>,
                         (const void*)k_topk_score<32>, (const void*)k_decide,
                         (const void*)k_compact_count, (const void*)k_compact_place, (const void*)k_select_pass};
     for (const void* kf : ks)
