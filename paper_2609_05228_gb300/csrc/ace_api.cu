@@ -42,7 +42,7 @@ void free_layer(ace_layer* L) {
     void* ptrs[] = {L->router_w, L->router_b, L->w_gate, L->w_up, L->w_gu, L->w_down, L->gamma, L->a_gsp,
                     L->a_rcr, L->ws.h, L->ws.logits, L->ws.ids, L->ws.gates, L->ws.cval, L->ws.keys, L->ws.skip,
                     L->ws.ghat, L->ws.tau, L->ws.chunk_counts, L->ws.offsets, L->ws.dlist, L->ws.perm,
-                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.act_bf16, L->ws.tt_off, L->ws.tt_tab, L->ws.tile_cnt, L->ws.sel_hist, L->ws.sel_state, L->ws.err, L->ws.x_stage, L->ws.out_stage};
+                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.act_bf16, L->ws.tt_off, L->ws.tt_tab, L->ws.tile_cnt, L->ws.sel_hist, L->ws.sel_cand, L->ws.err, L->ws.x_stage, L->ws.out_stage};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     for (cudaEvent_t e : L->ev)
@@ -190,8 +190,8 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     ALLOC(W.slot_pos, slots * sizeof(int32_t));
     ALLOC(W.meta, ace::kMetaCount * sizeof(int32_t));
     ALLOC(W.tile_cnt, (T / 8 + 1) * sizeof(int32_t));
-    ALLOC(W.sel_hist, 2048 * sizeof(int32_t));
-    ALLOC(W.sel_state, 8 * sizeof(int32_t));
+    ALLOC(W.sel_hist, (4096 + 1024) * sizeof(int32_t));
+    ALLOC(W.sel_cand, slots * sizeof(uint32_t));
     if (L->tc) {
         ALLOC(W.h_perm, slots * d * E);
         ALLOC(W.act_bf16, slots * m * E);
@@ -234,8 +234,7 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     CK(cudaMemcpyAsync(L->a_rcr, a_rcr, n * sizeof(float), cudaMemcpyHostToDevice, s), "copy a_rcr");
     CK(cudaMemsetAsync(W.meta, 0, ace::kMetaCount * sizeof(int32_t), s), "zero meta");
     CK(cudaMemsetAsync(W.tile_cnt, 0, (T / 8 + 1) * sizeof(int32_t), s), "zero tickets");
-    CK(cudaMemsetAsync(W.sel_hist, 0, 2048 * sizeof(int32_t), s), "zero select histogram");
-    CK(cudaMemsetAsync(W.sel_state, 0, 8 * sizeof(int32_t), s), "zero select state");
+    CK(cudaMemsetAsync(W.sel_hist, 0, (4096 + 1024) * sizeof(int32_t), s), "zero select histograms");
     CK(cudaMemsetAsync(W.err, 0, sizeof(int), s), "zero error word");
     CK(cudaMemsetAsync(W.offsets, 0, (n + 1) * sizeof(int32_t), s), "zero offsets");
     CK(ace::route_init(L), "route kernel attributes");
@@ -306,7 +305,8 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
         else
             ACE_CUDA(ace::launch_router(L, x, T, false, s), "router launch");
         if (ev) ACE_CUDA(ace::record_stage(ev[2], s), "event record");
-        ACE_CUDA(ace::launch_route(L, L->ws.logits, T, ctl, s), "route launch");
+        // split-K router: the top-k kernel sums the partials into ws.logits
+        ACE_CUDA(ace::launch_route(L, L->ws.logits, T, ctl, s, L->tc ? ace::router_splits(L, T) : 1), "route launch");
     }
     if (ev) ACE_CUDA(ace::record_stage(ev[3], s), "event record");
     if (L->tc) {

@@ -57,6 +57,8 @@ struct TcParams {
     int n_valid_cols;                   // columns of out that exist (EPI 2)
     const int32_t* perm;                // [R] slot of row r (GEMM 2 epilogue; direct token rows)
     int direct_rows;                    // SWAP: token rows loaded one by one from h (tm_tok: one-row boxes)
+    int k_splits;                       // router (EPI 2): K slices, each writing raw partials at split * split_stride
+    long long split_stride;
     const float* ghat;                  // [T*k] g_hat by slot (GEMM 2 reads ghat[perm[r]])
     int k;
 };
@@ -129,10 +131,15 @@ struct Tile {
     int nrows;    // valid token rows
     int wrow0;    // first weight row in the [N * w_rows] map
     int wt;       // weight tile index within the expert
+    int split;    // K slice (split-K router only, else 0)
+    int kb0;      // first K block of the slice
 };
 
+// Tiles run K slice major: tile = split * n_base + (token tile * w_tiles + weight tile).
 template <int TOKTILE, int WTILE>
-__device__ __forceinline__ Tile tile_at(const TcParams& p, int tile) {
+__device__ __forceinline__ Tile tile_at(const TcParams& p, int tile, int n_base, int kblocks) {
+    const int split = tile / n_base;
+    tile -= split * n_base;
     const int tt = tile / p.w_tiles;
     const int wt = tile - tt * p.w_tiles;
     Tile t;
@@ -148,6 +155,8 @@ __device__ __forceinline__ Tile tile_at(const TcParams& p, int tile) {
     }
     t.wrow0 = t.e * p.w_rows + wt * WTILE;
     t.wt = wt;
+    t.split = split;
+    t.kb0 = split * kblocks;
     return t;
 }
 
@@ -187,7 +196,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int kblocks = p.K / kBK;
+    const int splits = p.k_splits > 1 ? p.k_splits : 1;
+    const int kblocks = p.K / kBK / splits;          // K blocks per tile
     if (threadIdx.x == 0) {
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_tok)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_w)) : "memory");
@@ -216,8 +226,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
     const uint32_t tmem_base = *tmem_slot;
     // everything above overlaps the predecessor kernel (PDL); its results are read below
     pdl_wait();
-    const int n_tiles = (p.single_rows > 0 ? (p.single_rows + C::TOKTILE - 1) / C::TOKTILE : p.meta[kMetaTokTiles]) *
-                        p.w_tiles;
+    const int n_base = (p.single_rows > 0 ? (p.single_rows + C::TOKTILE - 1) / C::TOKTILE : p.meta[kMetaTokTiles]) *
+                       p.w_tiles;
+    const int n_tiles = n_base * splits;
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
@@ -231,7 +242,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
         bool ok = true;
         long long issued = 0;
         for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-            const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile);
+            const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile, n_base, kblocks);
             const int my_row = (direct && lane < t.nrows) ? p.perm[t.row0 + lane] / p.k : 0;
             const uint32_t bytes = direct ? (uint32_t)(C::A_BYTES + t.nrows * kBK * 2) : (uint32_t)C::STAGE_BYTES;
             for (int kb = 0; kb < kblocks; ++kb) {
@@ -242,17 +253,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                 unsigned char* sb = sa + C::A_BYTES;
                 if (lane == 0) {
                     mbar_expect_tx(&full[stage], bytes);
+                    const int kx = (t.kb0 + kb) * kBK;
                     if (SWAP) {
-                        tma_load_2d(sa, &p.tm_w, &full[stage], kb * kBK, t.wrow0);
-                        if (!direct) tma_load_2d(sb, &p.tm_tok, &full[stage], kb * kBK, t.row0);
+                        tma_load_2d(sa, &p.tm_w, &full[stage], kx, t.wrow0);
+                        if (!direct) tma_load_2d(sb, &p.tm_tok, &full[stage], kx, t.row0);
                     } else {
-                        tma_load_2d(sa, &p.tm_tok, &full[stage], kb * kBK, t.row0);
-                        tma_load_2d(sb, &p.tm_w, &full[stage], kb * kBK, t.wrow0);
+                        tma_load_2d(sa, &p.tm_tok, &full[stage], kx, t.row0);
+                        tma_load_2d(sb, &p.tm_w, &full[stage], kx, t.wrow0);
                     }
                 }
                 if (direct) {
                     __syncwarp();
-                    if (lane < t.nrows) tma_load_2d(sb + lane * (kBK * 2), &p.tm_tok, &full[stage], kb * kBK, my_row);
+                    if (lane < t.nrows)
+                        tma_load_2d(sb + lane * (kBK * 2), &p.tm_tok, &full[stage], (t.kb0 + kb) * kBK, my_row);
                 }
                 ++issued;
                 if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -310,7 +323,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
             ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
             if (!ok) break;
             tc_fence_after();
-            const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile);
+            const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile, n_base, kblocks);
             const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * C::ACC_COLS);
             if (SWAP) {
                 // lane = weight row (32 per warp), columns = TOKTILE (16) tokens
@@ -377,7 +390,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                         }
                     }
                 } else if (EPI == 2) {
-                    float* z = static_cast<float*>(p.out);
+                    // split-K: raw partial sums per slice (bias and temperature added by the consumer)
+                    float* z = static_cast<float*>(p.out) + (size_t)t.split * p.split_stride;
+                    const bool raw = splits > 1;
 #pragma unroll 1
                     for (int c0 = 0; c0 < C::WTILE; c0 += 16) {
                         const int col0 = t.wt * C::WTILE + c0;
@@ -386,14 +401,25 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                         tmem_ld16(tbase + c0, r);
                         tmem_ld_wait();
                         if (valid) {
+                            float v[16];
 #pragma unroll
                             for (int i = 0; i < 16; ++i) {
-                                const int col = col0 + i;
-                                if (col < p.n_valid_cols) {
-                                    float v = __uint_as_float(r[i]) + p.bias[col];
-                                    if (p.use_temp) v = v * p.inv_temp;
-                                    z[orow * p.out_ld + col] = v;
+                                const int col = min(col0 + i, p.n_valid_cols - 1);
+                                v[i] = __uint_as_float(r[i]);
+                                if (!raw) {
+                                    v[i] = v[i] + p.bias[col];
+                                    if (p.use_temp) v[i] = v[i] * p.inv_temp;
                                 }
+                            }
+                            float* zr = z + orow * p.out_ld + col0;
+                            if (col0 + 16 <= p.n_valid_cols && (p.out_ld & 3) == 0) {
+#pragma unroll
+                                for (int i = 0; i < 16; i += 4)
+                                    *reinterpret_cast<float4*>(zr + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+                            } else {
+#pragma unroll
+                                for (int i = 0; i < 16; ++i)
+                                    if (col0 + i < p.n_valid_cols) zr[i] = v[i];
                             }
                         }
                     }
@@ -656,12 +682,26 @@ cudaError_t tc_init(ace_layer* L) {
 // Router logits on the tensor cores for batches over 256 tokens (smaller
 // ones are routed by the fused kernel): 128 tokens x 256 experts per tile,
 // so W_r (N padded to 256 rows) is re-read from L2 once per 128 tokens.
+int router_splits(const ace_layer* L, int T) {
+    const ace_layer_desc& D = L->desc;
+    const int base = ((T + 127) / 128) * ((D.n_experts + 255) / 256);
+    const int kblocks = D.hidden / kBK;
+    int sp = 1;
+    // the partials [splits, T, N] fp32 live in act_bf16 ([T*k, m] bf16), idle while routing
+    while (sp < 8 && 2 * sp * base <= L->num_sms && kblocks % (2 * sp) == 0 && kblocks / (2 * sp) >= 4 &&
+           (size_t)2 * sp * D.n_experts * 4 <= (size_t)D.top_k * D.ffn * 2)
+        sp *= 2;
+    return sp;
+}
+
 cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s) {
     const ace_layer_desc& D = L->desc;
     TcParams p{};
     p.tm_tok = L->tcm.h_rows_big;
     p.tm_w = L->tcm.w_router_big;
-    p.out = L->ws.logits;
+    p.k_splits = router_splits(L, T);
+    p.split_stride = (long long)T * D.n_experts;
+    p.out = p.k_splits > 1 ? L->ws.act_bf16 : (void*)L->ws.logits;
     p.K = D.hidden;
     p.w_rows = D.n_experts;
     p.w_tiles = (D.n_experts + 255) / 256;

@@ -32,10 +32,14 @@ enum : int {
     kMetaTiles2 = 6,       // tensor-core GEMM 2 tiles
     kMetaTicket2 = 7,      // second ticket (fused small-T routing)
     kMetaTokTiles = 8,     // token tiles of the tensor-core expert schedule
+    kMetaSelCount = 9,     // large-T threshold select: candidates collected (kept zero between calls)
+    kMetaSelPrefix = 10,   //   first digit, as the key prefix
+    kMetaSelWant = 11,     //   rank still wanted inside the first digit
+    kMetaSelBelow = 12,    //   candidates below the first digit
     kMetaCount = 16,
 };
 
-constexpr int kChunk = 256;          // tokens per compaction block
+constexpr int kChunk = 64;            // tokens per compaction block (large-T route)
 constexpr int kTcSmallT = 256;       // tensor-core experts: decode tiling up to this many tokens
 constexpr int kMaxExperts = 1024;
 constexpr int kMaxTopK = 16;
@@ -65,8 +69,8 @@ struct Workspace {
     int32_t* tt_off = nullptr;   // [N+1] token-tile prefix over distinct experts
     int4* tt_tab = nullptr;      // [N + Tmax*k/16 + 1] token tiles: (expert, first row, rows, 0)
     int32_t* tile_cnt = nullptr; // [Tmax/8 + 1] per-token-tile tickets of the fused small-T kernel
-    int32_t* sel_hist = nullptr; // [2048] global histogram of the multi-block threshold select (kept zero)
-    int32_t* sel_state = nullptr;// [8] prefix / want / below / ticket of the multi-block select
+    int32_t* sel_hist = nullptr; // [4096 + 1024] digit histograms of the threshold keys (kept zero between calls)
+    uint32_t* sel_cand = nullptr;// [Tmax*k] keys of the chosen first digit (large-T threshold select)
     int* err = nullptr;          // device error word
     void* x_stage = nullptr;     // [Tmax, d] dtype: host-API staging
     void* out_stage = nullptr;   // [Tmax, d]
@@ -124,8 +128,8 @@ bool small_path(int T);
 cudaError_t launch_rmsnorm(const ace_layer* L, const void* x, int T, cudaStream_t s);
 cudaError_t launch_router(const ace_layer* L, const void* x, int T, bool fuse_norm, cudaStream_t s);
 // Runs top-k / gates / decision / threshold / compaction from `logits`.
-cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_skip_ctl ctl,
-                         cudaStream_t s);
+cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_skip_ctl ctl, cudaStream_t s,
+                         int n_split = 1);
 int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl);
 // T <= 256: RMSNorm + router + decision + compaction in one launch; with
 // x == nullptr the logits are taken from `logits` instead.
@@ -206,6 +210,9 @@ cudaError_t tc_pack_gate_up(ace_layer* L, const void* w_gate, const void* w_up, 
 // ev (nullable): recorded after gather, after gate/up, after down, after combine.
 cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
 // Router logits on the tensor cores (T > kTcSmallT): z = (h W_r^T + b) / temp.
+// With router_splits(L, T) > 1 it writes raw partial sums [splits, T, N] into
+// ws.act_bf16 and the top-k kernel forms the logits.
 cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s);
+int router_splits(const ace_layer* L, int T);
 
 }  // namespace ace

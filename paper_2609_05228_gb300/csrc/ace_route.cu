@@ -5,8 +5,8 @@
 // Two launch shapes share the same device functions (and so the same bits):
 //   T <= kSmallT: k_route_fused, one launch for RMSNorm, router, top-k,
 //                 decision, threshold and compaction;
-//   larger T:     k_rmsnorm, router GEMM, k_topk_score, [3 x k_select_pass, k_decide],
-//                 k_compact_count, k_compact_place.
+//   larger T:     k_rmsnorm, router GEMM, k_topk_score, [k_sel_collect, k_sel_final],
+//                 k_compact_count (+ the ratio-mode decision), k_compact_scan, k_compact_place.
 #include <math.h>
 
 #include "ace_device.cuh"
@@ -195,7 +195,6 @@ template <int NPL>
 __device__ __forceinline__ void warp_topk(const float* __restrict__ zrow, int n_exp, int k, int lane,
                                           int& my_id, float& my_z, bool& saw_nan) {
     uint32_t v[NPL];
-    unsigned taken = 0u;   // bit j: expert lane + 32*j chosen already (or absent)
     saw_nan = false;
 #pragma unroll
     for (int j = 0; j < NPL; ++j) {
@@ -205,23 +204,55 @@ __device__ __forceinline__ void warp_topk(const float* __restrict__ zrow, int n_
             if (z != z) { saw_nan = true; z = -INFINITY; }
             v[j] = order_key(z);
         } else {
-            v[j] = 0u;
-            taken |= 1u << j;
+            v[j] = 0u;                       // below every real key: never chosen
         }
     }
     my_id = -1;
     my_z = 0.f;
-    for (int r = 0; r < k; ++r) {
-        uint32_t bk = 0u;
-        int bj = -1;
+    if (NPL <= 8) {
+        // sort the lane's keys once (larger first, lower j first on ties: a
+        // stable insertion network), then each round takes the largest head
+        int jj[NPL];
 #pragma unroll
-        for (int j = 0; j < NPL; ++j)
-            if (!((taken >> j) & 1u) && (bj < 0 || v[j] > bk)) { bk = v[j]; bj = j; }
-        const uint32_t top = __reduce_max_sync(0xffffffffu, bj >= 0 ? bk : 0u);
-        const uint32_t e = __reduce_min_sync(0xffffffffu, (bj >= 0 && bk == top) ? (uint32_t)(lane + 32 * bj)
-                                                                                  : 0xffffffffu);
-        if ((int)(e & 31u) == lane) taken |= 1u << (e >> 5);
-        if (lane == r) { my_id = (int)e; my_z = key_value(top); }
+        for (int j = 0; j < NPL; ++j) jj[j] = j;
+#pragma unroll
+        for (int a = 1; a < NPL; ++a) {
+#pragma unroll
+            for (int b = a; b > 0; --b) {
+                const bool sw = v[b] > v[b - 1];
+                const uint32_t tv = sw ? v[b] : v[b - 1];
+                v[b] = sw ? v[b - 1] : v[b];
+                v[b - 1] = tv;
+                const int tj = sw ? jj[b] : jj[b - 1];
+                jj[b] = sw ? jj[b - 1] : jj[b];
+                jj[b - 1] = tj;
+            }
+        }
+        for (int r = 0; r < k; ++r) {
+            const uint32_t top = __reduce_max_sync(0xffffffffu, v[0]);
+            const uint32_t e = __reduce_min_sync(0xffffffffu, (v[0] == top && top != 0u) ? (uint32_t)(lane + 32 * jj[0])
+                                                                                       : 0xffffffffu);
+            if ((int)(e & 31u) == lane) {
+#pragma unroll
+                for (int j = 0; j < NPL - 1; ++j) { v[j] = v[j + 1]; jj[j] = jj[j + 1]; }
+                v[NPL - 1] = 0u;
+            }
+            if (lane == r) { my_id = (int)e; my_z = key_value(top); }
+        }
+    } else {
+        unsigned taken = 0u;   // bit j: expert lane + 32*j chosen already
+        for (int r = 0; r < k; ++r) {
+            uint32_t bk = 0u;
+            int bj = -1;
+#pragma unroll
+            for (int j = 0; j < NPL; ++j)
+                if (!((taken >> j) & 1u) && v[j] != 0u && (bj < 0 || v[j] > bk)) { bk = v[j]; bj = j; }
+            const uint32_t top = __reduce_max_sync(0xffffffffu, bj >= 0 ? bk : 0u);
+            const uint32_t e = __reduce_min_sync(0xffffffffu, (bj >= 0 && bk == top) ? (uint32_t)(lane + 32 * bj)
+                                                                                      : 0xffffffffu);
+            if ((int)(e & 31u) == lane) taken |= 1u << (e >> 5);
+            if (lane == r) { my_id = (int)e; my_z = key_value(top); }
+        }
     }
 }
 
@@ -484,116 +515,93 @@ __device__ void fill_tile_table(const int32_t* offsets, const int32_t* dlist, co
 // Large-T kernels
 // --------------------------------------------------------------------------
 
-// Pass 1: top-k, gates, c. THRESHOLD mode also decides; RATIO mode writes
-// candidate keys (float bits of c, or 0xffffffff for protected slots).
+// Pass 1: top-k, gates, c; one warp per token, 32 tokens per block.
+// THRESHOLD mode also decides. RATIO mode writes the candidate keys (float
+// bits of c, or 0xffffffff for protected slots) and adds the block's
+// histogram of their top 12 bits (shared memory first, then one global
+// atomic per non-empty bin) to ghist, the first digit of the threshold select.
+constexpr int kTopkWarps = 32;
+constexpr int kHistBins = 4096;
+
 template <int NPL>
-__global__ void __launch_bounds__(256) k_topk_score(const float* __restrict__ logits, int n_tokens,
-                                                    int n_exp, int k, const float* __restrict__ a_gsp,
-                                                    const float* __restrict__ a_rcr, float eps,
-                                                    int m_min, int mode, float tau,
-                                                    int32_t* __restrict__ ids, float* __restrict__ gates,
-                                                    float* __restrict__ cval, uint32_t* __restrict__ keys,
-                                                    uint8_t* __restrict__ skip, float* __restrict__ ghat,
-                                                    float* __restrict__ tau_out, int* __restrict__ err) {
+__global__ void __launch_bounds__(kTopkWarps * 32) k_topk_score(float* __restrict__ logits, int n_tokens,
+                                                                int n_exp, int k, const float* __restrict__ a_gsp,
+                                                                const float* __restrict__ a_rcr, float eps,
+                                                                int m_min, int mode, float tau,
+                                                                int32_t* __restrict__ ids, float* __restrict__ gates,
+                                                                float* __restrict__ cval, uint32_t* __restrict__ keys,
+                                                                uint8_t* __restrict__ skip, float* __restrict__ ghat,
+                                                                float* __restrict__ tau_out, int* __restrict__ err,
+                                                                int32_t* __restrict__ ghist,
+                                                                const float* __restrict__ part, int n_split,
+                                                                const float* __restrict__ bias, float inv_temp,
+                                                                int use_temp) {
+    __shared__ int hist[kHistBins];
+    const bool ratio = mode == ACE_SKIP_RATIO;
+    if (ratio)
+        for (int i = threadIdx.x; i < kHistBins; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
     pdl_wait();
-    if (mode == ACE_SKIP_THRESHOLD && blockIdx.x == 0 && threadIdx.x == 0) *tau_out = tau;
-    const int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (!ratio && blockIdx.x == 0 && threadIdx.x == 0) *tau_out = tau;
+    const int t = blockIdx.x * kTopkWarps + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
-    if (t >= n_tokens) return;
-    int id;
-    float zv;
-    bool nan;
-    warp_topk<NPL>(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
-    const float z0 = __shfl_sync(0xffffffffu, zv, 0);
-    if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(err, kErrNumeric);
-    const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a_gsp, a_rcr, eps);
-    const size_t base = (size_t)t * k;
-    if (lane < k) {
-        ids[base + lane] = id;
-        gates[base + lane] = sc.g;
-        cval[base + lane] = sc.c;
-    }
-    if (mode == ACE_SKIP_THRESHOLD) {
-        bool sk;
-        float gh;
-        decide_slot(lane, k, sc.g, sc.c, tau, m_min, eps, sk, gh);
+    if (t < n_tokens) {
+        if (n_split > 1) {
+            // split-K router: z = (sum of the slices in order + b) / temp
+            const size_t stride = (size_t)n_tokens * n_exp;
+            for (int e = lane; e < n_exp; e += 32) {
+                const size_t o = (size_t)t * n_exp + e;
+                float z = __ldcg(part + o);
+                for (int sp = 1; sp < n_split; ++sp) z += __ldcg(part + sp * stride + o);
+                z = z + bias[e];
+                if (use_temp) z = z * inv_temp;
+                logits[o] = z;
+            }
+            __syncwarp();
+        }
+        int id;
+        float zv;
+        bool nan;
+        warp_topk<NPL>(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
+        const float z0 = __shfl_sync(0xffffffffu, zv, 0);
+        if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(err, kErrNumeric);
+        const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a_gsp, a_rcr, eps);
+        const size_t base = (size_t)t * k;
         if (lane < k) {
-            skip[base + lane] = sk ? 1 : 0;
-            ghat[base + lane] = gh;
+            ids[base + lane] = id;
+            gates[base + lane] = sc.g;
+            cval[base + lane] = sc.c;
         }
-    } else {
-        const bool prot = slot_protected(lane, k, sc.c, m_min);
-        if (lane < k) keys[base + lane] = prot ? 0xffffffffu : __float_as_uint(sc.c);
+        if (!ratio) {
+            bool sk;
+            float gh;
+            decide_slot(lane, k, sc.g, sc.c, tau, m_min, eps, sk, gh);
+            if (lane < k) {
+                skip[base + lane] = sk ? 1 : 0;
+                ghat[base + lane] = gh;
+            }
+        } else {
+            const bool prot = slot_protected(lane, k, sc.c, m_min);
+            const uint32_t key = prot ? 0xffffffffu : __float_as_uint(sc.c);
+            if (lane < k) keys[base + lane] = key;
+            if (lane < k && !prot) {
+                const int bin = (int)(key >> 20);
+                const unsigned peers = __match_any_sync(__activemask(), bin);
+                if (lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+            }
+        }
+    }
+    if (ratio) {
+        __syncthreads();
+        for (int i = threadIdx.x; i < kHistBins; i += blockDim.x)
+            if (hist[i]) atomicAdd(&ghist[i], hist[i]);
     }
 }
 
-// Pass 2 (ratio mode): decide from stored g, c and the device tau, one
-// thread per token.
-__global__ void __launch_bounds__(256) k_decide(int n_tokens, int k, const float* __restrict__ gates,
-                                                const float* __restrict__ cval,
-                                                const float* __restrict__ tau_dev, int m_min, float eps,
-                                                uint8_t* __restrict__ skip, float* __restrict__ ghat) {
-    pdl_wait();
-    const int t = blockIdx.x * blockDim.x + threadIdx.x;
-    if (t >= n_tokens) return;
-    const size_t base = (size_t)t * k;
-    decide_token(gates + base, cval + base, k, __ldcg(tau_dev), m_min, eps, skip + base, ghat + base, nullptr);
-}
-
-// Multi-block App. B.1 threshold for large T: three passes over the
-// candidate keys with 11/11/10-bit digits (bits [31:21], [20:10], [9:0]).
-// Each block histograms its chunk in shared memory and adds the non-empty
-// bins to one global histogram; the last block of the pass (ticket) finds
-// the digit holding the (m+1)-th smallest key, records it in `state`, and
-// clears the histogram for the next pass. The last pass writes tau with the
-// same tie rule as block_select_tau.
-// state: [0] prefix, [1] want, [2] below, [3] ticket, [4] last bin count
-constexpr int kMsBins = 2048;
-constexpr int kMsKeysPerBlock = 4096;
-
-__global__ void __launch_bounds__(1024) k_select_pass(const uint32_t* __restrict__ keys, int n, int m, int pass,
-                                                      int32_t* __restrict__ ghist, int32_t* __restrict__ state,
-                                                      float* __restrict__ tau_out) {
-    __shared__ int hist[kMsBins];
-    __shared__ int wtot[32];
-    __shared__ bool is_last;
-    pdl_wait();
-    const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
-    const int bits = pass == 2 ? 10 : 11;
-    const uint32_t dmask = (1u << bits) - 1u;
-    const uint32_t pmask = pass == 0 ? 0u : (pass == 1 ? 0xFFE00000u : 0xFFFFFC00u);
-    const uint32_t prefix = pass == 0 ? 0u : (uint32_t)__ldcg(state + 0);
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    for (int i = tid; i < kMsBins; i += blockDim.x) hist[i] = 0;
-    __syncthreads();
-    const int lo = blockIdx.x * kMsKeysPerBlock, hi = min(n, lo + kMsKeysPerBlock);
-    for (int i0 = lo; i0 < hi; i0 += blockDim.x) {
-        const int i = i0 + tid;
-        const uint32_t key = i < hi ? keys[i] : 0xffffffffu;
-        if (key != 0xffffffffu && (key & pmask) == prefix) {
-            // keys cluster in few bins (c lies in [0, 1]): one atomic per distinct bin of the warp
-            const int bin = (int)((key >> shift) & dmask);
-            const unsigned peers = __match_any_sync(__activemask(), bin);
-            if (lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
-        }
-    }
-    __syncthreads();
-    for (int i = tid; i < kMsBins; i += blockDim.x)
-        if (hist[i]) atomicAdd(&ghist[i], hist[i]);
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) is_last = atomicAdd(&state[3], 1) == (int)gridDim.x - 1;
-    __syncthreads();
-    if (!is_last) return;
-    __threadfence();
-    // last block: thread i owns bins 2i, 2i+1 (blockDim.x == kMsBins / 2)
-    const int b0 = __ldcg(ghist + 2 * tid), b1 = __ldcg(ghist + 2 * tid + 1);
-    ghist[2 * tid] = 0;
-    ghist[2 * tid + 1] = 0;
-    const int want = pass == 0 ? m : __ldcg(state + 1);
-    const int below0 = pass == 0 ? 0 : __ldcg(state + 2);
-    const int loc = b0 + b1;
-    int inc = loc;
+// Exclusive prefix of v over a 1024-thread block (thread order); total = sum.
+__device__ __forceinline__ int block_exscan_1024(int v, int* wtot, int& total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int inc = v;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
         const int y = __shfl_up_sync(0xffffffffu, inc, o);
@@ -602,106 +610,261 @@ __global__ void __launch_bounds__(1024) k_select_pass(const uint32_t* __restrict
     if (lane == 31) wtot[warp] = inc;
     __syncthreads();
     if (warp == 0) {
-        const int v = wtot[lane];
-        int wi = v;
+        int wi = wtot[lane];
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int y = __shfl_up_sync(0xffffffffu, wi, o);
             if (lane >= o) wi += y;
         }
-        wtot[lane] = wi - v;            // exclusive prefix of the warp totals
+        wtot[lane] = wi;
     }
     __syncthreads();
-    const int exc = inc - loc + wtot[warp];
-    const int total = __shfl_sync(0xffffffffu, inc, 31) + wtot[warp];   // valid in the last warp
-    // the owner of `want`; the last thread if want lies past every count
-    const bool mine = (exc <= want && want < exc + loc) || (tid == (int)blockDim.x - 1 && want >= total);
-    if (mine) {
-        int cum = exc, dg = 2 * tid, cnt = b0;
-        if (cum + b0 <= want) { cum += b0; dg += 1; cnt = b1; }
-        const uint32_t pre = prefix | ((uint32_t)dg << shift);
-        const int below = below0 + cum;
-        state[0] = (int32_t)pre;
-        state[1] = want - cum;
-        state[2] = below;
-        state[4] = cnt;
-        state[3] = 0;
-        if (pass == 2) {
-            const int lo_c = below, hi_c = below + cnt;
-            float tau = __uint_as_float(pre);
-            if (!(lo_c == m || (m - lo_c) <= (hi_c - m))) tau = __uint_as_float(pre + 1u);
-            *tau_out = tau;
+    const int exc = inc - v + (warp ? wtot[warp - 1] : 0);
+    total = wtot[31];
+    __syncthreads();
+    return exc;
+}
+
+// App. B.1 threshold for large T: the (m+1)-th smallest candidate key v,
+// lo = #{c < v}, hi = #{c <= v}; tau = v when lo == m or lo is at least as
+// close to m as hi, else the next float above v. The key is taken as three
+// digits (bits 31..20, 19..10, 9..0):
+//   k_topk_score  adds the digit-1 histogram (4096 bins, hist1);
+//   k_sel_collect (many blocks) finds digit 1 from hist1 (every block, the
+//                 same way), appends the keys inside it to cand and adds
+//                 their digit-2 histogram (1024 bins, hist2);
+//   k_sel_final   (one block) finds digit 2, then digit 3 over cand, writes
+//                 tau and re-zeroes hist1, hist2 and the candidate count.
+constexpr int kSelKeysPerThread = 8;
+
+// Block-wide digit search over `bins` = 1024 * per counts held per thread:
+// the owner of rank `want` records prefix | digit << shift in S.
+struct SelShared {
+    int wtot[32];
+    uint32_t prefix;
+    int want, below, last;
+};
+
+template <int PER>
+__device__ __forceinline__ void find_digit(const int (&b)[PER], int want, uint32_t prefix, int shift, int below,
+                                           SelShared& S) {
+    int total;
+    int loc = 0;
+#pragma unroll
+    for (int j = 0; j < PER; ++j) loc += b[j];
+    const int exc = block_exscan_1024(loc, S.wtot, total);
+    if ((exc <= want && want < exc + loc) || (threadIdx.x == 1023 && want >= total)) {
+        int cum = exc, j = 0;
+        while (j < PER - 1 && cum + b[j] <= want) { cum += b[j]; ++j; }
+        S.prefix = prefix | ((uint32_t)(PER * threadIdx.x + j) << shift);
+        S.want = want - cum;
+        S.below = below + cum;
+        S.last = b[j];
+    }
+    __syncthreads();
+}
+
+__global__ void __launch_bounds__(1024) k_sel_collect(const uint32_t* __restrict__ keys, int n, int m,
+                                                      const int32_t* __restrict__ hist1,
+                                                      int32_t* __restrict__ hist2, uint32_t* __restrict__ cand,
+                                                      int32_t* __restrict__ meta) {
+    __shared__ SelShared S;
+    __shared__ int h2[1024];
+    const int tid = threadIdx.x, lane = tid & 31;
+    h2[tid] = 0;
+    pdl_wait();
+    int b[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) b[j] = __ldcg(hist1 + 4 * tid + j);
+    find_digit<4>(b, m, 0u, 20, 0, S);
+    const uint32_t prefix = S.prefix;
+    if (blockIdx.x == 0 && tid == 0) {
+        meta[kMetaSelPrefix] = (int32_t)prefix;
+        meta[kMetaSelWant] = S.want;
+        meta[kMetaSelBelow] = S.below;
+    }
+    // this block's keys: kSelKeysPerThread per thread, 16-byte loads
+    const int base = (blockIdx.x * 1024 + tid) * kSelKeysPerThread;
+    uint32_t kv[kSelKeysPerThread];
+    if (base + kSelKeysPerThread <= n) {
+#pragma unroll
+        for (int j = 0; j < kSelKeysPerThread; j += 4) {
+            const uint4 v = __ldcg(reinterpret_cast<const uint4*>(keys + base + j));
+            kv[j] = v.x; kv[j + 1] = v.y; kv[j + 2] = v.z; kv[j + 3] = v.w;
         }
+    } else {
+#pragma unroll
+        for (int j = 0; j < kSelKeysPerThread; ++j) kv[j] = base + j < n ? __ldcg(keys + base + j) : 0xffffffffu;
+    }
+#pragma unroll
+    for (int j = 0; j < kSelKeysPerThread; ++j) {
+        const bool in = kv[j] != 0xffffffffu && (kv[j] & 0xFFF00000u) == prefix;
+        const unsigned bal = __ballot_sync(0xffffffffu, in);
+        if (!bal) continue;
+        int pos = 0;
+        if (lane == 0) pos = atomicAdd(&meta[kMetaSelCount], __popc(bal));
+        pos = __shfl_sync(0xffffffffu, pos, 0) + __popc(bal & lanemask_lt());
+        if (in) {
+            cand[pos] = kv[j];
+            const int bin = (int)((kv[j] >> 10) & 1023u);
+            const unsigned peers = __match_any_sync(bal, bin);
+            if (lane == __ffs(peers) - 1) atomicAdd(&h2[bin], __popc(peers));
+        }
+    }
+    __syncthreads();
+    if (h2[tid]) atomicAdd(&hist2[tid], h2[tid]);
+}
+
+__global__ void __launch_bounds__(1024) k_sel_final(int m, int32_t* __restrict__ hist1, int32_t* __restrict__ hist2,
+                                                    const uint32_t* __restrict__ cand, int32_t* __restrict__ meta,
+                                                    float* __restrict__ tau_out) {
+    __shared__ SelShared S;
+    __shared__ int h3[1024];
+    const int tid = threadIdx.x, lane = tid & 31;
+    h3[tid] = 0;
+    pdl_wait();
+    const uint32_t prefix1 = (uint32_t)__ldcg(meta + kMetaSelPrefix);
+    const int want1 = __ldcg(meta + kMetaSelWant), below1 = __ldcg(meta + kMetaSelBelow);
+    const int nc = __ldcg(meta + kMetaSelCount);
+    int b[1] = {__ldcg(hist2 + tid)};
+    find_digit<1>(b, want1, prefix1, 10, below1, S);
+    const uint32_t prefix2 = S.prefix;
+    const int want2 = S.want, below2 = S.below;
+    for (int i0 = 0; i0 < nc; i0 += 1024 * 4) {
+        uint32_t kv[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int i = i0 + j * 1024 + tid;
+            kv[j] = i < nc ? __ldcg(cand + i) : 0xffffffffu;
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (kv[j] != 0xffffffffu && (kv[j] & 0xFFFFFC00u) == prefix2) {
+                const int bin = (int)(kv[j] & 1023u);
+                const unsigned peers = __match_any_sync(__activemask(), bin);
+                if (lane == __ffs(peers) - 1) atomicAdd(&h3[bin], __popc(peers));
+            }
+        }
+    }
+    __syncthreads();
+    int b3[1] = {h3[tid]};
+    find_digit<1>(b3, want2, prefix2, 0, below2, S);
+    // ready for the next call
+#pragma unroll
+    for (int j = 0; j < 4; ++j) hist1[4 * tid + j] = 0;
+    hist2[tid] = 0;
+    if (tid == 0) {
+        meta[kMetaSelCount] = 0;
+        const int lo = S.below, hi = S.below + S.last;
+        float tau = __uint_as_float(S.prefix);
+        if (!(lo == m || (m - lo) <= (hi - m))) tau = __uint_as_float(S.prefix + 1u);
+        *tau_out = tau;
     }
 }
 
 // Compaction (Algorithm 1 "evaluate only the experts indexed by I"): retained
 // slots grouped by expert, tokens increasing inside a group.
-// Pass A: per-chunk per-expert counts; the last block scans them into
-// offsets[N+1], per-chunk bases and the distinct-expert list.
-// Pass B: each chunk places its slots: rank within (chunk, expert) from a
-// per-expert token bitmap, so the order is deterministic.
+// Pass A (k_compact_count): per-chunk per-expert counts, stored expert-major
+//   (counts[e * n_chunks + c]).
+// Pass B (k_compact_scan, one block): exclusive scan of the counts in that
+//   order, so counts[e][c] becomes the first row of chunk c's expert-e slots;
+//   offsets[N+1], the distinct-expert list and the token-tile table.
+// Pass C (k_compact_place): each chunk places its slots: rank within
+//   (chunk, expert) from a per-expert token bitmap, so the order is deterministic.
+// With DECIDE (ratio mode) pass A first takes each token's decision from the
+// stored g, c and the device tau (decide_token).
+template <bool DECIDE>
 __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, int n_exp, int n_chunks,
                                                           const int32_t* __restrict__ ids,
-                                                          const uint8_t* __restrict__ skip,
-                                                          int32_t* __restrict__ chunk_counts,
-                                                          int32_t* __restrict__ offsets,
-                                                          int32_t* __restrict__ dlist,
-                                                          int32_t* __restrict__ meta, int tok_tile,
-                                                          int32_t* __restrict__ tt_off, int4* __restrict__ tt_tab) {
+                                                          uint8_t* __restrict__ skip,
+                                                          const float* __restrict__ gates,
+                                                          const float* __restrict__ cval,
+                                                          const float* __restrict__ tau_dev, int m_min, float eps,
+                                                          float* __restrict__ ghat,
+                                                          int32_t* __restrict__ chunk_counts) {
     __shared__ int cnt[kMaxExperts];
-    __shared__ bool is_last;
     for (int e = threadIdx.x; e < n_exp; e += blockDim.x) cnt[e] = 0;
     __syncthreads();
     pdl_wait();
     const int t = blockIdx.x * kChunk + threadIdx.x;
     if (t < n_tokens) {
+        const size_t base = (size_t)t * k;
+        if (DECIDE)
+            decide_token(gates + base, cval + base, k, __ldcg(tau_dev), m_min, eps, skip + base, ghat + base, nullptr);
         for (int i = 0; i < k; ++i)
-            if (!skip[(size_t)t * k + i]) atomicAdd(&cnt[ids[(size_t)t * k + i]], 1);
+            if (!skip[base + i]) atomicAdd(&cnt[ids[base + i]], 1);
     }
     __syncthreads();
     for (int e = threadIdx.x; e < n_exp; e += blockDim.x)
-        chunk_counts[(size_t)blockIdx.x * n_exp + e] = cnt[e];
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) is_last = atomicAdd(&meta[kMetaTicket], 1) == n_chunks - 1;
-    __syncthreads();
-    if (!is_last) return;
-    __threadfence();
-    // last block: per-expert running bases over chunks, totals in cnt[]
-    // (16 chunk counts in flight per thread, not one L2 round trip per chunk)
-    constexpr int kBatch = 16;
-    for (int e = threadIdx.x; e < n_exp; e += blockDim.x) {
-        int run = 0;
-        for (int c0 = 0; c0 < n_chunks; c0 += kBatch) {
-            int v[kBatch];
+        chunk_counts[(size_t)e * n_chunks + blockIdx.x] = cnt[e];
+}
+
+constexpr int kScanPer = 8;   // counts per thread per round of k_compact_scan
+
+// Rounds of 8192 counts: coalesced load into shared memory, each thread
+// scans its 8 consecutive counts, block scan of the thread sums, coalesced
+// store of the exclusive prefixes.
+__global__ void __launch_bounds__(1024) k_compact_scan(int n_exp, int n_chunks, int32_t* __restrict__ counts,
+                                                       int32_t* __restrict__ offsets, int32_t* __restrict__ dlist,
+                                                       int32_t* __restrict__ meta, int tok_tile,
+                                                       int32_t* __restrict__ tt_off, int4* __restrict__ tt_tab) {
+    __shared__ int wtot[32];
+    __shared__ int cnt[kMaxExperts];
+    __shared__ __align__(16) int buf[1024 * kScanPer];
+    pdl_wait();
+    const int n = n_exp * n_chunks;
+    const int tid = threadIdx.x;
+    int carry = 0;
+    for (int r0 = 0; r0 < n; r0 += 1024 * kScanPer) {
 #pragma unroll
-            for (int j = 0; j < kBatch; ++j)
-                v[j] = c0 + j < n_chunks ? __ldcg(chunk_counts + (size_t)(c0 + j) * n_exp + e) : 0;
+        for (int j = 0; j < kScanPer; ++j) {
+            const int i = r0 + j * 1024 + tid;
+            buf[j * 1024 + tid] = i < n ? __ldcg(counts + i) : 0;
+        }
+        __syncthreads();
+        int v[kScanPer];
+        const int4* b4 = reinterpret_cast<const int4*>(buf + tid * kScanPer);
 #pragma unroll
-            for (int j = 0; j < kBatch; ++j) {
-                if (c0 + j < n_chunks) {
-                    chunk_counts[(size_t)(c0 + j) * n_exp + e] = run;
-                    run += v[j];
-                }
+        for (int q = 0; q < kScanPer / 4; ++q) {
+            const int4 x = b4[q];
+            v[4 * q] = x.x; v[4 * q + 1] = x.y; v[4 * q + 2] = x.z; v[4 * q + 3] = x.w;
+        }
+        int loc = 0;
+#pragma unroll
+        for (int j = 0; j < kScanPer; ++j) loc += v[j];
+        int total;
+        int run = carry + block_exscan_1024(loc, wtot, total);   // (its barriers also order buf)
+#pragma unroll
+        for (int j = 0; j < kScanPer; ++j) {
+            buf[tid * kScanPer + j] = run;
+            run += v[j];
+        }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < kScanPer; ++j) {
+            const int i = r0 + j * 1024 + tid;
+            if (i < n) {
+                const int b = buf[j * 1024 + tid];
+                counts[i] = b;
+                if (i % n_chunks == 0) offsets[i / n_chunks] = b;
             }
         }
-        cnt[e] = run;
+        __syncthreads();
+        carry += total;
     }
+    if (tid == 0) offsets[n_exp] = carry;
     __syncthreads();
-    if (threadIdx.x < 32) {
-        scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, nullptr, tok_tile, tt_off);
-        if (threadIdx.x == 0) meta[kMetaTicket] = 0;
-    }
+    for (int e = tid; e < n_exp; e += blockDim.x) cnt[e] = __ldcg(offsets + e + 1) - __ldcg(offsets + e);
+    __syncthreads();
+    if (tid < 32) scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, nullptr, tok_tile, tt_off);
     __syncthreads();
     fill_tile_table(offsets, dlist, tt_off, meta, tok_tile, tt_tab);
 }
 
-__global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, int n_exp,
+__global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, int n_exp, int n_chunks,
                                                           const int32_t* __restrict__ ids,
                                                           const uint8_t* __restrict__ skip,
                                                           const int32_t* __restrict__ chunk_base,
-                                                          const int32_t* __restrict__ offsets,
                                                           int32_t* __restrict__ perm,
                                                           int32_t* __restrict__ slot_pos) {
     constexpr int W = kChunk / 32;
@@ -725,7 +888,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
             const int e = ids[s];
             int rank = __popc(bm[e * W + w] & lt);
             for (int ww = 0; ww < w; ++ww) rank += __popc(bm[e * W + ww]);
-            const int r = offsets[e] + chunk_base[(size_t)blockIdx.x * n_exp + e] + rank;
+            const int r = __ldcg(chunk_base + (size_t)e * n_chunks + blockIdx.x) + rank;
             perm[r] = (int32_t)s;
             slot_pos[s] = r;
         }
@@ -1159,8 +1322,8 @@ cudaError_t launch_router(const ace_layer* L, const void* x, int T, bool fuse_no
     return fuse_norm ? router_launch<float, true>(L, src, T, s) : router_launch<float, false>(L, src, T, s);
 }
 
-cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_skip_ctl ctl,
-                         cudaStream_t s) {
+cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_skip_ctl ctl, cudaStream_t s,
+                         int n_split) {
     const ace_layer_desc& D = L->desc;
     const Workspace& W = L->ws;
     const int k = D.top_k, n = D.n_experts;
@@ -1170,12 +1333,13 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     const int mode = need_select ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
     const int tok_tile = L->tc ? tc_token_tile(T) : 0;
     if (T <= kSmallT) return launch_route_fused(L, nullptr, logits, T, ctl, s);
-    const int blocks = cdiv(T, 8);
+    const int blocks = cdiv(T, kTopkWarps);
     cudaError_t e;
 #define ACE_TOPK(NPL)                                                                                             \
-    launch_pdl(k_topk_score<NPL>, dim3(blocks), dim3(256), 0, s, logits, T, n, k, (const float*)L->a_gsp,         \
-               (const float*)L->a_rcr, D.eps, D.min_active, mode, tau, W.ids, W.gates, W.cval, W.keys, W.skip,    \
-               W.ghat, W.tau, W.err)
+    launch_pdl(k_topk_score<NPL>, dim3(blocks), dim3(kTopkWarps * 32), 0, s, const_cast<float*>(logits), T, n, k, \
+               (const float*)L->a_gsp, (const float*)L->a_rcr, D.eps, D.min_active, mode, tau, W.ids, W.gates,    \
+               W.cval, W.keys, W.skip, W.ghat, W.tau, W.err, W.sel_hist, (const float*)W.act_bf16, n_split,        \
+               (const float*)L->router_b, 1.0f / D.router_temp, D.router_temp != 1.0f ? 1 : 0)
     if (n <= 128) e = ACE_TOPK(4);
     else if (n <= 256) e = ACE_TOPK(8);
     else e = ACE_TOPK(32);
@@ -1183,23 +1347,25 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     if (e != cudaSuccess) return e;
     if (mode == ACE_SKIP_RATIO) {
         const int nk = T * k;
-        const int sb = cdiv(nk, kMsKeysPerBlock);
-        for (int pass = 0; pass < 3; ++pass) {
-            e = launch_pdl(k_select_pass, dim3(sb), dim3(kMsBins / 2), 0, s, (const uint32_t*)W.keys, nk, m_q, pass,
-                           W.sel_hist, W.sel_state, W.tau);
-            if (e != cudaSuccess) return e;
-        }
-        e = launch_pdl(k_decide, dim3(cdiv(T, 256)), dim3(256), 0, s, T, k, (const float*)W.gates, (const float*)W.cval,
-                       (const float*)W.tau, D.min_active, D.eps, W.skip, W.ghat);
+        e = launch_pdl(k_sel_collect, dim3(cdiv(nk, 1024 * kSelKeysPerThread)), dim3(1024), 0, s,
+                       (const uint32_t*)W.keys, nk, m_q, (const int32_t*)W.sel_hist, W.sel_hist + kHistBins,
+                       W.sel_cand, W.meta);
+        if (e != cudaSuccess) return e;
+        e = launch_pdl(k_sel_final, dim3(1), dim3(1024), 0, s, m_q, W.sel_hist, W.sel_hist + kHistBins,
+                       (const uint32_t*)W.sel_cand, W.meta, W.tau);
         if (e != cudaSuccess) return e;
     }
     const int n_chunks = cdiv(T, kChunk);
-    e = launch_pdl(k_compact_count, dim3(n_chunks), dim3(kChunk), 0, s, T, k, n, n_chunks, (const int32_t*)W.ids,
-                   (const uint8_t*)W.skip, W.chunk_counts, W.offsets, W.dlist, W.meta, tok_tile, W.tt_off, W.tt_tab);
+    const bool dec = mode == ACE_SKIP_RATIO;
+    e = launch_pdl(dec ? k_compact_count<true> : k_compact_count<false>, dim3(n_chunks), dim3(kChunk), 0, s, T, k, n,
+                   n_chunks, (const int32_t*)W.ids, W.skip, (const float*)W.gates, (const float*)W.cval,
+                   (const float*)W.tau, D.min_active, D.eps, W.ghat, W.chunk_counts);
     if (e != cudaSuccess) return e;
-    return launch_pdl(k_compact_place, dim3(n_chunks), dim3(kChunk), 0, s, T, k, n, (const int32_t*)W.ids,
-                      (const uint8_t*)W.skip, (const int32_t*)W.chunk_counts, (const int32_t*)W.offsets, W.perm,
-                      W.slot_pos);
+    e = launch_pdl(k_compact_scan, dim3(1), dim3(1024), 0, s, n, n_chunks, W.chunk_counts, W.offsets, W.dlist, W.meta,
+                   tok_tile, W.tt_off, W.tt_tab);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(k_compact_place, dim3(n_chunks), dim3(kChunk), 0, s, T, k, n, n_chunks, (const int32_t*)W.ids,
+                      (const uint8_t*)W.skip, (const int32_t*)W.chunk_counts, W.perm, W.slot_pos);
 }
 
 int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl) {
@@ -1207,7 +1373,7 @@ int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl) {
     float tau;
     bool sel;
     select_mq(L, T, ctl, &tau, &sel);
-    return sel ? 7 : 3;
+    return sel ? 6 : 4;
 }
 
 cudaError_t route_init(const ace_layer* L) {
@@ -1222,8 +1388,9 @@ cudaError_t route_init(const ace_layer* L) {
                         (const void*)k_route_fused<__nv_bfloat16, 32, true>, (const void*)k_route_fused<float, 4, true>,
                         (const void*)k_route_fused<float, 8, true>, (const void*)k_route_fused<float, 32, true>,
                         (const void*)k_topk_score<4>, (const void*)k_topk_score<8>,
-                        (const void*)k_topk_score<32>, (const void*)k_decide,
-                        (const void*)k_compact_count, (const void*)k_compact_place, (const void*)k_select_pass};
+                        (const void*)k_topk_score<32>, (const void*)k_compact_count<true>,
+                        (const void*)k_compact_count<false>, (const void*)k_compact_place,
+                        (const void*)k_compact_scan};
     for (const void* kf : ks)
         if ((e = prefer_shared(kf)) != cudaSuccess) return e;
     return cudaSuccess;

@@ -120,6 +120,30 @@ def test_decision_bitexact(T, N, k, m_min):
     layer.close()
 
 
+@pytest.mark.parametrize("T,pattern", [(16384, "equal"), (8192, "two_values"), (300, "equal")])
+def test_decision_degenerate_scores(T, pattern):
+    """Every candidate score equal (or only two distinct values): the
+    threshold select meets one value held by far more keys than the select
+    stages in shared memory (and the App. B.1 tie rule decides tau)."""
+    N, k = 128, 8
+    z = np.zeros((T, N), np.float32)
+    if pattern == "two_values":
+        z[: T // 3, :] = np.linspace(0.0, -0.5, N, dtype=np.float32)[None, :]
+    tables = (np.ones(N, np.float32), np.ones(N, np.float32))
+    layer = _route_layer(N, k, T, 1, tables)
+    zd = torch.from_numpy(z).cuda()
+    ids_ref, g_ref = O.route_fp32(z, k)
+    for mode, val in [("ratio", 0.25), ("ratio", 0.5), ("ratio", 0.7)]:
+        ace.ace_route_logits(layer.handle, zd, T, mode, val)
+        skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, k)
+        ref = O.decide_fp32(ids_ref, g_ref, tables[0], tables[1], mode, val, 1, 1e-6)
+        assert (ids == ids_ref).all()
+        assert (skip.astype(bool) == ref["skip"]).all(), (mode, val, int(skip.sum()), int(ref["skip"].sum()))
+        assert (gh.view(np.uint32) == ref["g_hat"].view(np.uint32)).all()
+        assert np.float32(tau).view(np.uint32) == np.float32(ref["tau"]).view(np.uint32), (tau, ref["tau"])
+    layer.close()
+
+
 def test_decision_repeatable():
     T, N, k = 4096, 128, 8
     z = synth.make_logits(T, N, seed=3)
