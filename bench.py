@@ -387,11 +387,19 @@ def run_ours(args, rank, world, torch, dist):
 
 
 def sweep(torch, args):
-    """Tokens/s and speedup vs q=0 over the decode batches and prefill ratios."""
+    """Tokens/s and speedup vs q=0 over the configurations' batch sizes and
+    skip ratios: the d=2048 layer (decode batches, 4096-token prefill), or the
+    large layer (decode 1/16/128, prefill 2048/8192; q from 0 to 0.625 in
+    steps of 0.125) when the workload is a large-layer one."""
     from paper_2609_05228_gb300 import synth
+    if args.workload.startswith("large"):
+        qs = [0.0, 0.125, 0.25, 0.375, 0.5, 0.625]
+        plan = [("large_prefill", [1, 16, 128, 2048, 8192], qs)]
+    else:
+        plan = [("decode", [1, 8, 32, 64], [0.0, 0.25, 0.5]),
+                ("prefill", [4096], [0.0, 0.25, 0.5, 0.625])]
     pts = []
-    for wlname, Ts, qs in [("decode", [1, 8, 32, 64], [0.0, 0.25, 0.5]),
-                           ("prefill", [4096], [0.0, 0.25, 0.5, 0.625])]:
+    for wlname, Ts, qs in plan:
         model = Stack(WORKLOADS[wlname], max_tokens=max(Ts))
         flush = L2Flush(torch, "cuda")
         for T in Ts:

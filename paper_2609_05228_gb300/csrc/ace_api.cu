@@ -316,7 +316,7 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
         ACE_CUDA(ace::launch_experts_gemv(L, x, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
     }
     L->n_stages = ev ? ace::kNumStages : 0;
-    L->last_launches = (small ? 1 : 2 + ace::route_launch_count(L, T, ctl)) + (L->tc ? (small ? 3 : 4) : 3);
+    L->last_launches = (small ? 1 : 2 + ace::route_launch_count(L, T, ctl)) + (L->tc ? 4 : 3);
     return ACE_OK;
 }
 

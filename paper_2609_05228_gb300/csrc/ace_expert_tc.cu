@@ -55,8 +55,7 @@ struct TcParams {
     float inv_temp;
     int use_temp;
     int n_valid_cols;                   // columns of out that exist (EPI 2)
-    const int32_t* perm;                // [R] slot of row r (GEMM 2 epilogue; direct token rows)
-    int direct_rows;                    // SWAP: token rows loaded one by one from h (tm_tok: one-row boxes)
+    const int32_t* perm;                // [R] slot of row r (GEMM 2 epilogue)
     int k_splits;                       // router (EPI 2): K slices, each writing raw partials at split * split_stride
     long long split_stride;
     const float* ghat;                  // [T*k] g_hat by slot (GEMM 2 reads ghat[perm[r]])
@@ -232,19 +231,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
-        // Lane 0 waits for free stages and loads the A tile (and the B tile);
-        // with direct token rows (SWAP, GEMM 1) lane i < rows loads token row
-        // i of the tile from h itself (a one-row box; the 128-byte swizzle
-        // follows the shared-memory address, so the rows form the same tile).
-        const bool direct = SWAP && p.direct_rows;
+        // Lane 0 waits for free stages and loads the A and B tiles.
         int stage = 0;
         uint32_t phase = 0;
         bool ok = true;
         long long issued = 0;
         for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
             const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile, n_base, kblocks);
-            const int my_row = (direct && lane < t.nrows) ? p.perm[t.row0 + lane] / p.k : 0;
-            const uint32_t bytes = direct ? (uint32_t)(C::A_BYTES + t.nrows * kBK * 2) : (uint32_t)C::STAGE_BYTES;
             for (int kb = 0; kb < kblocks; ++kb) {
                 int go = 1;
                 if (lane == 0) go = mbar_wait(&empty[stage], phase ^ 1u, p.err) && !*abort_flag;
@@ -252,20 +245,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                 unsigned char* sa = smem + stage * C::STAGE_BYTES;
                 unsigned char* sb = sa + C::A_BYTES;
                 if (lane == 0) {
-                    mbar_expect_tx(&full[stage], bytes);
+                    mbar_expect_tx(&full[stage], C::STAGE_BYTES);
                     const int kx = (t.kb0 + kb) * kBK;
                     if (SWAP) {
                         tma_load_2d(sa, &p.tm_w, &full[stage], kx, t.wrow0);
-                        if (!direct) tma_load_2d(sb, &p.tm_tok, &full[stage], kx, t.row0);
+                        tma_load_2d(sb, &p.tm_tok, &full[stage], kx, t.row0);
                     } else {
                         tma_load_2d(sa, &p.tm_tok, &full[stage], kx, t.row0);
                         tma_load_2d(sb, &p.tm_w, &full[stage], kx, t.wrow0);
                     }
-                }
-                if (direct) {
-                    __syncwarp();
-                    if (lane < t.nrows)
-                        tma_load_2d(sb + lane * (kBK * 2), &p.tm_tok, &full[stage], (t.kb0 + kb) * kBK, my_row);
                 }
                 ++issued;
                 if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -674,7 +662,7 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = make_map(&L->tcm.wd_big, L->w_down, n * d, m, 256)) != cudaSuccess) return e;
     // router: h [Tmax, d] in 128-row boxes, W_r [N, d] in 256-row boxes
     if ((e = make_map(&L->tcm.h_rows_big, L->ws.h, h_rows, d, 128)) != cudaSuccess) return e;
-    if ((e = make_map(&L->tcm.h_row1, L->ws.h, h_rows, d, 1)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.tok1_small, L->ws.h_perm, rows, d, 16)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.w_router_big, L->router_w, n_pad, d, 256)) != cudaSuccess) return e;
     return cudaSuccess;
 }
@@ -722,17 +710,16 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     const int d = D.hidden, m = D.ffn, k = D.top_k;
     const bool small = T <= kTcSmallT;
     cudaError_t e = cudaSuccess;
-    // batches up to 256 tokens: GEMM 1 loads token rows straight from h; larger
-    // ones gather them into expert-grouped order first (128-row TMA tiles)
-    if (!small) {
+    // token rows in expert-grouped order for GEMM 1's TMA tiles (16 or 128 rows);
+    // loading them one row per TMA box from h instead measured slower
+    {
         e = launch_pdl(k_gather_rows, dim3(L->num_sms * 4), dim3(256), 0, s, (const __nv_bfloat16*)W.h,
                        (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k);
         if (e != cudaSuccess) return e;
     }
     if (ev) ace::record_stage(ev[0], s);
     TcParams p1{};
-    p1.tm_tok = small ? L->tcm.h_row1 : L->tcm.tok1_big;
-    p1.direct_rows = small ? 1 : 0;
+    p1.tm_tok = small ? L->tcm.tok1_small : L->tcm.tok1_big;
     p1.tm_w = small ? L->tcm.wgu_small : L->tcm.wgu_big;
     p1.offsets = W.offsets;
     p1.dlist = W.dlist;
@@ -751,7 +738,6 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     if (e != cudaSuccess) return e;
     if (ev) ace::record_stage(ev[1], s);
     TcParams p2 = p1;
-    p2.direct_rows = 0;
     p2.tm_tok = small ? L->tcm.tok2_small : L->tcm.tok2_big;
     p2.tm_w = small ? L->tcm.wd_small : L->tcm.wd_big;
     // y per slot: fp32 rows for SWAP tiles; bf16 rows otherwise, written over

@@ -78,12 +78,11 @@ struct Workspace {
 
 // Tensor maps of the tensor-core expert path (built once at create time).
 struct TcMaps {
-    CUtensorMap tok1_big;               // h_perm, boxes of 128 rows
+    CUtensorMap tok1_small, tok1_big;   // h_perm, boxes of 16 / 128 rows
     CUtensorMap tok2_small, tok2_big;   // act_bf16, boxes of 16 / 128 rows
     CUtensorMap wgu_small, wgu_big;     // W_gu, boxes of 128 / 256 rows
     CUtensorMap wd_small, wd_big;       // W_down
     CUtensorMap h_rows_big, w_router_big;   // router GEMM (batches over 256 tokens): 128-row / 256-row boxes
-    CUtensorMap h_row1;                 // h in one-row boxes: GEMM 1 token rows for batches <= 256
 };
 
 }  // namespace ace

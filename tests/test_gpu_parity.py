@@ -270,6 +270,21 @@ def test_forward_q0_matches_threshold0():
     assert torch.equal(o1, o2)
 
 
+@pytest.mark.parametrize("T", [1000, 4096])
+def test_forward_deterministic_large_batch(T):
+    """Batches over 256 tokens: per-slot output rows and a rank-order combine,
+    no atomics on the output, so every call returns the same bits."""
+    w, layer = _layer("qwen_zipf")
+    x = _dev(synth.make_tokens(w.spec, T, seed=6))
+    outs = []
+    for _ in range(3):
+        o = torch.empty_like(x)
+        layer.forward(x, o, T, "ratio", 0.5)
+        outs.append(o)
+    torch.cuda.synchronize()
+    assert all(torch.equal(outs[0], o) for o in outs[1:])
+
+
 def test_forward_deterministic_and_host_api():
     w, layer = _layer("qwen")
     T = 64
