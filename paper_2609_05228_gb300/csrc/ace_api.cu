@@ -223,12 +223,12 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     else
         CK(cudaMemsetAsync(L->router_b, 0, n * sizeof(float), s), "zero router_b");
     if (L->tc) {
-        CK(ace::tc_pack_gate_up(L, w_gate, w_up, s), "pack gate/up weights");
+        CK(ace::tc_pack_weights(L, w_gate, w_up, w_down, s), "pack expert weights");
     } else {
         CK(cudaMemcpyAsync(L->w_gate, w_gate, n * m * d * E, cudaMemcpyDeviceToDevice, s), "copy w_gate");
         CK(cudaMemcpyAsync(L->w_up, w_up, n * m * d * E, cudaMemcpyDeviceToDevice, s), "copy w_up");
+        CK(cudaMemcpyAsync(L->w_down, w_down, n * d * m * E, cudaMemcpyDeviceToDevice, s), "copy w_down");
     }
-    CK(cudaMemcpyAsync(L->w_down, w_down, n * d * m * E, cudaMemcpyDeviceToDevice, s), "copy w_down");
     CK(cudaMemcpyAsync(L->gamma, rms_gamma, d * E, cudaMemcpyDeviceToDevice, s), "copy gamma");
     CK(cudaMemcpyAsync(L->a_gsp, a_gsp, n * sizeof(float), cudaMemcpyHostToDevice, s), "copy a_gsp");
     CK(cudaMemcpyAsync(L->a_rcr, a_rcr, n * sizeof(float), cudaMemcpyHostToDevice, s), "copy a_rcr");

@@ -47,6 +47,8 @@ struct TcParams {
     int K;                              // reduction length
     int w_rows;                         // weight rows per expert (2m or d)
     int w_tiles;                        // w_rows / weight tile
+    const uint8_t* w_tiles_hbm;         // expert weights as pre-swizzled 16 KB tiles (nullptr: tm_w)
+    int w_kb;                           // 64-column K blocks per weight row (tiled weights)
     int out_ld;                         // row length of out
     int* err;
     // single-group schedule (router logits): rows > 0 replaces the expert groups
@@ -248,11 +250,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                     mbar_expect_tx(&full[stage], C::STAGE_BYTES);
                     const int kx = (t.kb0 + kb) * kBK;
                     if (SWAP) {
-                        tma_load_2d(sa, &p.tm_w, &full[stage], kx, t.wrow0);
+                        if (p.w_tiles_hbm)
+                            bulk_g2s(sa, p.w_tiles_hbm + (((size_t)t.e * (p.w_rows / 128) + t.wt) * p.w_kb + (t.kb0 + kb)) * 16384,
+                                     16384, &full[stage]);
+                        else
+                            tma_load_2d(sa, &p.tm_w, &full[stage], kx, t.wrow0);
                         tma_load_2d(sb, &p.tm_tok, &full[stage], kx, t.row0);
                     } else {
                         tma_load_2d(sa, &p.tm_tok, &full[stage], kx, t.row0);
-                        tma_load_2d(sb, &p.tm_w, &full[stage], kx, t.wrow0);
+                        if (p.w_tiles_hbm) {
+                            const unsigned char* wt0 =
+                                p.w_tiles_hbm + (((size_t)t.e * (p.w_rows / 128) + 2 * t.wt) * p.w_kb + (t.kb0 + kb)) * 16384;
+                            bulk_g2s(sb, wt0, 16384, &full[stage]);
+                            bulk_g2s(sb + 16384, wt0 + (size_t)p.w_kb * 16384, 16384, &full[stage]);
+                        } else {
+                            tma_load_2d(sb, &p.tm_w, &full[stage], kx, t.wrow0);
+                        }
                     }
                 }
                 ++issued;
@@ -601,30 +614,50 @@ cudaError_t launch_gemm(const ace_layer* L, const TcParams& p, cudaStream_t s) {
     return launch_pdl(k_expert_tc<SWAP, EPI, S>, dim3(L->num_sms), dim3(kThreads), TcCfg<SWAP, EPI, S>::SMEM, s, p);
 }
 
-// W_gu[e, 32b + i] = W_gate[e, 16b + i] (i < 16), W_up[e, 16b + i - 16] (i >= 16).
-__global__ void __launch_bounds__(256) k_pack_gate_up(const uint4* __restrict__ wg, const uint4* __restrict__ wu,
-                                                      uint4* __restrict__ wgu, int n_exp, int m, int d) {
-    const int nvec = d / 8;
-    const long long total = (long long)n_exp * 2 * m * nvec;
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const long long row = i / nvec;
-        const int c = (int)(i % nvec);
-        const int e = (int)(row / (2 * m));
-        const int pr = (int)(row % (2 * m));
-        const int b = pr >> 5, li = pr & 31;
-        const int j = b * 16 + (li & 15);
-        const uint4* src = li < 16 ? wg : wu;
-        wgu[i] = src[((long long)e * m + j) * nvec + c];
+// Expert weights as tiles in HBM: block (e, t, kb) holds weight rows
+// [128 t, 128 t + 128) x columns [64 kb, 64 kb + 64) of expert e, 16 KB,
+// already in the 128-byte-swizzled order of a shared-memory operand tile
+// (row r at 128 r, its 16-byte chunk c at chunk c ^ (r & 7)). A stage's
+// weights then arrive with one contiguous 16 KB bulk copy. Blocks are stored
+// [e][t][kb]. For W_gu the rows interleave gate and up in blocks of 16:
+// row 32b + i is W_gate row 16b + i (i < 16) or W_up row 16b + i - 16.
+template <bool GU>
+__global__ void __launch_bounds__(256) k_pack_tiles(const uint4* __restrict__ src0, const uint4* __restrict__ src1,
+                                                    uint4* __restrict__ dst, int n_exp, int rows, int cols) {
+    const int cv = cols / 8;                      // 16-byte chunks per source row
+    const int kbs = cols / 64, wts = rows / 128;
+    const long long total = (long long)n_exp * rows * cv;
+    for (long long q = (long long)blockIdx.x * blockDim.x + threadIdx.x; q < total;
+         q += (long long)gridDim.x * blockDim.x) {
+        const long long blk = q >> 10;            // 1024 chunks per 16 KB block
+        const int w = (int)(q & 1023);
+        const int r = w >> 3, c = (w & 7) ^ (r & 7);
+        const int kb = (int)(blk % kbs);
+        const long long et = blk / kbs;
+        const int t = (int)(et % wts), e = (int)(et / wts);
+        const int row = t * 128 + r, chunk = kb * 8 + c;
+        uint4 v;
+        if (GU) {
+            const int b = row >> 5, li = row & 31;
+            const int j = b * 16 + (li & 15);
+            v = (li < 16 ? src0 : src1)[((long long)e * (rows / 2) + j) * cv + chunk];
+        } else {
+            v = src0[((long long)e * rows + row) * cv + chunk];
+        }
+        dst[q] = v;
     }
 }
 
 }  // namespace
 
-cudaError_t tc_pack_gate_up(ace_layer* L, const void* w_gate, const void* w_up, cudaStream_t s) {
+cudaError_t tc_pack_weights(ace_layer* L, const void* w_gate, const void* w_up, const void* w_down, cudaStream_t s) {
     const ace_layer_desc& D = L->desc;
-    k_pack_gate_up<<<L->num_sms * 8, 256, 0, s>>>((const uint4*)w_gate, (const uint4*)w_up, (uint4*)L->w_gu,
-                                                  D.n_experts, D.ffn, D.hidden);
+    k_pack_tiles<true><<<L->num_sms * 8, 256, 0, s>>>((const uint4*)w_gate, (const uint4*)w_up, (uint4*)L->w_gu,
+                                                      D.n_experts, 2 * D.ffn, D.hidden);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    k_pack_tiles<false><<<L->num_sms * 8, 256, 0, s>>>((const uint4*)w_down, nullptr, (uint4*)L->w_down,
+                                                       D.n_experts, D.hidden, D.ffn);
     return cudaGetLastError();
 }
 
@@ -656,10 +689,6 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = make_map(&L->tcm.tok2_small, L->ws.act_bf16, rows, m, 16)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.tok2_big, L->ws.act_bf16, rows, m, 128)) != cudaSuccess) return e;
     // weight maps: W_gu [N * 2m, d] and W_down [N * d, m]
-    if ((e = make_map(&L->tcm.wgu_small, L->w_gu, n * 2 * m, d, 128)) != cudaSuccess) return e;
-    if ((e = make_map(&L->tcm.wgu_big, L->w_gu, n * 2 * m, d, 256)) != cudaSuccess) return e;
-    if ((e = make_map(&L->tcm.wd_small, L->w_down, n * d, m, 128)) != cudaSuccess) return e;
-    if ((e = make_map(&L->tcm.wd_big, L->w_down, n * d, m, 256)) != cudaSuccess) return e;
     // router: h [Tmax, d] in 128-row boxes, W_r [N, d] in 256-row boxes
     if ((e = make_map(&L->tcm.h_rows_big, L->ws.h, h_rows, d, 128)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.tok1_small, L->ws.h_perm, rows, d, 16)) != cudaSuccess) return e;
@@ -720,7 +749,8 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     if (ev) ace::record_stage(ev[0], s);
     TcParams p1{};
     p1.tm_tok = small ? L->tcm.tok1_small : L->tcm.tok1_big;
-    p1.tm_w = small ? L->tcm.wgu_small : L->tcm.wgu_big;
+    p1.w_tiles_hbm = static_cast<const uint8_t*>(L->w_gu);
+    p1.w_kb = d / kBK;
     p1.offsets = W.offsets;
     p1.dlist = W.dlist;
     p1.tt_tab = W.tt_tab;
@@ -739,7 +769,8 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     if (ev) ace::record_stage(ev[1], s);
     TcParams p2 = p1;
     p2.tm_tok = small ? L->tcm.tok2_small : L->tcm.tok2_big;
-    p2.tm_w = small ? L->tcm.wd_small : L->tcm.wd_big;
+    p2.w_tiles_hbm = static_cast<const uint8_t*>(L->w_down);
+    p2.w_kb = m / kBK;
     // y per slot: fp32 rows for SWAP tiles; bf16 rows otherwise, written over
     // h_perm, which GEMM 1 (complete before GEMM 2 reads anything) no longer needs
     p2.out = small ? (void*)W.yslot : W.h_perm;

@@ -80,8 +80,6 @@ struct Workspace {
 struct TcMaps {
     CUtensorMap tok1_small, tok1_big;   // h_perm, boxes of 16 / 128 rows
     CUtensorMap tok2_small, tok2_big;   // act_bf16, boxes of 16 / 128 rows
-    CUtensorMap wgu_small, wgu_big;     // W_gu, boxes of 128 / 256 rows
-    CUtensorMap wd_small, wd_big;       // W_down
     CUtensorMap h_rows_big, w_router_big;   // router GEMM (batches over 256 tokens): 128-row / 256-row boxes
 };
 
@@ -97,10 +95,11 @@ struct ace_layer {
     float* router_b = nullptr;   // [N] (zeros when there is no bias)
     void* w_gate = nullptr;      // [N, m, d] (CUDA-core path only)
     void* w_up = nullptr;        // [N, m, d] (CUDA-core path only)
-    void* w_gu = nullptr;        // [N, 2m, d] gate/up rows interleaved in blocks of 16 (tensor path)
+    void* w_gu = nullptr;        // tensor path: [N][2m/128][d/64] tiles of 128 x 64 bf16 (16 KB, 128-byte
+                                 // swizzled), gate/up rows interleaved in blocks of 16
     bool tc = false;             // tensor-core expert path in use
     ace::TcMaps tcm;
-    void* w_down = nullptr;      // [N, d, m]
+    void* w_down = nullptr;      // [N, d, m]; tensor path: [N][d/128][m/64] tiles like w_gu
     void* gamma = nullptr;       // [d]
     float* a_gsp = nullptr;      // [N]
     float* a_rcr = nullptr;      // [N]
@@ -205,7 +204,8 @@ constexpr int kNumStages = 7;
 bool tc_supported(const ace_layer* L);
 int tc_token_tile(int T);
 cudaError_t tc_init(ace_layer* L);
-cudaError_t tc_pack_gate_up(ace_layer* L, const void* w_gate, const void* w_up, cudaStream_t s);
+// Packs W_gate / W_up / W_down into the tiled, pre-swizzled layouts of w_gu and w_down.
+cudaError_t tc_pack_weights(ace_layer* L, const void* w_gate, const void* w_up, const void* w_down, cudaStream_t s);
 // ev (nullable): recorded after gather, after gate/up, after down, after combine.
 cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
 // Router logits on the tensor cores (T > kTcSmallT): z = (h W_r^T + b) / temp.
