@@ -593,7 +593,7 @@ cudaError_t make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t c
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-constexpr int kStagesSwap = 10;
+constexpr int kStagesSwap = 8;
 constexpr int kStagesWide = 4;
 
 template <bool SWAP, int EPI>
