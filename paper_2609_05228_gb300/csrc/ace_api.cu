@@ -310,7 +310,7 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
     }
     if (ev) ACE_CUDA(ace::record_stage(ev[3], s), "event record");
     if (L->tc) {
-        ACE_CUDA(ace::launch_experts_tc(L, x, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
+        ACE_CUDA(ace::launch_experts_tc(L, x, out, T, ctl, s, ev ? ev + 4 : nullptr), "expert launch");
     } else {
         if (ev) ACE_CUDA(ace::record_stage(ev[4], s), "event record");   // no gather stage
         ACE_CUDA(ace::launch_experts_gemv(L, x, out, T, s, ev ? ev + 4 : nullptr), "expert launch");

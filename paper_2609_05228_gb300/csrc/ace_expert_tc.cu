@@ -73,6 +73,58 @@ __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* m
         : "memory");
 }
 
+
+// ---------------------------------------------------------------- CTA-pair (cta_group::2) helpers
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// shared::cluster address of `p` (a shared::cta address) in CTA `rank` of the cluster
+__device__ __forceinline__ uint32_t mapa_shared(const void* p, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+    return r;
+}
+
+// Tensor load whose completion is counted on an mbarrier of either CTA of the pair.
+__device__ __forceinline__ void tma_load_2d_pair(void* smem_dst, const CUtensorMap* map, uint32_t bar_cluster, int x,
+                                                 int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];"
+        ::"r"(smem_u32(smem_dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y)
+        : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                              uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
+}
+
+// Arrives on the mbarrier at the same offset in both CTAs of the pair once
+// the pair's prior MMAs have completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t* bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;"
+        ::"r"(smem_u32(bar)), "h"((uint16_t)0x3)
+        : "memory");
+}
+
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -159,6 +211,64 @@ __device__ __forceinline__ Tile tile_at(const TcParams& p, int tile, int n_base,
     t.split = split;
     t.kb0 = split * kblocks;
     return t;
+}
+
+
+// Epilogue of a wide tile (this CTA's 128 token rows x 256 weight rows in
+// TMEM at tbase): EPI 0 writes SiLU(gate) * up as bf16 act (gate and up
+// columns interleaved in blocks of 16); EPI 1 writes the g_hat-scaled output
+// row of the slot, rounded to bf16, at its expert-grouped row (the combine
+// sums a token's rows in rank order). `row` is the token row in the tile.
+template <int EPI>
+__device__ __forceinline__ void epilogue_wide(const TcParams& p, const Tile& t, uint32_t tbase, int row) {
+    constexpr int WT = 256;
+    const bool valid = row < t.nrows;
+    const size_t orow = (size_t)(t.row0 + row);
+    if (EPI == 0) {
+        __nv_bfloat16* act = static_cast<__nv_bfloat16*>(p.out);
+#pragma unroll 1
+        for (int blk = 0; blk < WT / 32; ++blk) {
+            uint32_t g[16], u[16];
+            tmem_ld16(tbase + blk * 32, g);
+            tmem_ld16(tbase + blk * 32 + 16, u);
+            tmem_ld_wait();
+            if (valid) {
+                __align__(16) __nv_bfloat16 o[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    o[i] = __float2bfloat16_rn(silu(__uint_as_float(g[i])) * __uint_as_float(u[i]));
+                const int j0 = (t.wt * (WT / 32) + blk) * 16;
+                uint4* dst = reinterpret_cast<uint4*>(act + orow * p.out_ld + j0);
+                dst[0] = reinterpret_cast<const uint4*>(o)[0];
+                dst[1] = reinterpret_cast<const uint4*>(o)[1];
+            }
+        }
+    } else {
+        __nv_bfloat16* y = static_cast<__nv_bfloat16*>(p.out);
+        const float gh = valid ? p.ghat[p.perm[orow]] : 0.f;
+        uint4* dst = reinterpret_cast<uint4*>(y + orow * p.out_ld + t.wt * WT);
+#pragma unroll 1
+        for (int c0 = 0; c0 < WT; c0 += 64) {
+            uint32_t r[4][16];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) tmem_ld16(tbase + c0 + 16 * q, r[q]);
+            tmem_ld_wait();
+            if (valid) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    uint32_t w[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const __nv_bfloat162 b2 = __floats2bfloat162_rn(gh * __uint_as_float(r[q][2 * i]),
+                                                                        gh * __uint_as_float(r[q][2 * i + 1]));
+                        w[i] = *reinterpret_cast<const uint32_t*>(&b2);
+                    }
+                    dst[(c0 + 16 * q) / 8] = make_uint4(w[0], w[1], w[2], w[3]);
+                    dst[(c0 + 16 * q) / 8 + 1] = make_uint4(w[4], w[5], w[6], w[7]);
+                }
+            }
+        }
+    }
 }
 
 // ---------------------------------------------------------------- kernel
@@ -371,26 +481,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                 const int row = quad * 32 + lane;
                 const bool valid = row < t.nrows;
                 const size_t orow = (size_t)(t.row0 + row);
-                if (EPI == 0) {
-                    __nv_bfloat16* act = static_cast<__nv_bfloat16*>(p.out);
-#pragma unroll 1
-                    for (int blk = 0; blk < C::WTILE / 32; ++blk) {
-                        uint32_t g[16], u[16];
-                        tmem_ld16(tbase + blk * 32, g);
-                        tmem_ld16(tbase + blk * 32 + 16, u);
-                        tmem_ld_wait();
-                        if (valid) {
-                            __align__(16) __nv_bfloat16 o[16];
-#pragma unroll
-                            for (int i = 0; i < 16; ++i)
-                                o[i] = __float2bfloat16_rn(silu(__uint_as_float(g[i])) * __uint_as_float(u[i]));
-                            const int j0 = (t.wt * (C::WTILE / 32) + blk) * 16;
-                            uint4* dst = reinterpret_cast<uint4*>(act + orow * p.out_ld + j0);
-                            dst[0] = reinterpret_cast<const uint4*>(o)[0];
-                            dst[1] = reinterpret_cast<const uint4*>(o)[1];
-                        }
-                    }
-                } else if (EPI == 2) {
+                if (EPI != 2) {
+                    epilogue_wide<EPI>(p, t, tbase, row);
+                } else {
                     // split-K: raw partial sums per slice (bias and temperature added by the consumer)
                     float* z = static_cast<float*>(p.out) + (size_t)t.split * p.split_stride;
                     const bool raw = splits > 1;
@@ -424,33 +517,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                             }
                         }
                     }
-                } else {
-                    // g_hat-scaled output row of this slot, rounded to bf16, at its
-                    // expert-grouped row (the combine sums a token's rows in rank order)
-                    __nv_bfloat16* y = static_cast<__nv_bfloat16*>(p.out);
-                    const float gh = valid ? p.ghat[p.perm[orow]] : 0.f;
-                    uint4* dst = reinterpret_cast<uint4*>(y + orow * p.out_ld + t.wt * C::WTILE);
-#pragma unroll 1
-                    for (int c0 = 0; c0 < C::WTILE; c0 += 64) {
-                        uint32_t r[4][16];
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) tmem_ld16(tbase + c0 + 16 * q, r[q]);
-                        tmem_ld_wait();
-                        if (valid) {
-#pragma unroll
-                            for (int q = 0; q < 4; ++q) {
-                                uint32_t w[8];
-#pragma unroll
-                                for (int i = 0; i < 8; ++i) {
-                                    const __nv_bfloat162 b2 = __floats2bfloat162_rn(gh * __uint_as_float(r[q][2 * i]),
-                                                                                    gh * __uint_as_float(r[q][2 * i + 1]));
-                                    w[i] = *reinterpret_cast<const uint32_t*>(&b2);
-                                }
-                                dst[(c0 + 16 * q) / 8] = make_uint4(w[0], w[1], w[2], w[3]);
-                                dst[(c0 + 16 * q) / 8 + 1] = make_uint4(w[4], w[5], w[6], w[7]);
-                            }
-                        }
-                    }
                 }
             }
             tc_fence_before();
@@ -466,6 +532,161 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
     if (warp == 1) {
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
                      "r"((uint32_t)C::TMEM_COLS));
+    }
+}
+
+
+// ---------------------------------------------------------------- CTA-pair kernel
+//
+// Wide tiles of 256 token rows x 256 weight rows for batches whose experts
+// hold many tokens: a cluster of two CTAs issues tcgen05.mma.cta_group::2
+// (M = 256, N = 256). CTA r stages token rows [128 r, 128 r + 128) and weight
+// rows [128 r, 128 r + 128) of the tile, 32 KB per K block, and holds its 128
+// rows of the fp32 accumulator in its own TMEM, so each SM loads two thirds of
+// what a 128 x 256 tile on one SM loads for the same MACs.
+//   * Both CTAs' producers load their halves; every load completes on the
+//     leader's (rank 0) full barrier, which the leader arms for 64 KB.
+//   * The leader's single MMA thread issues the pair's MMAs; its commits
+//     arrive on the empty and acc_full barriers of both CTAs.
+//   * Each CTA's epilogue drains its own TMEM rows and arrives on the
+//     leader's acc_empty (count 8: four warps per CTA).
+// Every mbarrier wait is bounded as in k_expert_tc; TMEM is allocated and
+// freed by one warp in each CTA (cta_group::2).
+constexpr int kPairStages = 6;
+constexpr int kPairHalf = 128 * kBK * 2;                   // 16 KB: 128 rows x 64 bf16
+constexpr int kPairStage = 2 * kPairHalf;                  // this CTA's A + B halves
+constexpr int kPairSmem = kPairStages * kPairStage + 1024 + 256;
+
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1) k_expert_pair(const __grid_constant__ TcParams p) {
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + kPairStages * kPairStage);
+    uint64_t* empty = full + kPairStages;
+    uint64_t* acc_full = empty + kPairStages;
+    uint64_t* acc_empty = acc_full + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const bool leader = rank == 0;
+    const int unit = (int)(blockIdx.x >> 1), n_units = (int)(gridDim.x >> 1);
+    const int kblocks = p.K / kBK;
+    if (threadIdx.x == 0) {
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_tok)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_w)) : "memory");
+        for (int s = 0; s < kPairStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&acc_full[a], 1);
+            mbar_init(&acc_empty[a], 8);
+        }
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(512u));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();                                          // both CTAs' barriers exist
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    pdl_wait();
+    const int n_tiles = p.meta[kMetaTokTiles] * p.w_tiles;
+
+    if (warp == 0) {
+        // ------------------------------------------------ producer (both CTAs)
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            for (int tile = unit; tile < n_tiles && ok; tile += n_units) {
+                const Tile t = tile_at<256, 256>(p, tile, n_tiles, kblocks);
+                for (int kb = 0; kb < kblocks; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                    unsigned char* sa = smem + stage * kPairStage;
+                    unsigned char* sb = sa + kPairHalf;
+                    const uint32_t bar = mapa_shared(&full[stage], 0);
+                    if (leader) mbar_expect_tx(&full[stage], 2 * kPairStage);
+                    tma_load_2d_pair(sa, &p.tm_tok, bar, kb * kBK, t.row0 + 128 * (int)rank);
+                    // weight block (e, 2 wt + rank, kb) of the tiled layout: rows of 128 B, no swizzle
+                    const int blk = ((t.e * (p.w_rows / 128) + 2 * t.wt + (int)rank) * p.w_kb + kb);
+                    tma_load_2d_pair(sb, &p.tm_w, bar, 0, blk * 128);
+                    if (++stage == kPairStages) { stage = 0; phase ^= 1u; }
+                }
+            }
+            if (!ok) *abort_flag = 1;
+            // every fill's slot released again: no commit is still heading for this CTA
+            for (int s = 0; s < kPairStages && ok; ++s) {
+                if (!mbar_wait(&empty[stage], phase ^ 1u, p.err)) break;
+                if (++stage == kPairStages) { stage = 0; phase ^= 1u; }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer (leader only)
+        if (leader && lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16(256, 256);
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true;
+            for (int tile = unit; tile < n_tiles && ok; tile += n_units) {
+                if (!mbar_wait(&acc_empty[acc], acc_phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 256);
+                for (int kb = 0; kb < kblocks; ++kb) {
+                    if (!mbar_wait(&full[stage], phase, p.err) || *abort_flag) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t a_addr = smem_u32(smem + stage * kPairStage);
+                    const uint32_t b_addr = a_addr + kPairHalf;
+#pragma unroll
+                    for (int kk = 0; kk < kBK / kUmmaK; ++kk)
+                        mma_bf16_pair(d_tmem, smem_desc_sw128(a_addr + kk * kUmmaK * 2),
+                                      smem_desc_sw128(b_addr + kk * kUmmaK * 2), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                    mma_commit_pair(&empty[stage]);      // both CTAs may refill this stage
+                    if (++stage == kPairStages) { stage = 0; phase ^= 1u; }
+                }
+                if (!ok) break;
+                mma_commit_pair(&acc_full[acc]);         // both CTAs' accumulator rows are ready
+                if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+            }
+            if (!ok) *abort_flag = 1;
+        }
+    } else {
+        // ------------------------------------------------ epilogue (warps 2..5, both CTAs)
+        const int quad = warp & 3;
+        const uint32_t acc_empty_leader[2] = {mapa_shared(&acc_empty[0], 0), mapa_shared(&acc_empty[1], 0)};
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = unit; tile < n_tiles; tile += n_units) {
+            bool ok = true;
+            if (lane == 0) ok = mbar_wait(&acc_full[acc], acc_phase, p.err) && !*abort_flag;
+            ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+            if (!ok) break;
+            tc_fence_after();
+            const Tile t = tile_at<256, 256>(p, tile, n_tiles, kblocks);
+            const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * 256);
+            epilogue_wide<EPI>(p, t, tbase, 128 * (int)rank + quad * 32 + lane);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(acc_empty_leader[acc]);
+            if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();                                          // the pair is done with TMEM and barriers
+    pdl_trigger();
+    tc_fence_after();
+    if (warp == 1) {
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512u));
     }
 }
 
@@ -580,7 +801,10 @@ cudaError_t get_encoder() {
 }
 
 // 2-D bf16 map over [rows, cols] (row-major), box [box_rows, 64], 128-byte swizzle.
-cudaError_t make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+// With swizzle == false the map copies rows verbatim (the tiled expert weights
+// are stored already swizzled).
+cudaError_t make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                     bool swizzle = true) {
     cudaError_t e = get_encoder();
     if (e != cudaSuccess) return e;
     const cuuint64_t dims[2] = {cols, rows};
@@ -588,9 +812,50 @@ cudaError_t make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t c
     const cuuint32_t box[2] = {(cuuint32_t)kBK, box_rows};
     const cuuint32_t estr[2] = {1, 1};
     CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+cudaError_t set_pair_attr(const void* k) {
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmem);
+    if (e != cudaSuccess) return e;
+    return prefer_shared(k);
+}
+
+// Pair clusters that fit at once (one CTA per SM, clusters of two).
+cudaError_t max_pair_clusters(const void* k, int* n) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kPairSmem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaOccupancyMaxActiveClusters(n, k, &cfg);
+}
+
+template <int EPI>
+cudaError_t launch_pair(const ace_layer* L, const TcParams& p, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * L->pair_clusters);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kPairSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, k_expert_pair<EPI>, p);
 }
 
 constexpr int kStagesSwap = 8;
@@ -661,7 +926,20 @@ cudaError_t tc_pack_weights(ace_layer* L, const void* w_gate, const void* w_up, 
     return cudaGetLastError();
 }
 
-int tc_token_tile(int T) { return T <= kTcSmallT ? 16 : 128; }
+// Expected retained slots per expert (ratio mode: the requested skip ratio;
+// threshold mode: none skipped) decide the wide-tile kernel: CTA pairs with
+// 256-row tiles once experts average 256 or more slots, else one CTA per
+// 128-row tile.
+bool tc_use_pair(const ace_layer* L, int T, ace_skip_ctl ctl) {
+    if (T <= kTcSmallT || L->pair_clusters < 1) return false;
+    const ace_layer_desc& D = L->desc;
+    const double keep = ctl.mode == ACE_SKIP_RATIO ? 1.0 - (double)ctl.value : 1.0;
+    return (double)T * D.top_k * keep >= 256.0 * D.n_experts;
+}
+
+int tc_token_tile(const ace_layer* L, int T, ace_skip_ctl ctl) {
+    return T <= kTcSmallT ? 16 : (tc_use_pair(L, T, ctl) ? 256 : 128);
+}
 
 bool tc_supported(const ace_layer* L) {
     const ace_layer_desc& D = L->desc;
@@ -677,6 +955,12 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = set_attr<false, 0>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 1>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 2>()) != cudaSuccess) return e;
+    if ((e = set_pair_attr((const void*)k_expert_pair<0>)) != cudaSuccess) return e;
+    if ((e = set_pair_attr((const void*)k_expert_pair<1>)) != cudaSuccess) return e;
+    int c0 = 0, c1 = 0;
+    if ((e = max_pair_clusters((const void*)k_expert_pair<0>, &c0)) != cudaSuccess) return e;
+    if ((e = max_pair_clusters((const void*)k_expert_pair<1>, &c1)) != cudaSuccess) return e;
+    L->pair_clusters = c0 < c1 ? c0 : c1;
     if ((e = prefer_shared(k_gather_rows)) != cudaSuccess) return e;
 
     // row counts as allocated at create time (padded to at least 256 rows)
@@ -691,6 +975,9 @@ cudaError_t tc_init(ace_layer* L) {
     // weight maps: W_gu [N * 2m, d] and W_down [N * d, m]
     // router: h [Tmax, d] in 128-row boxes, W_r [N, d] in 256-row boxes
     if ((e = make_map(&L->tcm.h_rows_big, L->ws.h, h_rows, d, 128)) != cudaSuccess) return e;
+    // tiled expert weights as rows of 64 bf16 (16 KB tiles = 128 rows), copied verbatim
+    if ((e = make_map(&L->tcm.wgu_rows, L->w_gu, n * 2 * m * d / 64, 64, 128, false)) != cudaSuccess) return e;
+    if ((e = make_map(&L->tcm.wd_rows, L->w_down, n * d * m / 64, 64, 128, false)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.tok1_small, L->ws.h_perm, rows, d, 16)) != cudaSuccess) return e;
     if ((e = make_map(&L->tcm.w_router_big, L->router_w, n_pad, d, 256)) != cudaSuccess) return e;
     return cudaSuccess;
@@ -732,7 +1019,9 @@ cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s) {
     return launch_gemm<false, 2>(L, p, s);
 }
 
-cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, cudaStream_t s, cudaEvent_t* ev) {
+cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, ace_skip_ctl ctl, cudaStream_t s,
+                              cudaEvent_t* ev) {
+    const bool pair = tc_use_pair(L, T, ctl);
     const __nv_bfloat16* resid = L->desc.add_residual ? static_cast<const __nv_bfloat16*>(x) : nullptr;
     const ace_layer_desc& D = L->desc;
     const Workspace& W = L->ws;
@@ -764,7 +1053,14 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     p1.w_tiles = 2 * m / (small ? 128 : 256);
     p1.out_ld = m;
     p1.err = W.err;
-    e = small ? launch_gemm<true, 0>(L, p1, s) : launch_gemm<false, 0>(L, p1, s);
+    if (pair) {
+        TcParams q = p1;
+        q.tm_w = L->tcm.wgu_rows;
+        q.w_tiles = 2 * m / 256;
+        e = launch_pair<0>(L, q, s);
+    } else {
+        e = small ? launch_gemm<true, 0>(L, p1, s) : launch_gemm<false, 0>(L, p1, s);
+    }
     if (e != cudaSuccess) return e;
     if (ev) ace::record_stage(ev[1], s);
     TcParams p2 = p1;
@@ -778,7 +1074,14 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     p2.w_rows = d;
     p2.w_tiles = d / (small ? 128 : 256);
     p2.out_ld = d;
-    e = small ? launch_gemm<true, 1>(L, p2, s) : launch_gemm<false, 1>(L, p2, s);
+    if (pair) {
+        TcParams q = p2;
+        q.tm_w = L->tcm.wd_rows;
+        q.w_tiles = d / 256;
+        e = launch_pair<1>(L, q, s);
+    } else {
+        e = small ? launch_gemm<true, 1>(L, p2, s) : launch_gemm<false, 1>(L, p2, s);
+    }
     if (e != cudaSuccess) return e;
     if (ev) ace::record_stage(ev[2], s);
     const long long nthreads = (long long)T * (d / 8);

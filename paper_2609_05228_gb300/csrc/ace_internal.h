@@ -81,6 +81,7 @@ struct TcMaps {
     CUtensorMap tok1_small, tok1_big;   // h_perm, boxes of 16 / 128 rows
     CUtensorMap tok2_small, tok2_big;   // act_bf16, boxes of 16 / 128 rows
     CUtensorMap h_rows_big, w_router_big;   // router GEMM (batches over 256 tokens): 128-row / 256-row boxes
+    CUtensorMap wgu_rows, wd_rows;      // tiled W_gu / W_down as 128-B rows (CTA-pair kernel), no swizzle
 };
 
 }  // namespace ace
@@ -89,6 +90,7 @@ struct ace_layer {
     ace_layer_desc desc;
     int device = 0;
     int num_sms = 0;
+    int pair_clusters = 0;       // CTA pairs of the wide-tile expert kernel resident at once
     size_t elem = 2;             // bytes per element of dtype
     // layer-owned weights
     void* router_w = nullptr;    // [N, d]
@@ -202,12 +204,14 @@ constexpr int kNumStages = 7;
 
 // ---- tensor-core expert path (ace_expert_tc.cu) ----
 bool tc_supported(const ace_layer* L);
-int tc_token_tile(int T);
+int tc_token_tile(const ace_layer* L, int T, ace_skip_ctl ctl);
+bool tc_use_pair(const ace_layer* L, int T, ace_skip_ctl ctl);
 cudaError_t tc_init(ace_layer* L);
 // Packs W_gate / W_up / W_down into the tiled, pre-swizzled layouts of w_gu and w_down.
 cudaError_t tc_pack_weights(ace_layer* L, const void* w_gate, const void* w_up, const void* w_down, cudaStream_t s);
 // ev (nullable): recorded after gather, after gate/up, after down, after combine.
-cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, cudaStream_t s, cudaEvent_t* ev);
+cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, ace_skip_ctl ctl, cudaStream_t s,
+                              cudaEvent_t* ev);
 // Router logits on the tensor cores (T > kTcSmallT): z = (h W_r^T + b) / temp.
 // With router_splits(L, T) > 1 it writes raw partial sums [splits, T, N] into
 // ws.act_bf16 and the top-k kernel forms the logits.

@@ -1287,7 +1287,7 @@ cudaError_t launch_route_fused(const ace_layer* L, const void* x, const float* l
     a.slot_pos = W.slot_pos;
     a.meta = W.meta;
     a.err = W.err;
-    a.tok_tile = L->tc ? tc_token_tile(T) : 0;
+    a.tok_tile = L->tc ? tc_token_tile(L, T, ctl) : 0;
     a.tt_off = W.tt_off;
     a.tt_tab = W.tt_tab;
     a.tile_cnt = W.tile_cnt;
@@ -1331,7 +1331,7 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     bool need_select;
     const int m_q = select_mq(L, T, ctl, &tau, &need_select);
     const int mode = need_select ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
-    const int tok_tile = L->tc ? tc_token_tile(T) : 0;
+    const int tok_tile = L->tc ? tc_token_tile(L, T, ctl) : 0;
     if (T <= kSmallT) return launch_route_fused(L, nullptr, logits, T, ctl, s);
     const int blocks = cdiv(T, kTopkWarps);
     cudaError_t e;
