@@ -9,6 +9,7 @@ the same seeded inputs.
   within rounding distance of a decision boundary (top-k logit gap and
   |c - tau|); those boundary tokens are counted and must stay a minority.
 """
+import dataclasses
 import math
 
 import numpy as np
@@ -175,6 +176,9 @@ def _layer(kind):
             spec, seed = synth.spec_qwen(), 0
         elif kind == "qwen_zipf":
             spec, seed = synth.spec_qwen(zipf=True), 0
+        elif kind == "qwen_temp":
+            # router temperature != 1 and m_min = 2 (Algorithm 4's restore)
+            spec, seed = dataclasses.replace(synth.spec_qwen(zipf=True), router_temp=1.3, min_active=2), 7
         else:
             raise KeyError(kind)
         w = synth.make_layer(spec, seed)
@@ -184,7 +188,7 @@ def _layer(kind):
     return _LAYERS[kind]
 
 
-def _clear_tokens(dec, z_ref, k, dz, dc):
+def _clear_tokens(dec, z_ref, k, dz, dc, m_min=1):
     """Tokens whose top-k set, top-1 and every skip decision sit farther from
     a boundary than the GPU's rounding can move them. bf16 h rounding moves a
     logit by about 1e-3 (std) and c by about 1.5e-3 relative, so the bf16
@@ -196,13 +200,21 @@ def _clear_tokens(dec, z_ref, k, dz, dc):
     if dec["m_q"] is not None and 0 < dec["m_q"] and not math.isinf(tau):
         # ratio mode: tau is the (m+1)-th smallest candidate score itself, so
         # the boundary lies between the m-th and (m+1)-th candidate scores
-        prot = O.protected_mask(dec["c"], 1)
+        prot = O.protected_mask(dec["c"], m_min)
         cand = np.sort(dec["c"][~prot])
         tau = 0.5 * (cand[dec["m_q"] - 1] + cand[dec["m_q"]])
     if math.isinf(tau) or tau == 0:
         c_ok = np.ones(z_ref.shape[0], bool)
     else:
         c_ok = (np.abs(dec["c"] - tau) > dc * tau).all(axis=1)
+    if m_min > 1:
+        # which slots are protected (ratio mode) or restored (Algorithm 4) is
+        # decided by ranking c among the non-top-1 slots: keep tokens whose
+        # leading m_min such scores are separated by more than the margin
+        cs = np.sort(dec["c"][:, 1:], axis=1)[:, ::-1]
+        lead = cs[:, : min(m_min, cs.shape[1])]
+        gaps = lead[:, :-1] - cs[:, 1 : lead.shape[1]]
+        c_ok &= (gaps > dc * cs[:, :1]).all(axis=1)
     return (gap_k > dz) & (gap_1 > dz) & c_ok
 
 
@@ -229,6 +241,7 @@ FORWARD_CASES = [
     ("qwen", 64, "ratio", 0.0), ("qwen", 64, "ratio", 0.25), ("qwen", 64, "ratio", 0.5),
     ("qwen", 17, "threshold", 0.11), ("qwen", 129, "ratio", 0.5), ("qwen", 1000, "ratio", 0.625),
     ("qwen_zipf", 4096, "ratio", 0.0), ("qwen_zipf", 4096, "ratio", 0.5),
+    ("qwen_temp", 64, "ratio", 0.5), ("qwen_temp", 600, "ratio", 0.625), ("qwen_temp", 48, "threshold", 0.1),
 ]
 
 
@@ -237,7 +250,7 @@ def test_forward_parity(kind, T, mode, val):
     w, spec, x, y_gpu, y_ref, dec, z_ref, (skip, ids, gh, tau, R) = _run_layer(kind, T, mode, val)
     k = spec.top_k
     margin = 1e-4 if spec.dtype == "f32" else None
-    clear = _clear_tokens(dec, z_ref, k, margin or 6e-3, margin or 8e-3)
+    clear = _clear_tokens(dec, z_ref, k, margin or 6e-3, margin or 8e-3, spec.min_active)
     assert clear.mean() >= 0.4, clear.mean()
     # decisions agree on every clear token (compared per expert id)
     for t in np.nonzero(clear)[0]:
@@ -246,7 +259,7 @@ def test_forward_parity(kind, T, mode, val):
         assert gpu == ref, t
     if mode == "ratio":
         n_all = T * k
-        m_q = min(O.llround_pos(float(np.float32(val)) * n_all), T * (k - 1))
+        m_q = min(O.llround_pos(float(np.float32(val)) * n_all), T * (k - max(spec.min_active, 1)))
         assert n_all - R == m_q
     yr, yg = y_ref[clear], y_gpu[clear]
     rel = np.linalg.norm(yg - yr) / max(np.linalg.norm(yr), 1e-30)
