@@ -42,7 +42,7 @@ void free_layer(ace_layer* L) {
     void* ptrs[] = {L->router_w, L->router_b, L->w_gate, L->w_up, L->w_gu, L->w_down, L->gamma, L->a_gsp,
                     L->a_rcr, L->ws.h, L->ws.logits, L->ws.ids, L->ws.gates, L->ws.cval, L->ws.keys, L->ws.skip,
                     L->ws.ghat, L->ws.tau, L->ws.chunk_counts, L->ws.offsets, L->ws.dlist, L->ws.perm,
-                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.act_bf16, L->ws.tt_off, L->ws.tt_tab, L->ws.tile_cnt, L->ws.sel_hist, L->ws.sel_cand, L->ws.err, L->ws.x_stage, L->ws.out_stage};
+                    L->ws.slot_pos, L->ws.meta, L->ws.act, L->ws.yslot, L->ws.h_perm, L->ws.act_bf16, L->ws.tt_off, L->ws.tt_tab, L->ws.dec_done, L->ws.tile_cnt, L->ws.sel_hist, L->ws.sel_cand, L->ws.err, L->ws.x_stage, L->ws.out_stage};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     for (cudaEvent_t e : L->ev)
@@ -197,6 +197,7 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
         ALLOC(W.act_bf16, slots * m * E);
         ALLOC(W.tt_off, (n + 1) * sizeof(int32_t));
         ALLOC(W.tt_tab, (n + slots / 16 + 1) * sizeof(int4));
+        ALLOC(W.dec_done, (n + slots / 16 + 1) * sizeof(int32_t));
     } else {
         ALLOC(W.act, slots * m * sizeof(float));
     }
@@ -316,7 +317,7 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
         ACE_CUDA(ace::launch_experts_gemv(L, x, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
     }
     L->n_stages = ev ? ace::kNumStages : 0;
-    L->last_launches = (small ? 1 : 2 + ace::route_launch_count(L, T, ctl)) + (L->tc ? 4 : 3);
+    L->last_launches = (small ? 1 : 2 + ace::route_launch_count(L, T, ctl)) + (L->tc ? (small ? 3 : 4) : 3);
     return ACE_OK;
 }
 

@@ -536,6 +536,247 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
 }
 
 
+
+// ---------------------------------------------------------------- decode: both GEMMs in one launch
+//
+// For batches of at most 256 tokens (16-token tiles, weights as the 128-row
+// MMA operand) gate/up and down run in one persistent launch, so the SMs that
+// finish their gate/up tiles start on down tiles instead of idling through
+// the tail of a separate launch. Tiles 0 .. n1-1 are gate/up (token-tile
+// major, so one token tile's gate/up tiles run together), n1 .. are down. A
+// down tile's weights load at once; its act rows load after done[tt] shows
+// that every gate/up epilogue warp of that token tile has written its act
+// columns (release: store, proxy fence, fence, atomic; acquire: bounded spin
+// on an acquiring load, then a proxy fence before the TMA). Each CTA takes
+// its tiles in index order and issues all its gate/up tiles before any down
+// tile can wait, so the waits cannot form a cycle.
+struct DecParams {
+    CUtensorMap tm_h;                   // h_perm rows, 16-row boxes
+    CUtensorMap tm_act;                 // act rows, 16-row boxes
+    const uint8_t* w_gu;                // tiled W_gu
+    const uint8_t* w_down;              // tiled W_down
+    const int4* tt_tab;
+    const int32_t* meta;
+    const int32_t* perm;
+    const float* ghat;
+    __nv_bfloat16* act;                 // [R, m]
+    float* y;                           // [R, d]
+    int* done;                          // [token tiles] gate/up epilogue warps finished (zeroed by the gather)
+    int* err;
+    int d, m, k;
+};
+
+constexpr int kDecStages = 8;
+constexpr int kDecA = 128 * kBK * 2;
+constexpr int kDecB = 16 * kBK * 2;
+constexpr int kDecStage = kDecA + kDecB;
+constexpr int kDecSmem = kDecStages * kDecStage + 1024 + 256;
+
+__device__ __forceinline__ int ld_acquire(const int* p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+struct DecTile {
+    int phase;    // 0 gate/up, 1 down
+    int tt;       // token tile
+    int e, row0, nrows;
+    int wt;       // 128-row weight tile
+    int kblocks;
+};
+
+__device__ __forceinline__ DecTile dec_tile(const DecParams& p, int tile, int n1) {
+    DecTile t;
+    const int wt1 = 2 * p.m / 128, wt2 = p.d / 128;
+    if (tile < n1) {
+        t.phase = 0;
+        t.tt = tile / wt1;
+        t.wt = tile - t.tt * wt1;
+        t.kblocks = p.d / kBK;
+    } else {
+        const int j = tile - n1;
+        t.phase = 1;
+        t.tt = j / wt2;
+        t.wt = j - t.tt * wt2;
+        t.kblocks = p.m / kBK;
+    }
+    const int4 v = p.tt_tab[t.tt];
+    t.e = v.x;
+    t.row0 = v.y;
+    t.nrows = v.z;
+    return t;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_constant__ DecParams p) {
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + kDecStages * kDecStage);
+    uint64_t* empty = full + kDecStages;
+    uint64_t* acc_full = empty + kDecStages;
+    uint64_t* acc_empty = acc_full + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_h)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_act)) : "memory");
+        for (int s = 0; s < kDecStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&acc_full[a], 1);
+            mbar_init(&acc_empty[a], 4);
+        }
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(32u));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    pdl_wait();
+    const int ntt = p.meta[kMetaTokTiles];
+    const int wt1 = 2 * p.m / 128;
+    const int n1 = ntt * wt1, n_tiles = n1 + ntt * (p.d / 128);
+    const int done_target = 4 * wt1;
+
+    if (warp == 0) {
+        // ------------------------------------------------ producer
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            long long issued = 0;
+            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+                const DecTile t = dec_tile(p, tile, n1);
+                if (t.phase == 1) {
+                    // the token tile's act rows: every gate/up epilogue warp has written
+                    if (ld_acquire(p.done + t.tt) < done_target) {
+                        const long long t0 = clock64();
+                        while (ld_acquire(p.done + t.tt) < done_target) {
+                            if (clock64() - t0 > kSpinCycles || *abort_flag) {
+                                atomicOr(p.err, kErrTimeout);
+                                ok = false;
+                                break;
+                            }
+                        }
+                    }
+                    if (!ok) break;
+                    fence_proxy_async_global();
+                }
+                const uint8_t* wbase = t.phase == 0 ? p.w_gu : p.w_down;
+                const int wrows = t.phase == 0 ? 2 * p.m : p.d;
+                for (int kb = 0; kb < t.kblocks; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                    unsigned char* sa = smem + stage * kDecStage;
+                    mbar_expect_tx(&full[stage], kDecStage);
+                    bulk_g2s(sa, wbase + (((size_t)t.e * (wrows / 128) + t.wt) * t.kblocks + kb) * 16384, 16384,
+                             &full[stage]);
+                    tma_load_2d(sa + kDecA, t.phase == 0 ? &p.tm_h : &p.tm_act, &full[stage], kb * kBK, t.row0);
+                    ++issued;
+                    if (++stage == kDecStages) { stage = 0; phase ^= 1u; }
+                }
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                for (long long f = issued - 1; f >= 0 && f >= issued - kDecStages; --f) {
+                    if (!mbar_wait(&full[f % kDecStages], (uint32_t)((f / kDecStages) & 1), p.err)) break;
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16(128, 16);
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+                const DecTile t = dec_tile(p, tile, n1);
+                if (!mbar_wait(&acc_empty[acc], acc_phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 16);
+                for (int kb = 0; kb < t.kblocks; ++kb) {
+                    if (!mbar_wait(&full[stage], phase, p.err) || *abort_flag) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t a_addr = smem_u32(smem + stage * kDecStage);
+                    const uint32_t b_addr = a_addr + kDecA;
+#pragma unroll
+                    for (int kk = 0; kk < kBK / kUmmaK; ++kk)
+                        mma_bf16(d_tmem, smem_desc_sw128(a_addr + kk * kUmmaK * 2), smem_desc_sw128(b_addr + kk * kUmmaK * 2),
+                                 idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                    mma_commit(&empty[stage]);
+                    if (++stage == kDecStages) { stage = 0; phase ^= 1u; }
+                }
+                if (!ok) break;
+                mma_commit(&acc_full[acc]);
+                if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+            }
+            if (!ok) *abort_flag = 1;
+        }
+    } else {
+        // ------------------------------------------------ epilogue (warps 2..5)
+        const int quad = warp & 3;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+            bool ok = true;
+            if (lane == 0) ok = mbar_wait(&acc_full[acc], acc_phase, p.err) && !*abort_flag;
+            ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+            if (!ok) break;
+            tc_fence_after();
+            const DecTile t = dec_tile(p, tile, n1);
+            uint32_t r[16];
+            tmem_ld16(tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * 16), r);
+            tmem_ld_wait();
+            if (t.phase == 0) {
+                // rows: 16 gate then 16 up of FFN block (4 * wt + quad); SwiGLU into act
+                const int j = (t.wt * 4 + quad) * 16 + (lane & 15);
+#pragma unroll
+                for (int c = 0; c < 16; ++c) {
+                    const float v = __uint_as_float(r[c]);
+                    const float u = __shfl_xor_sync(0xffffffffu, v, 16);
+                    if (lane < 16 && c < t.nrows)
+                        p.act[(size_t)(t.row0 + c) * p.m + j] = __float2bfloat16_rn(silu(v) * u);
+                }
+                fence_proxy_async_global();          // act is read by the TMA of down tiles
+                __threadfence();
+                __syncwarp();
+                if (lane == 0) atomicAdd(p.done + t.tt, 1);
+            } else {
+                const int col = t.wt * 128 + quad * 32 + lane;
+#pragma unroll
+                for (int c = 0; c < 16; ++c) {
+                    if (c < t.nrows)
+                        p.y[(size_t)(t.row0 + c) * p.d + col] = p.ghat[p.perm[t.row0 + c]] * __uint_as_float(r[c]);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acc_empty[acc]);
+            if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    pdl_trigger();
+    tc_fence_after();
+    if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(32u));
+}
+
 // ---------------------------------------------------------------- CTA-pair kernel
 //
 // Wide tiles of 256 token rows x 256 weight rows for batches whose experts
@@ -698,8 +939,10 @@ __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __rest
                                                      const int32_t* __restrict__ perm,
                                                      const int32_t* __restrict__ meta,
                                                      __nv_bfloat16* __restrict__ h_perm,
-                                                     int d, int k) {
+                                                     int d, int k, int* __restrict__ done) {
     pdl_wait();
+    if (done && blockIdx.x == 0)                 // the decode kernel's per-token-tile counters
+        for (int i = threadIdx.x; i < meta[kMetaTokTiles]; i += blockDim.x) done[i] = 0;
     const int R = meta[kMetaRetained];
     const int nvec = d / 8;
     const int lane = threadIdx.x & 31;
@@ -955,6 +1198,9 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = set_attr<false, 0>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 1>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 2>()) != cudaSuccess) return e;
+    if ((e = cudaFuncSetAttribute(k_expert_decode, cudaFuncAttributeMaxDynamicSharedMemorySize, kDecSmem)) != cudaSuccess)
+        return e;
+    if ((e = prefer_shared(k_expert_decode)) != cudaSuccess) return e;
     if ((e = set_pair_attr((const void*)k_expert_pair<0>)) != cudaSuccess) return e;
     if ((e = set_pair_attr((const void*)k_expert_pair<1>)) != cudaSuccess) return e;
     int c0 = 0, c1 = 0;
@@ -1032,8 +1278,43 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     // loading them one row per TMA box from h instead measured slower
     {
         e = launch_pdl(k_gather_rows, dim3(L->num_sms * 4), dim3(256), 0, s, (const __nv_bfloat16*)W.h,
-                       (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k);
+                       (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k,
+                       small ? W.dec_done : (int*)nullptr);
         if (e != cudaSuccess) return e;
+    }
+    if (small) {
+        // both GEMMs in one persistent launch (k_expert_decode), then the combine
+        if (ev) ace::record_stage(ev[0], s);
+        DecParams q{};
+        q.tm_h = L->tcm.tok1_small;
+        q.tm_act = L->tcm.tok2_small;
+        q.w_gu = static_cast<const uint8_t*>(L->w_gu);
+        q.w_down = static_cast<const uint8_t*>(L->w_down);
+        q.tt_tab = W.tt_tab;
+        q.meta = W.meta;
+        q.perm = W.perm;
+        q.ghat = W.ghat;
+        q.act = static_cast<__nv_bfloat16*>(W.act_bf16);
+        q.y = W.yslot;
+        q.done = W.dec_done;
+        q.err = W.err;
+        q.d = d;
+        q.m = m;
+        q.k = k;
+        e = launch_pdl(k_expert_decode, dim3(L->num_sms), dim3(kThreads), kDecSmem, s, q);
+        if (e != cudaSuccess) return e;
+        if (ev) {                           // gate/up and down share one launch: the down stage reads 0
+            ace::record_stage(ev[1], s);
+            ace::record_stage(ev[2], s);
+        }
+        const long long nthreads = (long long)T * (d / 8);
+        const dim3 grid((unsigned)((nthreads + 255) / 256));
+        e = k <= 8 ? launch_pdl(k_combine_bf16<float, 8>, grid, dim3(256), 0, s, (const float*)W.yslot,
+                                (const int32_t*)W.slot_pos, resid, (__nv_bfloat16*)out, T, d, k)
+                   : launch_pdl(k_combine_bf16<float, kMaxTopK>, grid, dim3(256), 0, s, (const float*)W.yslot,
+                                (const int32_t*)W.slot_pos, resid, (__nv_bfloat16*)out, T, d, k);
+        if (ev) ace::record_stage(ev[3], s);
+        return e;
     }
     if (ev) ace::record_stage(ev[0], s);
     TcParams p1{};

@@ -67,6 +67,7 @@ struct Workspace {
                                  // batches over 256 tokens GEMM 2 then writes its bf16 y rows over it
     void* act_bf16 = nullptr;    // [Tmax*k, m] bf16 (tensor path)
     int32_t* tt_off = nullptr;   // [N+1] token-tile prefix over distinct experts
+    int32_t* dec_done = nullptr; // [tiles of tt_tab] gate/up warps finished per token tile (decode kernel)
     int4* tt_tab = nullptr;      // [N + Tmax*k/16 + 1] token tiles: (expert, first row, rows, 0)
     int32_t* tile_cnt = nullptr; // [Tmax/8 + 1] per-token-tile tickets of the fused small-T kernel
     int32_t* sel_hist = nullptr; // [4096 + 1024] digit histograms of the threshold keys (kept zero between calls)
