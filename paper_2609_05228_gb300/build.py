@@ -1,4 +1,5 @@
-"""Builds libace.so in-tree (paper_2609_05228_gb300/_lib/) with nvcc for sm_103a.
+"""Builds libace.so in-tree (paper_2609_05228_gb300/_lib/) with nvcc for sm_103a,
+and libace_offline.so (the host-only offline table tool) with g++.
 
 Each .cu file under csrc/ is compiled in parallel, then linked into one
 shared library (CUDA runtime linked statically). Run as
@@ -37,6 +38,23 @@ def sources() -> list[str]:
     return sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cu"))
 
 
+OFFLINE_SRC = os.path.join(PKG, "csrc_host", "ace_offline.cpp")
+OFFLINE_LIB = os.path.join(LIBDIR, "libace_offline.so")
+
+
+def build_offline() -> str:
+    """libace_offline.so: the host-only offline GSP/RCR tool (plain C++, no CUDA)."""
+    os.makedirs(LIBDIR, exist_ok=True)
+    cxx = shutil.which("g++") or "g++"
+    tmp = OFFLINE_LIB + ".tmp"
+    cmd = [cxx, "-O3", "-std=c++17", "-fPIC", "-shared", "-pthread", "-I", INCLUDE, "-o", tmp, OFFLINE_SRC]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"g++ failed for {OFFLINE_SRC}:\n{r.stdout}\n{r.stderr}")
+    os.replace(tmp, OFFLINE_LIB)
+    return OFFLINE_LIB
+
+
 def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
     os.makedirs(OBJDIR, exist_ok=True)
     cc = nvcc()
@@ -53,8 +71,10 @@ def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
         return obj
 
     srcs = sources()
-    with ThreadPoolExecutor(max(1, min(len(srcs), os.cpu_count() or 1))) as ex:
+    with ThreadPoolExecutor(max(1, min(len(srcs) + 1, os.cpu_count() or 1))) as ex:
+        host = ex.submit(build_offline)
         objs = list(ex.map(compile_one, srcs))
+        host.result()
     tmp = LIBPATH + ".tmp"
     cmd = [cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs]
     r = subprocess.run(cmd, capture_output=True, text=True)

@@ -1,83 +1,82 @@
 """Offline GSP and RCR tables (ACE Algorithms 2 and 3), host CPU.
 
 The tables are computed once per layer from the frozen weights and handed to
-ace_layer_create(). No calibration data is involved.
-
-GSP (§3.1, Eqs. gsp_up_path .. gsp_layer_normalization). With the paper's
-row-vector convention G = Gamma W_gate and U = Gamma W_up (d x m) and
-W_down (m x d):
-    a_up   = ||U||_F * ||G W_down||_F
-    a_gate = ||G||_F * ||U W_down||_F
-    a~     = sqrt(a_up * a_gate),   A(e) = a~_e / (mean_j a~_j + eps).
-The products G W_down are d x d; their Frobenius norms are taken through
-m x m Gram matrices instead, ||G W||_F^2 = <G^T G, W W^T>_F, which costs
-3 d m^2 multiply-adds per expert instead of 2 d^2 m.
-
-RCR (§3.2, Eqs. rcr_centered_router .. rcr_layer_normalization): centred
-router rows w~_e, prototypes q_e = w~_e / (RMS(w~_e) + eps) (rho = 1),
-a~_e = ||f_e(q_e)||_2 / (||q_e||_2 + eps), A(e) = a~_e / (mean a~ + eps).
-f is applied to q directly; apply_gamma=True scales q by gamma first.
+ace_layer_create(). No calibration data is involved. The computation is the
+host-only C++ library libace_offline.so (include/ace_offline.h: Gram-route
+GSP, prototype-forward RCR, fp64, one expert per thread); this module is its
+ctypes binding, with the C names.
 
 Weights are nn.Linear-shaped: w_gate, w_up [N, m, d]; w_down [N, d, m];
-bf16 arrays are uint16 bit patterns.
+bf16 arrays are uint16 bit patterns (passed as they are), others fp32.
 """
 from __future__ import annotations
 
+import ctypes
+import os
+
 import numpy as np
 
+from . import ace
 
-def _f32(a: np.ndarray) -> np.ndarray:
+LIBPATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libace_offline.so")
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIBPATH):       # host-only C++: built on first use (g++, a few seconds)
+            from . import build
+            build.build_offline()
+        L = ctypes.CDLL(LIBPATH)
+        L.ace_offline_tables.restype = ctypes.c_int
+        L.ace_offline_tables.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                         ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                         ctypes.c_void_p, ctypes.c_double, ctypes.c_int, ctypes.c_int,
+                                         ctypes.c_void_p, ctypes.c_void_p]
+        _lib = L
+    return _lib
+
+
+def _host(a: np.ndarray, bf16: bool) -> np.ndarray:
     a = np.asarray(a)
-    if a.dtype == np.uint16:
-        return (a.astype(np.uint32) << 16).view(np.float32)
-    return a.astype(np.float32, copy=False)
+    if bf16:
+        if a.dtype != np.uint16:
+            raise TypeError("bf16 weights are uint16 bit patterns")
+        return np.ascontiguousarray(a)
+    return np.ascontiguousarray(a, dtype=np.float32)
 
 
-def gsp_table(gamma, w_gate, w_up, w_down, eps: float = 1e-6) -> np.ndarray:
-    gam2 = _f32(gamma).astype(np.float64) ** 2
-    n = w_gate.shape[0]
-    raw = np.empty(n, dtype=np.float64)
-    for e in range(n):
-        wg = _f32(w_gate[e]).astype(np.float64)          # [m, d]
-        wu = _f32(w_up[e]).astype(np.float64)            # [m, d]
-        wd = _f32(w_down[e]).astype(np.float64)          # [d, m]
-        gram_g = (wg * gam2) @ wg.T                      # G^T G   [m, m]
-        gram_u = (wu * gam2) @ wu.T                      # U^T U   [m, m]
-        gram_d = wd.T @ wd                               # W_d W_d^T (paper W_d = wd.T)
-        fro_g2 = np.trace(gram_g)
-        fro_u2 = np.trace(gram_u)
-        fro_gd2 = float(np.vdot(gram_g, gram_d))
-        fro_ud2 = float(np.vdot(gram_u, gram_d))
-        a_up2 = fro_u2 * max(fro_gd2, 0.0)
-        a_gate2 = fro_g2 * max(fro_ud2, 0.0)
-        raw[e] = (a_up2 * a_gate2) ** 0.25
-    return (raw / (raw.mean() + eps)).astype(np.float32)
-
-
-def rcr_table(router_w, gamma, w_gate, w_up, w_down, eps: float = 1e-6,
-              apply_gamma: bool = False) -> np.ndarray:
-    wr = _f32(router_w).astype(np.float64)
-    n, d = wr.shape
-    centred = wr - wr.mean(axis=0)
-    rms = np.sqrt((centred ** 2).sum(axis=1) / d)
-    protos = centred / (rms + eps)[:, None]
-    raw = np.empty(n, dtype=np.float64)
-    gam = _f32(gamma).astype(np.float64)
-    for e in range(n):
-        q = protos[e]
-        xin = q * gam if apply_gamma else q
-        u = _f32(w_gate[e]).astype(np.float64) @ xin
-        v = _f32(w_up[e]).astype(np.float64) @ xin
-        a = u / (1.0 + np.exp(-u)) * v
-        y = _f32(w_down[e]).astype(np.float64) @ a
-        raw[e] = np.sqrt(y @ y) / (np.sqrt(q @ q) + eps)
-    return (raw / (raw.mean() + eps)).astype(np.float32)
+def ace_offline_tables(gamma, router_w, w_gate, w_up, w_down, eps: float = 1e-6, apply_gamma: bool = False,
+                       n_threads: int = 0):
+    """(A^GSP, A^RCR) float32 [N] from the layer's weights (see ace_offline.h)."""
+    bf16 = np.asarray(w_gate).dtype == np.uint16
+    n, m, d = np.asarray(w_gate).shape
+    arrs = [_host(x, bf16) for x in (gamma, router_w, w_gate, w_up, w_down)]
+    gsp = np.empty(n, np.float32)
+    rcr = np.empty(n, np.float32)
+    st = lib().ace_offline_tables(d, n, m, ace.ACE_BF16 if bf16 else ace.ACE_F32,
+                                  *[x.ctypes.data for x in arrs], float(eps), int(bool(apply_gamma)),
+                                  int(n_threads), gsp.ctypes.data, rcr.ctypes.data)
+    if st != 0:
+        raise ace.AceError(st, "ace_offline_tables failed")
+    return gsp, rcr
 
 
 def tables(layer, eps: float | None = None, apply_gamma: bool = False):
     """(A^GSP, A^RCR) as float32 arrays for a synth.LayerWeights-like layer."""
     e = layer.spec.eps if eps is None else eps
-    a = gsp_table(layer.gamma, layer.w_gate, layer.w_up, layer.w_down, e)
-    r = rcr_table(layer.router_w, layer.gamma, layer.w_gate, layer.w_up, layer.w_down, e,
-                  apply_gamma)
-    return a, r
+    return ace_offline_tables(layer.gamma, layer.router_w, layer.w_gate, layer.w_up, layer.w_down, e, apply_gamma)
+
+
+def gsp_table(gamma, w_gate, w_up, w_down, eps: float = 1e-6) -> np.ndarray:
+    """A^GSP alone (the router is not used by Algorithm 2)."""
+    n, m, d = np.asarray(w_gate).shape
+    bf16 = np.asarray(w_gate).dtype == np.uint16
+    wr = np.zeros((n, d), np.uint16 if bf16 else np.float32)
+    return ace_offline_tables(gamma, wr, w_gate, w_up, w_down, eps)[0]
+
+
+def rcr_table(router_w, gamma, w_gate, w_up, w_down, eps: float = 1e-6, apply_gamma: bool = False) -> np.ndarray:
+    """A^RCR alone."""
+    return ace_offline_tables(gamma, router_w, w_gate, w_up, w_down, eps, apply_gamma)[1]

@@ -34,3 +34,31 @@ def test_offline_tables_bf16_layer():
     a, r = offline.tables(w)
     np.testing.assert_allclose(a, O.gsp_table(w.gamma, w.w_gate, w.w_up, w.w_down, 1e-6), rtol=2e-6)
     np.testing.assert_allclose(r, O.rcr_table(w.router_w, w.gamma, w.w_gate, w.w_up, w.w_down, 1e-6), rtol=2e-6)
+
+
+def test_offline_tables_thread_count_does_not_change_bits():
+    w = _layer(11, d=64, n=9, m=24)
+    a1, r1 = offline.ace_offline_tables(w.gamma, w.router_w, w.w_gate, w.w_up, w.w_down, 1e-6, n_threads=1)
+    a4, r4 = offline.ace_offline_tables(w.gamma, w.router_w, w.w_gate, w.w_up, w.w_down, 1e-6, n_threads=4)
+    assert a1.tobytes() == a4.tobytes() and r1.tobytes() == r4.tobytes()
+
+
+def test_offline_library_boundary():
+    """libace_offline.so exports what include/ace_offline.h declares and
+    rejects bad arguments without writing."""
+    import ctypes
+    import os
+    import re
+    hdr = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "ace_offline.h")
+    text = re.sub(r"/\*.*?\*/", "", open(hdr).read(), flags=re.S)
+    names = sorted(set(re.findall(r"\b(ace_[a-z0-9_]+)\s*\(", text)))
+    L = offline.lib()
+    assert names == ["ace_offline_tables"] and all(hasattr(L, n) for n in names)
+    out = np.full(4, 7.0, np.float32)
+    z = np.zeros(16, np.float32)
+    st = L.ace_offline_tables(0, 4, 4, 1, z.ctypes.data, z.ctypes.data, z.ctypes.data, z.ctypes.data,
+                              z.ctypes.data, ctypes.c_double(1e-6), 0, 1, out.ctypes.data, out.ctypes.data)
+    assert st == 1 and (out == 7.0).all()
+    st = L.ace_offline_tables(4, 4, 4, 1, None, z.ctypes.data, z.ctypes.data, z.ctypes.data,
+                              z.ctypes.data, ctypes.c_double(1e-6), 0, 1, out.ctypes.data, out.ctypes.data)
+    assert st == 1 and (out == 7.0).all()
