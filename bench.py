@@ -183,6 +183,13 @@ class Stack:
             ace.ace_moe_forward(layer.handle, cur, out, T, "ratio", q, stream)
             cur = out
 
+    def forward_threshold(self, x, bufs, T, taus, stream=None):
+        from paper_2609_05228_gb300 import ace
+        cur = x
+        for layer, out, tau in zip(self.layers, bufs, taus):
+            ace.ace_moe_forward(layer.handle, cur, out, T, "threshold", tau, stream)
+            cur = out
+
     def close(self):
         for layer in self.layers:
             layer.close()
@@ -206,6 +213,31 @@ def time_point(torch, model, x, bufs, T, q, steps, warmup, flush):
             flush.zero_()
             g.replay()
         s.synchronize()
+        for i in range(steps):
+            flush.zero_()
+            starts[i].record(s)
+            g.replay()
+            ends[i].record(s)
+    s.synchronize()
+    return [a.elapsed_time(b) for a, b in zip(starts, ends)]
+
+
+def time_threshold(torch, model, x, bufs, T, taus, steps, warmup, flush):
+    """Device time per step (ms) of the graph-replayed forward in threshold mode."""
+    s = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(s):
+        model.forward_threshold(x, bufs, T, taus, s)
+    s.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        model.forward_threshold(x, bufs, T, taus, torch.cuda.current_stream())
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    with torch.cuda.stream(s):
+        for _ in range(warmup):
+            flush.zero_()
+            g.replay()
         for i in range(steps):
             flush.zero_()
             starts[i].record(s)
@@ -304,6 +336,7 @@ def run_ours(args, rank, world, torch, dist):
     if world > 1:
         dist.barrier()
     step_ms = float(np.mean(ms))
+    pct = {f"ms_p{p}": round(float(np.percentile(ms, p)), 5) for p in (10, 50, 90)}
     value, step_ms_max = aggregate(step_ms, T, world, dist, dev)
 
     # the dominant kernel's duration, from events on its own stream
@@ -311,6 +344,28 @@ def run_ours(args, rank, world, torch, dist):
     # skip ratio 0 with the same kernels, for the speedup
     ms0 = time_point(torch, model, x, bufs, T, 0.0, max(10, min(args.steps // 2, 200)), 3, flush)
     t0 = float(np.mean(ms0))
+
+    # threshold mode with tau calibrated on a separate seed-2 batch (App. B.1 mapping)
+    from paper_2609_05228_gb300 import calibrate
+    xc = torch.from_numpy(synth.make_tokens(spec, T, seed=2).view(np.int16)).view(torch.bfloat16).to(dev)
+    taus = [calibrate.calibrate_taus(l, xc, T, [q])[float(q)] for l in model.layers]
+    thr_ms = time_threshold(torch, model, x, bufs, T, taus, max(10, min(args.steps // 2, 200)), 3, flush)
+    model.forward_threshold(x, bufs, T, taus)
+    _, _, _, _, R_thr = ace.ace_last_skip_mask(layer.handle, T, spec.top_k)
+    threshold_point = {"tau_layer0": taus[0], "calibration": "seed-2 batch, ratio mode at q",
+                       "realised_skip_ratio": round((T * spec.top_k - R_thr) / (T * spec.top_k), 6),
+                       "ms_per_step": round(float(np.mean(thr_ms)), 5),
+                       "tokens_per_s": round(T / (float(np.mean(thr_ms)) * 1e-3), 1)}
+
+    # Zipf check: log-log slope of the sorted routed (top-k) slot counts over ranks 1..N/2
+    zipf_slope = None
+    if wl["zipf"]:
+        model.forward(x, bufs, T, q)
+        _, ids_r, _, _, _ = ace.ace_last_skip_mask(layer.handle, T, spec.top_k)
+        cnt = np.sort(np.bincount(ids_r.ravel(), minlength=spec.n_experts))[::-1][: spec.n_experts // 2]
+        ranks = np.arange(1, cnt.size + 1)
+        ok = cnt > 0
+        zipf_slope = round(float(np.polyfit(np.log(ranks[ok]), np.log(cnt[ok]), 1)[0]), 3)
 
     # end to end through the host-buffer C call (pinned buffers, copies included; one layer)
     xp = torch.from_numpy(xh.view(np.int16)).pin_memory()
@@ -375,7 +430,10 @@ def run_ours(args, rank, world, torch, dist):
         "realised_skip_ratio": round((T * spec.top_k - R) / (T * spec.top_k), 6),
         "retained_slots": R,
         "distinct_experts": D,
+        **pct,
         "speedup_vs_q0": round(t0 / step_ms, 4),
+        "threshold_mode": threshold_point,
+        "zipf_slope": zipf_slope,
         "q0_ms_per_step": round(t0, 5),
         "stage_us": stage_avg,
         "wall_s": round(wall, 3),

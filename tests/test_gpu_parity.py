@@ -335,3 +335,21 @@ def test_forward_edge_cases():
     skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, 4, w.spec.top_k)
     assert R == 4 and (skip[:, 0] == 0).all() and (skip[:, 1:] == 1).all()
     ace.ace_layer_sync(layer.handle)
+
+
+@pytest.mark.parametrize("T", [64, 2048])
+def test_calibrated_threshold_reproduces_ratio(T):
+    """App. B.1: a threshold calibrated on a batch in ratio mode, used in
+    threshold mode on that same batch, gives the same mask and g_hat."""
+    from paper_2609_05228_gb300 import calibrate
+    w, layer = _layer("qwen_zipf")
+    x = _dev(synth.make_tokens(w.spec, T, seed=12))
+    taus = calibrate.calibrate_taus(layer, x, T, [0.25, 0.5])
+    out = torch.empty_like(x)
+    for q, tau in taus.items():
+        layer.forward(x, out, T, "ratio", q)
+        ref = ace.ace_last_skip_mask(layer.handle, T, w.spec.top_k)
+        layer.forward(x, out, T, "threshold", tau)
+        got = ace.ace_last_skip_mask(layer.handle, T, w.spec.top_k)
+        assert (got[0] == ref[0]).all() and (got[2].view(np.uint32) == ref[2].view(np.uint32)).all()
+        assert got[4] == ref[4]
