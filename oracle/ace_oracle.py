@@ -11,6 +11,8 @@ Source: ACE, "Adaptive Calibration-Free Expert Skipping for MoE-based LLMs".
     rcr_contribution, rcr_probability; Algorithm 3 (RCR).
   * §3.2 fusion: Eqs. ace_contribution, ace_candidate_intersection;
     Algorithm 4 (online conservative skipping); Eq. ace_sparse_output.
+  * §4.1 Baselines (router-score skipping) and §4.3 ablations (single-view
+    GSP / RCR skipping, Min and Mean fusion): the skip-rule variants.
   * App. B.1 budget-to-threshold mapping (quantile rule for tau(q)).
 
 Two families of functions:
@@ -28,8 +30,11 @@ top-k, a dense brute-force evaluation of all experts on tiny inputs, the
 App. A.2.4 identities (max = intersection, skipped-mass ordering, the exact
 perturbation identity and its 2*alpha*F_max bound), the App. A.2.1 SwiGLU bound,
 router translation invariance (App. A.2.2), the closed-form table means and
-scaling laws, the realised skip count of the quantile rule, and the exp error
-bound against math.exp.
+scaling laws, the realised skip count of the quantile rule, the exp error
+bound against math.exp, and for the skip-rule variants a hand-worked example
+(tests/golden/fusion_worked.json), the nesting Max within Mean within Min,
+Max / Min as intersection / union of the single views, and router-score
+skipping as the GSP view with unit tables.
 
 Readings where the paper is silent (each also listed in the design notes):
   * gates g are the softmax over the top-k logits (softmax over all experts
@@ -52,7 +57,7 @@ import numpy as np
 
 __all__ = [
     "rmsnorm", "router_logits", "topk_gates", "silu", "swiglu_expert",
-    "ace_skip", "protected_mask", "tau_from_ratio", "ace_decide", "moe_forward",
+    "FUSIONS", "fused_contribution", "ace_skip", "protected_mask", "tau_from_ratio", "ace_decide", "moe_forward",
     "moe_stack_forward", "permutation", "gsp_table", "rcr_table",
     "exp32", "decide_fp32", "route_fp32", "tau_from_ratio_fp32", "llround_pos",
     "to_f64",
@@ -123,9 +128,40 @@ def swiglu_expert(x: np.ndarray, w_gate_e: np.ndarray, w_up_e: np.ndarray,
     return (silu(u) * v) @ to_f64(w_down_e).T
 
 
+# Skip rules. "max" is ACE (Eq. ace_contribution). The others are the
+# variants the paper compares against it: "min" and "mean" fusion
+# (§4.3, Tab. fusion_ablation), a single view "gsp" or "rcr" (§4.3,
+# Tab. ablation), and router-score skipping "score" (§4.1 Baselines), which
+# thresholds the routing gate itself.
+FUSIONS = ("max", "min", "mean", "gsp", "rcr", "score")
+
+
+def fused_contribution(p_gsp: np.ndarray, p_rcr: np.ndarray, g: np.ndarray, fusion: str) -> np.ndarray:
+    """Per-slot score c of a skip rule; a slot is a skip candidate when c < tau."""
+    if fusion == "max":
+        return np.maximum(p_gsp, p_rcr)                 # Eq. ace_contribution
+    if fusion == "min":
+        return np.minimum(p_gsp, p_rcr)
+    if fusion == "mean":
+        return (p_gsp + p_rcr) / 2.0
+    if fusion == "gsp":
+        return p_gsp
+    if fusion == "rcr":
+        return p_rcr
+    if fusion == "score":
+        return np.asarray(g, dtype=np.float64)
+    raise ValueError(f"unknown fusion {fusion!r}")
+
+
 def ace_skip(ids: np.ndarray, g: np.ndarray, a_gsp: np.ndarray, a_rcr: np.ndarray,
-             tau: float, m_min: int, eps: float):
+             tau: float, m_min: int, eps: float, fusion: str = "max"):
     """Algorithm 4 (online conservative expert skipping), vectorised over tokens.
+
+    The candidate set of each rule is formed from the per-view sets as the
+    paper describes it: ACE skips a slot only when both views call it
+    dispensable (intersection, Eq. ace_candidate_intersection); "min" when
+    either does (union); "gsp" / "rcr" use one view; "mean" and "score"
+    threshold their score directly.
 
     Returns (skip [T,k] bool, g_hat [T,k] (0 where skipped), c [T,k],
     p_gsp [T,k], p_rcr [T,k]).
@@ -140,10 +176,19 @@ def ace_skip(ids: np.ndarray, g: np.ndarray, a_gsp: np.ndarray, a_rcr: np.ndarra
     z_rcr = s_rcr.sum(axis=1, keepdims=True) + eps
     p_gsp = s_gsp / z_gsp                               # Eq. gsp_probability
     p_rcr = s_rcr / z_rcr                               # Eq. rcr_probability
-    c = np.maximum(p_gsp, p_rcr)                        # Eq. ace_contribution
+    c = fused_contribution(p_gsp, p_rcr, g, fusion)
     low_gsp = p_gsp < tau                               # Eq. gsp_candidate_set
     low_rcr = p_rcr < tau                               # Eq. rcr_candidate_set
-    skip = low_gsp & low_rcr                            # Eq. ace_candidate_intersection
+    if fusion == "max":
+        skip = low_gsp & low_rcr                        # Eq. ace_candidate_intersection
+    elif fusion == "min":
+        skip = low_gsp | low_rcr
+    elif fusion == "gsp":
+        skip = low_gsp
+    elif fusion == "rcr":
+        skip = low_rcr
+    else:
+        skip = c < tau
     top1 = np.argmax(g, axis=1)                         # top-1 by original gate
     skip[np.arange(T), top1] = False
     if m_min > 1:
@@ -215,24 +260,24 @@ def tau_from_ratio(c: np.ndarray, prot: np.ndarray, q: float):
 
 
 def ace_decide(z: np.ndarray, k: int, a_gsp, a_rcr, mode: str, value: float,
-               m_min: int = 1, eps: float = 1e-6) -> dict:
+               m_min: int = 1, eps: float = 1e-6, fusion: str = "max") -> dict:
     """Routing + skipping decision in fp64 from logits z [T, N]."""
     ids, g = topk_gates(z, k)
     # scores at tau = 0 (no skip) give c for the threshold search
-    _, _, c, _, _ = ace_skip(ids, g, a_gsp, a_rcr, 0.0, 1, eps)
+    _, _, c, _, _ = ace_skip(ids, g, a_gsp, a_rcr, 0.0, 1, eps, fusion)
     if mode == "ratio":
         prot = protected_mask(c, m_min)
         tau, m_q, cnt = tau_from_ratio(c, prot, value)
     else:
         tau, m_q, cnt = float(value), None, None
-    skip, g_hat, c, p_gsp, p_rcr = ace_skip(ids, g, a_gsp, a_rcr, tau, m_min, eps)
+    skip, g_hat, c, p_gsp, p_rcr = ace_skip(ids, g, a_gsp, a_rcr, tau, m_min, eps, fusion)
     return dict(ids=ids, g=g, skip=skip, g_hat=g_hat, c=c, p_gsp=p_gsp, p_rcr=p_rcr,
                 tau=tau, m_q=m_q, count=cnt)
 
 
 def moe_forward(x: np.ndarray, w, mode: str = "threshold", value: float = 0.0,
                 decision: dict | None = None, return_decision: bool = False,
-                tokens: np.ndarray | None = None):
+                tokens: np.ndarray | None = None, fusion: str = "max"):
     """ACE MoE layer output y_t = sum_{i in I_t} g_hat_i f_{e_i}(x_t)
     (Eq. ace_sparse_output; Algorithm 1 online loop for one layer), fp64.
 
@@ -248,7 +293,7 @@ def moe_forward(x: np.ndarray, w, mode: str = "threshold", value: float = 0.0,
     if decision is None:
         z = router_logits(h, w.router_w, w.router_b, spec.router_temp)
         decision = ace_decide(z, spec.top_k, w.extra["a_gsp"], w.extra["a_rcr"], mode,
-                              value, spec.min_active, spec.eps)
+                              value, spec.min_active, spec.eps, fusion)
     ids, skip, g_hat = decision["ids"], decision["skip"], decision["g_hat"]
     rows = np.arange(h.shape[0]) if tokens is None else np.asarray(tokens)
     hs, ids_s, skip_s, gh_s = h[rows], ids[rows], skip[rows], g_hat[rows]
@@ -390,7 +435,7 @@ def route_fp32(z: np.ndarray, k: int):
     return ids.astype(np.int32), g
 
 
-def _scores_fp32(ids, g, a_gsp, a_rcr, eps32):
+def _scores_fp32(ids, g, a_gsp, a_rcr, eps32, fusion="max"):
     k = g.shape[1]
     sg = (g * a_gsp[ids]).astype(np.float32)
     sr = (g * a_rcr[ids]).astype(np.float32)
@@ -403,7 +448,21 @@ def _scores_fp32(ids, g, a_gsp, a_rcr, eps32):
     zr = (zr + eps32).astype(np.float32)
     pg = (sg / zg[:, None]).astype(np.float32)
     pr = (sr / zr[:, None]).astype(np.float32)
-    return np.maximum(pg, pr).astype(np.float32), pg, pr
+    if fusion == "max":
+        c = np.maximum(pg, pr)
+    elif fusion == "min":
+        c = np.minimum(pg, pr)
+    elif fusion == "mean":
+        c = (pg + pr).astype(np.float32) * np.float32(0.5)
+    elif fusion == "gsp":
+        c = pg
+    elif fusion == "rcr":
+        c = pr
+    elif fusion == "score":
+        c = g
+    else:
+        raise ValueError(f"unknown fusion {fusion!r}")
+    return np.asarray(c, dtype=np.float32), pg, pr
 
 
 def _protected_fp32(c: np.ndarray, m_min: int) -> np.ndarray:
@@ -440,12 +499,13 @@ def tau_from_ratio_fp32(c: np.ndarray, prot: np.ndarray, q: float):
 
 
 def decide_fp32(ids: np.ndarray, g: np.ndarray, a_gsp, a_rcr, mode: str, value: float,
-                m_min: int = 1, eps: float = 1e-6) -> dict:
+                m_min: int = 1, eps: float = 1e-6, fusion: str = "max") -> dict:
     """Algorithm 4 in the fixed float32 operation order, from rank-ordered
     (ids, g). tau: the given float32 threshold, or tau_from_ratio_fp32.
 
     Order: s = g * A[e]; Z = (sum in rank order) + eps; p = s / Z;
-    c = max(p_gsp, p_rcr); skip = rank != 0 and c < tau; minimum-active
+    c = max(p_gsp, p_rcr) (other rules: min, (p_gsp + p_rcr) * 0.5, p_gsp,
+    p_rcr, or g); skip = rank != 0 and c < tau; minimum-active
     restore in c-descending order (lower rank first on ties);
     Z_gate = (sum of kept g in rank order) + eps; g_hat = g / Z_gate.
     """
@@ -454,7 +514,7 @@ def decide_fp32(ids: np.ndarray, g: np.ndarray, a_gsp, a_rcr, mode: str, value: 
     eps32 = np.float32(eps)
     a_gsp = np.asarray(a_gsp, dtype=np.float32)
     a_rcr = np.asarray(a_rcr, dtype=np.float32)
-    c, pg, pr = _scores_fp32(ids, g, a_gsp, a_rcr, eps32)
+    c, pg, pr = _scores_fp32(ids, g, a_gsp, a_rcr, eps32, fusion)
     if mode == "ratio":
         prot = _protected_fp32(c, m_min)
         tau, m_q, cnt = tau_from_ratio_fp32(c, prot, value)

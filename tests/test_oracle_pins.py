@@ -204,6 +204,109 @@ def test_skip_requires_both_views_and_mass_ordering():
     assert skip.any()
 
 
+# ---------------------------------------------------------------- skip-rule variants
+
+
+@pytest.mark.parametrize("fp32", [False, True])
+def test_fusion_worked_example(fp32):
+    ex = _load("fusion_worked.json")
+    g = np.array([ex["g"]], dtype=np.float32 if fp32 else np.float64)
+    ids = np.array([ex["ids"]], dtype=np.int32)
+    for case in ex["cases"]:
+        fu = case["fusion"]
+        if fp32:
+            d = O.decide_fp32(ids, g, ex["a_gsp"], ex["a_rcr"], "threshold", case["tau"], case["m_min"],
+                              ex["eps"], fusion=fu)
+            skip, g_hat, c = d["skip"], d["g_hat"], d["c"]
+            np.testing.assert_allclose(c[0], ex["c"][fu], rtol=3e-7)
+        else:
+            skip, g_hat, c, _, _ = O.ace_skip(ids, g, np.array(ex["a_gsp"]), np.array(ex["a_rcr"]),
+                                              case["tau"], case["m_min"], ex["eps"], fu)
+            np.testing.assert_allclose(c[0], ex["c"][fu], rtol=1e-15)
+        assert skip[0].astype(int).tolist() == case["skip"], case
+        kept = 1 - np.array(case["skip"])
+        want = np.array(ex["g"]) * kept / float(np.dot(ex["g"], kept))
+        np.testing.assert_allclose(g_hat[0], want, rtol=3e-7 if fp32 else 1e-15, atol=0)
+
+
+def _random_route(seed, T=500, N=24, k=6):
+    rng = np.random.Generator(np.random.PCG64(seed))
+    z = rng.standard_normal((T, N))
+    ids, g = O.topk_gates(z, k)
+    a_gsp = np.abs(1 + 0.5 * rng.standard_normal(N))
+    a_rcr = np.abs(1 + 0.5 * rng.standard_normal(N))
+    return ids, g, a_gsp, a_rcr
+
+
+def test_fusion_candidate_sets_nest():
+    """min(p) <= mean(p) <= max(p) slot by slot, so at one tau the skip sets
+    nest: Max (intersection) within Mean within Min (union); each single
+    view lies between intersection and union."""
+    ids, g, a_gsp, a_rcr = _random_route(21)
+    for tau in [0.05, 0.1, 0.15, 0.2, 0.3]:
+        sk = {f: O.ace_skip(ids, g, a_gsp, a_rcr, tau, 1, 1e-6, f)[0] for f in O.FUSIONS}
+        assert not (sk["max"] & ~sk["mean"]).any()
+        assert not (sk["mean"] & ~sk["min"]).any()
+        for single in ("gsp", "rcr"):
+            assert not (sk["max"] & ~sk[single]).any()
+            assert not (sk[single] & ~sk["min"]).any()
+        # union / intersection of the single views, formed independently
+        assert (sk["max"] == (sk["gsp"] & sk["rcr"])).all()
+        assert (sk["min"] == (sk["gsp"] | sk["rcr"])).all()
+        assert sk["min"].sum() > sk["max"].sum()
+
+
+def test_fusion_threshold_form_equals_candidate_sets():
+    """Every rule's candidate set equals {rank != 0 : c < tau} for its c
+    (for Max this is the App. A.2 equivalence to the intersection)."""
+    ids, g, a_gsp, a_rcr = _random_route(22)
+    for fu in O.FUSIONS:
+        _, _, c, _, _ = O.ace_skip(ids, g, a_gsp, a_rcr, 0.0, 1, 1e-6, fu)
+        for tau in [0.07, 0.12, 0.2]:
+            skip, *_ = O.ace_skip(ids, g, a_gsp, a_rcr, tau, 1, 1e-6, fu)
+            want = c < tau
+            want[:, 0] = False
+            assert (skip == want).all(), (fu, tau)
+
+
+def test_single_view_rules_reduce_to_max_with_equal_tables():
+    """With both tables equal the two views coincide, so Max, Min and Mean
+    equal the single view; GSP-only ignores A^RCR and RCR-only ignores A^GSP."""
+    ids, g, a_gsp, a_rcr = _random_route(23)
+    junk = np.abs(np.random.Generator(np.random.PCG64(99)).standard_normal(a_gsp.size)) * 7
+    for tau in [0.08, 0.15]:
+        ref_g = O.ace_skip(ids, g, a_gsp, a_gsp, tau, 2, 1e-6, "max")
+        ref_r = O.ace_skip(ids, g, a_rcr, a_rcr, tau, 2, 1e-6, "max")
+        for fu in ("max", "min", "mean"):
+            out = O.ace_skip(ids, g, a_gsp, a_gsp, tau, 2, 1e-6, fu)
+            assert (out[0] == ref_g[0]).all()
+            np.testing.assert_allclose(out[2], ref_g[2], rtol=1e-15)
+        out_g = O.ace_skip(ids, g, a_gsp, junk, tau, 2, 1e-6, "gsp")
+        out_r = O.ace_skip(ids, g, junk, a_rcr, tau, 2, 1e-6, "rcr")
+        assert (out_g[0] == ref_g[0]).all() and (out_r[0] == ref_r[0]).all()
+        np.testing.assert_allclose(out_g[1], ref_g[1], rtol=1e-15)
+        np.testing.assert_allclose(out_r[1], ref_r[1], rtol=1e-15)
+
+
+def test_score_rule_is_unit_tables():
+    """Router-score skipping thresholds the routing gate: it is the single
+    GSP view with every table entry 1 and eps = 0 (then p = g / sum g = g)."""
+    ids, g, a_gsp, a_rcr = _random_route(24)
+    ones = np.ones(a_gsp.size)
+    _, _, c_s, _, _ = O.ace_skip(ids, g, a_gsp, a_rcr, 0.0, 1, 0.0, "score")
+    _, _, c_1, _, _ = O.ace_skip(ids, g, ones, ones, 0.0, 1, 0.0, "gsp")
+    np.testing.assert_allclose(c_s, g, rtol=0, atol=0)
+    np.testing.assert_allclose(c_s, c_1, rtol=1e-14)
+    for tau in [0.05, 0.1, 0.17]:
+        margin = np.abs(g - tau) > 1e-12
+        s_s = O.ace_skip(ids, g, a_gsp, a_rcr, tau, 1, 0.0, "score")[0]
+        s_1 = O.ace_skip(ids, g, ones, ones, tau, 1, 0.0, "gsp")[0]
+        assert (s_s[margin] == s_1[margin]).all()
+        # the result does not depend on the tables at all
+        s_t = O.ace_skip(ids, g, a_gsp * 3 + 1, a_rcr * 0.1, tau, 1, 0.0, "score")[0]
+        assert (s_t == s_s).all()
+
+
 def test_perturbation_identity_and_bound():
     w = _tiny_layer(5, eps=0.0)
     x = np.random.Generator(np.random.PCG64(10)).standard_normal((20, w.spec.hidden))
@@ -301,7 +404,8 @@ def test_rmsnorm_closed_form():
 # ---------------------------------------------------------------- ratio mode
 
 
-def test_realised_ratio_matches_request():
+@pytest.mark.parametrize("fusion", O.FUSIONS)
+def test_realised_ratio_matches_request(fusion):
     rng = np.random.Generator(np.random.PCG64(14))
     T, N, k = 300, 32, 8
     z = rng.standard_normal((T, N))
@@ -309,7 +413,7 @@ def test_realised_ratio_matches_request():
     a_rcr = np.abs(1 + 0.3 * rng.standard_normal(N))
     for m_min in [1, 3]:
         for q in [0.0, 0.125, 0.25, 0.5, 0.625, 0.9]:
-            dec = O.ace_decide(z, k, a_gsp, a_rcr, "ratio", q, m_min)
+            dec = O.ace_decide(z, k, a_gsp, a_rcr, "ratio", q, m_min, fusion=fusion)
             n_cand = T * (k - m_min)
             m_q = min(int(math.floor(q * T * k + 0.5)), n_cand)
             assert dec["m_q"] == m_q
@@ -317,7 +421,8 @@ def test_realised_ratio_matches_request():
             assert (k - dec["skip"].sum(1) >= m_min).all()
 
 
-def test_decide_fp32_matches_fp64_off_boundary():
+@pytest.mark.parametrize("fusion", O.FUSIONS)
+def test_decide_fp32_matches_fp64_off_boundary(fusion):
     z32 = synth.make_logits(2000, 128, seed=3)
     a_gsp, a_rcr = synth.make_tables(128, seed=4, spread=0.2)
     k = 8
@@ -328,9 +433,12 @@ def test_decide_fp32_matches_fp64_off_boundary():
     assert (ids32[clear] == ids64[clear]).all()
     np.testing.assert_allclose(g32, g64, rtol=3e-6)
     for tau in [0.08, 0.11, 0.13]:
-        d32 = O.decide_fp32(ids32, g32, a_gsp, a_rcr, "threshold", tau)
-        _, _, c64, _, _ = O.ace_skip(ids64, g64, a_gsp.astype(np.float64), a_rcr.astype(np.float64), 0.0, 1, 1e-6)
-        s64, gh64, *_ = O.ace_skip(ids64, g64, a_gsp.astype(np.float64), a_rcr.astype(np.float64), tau, 1, 1e-6)
+        d32 = O.decide_fp32(ids32, g32, a_gsp, a_rcr, "threshold", tau, fusion=fusion)
+        _, _, c64, _, _ = O.ace_skip(ids64, g64, a_gsp.astype(np.float64), a_rcr.astype(np.float64), 0.0, 1, 1e-6,
+                                     fusion)
+        s64, gh64, *_ = O.ace_skip(ids64, g64, a_gsp.astype(np.float64), a_rcr.astype(np.float64), tau, 1, 1e-6,
+                                   fusion)
+        np.testing.assert_allclose(d32["c"][clear], c64[clear], rtol=3e-6)
         margin = np.abs(c64 - tau) > 1e-5 * tau
         ok = clear[:, None] & margin
         assert (d32["skip"][ok] == s64[ok]).all()
