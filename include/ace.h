@@ -71,9 +71,27 @@ typedef struct ace_layer_desc {
                             the MoE layer), added in fp32 before rounding to dtype */
 } ace_layer_desc;
 
+/*
+ * Skip rule: the per-slot score c that is compared with tau (a slot of rank
+ * > 0 is a skip candidate when c < tau). p_gsp and p_rcr are the two views
+ * of Eqs. gsp_probability and rcr_probability, g the routing gate.
+ */
+typedef enum ace_fusion {
+    ACE_FUSION_MAX = 0,    /* c = max(p_gsp, p_rcr): ACE, skip only when both views
+                              are low (Eqs. ace_contribution, ace_candidate_intersection) */
+    ACE_FUSION_MIN = 1,    /* c = min(p_gsp, p_rcr): skip when either view is low
+                              (§4.3, Tab. fusion_ablation "Min") */
+    ACE_FUSION_MEAN = 2,   /* c = (p_gsp + p_rcr) * 0.5 (Tab. fusion_ablation "Mean") */
+    ACE_FUSION_GSP = 3,    /* c = p_gsp, the GSP view alone (§4.3, Tab. ablation) */
+    ACE_FUSION_RCR = 4,    /* c = p_rcr, the RCR view alone (Tab. ablation) */
+    ACE_FUSION_SCORE = 5   /* c = g, router-score skipping (§4.1 Baselines, "Score");
+                              the tables are not read */
+} ace_fusion;
+
 typedef struct ace_skip_ctl {
     int mode;            /* ace_skip_mode */
     float value;         /* tau (>= 0, may be +inf) or q (in [0,1]) */
+    int fusion;          /* ace_fusion; 0 (zero-initialised) is the ACE rule */
 } ace_skip_ctl;
 
 typedef struct ace_layer ace_layer;   /* opaque */
@@ -121,7 +139,7 @@ void ace_layer_destroy(ace_layer* layer);
  * Stream-ordered and asynchronous; allocates nothing; the sequence of
  * launches depends only on (T, ctl.mode), so it can be captured in a CUDA graph.
  * Errors: INVALID_ARG (NULL, T out of range, ratio outside [0,1], negative
- * or NaN tau), CUDA.
+ * or NaN tau, unknown fusion), CUDA.
  */
 ace_status ace_moe_forward(ace_layer* layer, const void* x, void* out, int T,
                            ace_skip_ctl ctl, void* stream);

@@ -17,6 +17,9 @@ LIBPATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "liba
 
 ACE_BF16, ACE_F32 = 0, 1
 ACE_SKIP_THRESHOLD, ACE_SKIP_RATIO = 0, 1
+# Skip rules (ace_fusion): index = enum value. "max" is ACE.
+FUSIONS = ("max", "min", "mean", "gsp", "rcr", "score")
+ACE_FUSION_MAX, ACE_FUSION_MIN, ACE_FUSION_MEAN, ACE_FUSION_GSP, ACE_FUSION_RCR, ACE_FUSION_SCORE = range(6)
 STATUS = {0: "ACE_OK", 1: "ACE_ERR_INVALID_ARG", 2: "ACE_ERR_UNSUPPORTED", 3: "ACE_ERR_OOM",
           4: "ACE_ERR_CUDA", 5: "ACE_ERR_TIMEOUT", 6: "ACE_ERR_NUMERIC", 7: "ACE_ERR_STATE"}
 
@@ -35,7 +38,7 @@ class ace_layer_desc(ctypes.Structure):
 
 
 class ace_skip_ctl(ctypes.Structure):
-    _fields_ = [("mode", ctypes.c_int), ("value", ctypes.c_float)]
+    _fields_ = [("mode", ctypes.c_int), ("value", ctypes.c_float), ("fusion", ctypes.c_int)]
 
 
 _lib = None
@@ -106,10 +109,18 @@ def _check(st: int) -> None:
         raise AceError(st, lib().ace_last_error_message().decode())
 
 
-def _ctl(mode, value) -> ace_skip_ctl:
+def _fusion(fusion) -> int:
+    if isinstance(fusion, str):
+        if fusion not in FUSIONS:
+            raise ValueError(f"unknown fusion {fusion!r}; one of {FUSIONS}")
+        return FUSIONS.index(fusion)
+    return int(fusion)
+
+
+def _ctl(mode, value, fusion=ACE_FUSION_MAX) -> ace_skip_ctl:
     if isinstance(mode, str):
         mode = ACE_SKIP_RATIO if mode == "ratio" else ACE_SKIP_THRESHOLD
-    return ace_skip_ctl(int(mode), float(value))
+    return ace_skip_ctl(int(mode), float(value), _fusion(fusion))
 
 
 def ace_layer_create(desc: ace_layer_desc, router_w, router_b, w_gate, w_up, w_down, rms_gamma,
@@ -128,17 +139,17 @@ def ace_layer_destroy(layer: int) -> None:
         lib().ace_layer_destroy(layer)
 
 
-def ace_moe_forward(layer: int, x, out, T: int, mode, value: float, stream=None) -> None:
-    _check(lib().ace_moe_forward(layer, _ptr(x), _ptr(out), int(T), _ctl(mode, value), _stream(stream)))
+def ace_moe_forward(layer: int, x, out, T: int, mode, value: float, stream=None, fusion=ACE_FUSION_MAX) -> None:
+    _check(lib().ace_moe_forward(layer, _ptr(x), _ptr(out), int(T), _ctl(mode, value, fusion), _stream(stream)))
 
 
-def ace_moe_forward_host(layer: int, x_host, out_host, T: int, mode, value: float, stream=None) -> None:
-    _check(lib().ace_moe_forward_host(layer, _ptr(x_host), _ptr(out_host), int(T), _ctl(mode, value),
+def ace_moe_forward_host(layer: int, x_host, out_host, T: int, mode, value: float, stream=None, fusion=ACE_FUSION_MAX) -> None:
+    _check(lib().ace_moe_forward_host(layer, _ptr(x_host), _ptr(out_host), int(T), _ctl(mode, value, fusion),
                                       _stream(stream)))
 
 
-def ace_route_logits(layer: int, logits, T: int, mode, value: float, stream=None) -> None:
-    _check(lib().ace_route_logits(layer, _ptr(logits), int(T), _ctl(mode, value), _stream(stream)))
+def ace_route_logits(layer: int, logits, T: int, mode, value: float, stream=None, fusion=ACE_FUSION_MAX) -> None:
+    _check(lib().ace_route_logits(layer, _ptr(logits), int(T), _ctl(mode, value, fusion), _stream(stream)))
 
 
 def ace_last_skip_mask(layer: int, T: int, k: int):
@@ -189,10 +200,11 @@ def ace_last_stage_times(layer: int) -> dict:
 
 
 def ace_route_decide_noalloc(logits, T: int, n_experts: int, top_k: int, a_gsp, a_rcr, eps: float,
-                             min_active: int, mode, value: float, ids, skip, gates_hat, tau, stream=None) -> None:
+                             min_active: int, mode, value: float, ids, skip, gates_hat, tau, stream=None,
+                             fusion=ACE_FUSION_MAX) -> None:
     """Routing decision without a layer or any device allocation (all pointers are device buffers)."""
     _check(lib().ace_route_decide_noalloc(_ptr(logits), int(T), int(n_experts), int(top_k), _ptr(a_gsp), _ptr(a_rcr),
-                                          float(eps), int(min_active), _ctl(mode, value), _ptr(ids), _ptr(skip),
+                                          float(eps), int(min_active), _ctl(mode, value, fusion), _ptr(ids), _ptr(skip),
                                           _ptr(gates_hat), _ptr(tau), _stream(stream)))
 
 
@@ -243,8 +255,9 @@ class AceLayer:
         self.spec = spec
         self.torch_dtype = tdt
 
-    def forward(self, x, out, T: int, mode="threshold", value: float = 0.0, stream=None) -> None:
-        ace_moe_forward(self.handle, x, out, T, mode, value, stream)
+    def forward(self, x, out, T: int, mode="threshold", value: float = 0.0, stream=None,
+                fusion=ACE_FUSION_MAX) -> None:
+        ace_moe_forward(self.handle, x, out, T, mode, value, stream, fusion)
 
     def close(self) -> None:
         if getattr(self, "handle", None):

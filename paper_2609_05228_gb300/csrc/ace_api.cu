@@ -77,6 +77,8 @@ ace_status check_ctl(ace_skip_ctl ctl) {
     } else {
         return fail(ACE_ERR_INVALID_ARG, "unknown skip mode");
     }
+    if (ctl.fusion < ACE_FUSION_MAX || ctl.fusion > ACE_FUSION_SCORE)
+        return fail(ACE_ERR_INVALID_ARG, "unknown fusion rule");
     return ACE_OK;
 }
 

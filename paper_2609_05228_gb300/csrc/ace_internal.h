@@ -50,7 +50,7 @@ struct Workspace {
     float* logits = nullptr;     // [Tmax, N]
     int32_t* ids = nullptr;      // [Tmax, k] rank order
     float* gates = nullptr;      // [Tmax, k] g
-    float* cval = nullptr;       // [Tmax, k] c = max(p_gsp, p_rcr)
+    float* cval = nullptr;       // [Tmax, k] c of the skip rule (ACE: max(p_gsp, p_rcr))
     uint32_t* keys = nullptr;    // [Tmax, k] ratio-mode candidate keys
     uint8_t* skip = nullptr;     // [Tmax, k]
     float* ghat = nullptr;       // [Tmax, k]

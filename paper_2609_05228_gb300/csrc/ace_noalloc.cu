@@ -84,6 +84,8 @@ extern "C" ace_status ace_route_decide_noalloc(const float* logits, int T, int n
     } else {
         return na_fail(ACE_ERR_INVALID_ARG, "ace_route_decide_noalloc: unknown skip mode");
     }
+    if (ctl.fusion < ACE_FUSION_MAX || ctl.fusion > ACE_FUSION_SCORE)
+        return na_fail(ACE_ERR_INVALID_ARG, "ace_route_decide_noalloc: unknown fusion rule");
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return na_fail(ACE_ERR_CUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));

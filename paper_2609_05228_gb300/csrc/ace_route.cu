@@ -174,7 +174,7 @@ __global__ void __launch_bounds__(256) k_router(const T* __restrict__ src, const
 // --------------------------------------------------------------------------
 struct SlotScore {
     float g;   // gate
-    float c;   // max(p_gsp, p_rcr)
+    float c;   // score of the skip rule (ACE: max(p_gsp, p_rcr))
 };
 
 // Top-k over one token's logits (one warp). Lane l owns experts l + 32 j,
@@ -256,10 +256,22 @@ __device__ __forceinline__ void warp_topk(const float* __restrict__ zrow, int n_
     }
 }
 
+// c of a skip rule from the two views and the gate (ace_fusion).
+__device__ __forceinline__ float fuse_views(float pg, float pr, float g, int fusion) {
+    switch (fusion) {
+        case ACE_FUSION_MIN: return fminf(pg, pr);
+        case ACE_FUSION_MEAN: return __fmul_rn(__fadd_rn(pg, pr), 0.5f);
+        case ACE_FUSION_GSP: return pg;
+        case ACE_FUSION_RCR: return pr;
+        case ACE_FUSION_SCORE: return g;
+        default: return fmaxf(pg, pr);                          // Eq. ace_contribution
+    }
+}
+
 // Gates and c for the slot held by this lane (lanes >= k return zeros).
 __device__ __forceinline__ SlotScore score_slot(int lane, int k, float z_i, float z_0, int id,
                                                 const float* __restrict__ a_gsp,
-                                                const float* __restrict__ a_rcr, float eps) {
+                                                const float* __restrict__ a_rcr, float eps, int fusion) {
     const bool on = lane < k;
     const float e_i = on ? ace_exp32(__fsub_rn(z_i, z_0)) : 0.f;
     float s = __shfl_sync(0xffffffffu, e_i, 0);
@@ -277,7 +289,7 @@ __device__ __forceinline__ SlotScore score_slot(int lane, int k, float z_i, floa
     zr = __fadd_rn(zr, eps);
     const float pg = on ? __fdiv_rn(sg, zg) : 0.f;              // Eq. gsp_probability
     const float pr = on ? __fdiv_rn(sr, zr) : 0.f;              // Eq. rcr_probability
-    return SlotScore{g, fmaxf(pg, pr)};                         // Eq. ace_contribution
+    return SlotScore{g, on ? fuse_views(pg, pr, g, fusion) : 0.f};
 }
 
 // Slots excluded from the threshold search (App. B.1): rank 0 (the top-1)
@@ -300,7 +312,8 @@ __device__ __forceinline__ bool slot_protected(int lane, int k, float c, int m_m
 __device__ __forceinline__ void decide_slot(int lane, int k, float g, float c, float tau, int m_min,
                                             float eps, bool& skip_out, float& ghat_out) {
     const bool on = lane < k;
-    // Eq. ace_candidate_intersection via max; slot 0 is the top-1 and is kept.
+    // candidate when c < tau (for ACE, Eq. ace_candidate_intersection via max);
+    // slot 0 is the top-1 and is kept.
     bool skip = on && lane != 0 && (c < tau);
     const unsigned sk = __ballot_sync(0xffffffffu, skip);
     const int active = k - __popc(sk);
@@ -345,7 +358,7 @@ __device__ __forceinline__ void decide_token(const float* g_in, const float* c_i
     for (int j = 0; j < kMaxTopK; ++j) {
         g[j] = j < k ? g_in[j] : 0.f;
         c[j] = j < k ? c_in[j] : 0.f;
-        if (j < k && j != 0 && c[j] < tau) sk |= 1u << j;   // Eq. ace_candidate_intersection via max
+        if (j < k && j != 0 && c[j] < tau) sk |= 1u << j;   // candidate: c < tau
     }
     int need = m_min - (k - __popc(sk));
     while (need > 0 && sk) {
@@ -535,7 +548,7 @@ __global__ void __launch_bounds__(kTopkWarps * 32) k_topk_score(float* __restric
                                                                 int32_t* __restrict__ ghist,
                                                                 const float* __restrict__ part, int n_split,
                                                                 const float* __restrict__ bias, float inv_temp,
-                                                                int use_temp) {
+                                                                int use_temp, int fusion) {
     __shared__ int hist[kHistBins];
     const bool ratio = mode == ACE_SKIP_RATIO;
     if (ratio)
@@ -565,7 +578,7 @@ __global__ void __launch_bounds__(kTopkWarps * 32) k_topk_score(float* __restric
         warp_topk<NPL>(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
         const float z0 = __shfl_sync(0xffffffffu, zv, 0);
         if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(err, kErrNumeric);
-        const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a_gsp, a_rcr, eps);
+        const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a_gsp, a_rcr, eps, fusion);
         const size_t base = (size_t)t * k;
         if (lane < k) {
             ids[base + lane] = id;
@@ -926,7 +939,7 @@ struct FusedArgs {
     const float* a_gsp;
     const float* a_rcr;
     float eps;
-    int m_min, mode;
+    int m_min, mode, fusion;
     float tau_in;
     int m_q;
     int32_t* ids;
@@ -1074,7 +1087,7 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         warp_topk<NPL>(a.logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
         const float z0 = __shfl_sync(0xffffffffu, zv, 0);
         if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(a.err, kErrNumeric);
-        const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a.a_gsp, a.a_rcr, a.eps);
+        const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a.a_gsp, a.a_rcr, a.eps, a.fusion);
         const size_t base = (size_t)t * k;
         if (lane < k) {
             a.ids[base + lane] = id;
@@ -1256,6 +1269,7 @@ cudaError_t launch_route_fused(const ace_layer* L, const void* x, const float* l
     bool need_select;
     a.m_q = select_mq(L, T, ctl, &tau, &need_select);
     a.mode = need_select ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
+    a.fusion = ctl.fusion;
     a.tau_in = tau;
     a.x = x;
     a.gamma = L->gamma;
@@ -1339,7 +1353,7 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     launch_pdl(k_topk_score<NPL>, dim3(blocks), dim3(kTopkWarps * 32), 0, s, const_cast<float*>(logits), T, n, k, \
                (const float*)L->a_gsp, (const float*)L->a_rcr, D.eps, D.min_active, mode, tau, W.ids, W.gates,    \
                W.cval, W.keys, W.skip, W.ghat, W.tau, W.err, W.sel_hist, (const float*)W.act_bf16, n_split,        \
-               (const float*)L->router_b, 1.0f / D.router_temp, D.router_temp != 1.0f ? 1 : 0)
+               (const float*)L->router_b, 1.0f / D.router_temp, D.router_temp != 1.0f ? 1 : 0, ctl.fusion)
     if (n <= 128) e = ACE_TOPK(4);
     else if (n <= 256) e = ACE_TOPK(8);
     else e = ACE_TOPK(32);
@@ -1431,6 +1445,7 @@ cudaError_t launch_route_decide_scratch(const float* logits, int T, int n_exp, i
         else need_select = true;
     }
     a.mode = need_select ? ACE_SKIP_RATIO : ACE_SKIP_THRESHOLD;
+    a.fusion = ctl.fusion;
     a.tau_in = tau;
     a.m_q = m_q;
     a.logits = const_cast<float*>(logits);

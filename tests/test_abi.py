@@ -54,3 +54,37 @@ def test_host_side_argument_checks(libace):
     assert st == 2
     assert L.ace_moe_forward(None, None, None, 1, ace.ace_skip_ctl(0, 0.1), None) == 1
     assert L.ace_last_skip_mask(None, None, None, None, None, None) == 1
+
+
+def test_struct_layouts_match_header(tmp_path):
+    """The binding's ctypes structs have the sizes and field offsets that a C
+    compiler gives the header's structs."""
+    src = tmp_path / "layout.c"
+    src.write_text(
+        '#include <stdio.h>\n#include <stddef.h>\n#include "ace.h"\n'
+        "int main(void) {\n"
+        '  printf("%zu %zu %zu %zu\\n", sizeof(ace_skip_ctl), offsetof(ace_skip_ctl, value),'
+        " offsetof(ace_skip_ctl, fusion), sizeof(ace_layer_desc));\n"
+        '  printf("%zu %zu\\n", offsetof(ace_layer_desc, eps), offsetof(ace_layer_desc, add_residual));\n'
+        "  return 0;\n}\n")
+    exe = tmp_path / "layout"
+    import subprocess
+    subprocess.run(["gcc", "-I", os.path.dirname(HEADER), str(src), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()
+    got = [int(v) for v in out]
+    want = [ctypes.sizeof(ace.ace_skip_ctl), ace.ace_skip_ctl.value.offset, ace.ace_skip_ctl.fusion.offset,
+            ctypes.sizeof(ace.ace_layer_desc), ace.ace_layer_desc.eps.offset, ace.ace_layer_desc.add_residual.offset]
+    assert got == want
+
+
+def test_unknown_fusion_rejected_on_host(libace):
+    ace._lib = None
+    L = ace.lib()
+    bad = ace.ace_skip_ctl(ace.ACE_SKIP_RATIO, 0.5, 6)
+    fake = ctypes.c_void_p(16)
+    st = L.ace_route_decide_noalloc(fake, 4, 8, 2, fake, fake, ctypes.c_float(1e-6), 1, bad, fake, fake, fake,
+                                    fake, None)
+    assert st == 1 and b"fusion" in L.ace_last_error_message()
+    with pytest.raises(ValueError):
+        ace._ctl("ratio", 0.5, "median")
+    assert ace._ctl("ratio", 0.5, "score").fusion == ace.ACE_FUSION_SCORE

@@ -121,6 +121,37 @@ def test_decision_bitexact(T, N, k, m_min):
     layer.close()
 
 
+FUSION_ROUTE_CASES = [(64, 128, 8, 1), (257, 100, 6, 2), (4096, 128, 8, 1), (200, 1024, 16, 3), (2048, 256, 8, 3)]
+
+
+@pytest.mark.parametrize("fusion", ["min", "mean", "gsp", "rcr", "score"])
+@pytest.mark.parametrize("T,N,k,m_min", FUSION_ROUTE_CASES)
+def test_decision_bitexact_fusion(T, N, k, m_min, fusion):
+    """The skip-rule variants (Min / Mean fusion, single views, router score)
+    through the fused small-batch route and the large-batch chain."""
+    z = synth.make_logits(T, N, seed=500 + T + N, tie_fraction=0.05)
+    tables = synth.make_tables(N, seed=9 + N, spread=0.2)
+    layer = _route_layer(N, k, T, m_min, tables)
+    zd = torch.from_numpy(z).cuda()
+    ids_ref, g_ref = O.route_fp32(z, k)
+    for mode, val in [("threshold", 0.09), ("ratio", 0.25), ("ratio", 0.5), ("ratio", 0.625)]:
+        ace.ace_route_logits(layer.handle, zd, T, mode, val, fusion=fusion)
+        skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, k)
+        ref = O.decide_fp32(ids_ref, g_ref, tables[0], tables[1], mode, val, m_min, 1e-6, fusion=fusion)
+        assert (ids == ids_ref).all(), (mode, val)
+        assert (skip.astype(bool) == ref["skip"]).all(), (mode, val, int(skip.sum()), int(ref["skip"].sum()))
+        assert (gh.view(np.uint32) == ref["g_hat"].view(np.uint32)).all(), (mode, val)
+        assert np.float32(tau).view(np.uint32) == np.float32(ref["tau"]).view(np.uint32), (mode, val, tau, ref["tau"])
+        if mode == "ratio":
+            assert T * k - R == ref["count"]
+        off, perm = ace.ace_last_permutation(layer.handle, N, R)
+        off_ref, perm_ref = O.permutation(ids_ref, ref["skip"], N)
+        assert (off == off_ref).all() and (perm == perm_ref).all(), (mode, val)
+    with pytest.raises(ace.AceError):
+        ace.ace_route_logits(layer.handle, zd, T, "ratio", 0.5, fusion=6)
+    layer.close()
+
+
 @pytest.mark.parametrize("T,pattern", [(16384, "equal"), (8192, "two_values"), (300, "equal")])
 def test_decision_degenerate_scores(T, pattern):
     """Every candidate score equal (or only two distinct values): the
@@ -218,17 +249,17 @@ def _clear_tokens(dec, z_ref, k, dz, dc, m_min=1):
     return (gap_k > dz) & (gap_1 > dz) & c_ok
 
 
-def _run_layer(kind, T, mode, val, x_seed=1):
+def _run_layer(kind, T, mode, val, x_seed=1, fusion="max"):
     w, layer = _layer(kind)
     spec = w.spec
     x = synth.make_tokens(spec, T, seed=x_seed)
     xd = _dev(x)
     out = torch.empty_like(xd)
-    layer.forward(xd, out, T, mode, val)
+    layer.forward(xd, out, T, mode, val, fusion=fusion)
     torch.cuda.synchronize()
     skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, spec.top_k)
     y_gpu = _host(out).astype(np.float64)
-    y_ref, dec = O.moe_forward(x, w, mode, val, return_decision=True)
+    y_ref, dec = O.moe_forward(x, w, mode, val, return_decision=True, fusion=fusion)
     h = O.rmsnorm(x, w.gamma, spec.rms_eps)
     z_ref = O.router_logits(h, w.router_w, w.router_b, spec.router_temp)
     return w, spec, x, y_gpu, y_ref, dec, z_ref, (skip, ids, gh, tau, R)
@@ -245,9 +276,23 @@ FORWARD_CASES = [
 ]
 
 
+FUSION_FORWARD_CASES = [(f, kind, T, "ratio", 0.5) for f in ("min", "mean", "gsp", "rcr", "score")
+                        for kind, T in (("qwen", 64), ("qwen_zipf", 4096))] + [
+    ("score", "qwen_temp", 600, "ratio", 0.625), ("min", "qwen", 17, "threshold", 0.11)]
+
+
 @pytest.mark.parametrize("kind,T,mode,val", FORWARD_CASES)
 def test_forward_parity(kind, T, mode, val):
-    w, spec, x, y_gpu, y_ref, dec, z_ref, (skip, ids, gh, tau, R) = _run_layer(kind, T, mode, val)
+    _check_forward(kind, T, mode, val, "max")
+
+
+@pytest.mark.parametrize("fusion,kind,T,mode,val", FUSION_FORWARD_CASES)
+def test_forward_parity_fusion(fusion, kind, T, mode, val):
+    _check_forward(kind, T, mode, val, fusion)
+
+
+def _check_forward(kind, T, mode, val, fusion):
+    w, spec, x, y_gpu, y_ref, dec, z_ref, (skip, ids, gh, tau, R) = _run_layer(kind, T, mode, val, fusion=fusion)
     k = spec.top_k
     margin = 1e-4 if spec.dtype == "f32" else None
     clear = _clear_tokens(dec, z_ref, k, margin or 6e-3, margin or 8e-3, spec.min_active)

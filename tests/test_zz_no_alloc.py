@@ -14,6 +14,7 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
+import oracle as O
 from paper_2609_05228_gb300 import ace, synth
 
 pytestmark = pytest.mark.gpu
@@ -61,6 +62,29 @@ def test_noalloc_matches_route_logits(T, N, k, m_min, calls):
         assert (gh.cpu().numpy().view(np.uint32) == r_gh.view(np.uint32)).all()
         assert tau.cpu().numpy().view(np.uint32)[0] == np.float32(r_tau).view(np.uint32)
     layer.close()
+
+
+@pytest.mark.parametrize("fusion", ["min", "mean", "gsp", "rcr", "score"])
+def test_noalloc_fusion_matches_oracle(fusion):
+    T, N, k, m_min = 128, 128, 8, 2
+    tables = synth.make_tables(N, seed=12, spread=0.2)
+    a_gsp = torch.from_numpy(tables[0]).cuda()
+    a_rcr = torch.from_numpy(tables[1]).cuda()
+    ids = torch.empty((T, k), dtype=torch.int32, device="cuda")
+    skip = torch.empty((T, k), dtype=torch.uint8, device="cuda")
+    gh = torch.empty((T, k), dtype=torch.float32, device="cuda")
+    tau = torch.empty(1, dtype=torch.float32, device="cuda")
+    z = synth.make_logits(T, N, seed=41, tie_fraction=0.05)
+    ids_ref, g_ref = O.route_fp32(z, k)
+    for mode, val in [("ratio", 0.5), ("threshold", 0.1)]:
+        ace.ace_route_decide_noalloc(torch.from_numpy(z).cuda(), T, N, k, a_gsp, a_rcr, 1e-6, m_min, mode, val,
+                                     ids, skip, gh, tau, fusion=fusion)
+        torch.cuda.synchronize()
+        ref = O.decide_fp32(ids_ref, g_ref, tables[0], tables[1], mode, val, m_min, 1e-6, fusion=fusion)
+        assert (ids.cpu().numpy() == ids_ref).all()
+        assert (skip.cpu().numpy().astype(bool) == ref["skip"]).all(), (mode, val)
+        assert (gh.cpu().numpy().view(np.uint32) == ref["g_hat"].view(np.uint32)).all()
+        assert tau.cpu().numpy().view(np.uint32)[0] == np.float32(ref["tau"]).view(np.uint32)
 
 
 def test_noalloc_rejects_sizes_beyond_limits():
