@@ -43,10 +43,10 @@ WORKLOADS = {
     "stack_decode": dict(spec="qwen", zipf=False, T=32, q=0.5, layers=4, tables="offline",
                          name="4-layer stack of the d=2048 N=128 top-8 m=768 layer (residual), decode 32 tokens, "
                               "skip ratio 0.5"),
-    "large_prefill": dict(spec="large", zipf=True, T=8192, q=0.5, layers=1, tables="random",
+    "large_prefill": dict(spec="large", zipf=True, T=8192, q=0.5, layers=1, tables="gpu",
                           name="large MoE layer d=4096 N=256 top-8 m=2048 bf16, prefill 8192 tokens Zipf routing, "
                                "skip ratio 0.5"),
-    "large_decode": dict(spec="large", zipf=True, T=128, q=0.5, layers=1, tables="random",
+    "large_decode": dict(spec="large", zipf=True, T=128, q=0.5, layers=1, tables="gpu",
                          name="large MoE layer d=4096 N=256 top-8 m=2048 bf16, decode 128 tokens, skip ratio 0.5"),
 }
 METRIC = "ACE MoE-layer tokens/s (prefill, decode) + speedup vs skip=0; % of roofline"
@@ -163,10 +163,10 @@ class Stack:
         n = wl["layers"]
         for l in range(n):
             w = synth.make_layer(spec, seed=0 if n == 1 else 100 + l)
-            if wl["tables"] == "offline":
+            if wl["tables"] == "offline":     # host library (fp64)
                 w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables(w)
-            else:   # the large layer: seeded positive tables stand in (the forward takes any valid tables)
-                w.extra["a_gsp"], w.extra["a_rcr"] = synth.make_tables(spec.n_experts, seed=5, spread=0.1)
+            else:                             # the GPU tables (ace_offline_tables_device)
+                w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables_device(w)
             self.ws.append(w)
             self.layers.append(ace.AceLayer(w, w.extra["a_gsp"], w.extra["a_rcr"], max_tokens=max_tokens,
                                             residual=n > 1))
@@ -423,7 +423,8 @@ def run_ours(args, rank, world, torch, dist):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) tokens, N(0,0.02^2) weights, " +
-                ("offline GSP/RCR tables)" if wl["tables"] == "offline" else "seeded positive tables)"),
+                ("offline GSP/RCR tables from the host library)" if wl["tables"] == "offline"
+                 else "offline GSP/RCR tables computed on the GPU)"),
         "config": {"workload": wl["name"], "tokens_per_step": T, "layers": n_layers, "skip_ratio": q,
                    "parallelism": f"replicas{world}" if world > 1 else "single GPU",
                    "l2": "flushed between timed steps (512 MB write, then a 256 MB read)", "graph": "CUDA graph replay"},
@@ -446,6 +447,7 @@ def run_ours(args, rank, world, torch, dist):
                 "d2h_bytes_per_step": int(n_layers * T * spec.hidden * 2)},
         "gpu_launches": args.steps * launches,
         "clocks": clk,
+        "offline_tables": time_tables(torch, w) if rank == 0 else None,
     }
     if rank == 0 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(model.ws, wl, budget_s=args.cpu_seconds)
@@ -487,6 +489,35 @@ def sweep(torch, args):
     return pts
 
 
+def time_tables(torch, w, reps=3):
+    """Wall time of ace_offline_tables_device (Algorithms 2 and 3 on the GPU)
+    for layer `w`, weights resident on the device; the call allocates its
+    scratch, packs, runs and synchronises. GSP GEMM FLOPs: two d x d x m
+    products per expert."""
+    from paper_2609_05228_gb300 import ace
+    spec = w.spec
+    d, n, m = spec.hidden, spec.n_experts, spec.ffn
+
+    def up(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).cuda()
+
+    ts = [up(a) for a in (w.gamma, w.router_w, w.w_gate, w.w_up, w.w_down)]
+    torch.cuda.synchronize()
+    ace.ace_offline_tables_device(d, n, m, *ts, spec.eps)
+    times = []
+    for _ in range(reps):
+        t = time.perf_counter()
+        ace.ace_offline_tables_device(d, n, m, *ts, spec.eps)
+        times.append(time.perf_counter() - t)
+    del ts
+    torch.cuda.empty_cache()
+    t = float(np.median(times))
+    flops = 2 * 2 * d * d * m * n
+    return {"call_ms": round(t * 1e3, 3), "gsp_gemm_tflop": round(flops / 1e12, 4),
+            "gsp_gemm_tflops_over_call": round(flops / t / 1e12, 1),
+            "note": "whole call: scratch allocation, packing, GSP GEMM, norms, RCR GEMV, normalisation"}
+
+
 def cpu_baseline(ws, wl, budget_s=12.0):
     """The CPU oracle (fp64) on a bounded sample of the same workload: the
     stacked layers over a sample of tokens (64, or 256 for prefill)."""
@@ -522,7 +553,7 @@ def run_reference(args):
         w = synth.make_layer(spec, seed=0 if wl["layers"] == 1 else 100 + l)
         if wl["tables"] == "offline":
             w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables(w)
-        else:
+        else:   # the arm stays on the host: seeded positive tables stand in for the GPU tables
             w.extra["a_gsp"], w.extra["a_rcr"] = synth.make_tables(spec.n_experts, seed=5, spread=0.1)
         ws.append(w)
     T = wl["T"] if wl["T"] <= 64 else 256
@@ -563,6 +594,8 @@ def main():
     ap.add_argument("--workload", default="decode", choices=sorted(WORKLOADS))
     ap.add_argument("--sweep", action="store_true", help="add decode/prefill sweep points")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--tables-only", action="store_true",
+                    help="time only the GPU offline tables (ace_offline_tables_device) of the workload's layer")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -576,6 +609,15 @@ def main():
 
     import torch
     import torch.distributed as dist
+    if args.tables_only:
+        if rank == 0:
+            from paper_2609_05228_gb300 import synth
+            wl = WORKLOADS[args.workload]
+            spec = synth.spec_qwen(zipf=wl["zipf"]) if wl["spec"] == "qwen" else synth.spec_large(zipf=wl["zipf"])
+            w = synth.make_layer(spec, seed=0)
+            print(json.dumps({"workload": wl["name"], "offline_tables": time_tables(torch, w, reps=args.steps)}),
+                  flush=True)
+        return
     if world > 1:
         dist.init_process_group("nccl")
     try:

@@ -256,6 +256,43 @@ ace_status ace_route_decide_noalloc(const float* logits, int T, int n_experts, i
                                     ace_skip_ctl ctl, int32_t* ids, uint8_t* skip, float* gates_hat,
                                     float* tau, void* stream);
 
+/*
+ * ace_offline_tables_device — the offline GSP and RCR tables (Algorithms 2
+ * and 3) computed on the GPU from bf16 weights already in device memory, in
+ * the layouts ace_layer_create takes. Needs no layer.
+ *   GSP: a_up = ||U||_F ||G W_down||_F, a_gate = ||G||_F ||U W_down||_F with
+ *        G = Gamma W_gate, U = Gamma W_up; a~ = sqrt(a_up a_gate);
+ *        A^GSP = a~ / (mean a~ + eps)  (Eqs. gsp_up_path, gsp_gate_path,
+ *        gsp_geometric_mean, gsp_layer_normalization). The two d x d x m
+ *        products per expert run on the tensor cores with bf16 operands
+ *        exactly as stored and fp32 accumulation; Gamma is applied in fp64
+ *        to the row sums of squares.
+ *   RCR: centred router rows, prototype q_e = w~_e / (RMS(w~_e) + eps),
+ *        a~ = ||f_e(q_e)||_2 / (||q_e||_2 + eps), A^RCR = a~ / (mean a~ + eps)
+ *        (Eqs. rcr_centered_router, rcr_direction_prototype,
+ *        rcr_raw_amplification, rcr_layer_normalization); q_e is scaled by
+ *        gamma first when rcr_apply_gamma != 0. fp32 FMA on the CUDA cores.
+ *   d, N, m        hidden size (multiple of 256, <= 16384), experts (1..1024),
+ *                  FFN width (multiple of 64)
+ *   gamma [d], router_w [N, d], w_gate / w_up [N, m, d], w_down [N, d, m]
+ *                  device, bf16
+ *   eps            the paper's epsilon (>= 0)
+ *   tile_budget    device bytes for the repacked weight tiles (3 d m 2 bytes
+ *                  per expert; experts are processed in chunks that fit, at
+ *                  least one at a time); 0 = 1.5 GiB
+ *   gsp_out, rcr_out [N] host float32, written on success
+ * Allocates its device scratch (the tiles plus O(N d) bytes) for the call
+ * and frees it before returning; synchronises `stream`. Sums are taken in a
+ * fixed order, so the result is the same bits on every run and for every
+ * tile_budget.
+ * Errors: INVALID_ARG (NULL, non-positive size, eps < 0), UNSUPPORTED (shape),
+ * OOM, CUDA, TIMEOUT (a bounded device wait ran out).
+ */
+ace_status ace_offline_tables_device(int d, int N, int m, const void* gamma, const void* router_w,
+                                     const void* w_gate, const void* w_up, const void* w_down, double eps,
+                                     int rcr_apply_gamma, size_t tile_budget, float* gsp_out, float* rcr_out,
+                                     void* stream);
+
 /* Fills *desc with the layer's descriptor (after defaults were applied). */
 ace_status ace_layer_get_desc(const ace_layer* layer, ace_layer_desc* desc);
 

@@ -73,6 +73,8 @@ def lib() -> ctypes.CDLL:
             "ace_last_launch_count": (_S, [_P, _P]),
             "ace_route_decide_noalloc": (_S, [_P, _I, _I, _I, _P, _P, ctypes.c_float, _I, ace_skip_ctl, _P, _P, _P,
                                               _P, _P]),
+            "ace_offline_tables_device": (_S, [_I, _I, _I, _P, _P, _P, _P, _P, ctypes.c_double, _I, ctypes.c_size_t,
+                                               _P, _P, _P]),
             "ace_status_string": (ctypes.c_char_p, [_S]),
             "ace_last_error_message": (ctypes.c_char_p, []),
         }
@@ -206,6 +208,17 @@ def ace_route_decide_noalloc(logits, T: int, n_experts: int, top_k: int, a_gsp, 
     _check(lib().ace_route_decide_noalloc(_ptr(logits), int(T), int(n_experts), int(top_k), _ptr(a_gsp), _ptr(a_rcr),
                                           float(eps), int(min_active), _ctl(mode, value, fusion), _ptr(ids), _ptr(skip),
                                           _ptr(gates_hat), _ptr(tau), _stream(stream)))
+
+
+def ace_offline_tables_device(d: int, N: int, m: int, gamma, router_w, w_gate, w_up, w_down, eps: float = 1e-6,
+                              rcr_apply_gamma: bool = False, tile_budget: int = 0, stream=None):
+    """(A^GSP, A^RCR) float32 [N] computed on the GPU from bf16 device weights."""
+    gsp = np.empty(N, np.float32)
+    rcr = np.empty(N, np.float32)
+    _check(lib().ace_offline_tables_device(int(d), int(N), int(m), _ptr(gamma), _ptr(router_w), _ptr(w_gate),
+                                           _ptr(w_up), _ptr(w_down), float(eps), int(bool(rcr_apply_gamma)),
+                                           int(tile_budget), gsp.ctypes.data, rcr.ctypes.data, _stream(stream)))
+    return gsp, rcr
 
 
 def ace_last_launch_count(layer: int) -> int:

@@ -1,4 +1,5 @@
-"""Offline GSP and RCR tables (ACE Algorithms 2 and 3), host CPU.
+"""Offline GSP and RCR tables (ACE Algorithms 2 and 3): host CPU, and GPU
+(tables_device, through libace.so's ace_offline_tables_device).
 
 The tables are computed once per layer from the frozen weights and handed to
 ace_layer_create(). No calibration data is involved. The computation is the
@@ -67,6 +68,29 @@ def tables(layer, eps: float | None = None, apply_gamma: bool = False):
     """(A^GSP, A^RCR) as float32 arrays for a synth.LayerWeights-like layer."""
     e = layer.spec.eps if eps is None else eps
     return ace_offline_tables(layer.gamma, layer.router_w, layer.w_gate, layer.w_up, layer.w_down, e, apply_gamma)
+
+
+def tables_device(layer, eps: float | None = None, apply_gamma: bool = False, device: int = 0,
+                  tile_budget: int = 0):
+    """(A^GSP, A^RCR) for a bf16 synth.LayerWeights-like layer, computed on the
+    GPU by ace_offline_tables_device (libace.so); torch only holds the device
+    copies of the weights for the call."""
+    import torch
+
+    if np.asarray(layer.w_gate).dtype != np.uint16:
+        raise TypeError("the GPU tables take bf16 weights")
+    dev = torch.device("cuda", device)
+
+    def up(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    n, m, d = np.asarray(layer.w_gate).shape
+    ts = [up(x) for x in (layer.gamma, layer.router_w, layer.w_gate, layer.w_up, layer.w_down)]
+    torch.cuda.synchronize(dev)
+    e = layer.spec.eps if eps is None else eps
+    out = ace.ace_offline_tables_device(d, n, m, *ts, e, apply_gamma, tile_budget)
+    del ts
+    return out
 
 
 def gsp_table(gamma, w_gate, w_up, w_down, eps: float = 1e-6) -> np.ndarray:

@@ -113,8 +113,8 @@ def _large():
     if not _LARGE:
         spec = synth.spec_large(zipf=True)
         w = synth.make_layer(spec, seed=0)
-        # any finite non-negative tables are valid inputs to the forward
-        w.extra["a_gsp"], w.extra["a_rcr"] = synth.make_tables(spec.n_experts, seed=5, spread=0.1)
+        # the GPU tables (checked against the oracle in test_large_layer_tables_device)
+        w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables_device(w)
         _LARGE["w"] = w
         _LARGE["layer"] = ace.AceLayer(w, w.extra["a_gsp"], w.extra["a_rcr"], max_tokens=2048)
     return _LARGE["w"], _LARGE["layer"]
@@ -140,3 +140,17 @@ def test_large_layer(T, q):
     y_ref = O.moe_forward(x, w, decision=dec, tokens=sample)
     clear = _clear(dec, z, spec.top_k, 6e-3, 8e-3)[sample]
     _compare(y_gpu[sample], y_ref, clear, min_frac=0.3 if T > 1 else 0.0)
+
+
+def test_large_layer_tables_device():
+    """GPU tables of the large layer (256 experts in nine chunks of the tile
+    budget, the last one ragged): A^GSP ratios of sampled experts against the
+    oracle's direct fp64 products on those experts (the normalisation is one
+    constant, so A[e] / A[e'] = a~_e / a~_e'), and the whole A^RCR table."""
+    w, _ = _large()
+    a, r = w.extra["a_gsp"], w.extra["a_rcr"]
+    idx = [0, 31, 137, 255]
+    sub = O.gsp_table(w.gamma, w.w_gate[idx], w.w_up[idx], w.w_down[idx], 0.0)
+    np.testing.assert_allclose(a[idx] / a[idx[0]], sub / sub[0], rtol=3e-5)
+    r_ref = O.rcr_table(w.router_w, w.gamma, w.w_gate, w.w_up, w.w_down, w.spec.eps)
+    np.testing.assert_allclose(r, r_ref, rtol=3e-5)
