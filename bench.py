@@ -80,9 +80,12 @@ def _recorded_traffic(path="profiles/decode_T64_q0.5_expert_decode_full.md"):
                 if "=" in line and " " not in line.split("=", 1)[0]:
                     k, v = line.split("=", 1)
                     rec[k] = v
-        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
-            if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
-                return None
+        h = hashlib.sha256()          # the listed sources, concatenated in order
+        for src in rec["source"].split(","):
+            with open(os.path.join(ROOT, src), "rb") as f:
+                h.update(f.read())
+        if h.hexdigest() != rec["source_sha256"]:
+            return None
         return int(rec["dram_bytes_per_launch"])
     except Exception:
         return None

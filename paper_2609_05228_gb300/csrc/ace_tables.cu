@@ -46,7 +46,19 @@ constexpr int kTabB = 256 * kBK * 2;            // 32 KB: 256 rows j x 64 r
 constexpr int kTabStage = kTabA + kTabB;
 constexpr int kTabSmem = kTabStages * kTabStage + 1024 + 256;
 constexpr int kTile = 16384;                    // bytes of one 128 x 64 bf16 tile
-constexpr int kNormSlices = 16;                 // row slices per (expert, path) in k_gsp_norms
+
+// Fixed-order block sum of one double per thread (blockDim.x = 256).
+__device__ __forceinline__ double block_sum_256(double v, double* sh) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = v;
+    __syncthreads();
+    double t = 0.0;
+    if (threadIdx.x == 0)
+        for (int w = 0; w < 8; ++w) t += sh[w];
+    __syncthreads();
+    return t;   // valid in thread 0
+}
 
 // ---------------------------------------------------------------- packing
 //
@@ -74,25 +86,47 @@ __global__ void __launch_bounds__(256) k_pack_rows(const uint4* __restrict__ src
 }
 
 // A operand: w_p[e] is [m][d] (K = m is the slow index), so each block
-// transposes a 64 (r) x 128 (i) sub-matrix through shared memory into one tile.
-constexpr int kTrLd = 128 + 8;                  // padded row of the staging buffer (bf16)
+// transposes a 64 (r) x 128 (i) sub-matrix into one tile through shared
+// memory: coalesced 16-byte reads into a row-major staging buffer; each warp
+// then builds the 16-byte chunks of 32 consecutive tile rows i (one logical
+// chunk c at a time, conflict-free column reads) and stores them at their
+// swizzled positions in a second buffer (8 consecutive rows hit 8 distinct
+// 16-byte bank groups); the finished tile leaves in coalesced 16-byte writes.
+// The same pass accumulates the block's share of ||Gamma W_p||_F^2 =
+// sum_{r,i} gamma_i^2 W_p[i, r]^2 (one fp64 partial per block, fixed order).
+constexpr int kTrLd = 128 + 2;                  // staging row (bf16): 65 words, odd
 
 __global__ void __launch_bounds__(256) k_pack_transposed(const __nv_bfloat16* __restrict__ src,
-                                                         uint4* __restrict__ dst, int d, int m) {
+                                                         const float* __restrict__ gamma2,
+                                                         uint4* __restrict__ dst, double* __restrict__ norm_part,
+                                                         int d, int m) {
     __shared__ __align__(16) __nv_bfloat16 buf[64 * kTrLd];
+    __shared__ __align__(16) uint4 tile[1024];
+    __shared__ double sh[8];
     const int kbs = m / 64, ts = d / 128;
     const int kb = blockIdx.x % kbs;
     const int t = (blockIdx.x / kbs) % ts;
     const long long e = blockIdx.x / ((long long)kbs * ts);
     const __nv_bfloat16* s = src + (e * m + (long long)kb * 64) * d + (long long)t * 128;
+    double acc = 0.0;
     for (int q = threadIdx.x; q < 64 * 16; q += 256) {
         const int r = q >> 4, c = q & 15;          // 16 chunks of 8 along i
-        *reinterpret_cast<uint4*>(&buf[r * kTrLd + c * 8]) = *reinterpret_cast<const uint4*>(s + (long long)r * d + c * 8);
+        const uint4 v = *reinterpret_cast<const uint4*>(s + (long long)r * d + c * 8);
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+        float f[8];
+        Vec16<__nv_bfloat16>::to_float(v, f);
+        float sq = 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) sq = fmaf(gamma2[t * 128 + c * 8 + j] * f[j], f[j], sq);
+        acc += (double)sq;
+        uint32_t* row = reinterpret_cast<uint32_t*>(&buf[r * kTrLd + c * 8]);   // 4-byte aligned (kTrLd even)
+#pragma unroll
+        for (int h = 0; h < 4; ++h) row[h] = w[h];
     }
     __syncthreads();
-    uint4* out = dst + (long long)blockIdx.x * 1024;
-    for (int q = threadIdx.x; q < 1024; q += 256) {
-        const int i = q >> 3, c = (q & 7) ^ (i & 7);   // tile row i, logical chunk c: r = 8c .. 8c + 7
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int job = warp; job < 32; job += 8) {      // 4 groups of 32 rows x 8 logical chunks
+        const int i = (job & 3) * 32 + lane, c = job >> 2;
         uint32_t w[4];
 #pragma unroll
         for (int h = 0; h < 4; ++h) {
@@ -100,8 +134,13 @@ __global__ void __launch_bounds__(256) k_pack_transposed(const __nv_bfloat16* __
             const uint32_t hi = __bfloat16_as_ushort(buf[(8 * c + 2 * h + 1) * kTrLd + i]);
             w[h] = lo | (hi << 16);
         }
-        out[q] = make_uint4(w[0], w[1], w[2], w[3]);
+        tile[i * 8 + (c ^ (i & 7))] = make_uint4(w[0], w[1], w[2], w[3]);
     }
+    __syncthreads();
+    uint4* out = dst + (long long)blockIdx.x * 1024;
+    for (int q = threadIdx.x; q < 1024; q += 256) out[q] = tile[q];
+    const double tot = block_sum_256(acc, sh);
+    if (threadIdx.x == 0) norm_part[blockIdx.x] = tot;
 }
 
 // ---------------------------------------------------------------- GSP: Frobenius norms of the products
@@ -279,44 +318,6 @@ __global__ void __launch_bounds__(kTabThreads, 1) k_gsp_frob(const __grid_consta
     if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512u));
 }
 
-// Fixed-order block sum of one double per thread (blockDim.x = 256).
-__device__ __forceinline__ double block_sum_256(double v, double* sh) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = v;
-    __syncthreads();
-    double t = 0.0;
-    if (threadIdx.x == 0)
-        for (int w = 0; w < 8; ++w) t += sh[w];
-    __syncthreads();
-    return t;   // valid in thread 0
-}
-
-// ||Gamma W_p||_F^2 over one slice of rows: grid (kNormSlices, 2 paths, N).
-__global__ void __launch_bounds__(256) k_gsp_norms(const __nv_bfloat16* __restrict__ w_gate,
-                                                   const __nv_bfloat16* __restrict__ w_up,
-                                                   const float* __restrict__ gamma2, int d, int m,
-                                                   double* __restrict__ out) {
-    __shared__ double sh[8];
-    const int slice = blockIdx.x, path = blockIdx.y;
-    const long long e = blockIdx.z;
-    const __nv_bfloat16* w = (path == 0 ? w_gate : w_up) + e * m * (long long)d;
-    const int rows = m / kNormSlices, cv = d / 8;
-    const uint4* src = reinterpret_cast<const uint4*>(w + (long long)slice * rows * d);
-    double acc = 0.0;
-    for (int q = threadIdx.x; q < rows * cv; q += 256) {
-        float f[8];
-        Vec16<__nv_bfloat16>::to_float(ld_stream(src + q), f);
-        const int i0 = (q % cv) * 8;
-        float s = 0.f;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) s = fmaf(gamma2[i0 + j] * f[j], f[j], s);
-        acc += (double)s;
-    }
-    const double t = block_sum_256(acc, sh);
-    if (threadIdx.x == 0) out[(e * 2 + path) * kNormSlices + slice] = t;
-}
-
 // ---------------------------------------------------------------- RCR
 
 // Column means of the router weight: mean_i = (1/N) sum_e w_r[e, i].
@@ -425,30 +426,39 @@ __global__ void __launch_bounds__(256) k_rcr_down(const float* __restrict__ act,
 
 // ---------------------------------------------------------------- final normalisation
 
-// One block of 1024 threads; thread e combines expert e's partials in a fixed order.
-__global__ void __launch_bounds__(1024) k_tables_final(const double* __restrict__ frob, int frob_per,
-                                                       const double* __restrict__ norms,
-                                                       const double* __restrict__ rcr_part, int rcr_per,
+// Block e sums expert e's partials, each list in a fixed order (strided
+// per-thread sums, then block_sum_256): raw[e] = {||G W_down||^2,
+// ||U W_down||^2, ||G||^2, ||U||^2, ||f_e(q_e)||^2}.
+__global__ void __launch_bounds__(256) k_tables_reduce(const double* __restrict__ frob, int frob_per,
+                                                       const double* __restrict__ norms, int norm_per,
+                                                       const double* __restrict__ rcr_part, int rcr_per, int n,
+                                                       double* __restrict__ raw) {
+    __shared__ double sh[8];
+    const size_t e = blockIdx.x;
+    const double* lists[5] = {frob + (e * 2 + 0) * frob_per, frob + (e * 2 + 1) * frob_per, norms + e * norm_per,
+                              norms + ((size_t)n + e) * norm_per, rcr_part + e * rcr_per};
+    const int lens[5] = {frob_per, frob_per, norm_per, norm_per, rcr_per};
+    for (int l = 0; l < 5; ++l) {
+        double v = 0.0;
+        for (int i = threadIdx.x; i < lens[l]; i += 256) v += lists[l][i];
+        const double t = block_sum_256(v, sh);
+        if (threadIdx.x == 0) raw[e * 5 + l] = t;
+    }
+}
+
+// One block of 1024 threads: the per-expert scores and the layer normalisation.
+__global__ void __launch_bounds__(1024) k_tables_final(const double* __restrict__ raw,
                                                        const double* __restrict__ qnorm, int n, double eps,
                                                        float* __restrict__ gsp_out, float* __restrict__ rcr_out) {
     __shared__ double sg[1024], sr[1024];
     const int e = threadIdx.x;
     double ag = 0.0, ar = 0.0;
     if (e < n) {
-        double pg = 0.0, pu = 0.0, ng = 0.0, nu = 0.0, y2 = 0.0;
-        for (int t = 0; t < frob_per; ++t) {
-            pg += frob[((size_t)e * 2 + 0) * frob_per + t];
-            pu += frob[((size_t)e * 2 + 1) * frob_per + t];
-        }
-        for (int s = 0; s < kNormSlices; ++s) {
-            ng += norms[((size_t)e * 2 + 0) * kNormSlices + s];
-            nu += norms[((size_t)e * 2 + 1) * kNormSlices + s];
-        }
-        for (int b = 0; b < rcr_per; ++b) y2 += rcr_part[(size_t)e * rcr_per + b];
-        const double a_up = sqrt(nu) * sqrt(pg);      // ||U||_F ||G W_down||_F   (Eq. gsp_up_path)
-        const double a_gate = sqrt(ng) * sqrt(pu);    // ||G||_F ||U W_down||_F   (Eq. gsp_gate_path)
-        ag = sqrt(a_up * a_gate);                     // Eq. gsp_geometric_mean
-        ar = sqrt(y2) / (qnorm[e] + eps);             // Eq. rcr_raw_amplification
+        const double* r = raw + (size_t)e * 5;
+        const double a_up = sqrt(r[3]) * sqrt(r[0]);      // ||U||_F ||G W_down||_F   (Eq. gsp_up_path)
+        const double a_gate = sqrt(r[2]) * sqrt(r[1]);    // ||G||_F ||U W_down||_F   (Eq. gsp_gate_path)
+        ag = sqrt(a_up * a_gate);                         // Eq. gsp_geometric_mean
+        ar = sqrt(r[4]) / (qnorm[e] + eps);               // Eq. rcr_raw_amplification
     }
     sg[e] = ag;
     sr[e] = ar;
@@ -491,7 +501,7 @@ extern "C" ace_status ace_offline_tables_device(int d, int N, int m, const void*
         return tab_fail(ACE_ERR_INVALID_ARG, "ace_offline_tables_device: NULL pointer");
     if (d <= 0 || N <= 0 || m <= 0) return tab_fail(ACE_ERR_INVALID_ARG, "ace_offline_tables_device: sizes must be > 0");
     if (N > kMaxExperts) return tab_fail(ACE_ERR_UNSUPPORTED, "ace_offline_tables_device: N > 1024");
-    if (d % 256 || m % 64 || m % kNormSlices || d > 16384)
+    if (d % 256 || m % 64 || d > 16384)
         return tab_fail(ACE_ERR_UNSUPPORTED,
                         "ace_offline_tables_device: d must be a multiple of 256 (<= 16384), m a multiple of 64");
     if (!(eps >= 0.0)) return tab_fail(ACE_ERR_INVALID_ARG, "ace_offline_tables_device: eps must be >= 0");
@@ -508,12 +518,14 @@ extern "C" ace_status ace_offline_tables_device(int d, int N, int m, const void*
     int chunk = chunk_ll > N ? N : (int)chunk_ll;
     chunk = chunk < 1 ? 1 : chunk;
     const int ti_n = d / 128, tj_n = d / 256, frob_per = ti_n * tj_n * 4, rcr_per = d / 64;
+    const int norm_per = ti_n * (m / 64);        // k_pack_transposed blocks per expert
 
     const size_t tiles_bytes = (size_t)chunk * d * m * 2;
     size_t off = 0;
     auto take = [&](size_t bytes) { const size_t o = off; off += (bytes + 255) & ~(size_t)255; return o; };
     const size_t o_a0 = take(tiles_bytes), o_a1 = take(tiles_bytes), o_b = take(tiles_bytes);
-    const size_t o_frob = take((size_t)N * 2 * frob_per * 8), o_norm = take((size_t)N * 2 * kNormSlices * 8);
+    const size_t o_frob = take((size_t)N * 2 * frob_per * 8), o_norm = take((size_t)N * 2 * norm_per * 8);
+    const size_t o_raw = take((size_t)N * 5 * 8);
     const size_t o_mean = take((size_t)d * 8), o_x = take((size_t)N * d * 4), o_qn = take((size_t)N * 8);
     const size_t o_act = take((size_t)N * m * 4), o_rcr = take((size_t)N * rcr_per * 8);
     const size_t o_g2 = take((size_t)d * 4), o_out = take((size_t)2 * N * 4), o_err = take(4);
@@ -542,15 +554,16 @@ extern "C" ace_status ace_offline_tables_device(int d, int N, int m, const void*
     TAB_CK(cudaMemsetAsync(err, 0, 4, s));
     k_gamma2<<<(d + 255) / 256, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(gamma), g2, d);
     TAB_CK(cudaGetLastError());
-    k_gsp_norms<<<dim3(kNormSlices, 2, N), 256, 0, s>>>(wg, wu, g2, d, m, reinterpret_cast<double*>(base + o_norm));
-    TAB_CK(cudaGetLastError());
     for (int e0 = 0; e0 < N; e0 += chunk) {
         const int n_e = N - e0 < chunk ? N - e0 : chunk;
         const size_t eo = (size_t)e0 * m * d;
         const int tblocks = n_e * ti_n * (m / 64);
-        k_pack_transposed<<<tblocks, 256, 0, s>>>(wg + eo, reinterpret_cast<uint4*>(base + o_a0), d, m);
+        double* norm = reinterpret_cast<double*>(base + o_norm);   // [path][e][norm_per]
+        k_pack_transposed<<<tblocks, 256, 0, s>>>(wg + eo, g2, reinterpret_cast<uint4*>(base + o_a0),
+                                                  norm + (size_t)e0 * norm_per, d, m);
         TAB_CK(cudaGetLastError());
-        k_pack_transposed<<<tblocks, 256, 0, s>>>(wu + eo, reinterpret_cast<uint4*>(base + o_a1), d, m);
+        k_pack_transposed<<<tblocks, 256, 0, s>>>(wu + eo, g2, reinterpret_cast<uint4*>(base + o_a1),
+                                                  norm + ((size_t)N + e0) * norm_per, d, m);
         TAB_CK(cudaGetLastError());
         k_pack_rows<<<sms * 8, 256, 0, s>>>(reinterpret_cast<const uint4*>(wd + eo), reinterpret_cast<uint4*>(base + o_b),
                                             n_e, d, m);
@@ -583,9 +596,12 @@ extern "C" ace_status ace_offline_tables_device(int d, int N, int m, const void*
     k_rcr_down<<<dim3(d / 64, N), 256, m * 4, s>>>(reinterpret_cast<const float*>(base + o_act), wd, d, m,
                                                    reinterpret_cast<double*>(base + o_rcr));
     TAB_CK(cudaGetLastError());
-    k_tables_final<<<1, 1024, 0, s>>>(reinterpret_cast<const double*>(base + o_frob), frob_per,
-                                      reinterpret_cast<const double*>(base + o_norm),
-                                      reinterpret_cast<const double*>(base + o_rcr), rcr_per,
+    k_tables_reduce<<<N, 256, 0, s>>>(reinterpret_cast<const double*>(base + o_frob), frob_per,
+                                      reinterpret_cast<const double*>(base + o_norm), norm_per,
+                                      reinterpret_cast<const double*>(base + o_rcr), rcr_per, N,
+                                      reinterpret_cast<double*>(base + o_raw));
+    TAB_CK(cudaGetLastError());
+    k_tables_final<<<1, 1024, 0, s>>>(reinterpret_cast<const double*>(base + o_raw),
                                       reinterpret_cast<const double*>(base + o_qn), N, eps, out, out + N);
     TAB_CK(cudaGetLastError());
     TAB_CK(cudaMemcpyAsync(gsp_out, out, (size_t)N * 4, cudaMemcpyDeviceToHost, s));
