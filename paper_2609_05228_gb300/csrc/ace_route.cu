@@ -923,6 +923,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
 // --------------------------------------------------------------------------
 constexpr int kFuseTok = 8;
 constexpr int kFuseWarps = 8;
+constexpr long long kRoutePrefetchBytes = 48LL << 20;   // decode: leading W_gu bytes pulled towards L2 while routing
 
 struct FusedArgs {
     const void* x;
@@ -959,6 +960,8 @@ struct FusedArgs {
     int32_t* tt_off;
     int4* tt_tab;
     int32_t* tile_cnt;
+    const uint8_t* pf_base;     // expert weights to start pulling into L2 while routing runs
+    long long pf_bytes;         // (a multiple of 256 bytes; 0 = none)
 };
 
 __host__ __device__ inline size_t fused_phase_c_bytes(int T, int k, int n_exp) {
@@ -1004,6 +1007,16 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         pdl_wait();                                               // x is the predecessor's output
         if (threadIdx.x == 0) bulk_g2s(xs, static_cast<const T*>(a.x) + (size_t)t0 * d, (uint32_t)nt * row_bytes, bar);
         if (!mbar_wait(bar, 0, a.err)) return;
+        if (a.pf_bytes > 0) {
+            // HBM idles while routing runs: pull the leading expert-weight
+            // tiles towards L2 (per-thread line prefetches; a bulk prefetch
+            // holds up the SM's copy engine and delays this kernel)
+            const long long units = a.pf_bytes >> 8;
+            const long long nthr = (long long)gridDim.x * gridDim.y * blockDim.x;
+            for (long long u = ((long long)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x; u < units;
+                 u += nthr)
+                asm volatile("prefetch.global.L2::evict_last [%0];" ::"l"(a.pf_base + (u << 8)) : "memory");
+        }
         const uint4* gv = reinterpret_cast<const uint4*>(gs);
         if (warp < nt) {
             // h = x / sqrt(mean(x^2) + eps) * gamma, rounded to T (the stored h feeds the router)
@@ -1305,6 +1318,12 @@ cudaError_t launch_route_fused(const ace_layer* L, const void* x, const float* l
     a.tt_off = W.tt_off;
     a.tt_tab = W.tt_tab;
     a.tile_cnt = W.tile_cnt;
+    if (x && L->tc && L->w_gu) {
+        const long long gu_bytes = 2LL * D.ffn * D.hidden * 2 * D.n_experts;
+        const long long want = kRoutePrefetchBytes;
+        a.pf_base = static_cast<const uint8_t*>(L->w_gu);
+        a.pf_bytes = (want < gu_bytes ? want : gu_bytes) & ~255LL;
+    }
     const bool bf = D.dtype == ACE_BF16;
     if (x) return bf ? fused_dispatch<__nv_bfloat16, true>(L, a, T, s) : fused_dispatch<float, true>(L, a, T, s);
     return bf ? fused_dispatch<__nv_bfloat16, false>(L, a, T, s) : fused_dispatch<float, false>(L, a, T, s);
