@@ -460,57 +460,79 @@ __device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem
     return tau;
 }
 
-// Exclusive scan of cnt[0..n_exp) by warp 0 of the block: offsets[e],
-// offsets[n_exp] = total, the distinct-expert list and the meta totals.
-// Also fills off_s (shared) when given.
-// With tok_tile > 0 it also writes tt_off[j] = sum over distinct experts
-// before j of ceil(count / tok_tile) (the token-tile schedule of the
-// tensor-core experts) and tt_off[D].
-__device__ void scan_counts_warp0(const int* cnt, int n_exp, int32_t* __restrict__ offsets,
+// Exclusive scan of cnt[0..n_exp) by the whole block (called by every
+// thread; blockDim.x a multiple of 32, at most 1024): offsets[e],
+// offsets[n_exp] = total, the distinct-expert list (increasing) and the meta
+// totals; also off_s (shared) when given. With tok_tile > 0 it also writes
+// tt_off[j] = sum over distinct experts before j of ceil(count / tok_tile)
+// (the token-tile schedule of the tensor-core experts) and tt_off[D].
+// Each thread scans a contiguous run of experts; the three running sums are
+// combined by warp shuffles and one pass over the per-warp totals in wsum
+// (shared, 3 x 32 ints).
+__device__ void scan_counts_block(const int* cnt, int n_exp, int32_t* __restrict__ offsets,
                                   int32_t* __restrict__ dlist, int32_t* __restrict__ meta, int* off_s,
-                                  int tok_tile, int32_t* __restrict__ tt_off) {
-    const int lane = threadIdx.x;
-    const int per = (n_exp + 31) / 32;
-    const int e0 = min(lane * per, n_exp), e1 = min(e0 + per, n_exp);
+                                  int tok_tile, int32_t* __restrict__ tt_off, int* wsum) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+    const int per = (n_exp + blockDim.x - 1) / blockDim.x;
+    const int e0 = min(tid * per, n_exp), e1 = min(e0 + per, n_exp);
     const int tt = tok_tile > 0 ? tok_tile : 1;
     int s = 0, dcount = 0, tiles = 0;
     for (int e = e0; e < e1; ++e) {
-        s += cnt[e];
-        dcount += cnt[e] > 0;
-        tiles += (cnt[e] + tt - 1) / tt;
+        const int c = cnt[e];
+        s += c;
+        dcount += c > 0;
+        tiles += (c + tt - 1) / tt;
     }
     int xs = s, xd = dcount, xt = tiles;
+#pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
         const int ys = __shfl_up_sync(0xffffffffu, xs, o);
         const int yd = __shfl_up_sync(0xffffffffu, xd, o);
         const int yt = __shfl_up_sync(0xffffffffu, xt, o);
         if (lane >= o) { xs += ys; xd += yd; xt += yt; }
     }
-    int run = xs - s, drun = xd - dcount, trun = xt - tiles;
+    if (lane == 31) { wsum[warp] = xs; wsum[32 + warp] = xd; wsum[64 + warp] = xt; }
+    __syncthreads();
+    if (warp == 0) {
+        int vs = lane < nw ? wsum[lane] : 0, vd = lane < nw ? wsum[32 + lane] : 0, vt = lane < nw ? wsum[64 + lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int ys = __shfl_up_sync(0xffffffffu, vs, o);
+            const int yd = __shfl_up_sync(0xffffffffu, vd, o);
+            const int yt = __shfl_up_sync(0xffffffffu, vt, o);
+            if (lane >= o) { vs += ys; vd += yd; vt += yt; }
+        }
+        wsum[lane] = vs;
+        wsum[32 + lane] = vd;
+        wsum[64 + lane] = vt;
+    }
+    __syncthreads();
+    int run = xs - s + (warp ? wsum[warp - 1] : 0);
+    int drun = xd - dcount + (warp ? wsum[32 + warp - 1] : 0);
+    int trun = xt - tiles + (warp ? wsum[64 + warp - 1] : 0);
     for (int e = e0; e < e1; ++e) {
+        const int c = cnt[e];
         offsets[e] = run;
         if (off_s) off_s[e] = run;
-        run += cnt[e];
-        if (cnt[e] > 0) {
+        run += c;
+        if (c > 0) {
             if (tok_tile > 0) tt_off[drun] = trun;
-            trun += (cnt[e] + tt - 1) / tt;
+            trun += (c + tt - 1) / tt;
             dlist[drun++] = e;
         }
     }
-    const int total = __shfl_sync(0xffffffffu, xs, 31);
-    const int dtotal = __shfl_sync(0xffffffffu, xd, 31);
-    const int ttotal = __shfl_sync(0xffffffffu, xt, 31);
-    if (lane == 31) {
-        offsets[n_exp] = total;
-        if (off_s) off_s[n_exp] = total;
-        if (tok_tile > 0) tt_off[dtotal] = ttotal;
-        meta[kMetaRetained] = total;
-        meta[kMetaDistinct] = dtotal;
-        meta[kMetaTokTiles] = tok_tile > 0 ? ttotal : 0;
+    if (tid == blockDim.x - 1) {       // its running sums end at the totals
+        offsets[n_exp] = run;
+        if (off_s) off_s[n_exp] = run;
+        if (tok_tile > 0) tt_off[drun] = trun;
+        meta[kMetaRetained] = run;
+        meta[kMetaDistinct] = drun;
+        meta[kMetaTokTiles] = tok_tile > 0 ? trun : 0;
     }
+    __syncthreads();                   // wsum may be reused by the caller
 }
 
-// After scan_counts_warp0 and a block barrier: the flat token-tile table of
+// After scan_counts_block and a block barrier: the flat token-tile table of
 // the tensor-core experts, tt_tab[tt] = (expert, first row, rows, 0).
 __device__ void fill_tile_table(const int32_t* offsets, const int32_t* dlist, const int32_t* tt_off,
                                 const int32_t* meta, int tok_tile, int4* tt_tab) {
@@ -822,6 +844,7 @@ __global__ void __launch_bounds__(1024) k_compact_scan(int n_exp, int n_chunks, 
                                                        int32_t* __restrict__ meta, int tok_tile,
                                                        int32_t* __restrict__ tt_off, int4* __restrict__ tt_tab) {
     __shared__ int wtot[32];
+    __shared__ int wsum[96];
     __shared__ int cnt[kMaxExperts];
     __shared__ __align__(16) int buf[1024 * kScanPer];
     pdl_wait();
@@ -869,7 +892,7 @@ __global__ void __launch_bounds__(1024) k_compact_scan(int n_exp, int n_chunks, 
     __syncthreads();
     for (int e = tid; e < n_exp; e += blockDim.x) cnt[e] = __ldcg(offsets + e + 1) - __ldcg(offsets + e);
     __syncthreads();
-    if (tid < 32) scan_counts_warp0(cnt, n_exp, offsets, dlist, meta, nullptr, tok_tile, tt_off);
+    scan_counts_block(cnt, n_exp, offsets, dlist, meta, nullptr, tok_tile, tt_off, wsum);
     __syncthreads();
     fill_tile_table(offsets, dlist, tt_off, meta, tok_tile, tt_tab);
 }
@@ -1007,16 +1030,6 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         pdl_wait();                                               // x is the predecessor's output
         if (threadIdx.x == 0) bulk_g2s(xs, static_cast<const T*>(a.x) + (size_t)t0 * d, (uint32_t)nt * row_bytes, bar);
         if (!mbar_wait(bar, 0, a.err)) return;
-        if (a.pf_bytes > 0) {
-            // HBM idles while routing runs: pull the leading expert-weight
-            // tiles towards L2 (per-thread line prefetches; a bulk prefetch
-            // holds up the SM's copy engine and delays this kernel)
-            const long long units = a.pf_bytes >> 8;
-            const long long nthr = (long long)gridDim.x * gridDim.y * blockDim.x;
-            for (long long u = ((long long)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x; u < units;
-                 u += nthr)
-                asm volatile("prefetch.global.L2::evict_last [%0];" ::"l"(a.pf_base + (u << 8)) : "memory");
-        }
         const uint4* gv = reinterpret_cast<const uint4*>(gs);
         if (warp < nt) {
             // h = x / sqrt(mean(x^2) + eps) * gamma, rounded to T (the stored h feeds the router)
@@ -1085,7 +1098,21 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
             if (s_last) a.tile_cnt[blockIdx.x] = 0;
         }
         __syncthreads();
-        if (!s_last) return;
+        if (!s_last) {
+            if (a.pf_bytes > 0) {
+                // HBM idles while the rest of the routing runs: the blocks
+                // that leave here pull the leading expert-weight tiles towards
+                // L2 (per-thread line prefetches: a bulk prefetch occupies the
+                // SM's copy engine), off the path of the blocks that go on
+                // (the lines of the continuing blocks' shares are left out)
+                const long long units = a.pf_bytes >> 8;
+                const long long nthr = (long long)gridDim.x * gridDim.y * blockDim.x;
+                const long long b = (long long)blockIdx.y * gridDim.x + blockIdx.x;
+                for (long long u = b * blockDim.x + threadIdx.x; u < units; u += nthr)
+                    asm volatile("prefetch.global.L2::evict_last [%0];" ::"l"(a.pf_base + (u << 8)) : "memory");
+            }
+            return;
+        }
         __threadfence();
     } else {
         pdl_wait();                                               // logits are the predecessor's output
@@ -1172,7 +1199,7 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         atomicOr(&bm[e * 8 + (t >> 5)], 1u << (t & 31));
     }
     __syncthreads();
-    if (threadIdx.x < 32) scan_counts_warp0(cnt, n_exp, a.offsets, a.dlist, a.meta, off_s, a.tok_tile, a.tt_off);
+    scan_counts_block(cnt, n_exp, a.offsets, a.dlist, a.meta, off_s, a.tok_tile, a.tt_off, S.hist);
     __syncthreads();
     fill_tile_table(a.offsets, a.dlist, a.tt_off, a.meta, a.tok_tile, a.tt_tab);
     for (int s = threadIdx.x; s < ns; s += blockDim.x) {
