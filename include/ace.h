@@ -130,9 +130,8 @@ void ace_layer_destroy(ace_layer* layer);
  * (Eq. ace_sparse_output), with RMSNorm, router, top-k, the skip decision of
  * Algorithm 4, compaction of the retained slots and the SwiGLU experts all on
  * the GPU. out = y, or x + y when the layer was created with add_residual.
- * Batches of T <= 256 sum a token's slot outputs in rank order (bitwise
- * reproducible); larger batches accumulate them with fp32 atomics (results
- * may differ between runs in the last bit).
+ * The combine sums a token's slot outputs in rank order (fp32 slot rows for
+ * T <= 256, bf16 slot rows above), so repeated calls give the same bits.
  *   x    [T, d]  device, dtype     layer input (pre-RMSNorm hidden states)
  *   out  [T, d]  device, dtype     layer output; must not alias x
  *   T    0..max_tokens             T = 0 is a no-op

@@ -71,6 +71,27 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
     return v;
 }
 
+// L2 cache policy that marks the lines a load touches as evict-last.
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
+// 16-byte load with an L2 cache policy.
+__device__ __forceinline__ uint4 ld_l2_keep(const void* p, uint64_t policy) {
+    uint4 v;
+    asm volatile("ld.global.L2::cache_hint.v4.u32 {%0,%1,%2,%3}, [%4], %5;"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p), "l"(policy));
+    return v;
+}
+
+// 16-byte streaming store (data read once later: evict first).
+__device__ __forceinline__ void st_stream(void* p, const uint4& v) {
+    asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
 // exp(x) for float32 x <= 0 in a fixed operation sequence (each multiply and
 // add rounded to nearest even, none fused), so that the gates are
 // reproducible bit for bit by any implementation following the same steps:

@@ -889,6 +889,9 @@ __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __rest
     const int nvec = d / 8;
     const int lane = threadIdx.x & 31;
     const int wpb = blockDim.x >> 5;
+    // h rows are read once per retained slot (k times a token at most): keep
+    // them in L2; the h_perm rows are read once, by GEMM 1's TMA: stream them
+    const uint64_t keep = l2_policy_evict_last();
     for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < R; r += gridDim.x * wpb) {
         const int tok = perm[r] / k;
         const uint4* src = reinterpret_cast<const uint4*>(h + (size_t)tok * d);
@@ -897,12 +900,12 @@ __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __rest
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
             const int c = lane + 32 * i;
-            if (c < nvec) v[i] = src[c];
+            if (c < nvec) v[i] = ld_l2_keep(src + c, keep);
         }
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
             const int c = lane + 32 * i;
-            if (c < nvec) dst[c] = v[i];
+            if (c < nvec) st_stream(dst + c, v[i]);
         }
     }
 }
