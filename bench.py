@@ -559,21 +559,26 @@ def run_reference(args):
         else:   # the arm stays on the host: seeded positive tables stand in for the GPU tables
             w.extra["a_gsp"], w.extra["a_rcr"] = synth.make_tables(spec.n_experts, seed=5, spread=0.1)
         ws.append(w)
-    T = wl["T"] if wl["T"] <= 64 else 256
-    x = synth.make_tokens(spec, T, seed=1)
+    xall = synth.make_tokens(spec, min(wl["T"], 256), seed=1)
 
-    def step():
-        cur = O.to_f64(x)
+    def step(T):
+        cur = O.to_f64(xall[:T])
         for w in ws:
             y = O.moe_forward(cur, w, "ratio", wl["q"])
             cur = cur + y if len(ws) > 1 else y
 
+    # tokens per step: the whole run (warm-up + steps) is sized to about two
+    # minutes of oracle time, from a one-step rate estimate on 8 tokens
+    t = time.perf_counter()
+    step(min(8, xall.shape[0]))
+    rate = min(8, xall.shape[0]) / (time.perf_counter() - t)
+    T = int(max(1, min(xall.shape[0], rate * 120.0 / (args.steps + args.warmup))))
     for _ in range(args.warmup):
-        step()
+        step(T)
     times = []
     for _ in range(args.steps):
         t = time.perf_counter()
-        step()
+        step(T)
         times.append(time.perf_counter() - t)
     st = float(np.mean(times))
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
