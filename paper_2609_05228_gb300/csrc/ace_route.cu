@@ -946,6 +946,8 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
 // --------------------------------------------------------------------------
 constexpr int kFuseTok = 8;
 constexpr int kFuseWarps = 8;
+constexpr int kRowPad = 16;    // bytes appended to each row staged by phase A
+static_assert(kFuseTok == 8 && kFuseWarps == 8, "phase A's MMA takes 8 token rows x 8 router rows");
 constexpr long long kRoutePrefetchBytes = 48LL << 20;   // decode: leading W_gu bytes pulled towards L2 while routing
 
 struct FusedArgs {
@@ -1003,37 +1005,48 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
     const int n_exp = a.n_exp, k = a.k;
     if (LOGITS) {
         // ---------------- phase A: RMSNorm + logits for 8 tokens x 8 experts.
-        // One thread bulk-copies gamma and the block's 8 router rows (layer
+        // Warp 0 bulk-copies gamma and the block's 8 router rows (layer
         // constants, before the dependency wait) and the tile's x rows into
-        // shared memory, so the block waits for one round trip; the rows
-        // are then normalised in place and the dot products read shared memory.
+        // shared memory, one row per lane, so the block waits for one round
+        // trip; the rows are then normalised in place and the dot products
+        // read shared memory. Staged rows are kRowPad bytes longer than a row,
+        // which spreads the 8 rows of an MMA operand load over all 32 banks.
         const int d = a.d;
         constexpr int V = Vec16<T>::N;
         const int nvec = d / V;
+        const uint32_t row_bytes = (uint32_t)(d * sizeof(T));
+        const uint32_t rs = row_bytes + kRowPad;                  // staged row stride
         uint64_t* bar = reinterpret_cast<uint64_t*>(smem_raw);
-        T* xs = reinterpret_cast<T*>(smem_raw + 16);             // [kFuseTok][d] -> h in place
-        T* gs = xs + (size_t)kFuseTok * d;                        // [d]
-        T* wsm = gs + d;                                          // [kFuseWarps][d]
+        unsigned char* xs = smem_raw + 16;                        // [kFuseTok] rows -> h in place
+        unsigned char* gs = xs + (size_t)kFuseTok * rs;           // gamma
+        unsigned char* wsm = gs + rs;                             // [kFuseWarps] router rows
+        float* red = reinterpret_cast<float*>(wsm + (size_t)kFuseWarps * rs);   // [warps][8][8] partial logits
         const int e0 = blockIdx.y * kFuseWarps;
         const int ne = min(kFuseWarps, n_exp - e0);
-        const uint32_t row_bytes = (uint32_t)(d * sizeof(T));
         if (threadIdx.x == 0) {
             mbar_init(bar, 1);
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         }
         __syncthreads();
-        if (threadIdx.x == 0) {
-            mbar_expect_tx(bar, (uint32_t)(nt + 1 + ne) * row_bytes);
-            bulk_g2s(gs, a.gamma, row_bytes, bar);
-            bulk_g2s(wsm, static_cast<const T*>(a.w_r) + (size_t)e0 * d, (uint32_t)ne * row_bytes, bar);
+        if (warp == 0) {
+            if (lane == 0) {
+                mbar_expect_tx(bar, (uint32_t)(nt + 1 + ne) * row_bytes);
+                bulk_g2s(gs, a.gamma, row_bytes, bar);
+            }
+            __syncwarp();
+            if (lane < ne) bulk_g2s(wsm + (size_t)lane * rs, static_cast<const T*>(a.w_r) + (size_t)(e0 + lane) * d,
+                                    row_bytes, bar);
+            pdl_wait();                                           // x is the predecessor's output
+            if (lane < nt) bulk_g2s(xs + (size_t)lane * rs, static_cast<const T*>(a.x) + (size_t)(t0 + lane) * d,
+                                    row_bytes, bar);
+        } else {
+            pdl_wait();
         }
-        pdl_wait();                                               // x is the predecessor's output
-        if (threadIdx.x == 0) bulk_g2s(xs, static_cast<const T*>(a.x) + (size_t)t0 * d, (uint32_t)nt * row_bytes, bar);
         if (!mbar_wait(bar, 0, a.err)) return;
         const uint4* gv = reinterpret_cast<const uint4*>(gs);
         if (warp < nt) {
             // h = x / sqrt(mean(x^2) + eps) * gamma, rounded to T (the stored h feeds the router)
-            uint4* xr = reinterpret_cast<uint4*>(xs) + (size_t)warp * nvec;
+            uint4* xr = reinterpret_cast<uint4*>(xs + (size_t)warp * rs);
             float ss = 0.f;
 #pragma unroll 1
             for (int c = lane; c < nvec; c += 32) {
@@ -1061,10 +1074,47 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         }
         __syncthreads();
         if (threadIdx.x == 0) mbar_inval(bar);
-        if (warp < ne) {
+        if (sizeof(T) == 2 && d % (16 * kFuseWarps) == 0) {
+            // bf16: warp w takes K slice w and runs mma.sync m16n8k16 over it
+            // (A = the 8 token rows, zero-padded to 16; B = the 8 router rows;
+            // products exact, fp32 accumulation); the 8 partial 8 x 8 blocks
+            // are summed in warp order
+            const int g = lane >> 2, tq = lane & 3;
+            const int kslice = d / kFuseWarps;
+            const unsigned char* xrow = xs + (size_t)g * rs;
+            const unsigned char* wrow = wsm + (size_t)g * rs;
+            float c0 = 0.f, c1 = 0.f, c2 = 0.f, c3 = 0.f;
+#pragma unroll 4
+            for (int ks = 0; ks < kslice; ks += 16) {
+                const int kb = (warp * kslice + ks + 2 * tq) * 2;     // byte offset in the row
+                const uint32_t a0 = *reinterpret_cast<const uint32_t*>(xrow + kb);
+                const uint32_t a2 = *reinterpret_cast<const uint32_t*>(xrow + kb + 16);
+                const uint32_t b0 = *reinterpret_cast<const uint32_t*>(wrow + kb);
+                const uint32_t b1 = *reinterpret_cast<const uint32_t*>(wrow + kb + 16);
+                asm volatile(
+                    "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+                    "{%0,%1,%2,%3};"
+                    : "+f"(c0), "+f"(c1), "+f"(c2), "+f"(c3)
+                    : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+            }
+            // c0, c1: token g, experts 2 tq and 2 tq + 1 (rows 8..15 are padding)
+            red[(warp * 8 + g) * 8 + 2 * tq] = c0;
+            red[(warp * 8 + g) * 8 + 2 * tq + 1] = c1;
+            __syncthreads();
+            if (threadIdx.x < 64) {
+                const int r = threadIdx.x >> 3, j = threadIdx.x & 7;
+                float v = 0.f;
+#pragma unroll
+                for (int w = 0; w < kFuseWarps; ++w) v += red[(w * 8 + r) * 8 + j];
+                if (r < nt && j < ne) {
+                    v = v + a.b_r[e0 + j];
+                    if (a.use_temp) v = v * a.inv_temp;
+                    a.logits[(size_t)(t0 + r) * n_exp + e0 + j] = v;
+                }
+            }
+        } else if (warp < ne) {
             const int e = e0 + warp;
-            const uint4* wr = reinterpret_cast<const uint4*>(wsm) + (size_t)warp * nvec;
-            const uint4* hx = reinterpret_cast<const uint4*>(xs);
+            const uint4* wr = reinterpret_cast<const uint4*>(wsm + (size_t)warp * rs);
             float acc[kFuseTok];
 #pragma unroll
             for (int r = 0; r < kFuseTok; ++r) acc[r] = 0.f;
@@ -1075,7 +1125,7 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
 #pragma unroll
                 for (int r = 0; r < kFuseTok; ++r) {
                     float hf[V];
-                    Vec16<T>::to_float(hx[(size_t)r * nvec + c], hf);
+                    Vec16<T>::to_float(reinterpret_cast<const uint4*>(xs + (size_t)r * rs)[c], hf);
 #pragma unroll
                     for (int j = 0; j < V; ++j) acc[r] = fmaf(hf[j], wf[j], acc[r]);
                 }
@@ -1214,7 +1264,8 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
 }
 
 size_t fused_smem_bytes(const ace_layer* L, int T) {
-    const size_t a = 16 + (size_t)(kFuseTok + 1 + kFuseWarps) * L->desc.hidden * L->elem;
+    const size_t a = 16 + (size_t)(kFuseTok + 1 + kFuseWarps) * (L->desc.hidden * L->elem + kRowPad) +
+                     (size_t)kFuseWarps * 64 * sizeof(float);
     const size_t c = fused_phase_c_bytes(T, L->desc.top_k, L->desc.n_experts);
     return a > c ? a : c;
 }
