@@ -144,6 +144,35 @@ ace_status ace_moe_forward(ace_layer* layer, const void* x, void* out, int T,
                            ace_skip_ctl ctl, void* stream);
 
 /*
+ * Stacks of layers (a decoder block's MoE layers in sequence):
+ *   x_{l+1} = x_l + MoE_l(x_l),  out = x_L
+ * ace_stack_create takes n_layers distinct layers, each created with
+ * add_residual, bf16 and on the tensor-core path (d a multiple of 256, m a
+ * multiple of 128), sharing d and the device; the stack holds pointers to
+ * them (they must outlive it) and two [max_tokens, d] buffers for the
+ * intermediate outputs, max_tokens being the smallest of the layers'.
+ * ace_stack_forward runs the layers on `stream` with one skip control for
+ * all. For T > 256 each layer's combine also computes the next layer's
+ * RMSNorm from the rounded output it writes, so the next layer starts at its
+ * router (one kernel and one read of the [T, d] activations fewer per layer);
+ * the result is bit-identical to chaining ace_moe_forward calls. After the
+ * call, each layer's ace_last_* functions describe its own part.
+ * Errors: INVALID_ARG (NULL, duplicates, mismatched layers, T out of range,
+ * aliasing, bad control), UNSUPPORTED (a layer not on the tensor-core
+ * path), OOM, CUDA.
+ */
+typedef struct ace_stack ace_stack;   /* opaque */
+ace_status ace_stack_create(ace_layer* const* layers, int n_layers, ace_stack** out_stack);
+ace_status ace_stack_forward(ace_stack* stack, const void* x, void* out, int T, ace_skip_ctl ctl, void* stream);
+/* The same from HOST buffers x_host, out_host [T, d] bf16: one copy in, the
+ * stack, one copy out; synchronises `stream` and reports the layers' device
+ * error words. */
+ace_status ace_stack_forward_host(ace_stack* stack, const void* x_host, void* out_host, int T, ace_skip_ctl ctl,
+                                  void* stream);
+/* Frees the stack's buffers (not the layers). NULL is a no-op. Synchronises the device. */
+void ace_stack_destroy(ace_stack* stack);
+
+/*
  * ace_moe_forward_host — the same forward from HOST buffers: copies x to a
  * layer-owned device buffer, runs ace_moe_forward, copies the result back
  * and synchronises `stream` before returning.

@@ -73,6 +73,10 @@ def lib() -> ctypes.CDLL:
             "ace_last_launch_count": (_S, [_P, _P]),
             "ace_route_decide_noalloc": (_S, [_P, _I, _I, _I, _P, _P, ctypes.c_float, _I, ace_skip_ctl, _P, _P, _P,
                                               _P, _P]),
+            "ace_stack_create": (_S, [ctypes.POINTER(_P), _I, ctypes.POINTER(_P)]),
+            "ace_stack_forward": (_S, [_P, _P, _P, _I, ace_skip_ctl, _P]),
+            "ace_stack_destroy": (None, [_P]),
+            "ace_stack_forward_host": (_S, [_P, _P, _P, _I, ace_skip_ctl, _P]),
             "ace_offline_tables_device": (_S, [_I, _I, _I, _P, _P, _P, _P, _P, ctypes.c_double, _I, ctypes.c_size_t,
                                                _P, _P, _P]),
             "ace_status_string": (ctypes.c_char_p, [_S]),
@@ -152,6 +156,29 @@ def ace_moe_forward_host(layer: int, x_host, out_host, T: int, mode, value: floa
 
 def ace_route_logits(layer: int, logits, T: int, mode, value: float, stream=None, fusion=ACE_FUSION_MAX) -> None:
     _check(lib().ace_route_logits(layer, _ptr(logits), int(T), _ctl(mode, value, fusion), _stream(stream)))
+
+
+def ace_stack_create(layers) -> int:
+    """A stack over layer handles (ints); the layers must outlive it."""
+    arr = (_P * len(layers))(*[int(h) for h in layers])
+    out = _P()
+    _check(lib().ace_stack_create(arr, len(layers), ctypes.byref(out)))
+    return out.value
+
+
+def ace_stack_forward(stack: int, x, out, T: int, mode, value: float, stream=None, fusion=ACE_FUSION_MAX) -> None:
+    _check(lib().ace_stack_forward(stack, _ptr(x), _ptr(out), int(T), _ctl(mode, value, fusion), _stream(stream)))
+
+
+def ace_stack_forward_host(stack: int, x_host, out_host, T: int, mode, value: float, stream=None,
+                           fusion=ACE_FUSION_MAX) -> None:
+    _check(lib().ace_stack_forward_host(stack, _ptr(x_host), _ptr(out_host), int(T), _ctl(mode, value, fusion),
+                                        _stream(stream)))
+
+
+def ace_stack_destroy(stack: int) -> None:
+    if stack:
+        lib().ace_stack_destroy(stack)
 
 
 def ace_last_skip_mask(layer: int, T: int, k: int):

@@ -279,14 +279,16 @@ ace_status ace_route_logits(ace_layer* L, const float* logits, int T, ace_skip_c
     return ACE_OK;
 }
 
-ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_skip_ctl ctl, void* stream) {
-    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
-    if (T < 0 || T > L->desc.max_tokens) return fail(ACE_ERR_INVALID_ARG, "T out of range [0, max_tokens]");
-    if (T > 0 && (!x || !out)) return fail(ACE_ERR_INVALID_ARG, "x and out must be non-NULL");
-    if (T > 0 && x == out) return fail(ACE_ERR_INVALID_ARG, "out must not alias x");
-    ace_status st = check_ctl(ctl);
-    if (st != ACE_OK) return st;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
+}  // extern "C"
+
+namespace {
+
+// One layer's forward. In a stack (T > 256 only): h_ready = the previous
+// layer's combine has already written RMSNorm(x) into L->ws.h, so the
+// RMSNorm launch is left out; next = the following layer, whose RMSNorm of
+// `out` this layer's combine writes into next->ws.h.
+ace_status forward_impl(ace_layer* L, const void* x, void* out, int T, ace_skip_ctl ctl, cudaStream_t s,
+                        const ace_layer* next, bool h_ready) {
     L->last_T = T;
     L->last_ctl = ctl;
     L->last_stream = s;
@@ -295,8 +297,9 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
     if (T == 0) return ACE_OK;
     cudaEvent_t* ev = L->profiling ? L->ev : nullptr;
     const bool small = ace::small_path(T);
+    if (small) next = nullptr, h_ready = false;
     if (ev) ACE_CUDA(ace::record_stage(ev[0], s), "event record");
-    if (!small) ACE_CUDA(ace::launch_rmsnorm(L, x, T, s), "rmsnorm launch");
+    if (!small && !h_ready) ACE_CUDA(ace::launch_rmsnorm(L, x, T, s), "rmsnorm launch");
     if (ev) ACE_CUDA(ace::record_stage(ev[1], s), "event record");
     if (small) {
         // router and routing in one launch (stage "router" holds both)
@@ -313,13 +316,120 @@ ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_sk
     }
     if (ev) ACE_CUDA(ace::record_stage(ev[3], s), "event record");
     if (L->tc) {
-        ACE_CUDA(ace::launch_experts_tc(L, x, out, T, ctl, s, ev ? ev + 4 : nullptr), "expert launch");
+        ACE_CUDA(ace::launch_experts_tc(L, x, out, T, ctl, s, ev ? ev + 4 : nullptr, next), "expert launch");
     } else {
         if (ev) ACE_CUDA(ace::record_stage(ev[4], s), "event record");   // no gather stage
         ACE_CUDA(ace::launch_experts_gemv(L, x, out, T, s, ev ? ev + 4 : nullptr), "expert launch");
     }
     L->n_stages = ev ? ace::kNumStages : 0;
-    L->last_launches = (small ? 1 : 2 + ace::route_launch_count(L, T, ctl)) + (L->tc ? (small ? 3 : 4) : 3);
+    L->last_launches = (small ? 1 : (h_ready ? 1 : 2) + ace::route_launch_count(L, T, ctl)) +
+                       (L->tc ? (small ? 3 : 4) : 3);
+    return ACE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+ace_status ace_moe_forward(ace_layer* L, const void* x, void* out, int T, ace_skip_ctl ctl, void* stream) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    if (T < 0 || T > L->desc.max_tokens) return fail(ACE_ERR_INVALID_ARG, "T out of range [0, max_tokens]");
+    if (T > 0 && (!x || !out)) return fail(ACE_ERR_INVALID_ARG, "x and out must be non-NULL");
+    if (T > 0 && x == out) return fail(ACE_ERR_INVALID_ARG, "out must not alias x");
+    ace_status st = check_ctl(ctl);
+    if (st != ACE_OK) return st;
+    return forward_impl(L, x, out, T, ctl, static_cast<cudaStream_t>(stream), nullptr, false);
+}
+
+ace_status ace_stack_create(ace_layer* const* layers, int n_layers, ace_stack** out_stack) {
+    if (!out_stack) return fail(ACE_ERR_INVALID_ARG, "out_stack is NULL");
+    *out_stack = nullptr;
+    if (!layers || n_layers < 1) return fail(ACE_ERR_INVALID_ARG, "need at least one layer");
+    int max_tokens = 0, d = 0;
+    for (int l = 0; l < n_layers; ++l) {
+        const ace_layer* L = layers[l];
+        if (!L) return fail(ACE_ERR_INVALID_ARG, "a layer is NULL");
+        for (int j = 0; j < l; ++j)
+            if (layers[j] == L) return fail(ACE_ERR_INVALID_ARG, "a layer appears twice in the stack");
+        if (!L->tc) return fail(ACE_ERR_UNSUPPORTED, "stacks take bf16 layers on the tensor-core path");
+        if (!L->desc.add_residual) return fail(ACE_ERR_INVALID_ARG, "stack layers must be created with add_residual");
+        if (l == 0) {
+            d = L->desc.hidden;
+            max_tokens = L->desc.max_tokens;
+        } else {
+            if (L->desc.hidden != d) return fail(ACE_ERR_INVALID_ARG, "stack layers must share the hidden size");
+            if (L->device != layers[0]->device) return fail(ACE_ERR_INVALID_ARG, "stack layers must share a device");
+            max_tokens = L->desc.max_tokens < max_tokens ? L->desc.max_tokens : max_tokens;
+        }
+    }
+    ace_stack* st = new ace_stack();
+    st->layers.assign(layers, layers + n_layers);
+    st->max_tokens = max_tokens;
+    st->hidden = d;
+    const size_t bytes = (size_t)max_tokens * d * 2;
+    int prev = 0;
+    cudaGetDevice(&prev);
+    cudaSetDevice(layers[0]->device);
+    for (int i = 0; i < 2 && n_layers > 1; ++i) {
+        if (cudaMalloc(&st->buf[i], bytes ? bytes : 16) != cudaSuccess) {
+            for (int j = 0; j < i; ++j) cudaFree(st->buf[j]);
+            cudaSetDevice(prev);
+            delete st;
+            return fail(ACE_ERR_OOM, "stack buffer allocation failed");
+        }
+    }
+    cudaSetDevice(prev);
+    *out_stack = st;
+    return ACE_OK;
+}
+
+void ace_stack_destroy(ace_stack* st) {
+    if (!st) return;
+    cudaDeviceSynchronize();
+    for (void* b : st->buf)
+        if (b) cudaFree(b);
+    delete st;
+}
+
+ace_status ace_stack_forward_host(ace_stack* st, const void* x_host, void* out_host, int T, ace_skip_ctl ctl,
+                                  void* stream) {
+    if (!st) return fail(ACE_ERR_INVALID_ARG, "stack is NULL");
+    if (T < 0 || T > st->max_tokens) return fail(ACE_ERR_INVALID_ARG, "T out of range [0, max_tokens]");
+    if (T > 0 && (!x_host || !out_host)) return fail(ACE_ERR_INVALID_ARG, "x_host and out_host must be non-NULL");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    ace_layer* first = st->layers.front();
+    ace_layer* last = st->layers.back();
+    const size_t bytes = (size_t)T * st->hidden * 2;
+    if (T > 0)
+        ACE_CUDA(cudaMemcpyAsync(first->ws.x_stage, x_host, bytes, cudaMemcpyHostToDevice, s), "copy x to device");
+    ace_status rc = ace_stack_forward(st, first->ws.x_stage, last->ws.out_stage, T, ctl, stream);
+    if (rc != ACE_OK) return rc;
+    if (T > 0)
+        ACE_CUDA(cudaMemcpyAsync(out_host, last->ws.out_stage, bytes, cudaMemcpyDeviceToHost, s), "copy out to host");
+    ACE_CUDA(cudaStreamSynchronize(s), "stack forward_host: synchronize");
+    for (ace_layer* L : st->layers) {
+        rc = check_device_word(L);
+        if (rc != ACE_OK) return rc;
+    }
+    return ACE_OK;
+}
+
+ace_status ace_stack_forward(ace_stack* st, const void* x, void* out, int T, ace_skip_ctl ctl, void* stream) {
+    if (!st) return fail(ACE_ERR_INVALID_ARG, "stack is NULL");
+    if (T < 0 || T > st->max_tokens) return fail(ACE_ERR_INVALID_ARG, "T out of range [0, max_tokens]");
+    if (T > 0 && (!x || !out)) return fail(ACE_ERR_INVALID_ARG, "x and out must be non-NULL");
+    if (T > 0 && x == out) return fail(ACE_ERR_INVALID_ARG, "out must not alias x");
+    ace_status rc = check_ctl(ctl);
+    if (rc != ACE_OK) return rc;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int n = (int)st->layers.size();
+    for (int l = 0; l < n; ++l) {
+        const void* in = l == 0 ? x : st->buf[(l - 1) & 1];
+        void* o = l == n - 1 ? out : st->buf[l & 1];
+        const ace_layer* next = l + 1 < n ? st->layers[l + 1] : nullptr;
+        rc = forward_impl(st->layers[l], in, o, T, ctl, s, next, l > 0);
+        if (rc != ACE_OK) return rc;
+    }
     return ACE_OK;
 }
 

@@ -973,6 +973,79 @@ __global__ void __launch_bounds__(256) k_combine_bf16(const Y* __restrict__ y, c
     reinterpret_cast<uint4*>(out + (size_t)t * d)[c8] = *reinterpret_cast<const uint4*>(o);
 }
 
+// The combine of a layer in a stack fused with the next layer's RMSNorm
+// (bf16 slot rows, T > 256): one block per token and one thread per 8-element
+// chunk (blockDim = d / 8). Each thread forms its chunk of the output row as
+// k_combine_bf16 does (slot rows in rank order, then the residual, rounded to
+// bf16) and the sum of squares of the rounded values as one fma chain; warp 0
+// then adds, for lane l, the partials of chunks l, l + 32, l + 64, ... in that
+// order and reduces across lanes by the butterfly -- the order of the
+// stand-alone RMSNorm, so h_next = out / sqrt(mean(out^2) + eps) * gamma_next
+// has the same bits as that kernel applied to the output.
+template <int KMAX>
+__global__ void __launch_bounds__(512) k_combine_norm(const __nv_bfloat16* __restrict__ y,
+                                                      const int32_t* __restrict__ slot_pos,
+                                                      const __nv_bfloat16* __restrict__ resid,
+                                                      __nv_bfloat16* __restrict__ out,
+                                                      const __nv_bfloat16* __restrict__ gamma_next,
+                                                      __nv_bfloat16* __restrict__ h_next, float eps_next, int d,
+                                                      int k) {
+    __shared__ float part_s[512];
+    __shared__ float inv_s;
+    pdl_wait();
+    const int t = blockIdx.x, c8 = threadIdx.x;
+    int r[KMAX];
+#pragma unroll
+    for (int i = 0; i < KMAX; ++i) r[i] = i < k ? __ldg(slot_pos + (size_t)t * k + i) : -1;
+    Row8<__nv_bfloat16> v[KMAX];
+#pragma unroll
+    for (int i = 0; i < KMAX; ++i)
+        if (r[i] >= 0) v[i].load(y + (size_t)r[i] * d + 8 * c8);
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int i = 0; i < KMAX; ++i)
+        if (r[i] >= 0) v[i].add_to(acc);
+    if (resid) {
+        float xr[8];
+        Vec16<__nv_bfloat16>::to_float(reinterpret_cast<const uint4*>(resid + (size_t)t * d)[c8], xr);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[j] = xr[j] + acc[j];
+    }
+    __align__(16) __nv_bfloat16 o[8];
+    float f[8], part = 0.f;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        o[j] = __float2bfloat16_rn(acc[j]);
+        f[j] = __bfloat162float(o[j]);
+        part = fmaf(f[j], f[j], part);
+    }
+    reinterpret_cast<uint4*>(out + (size_t)t * d)[c8] = *reinterpret_cast<const uint4*>(o);
+    part_s[c8] = part;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        float ss = 0.f;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) ss += part_s[threadIdx.x + 32 * w];
+        ss = warp_sum(ss);
+        if (threadIdx.x == 0) inv_s = 1.0f / sqrtf(ss / (float)d + eps_next);
+    }
+    __syncthreads();
+    const float inv = inv_s;
+    float gm[8];
+    Vec16<__nv_bfloat16>::to_float(reinterpret_cast<const uint4*>(gamma_next)[c8], gm);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) o[j] = __float2bfloat16_rn(f[j] * inv * gm[j]);
+    reinterpret_cast<uint4*>(h_next + (size_t)t * d)[c8] = *reinterpret_cast<const uint4*>(o);
+}
+
+template <int KMAX>
+cudaError_t launch_combine_norm(const __nv_bfloat16* y, const int32_t* sp, const __nv_bfloat16* resid,
+                                __nv_bfloat16* out, const ace_layer* next, int T, int d, int k, cudaStream_t s) {
+    // d is a multiple of 256 (tensor-core layers) and at most 4096: d / 8 threads, whole warps
+    return launch_pdl(k_combine_norm<KMAX>, dim3(T), dim3(d / 8), 0, s, y, sp, resid, out,
+                      static_cast<const __nv_bfloat16*>(next->gamma), static_cast<__nv_bfloat16*>(next->ws.h),
+                      next->desc.rms_eps, d, k);
+}
+
 // ---------------------------------------------------------------- host side
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
@@ -1211,7 +1284,7 @@ cudaError_t launch_router_tc(const ace_layer* L, int T, cudaStream_t s) {
 }
 
 cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, ace_skip_ctl ctl, cudaStream_t s,
-                              cudaEvent_t* ev) {
+                              cudaEvent_t* ev, const ace_layer* next) {
     const bool pair = tc_use_pair(L, T, ctl);
     const __nv_bfloat16* resid = L->desc.add_residual ? static_cast<const __nv_bfloat16*>(x) : nullptr;
     const ace_layer_desc& D = L->desc;
@@ -1318,6 +1391,10 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
         const float* y = W.yslot;
         e = k <= 8 ? launch_pdl(k_combine_bf16<float, 8>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k)
                    : launch_pdl(k_combine_bf16<float, kMaxTopK>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k);
+    } else if (next) {
+        const __nv_bfloat16* y = static_cast<const __nv_bfloat16*>(W.h_perm);
+        e = k <= 8 ? launch_combine_norm<8>(y, sp, resid, o, next, T, d, k, s)
+                   : launch_combine_norm<kMaxTopK>(y, sp, resid, o, next, T, d, k, s);
     } else {
         const __nv_bfloat16* y = static_cast<const __nv_bfloat16*>(W.h_perm);
         e = k <= 8 ? launch_pdl(k_combine_bf16<__nv_bfloat16, 8>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k)

@@ -9,6 +9,7 @@
 #include <stdint.h>
 
 #include <utility>
+#include <vector>
 
 #include "ace.h"
 
@@ -86,6 +87,13 @@ struct TcMaps {
 };
 
 }  // namespace ace
+
+struct ace_stack {
+    std::vector<ace_layer*> layers;
+    void* buf[2] = {nullptr, nullptr};   // [max_tokens, d] bf16: alternating layer outputs
+    int max_tokens = 0;
+    int hidden = 0;
+};
 
 struct ace_layer {
     ace_layer_desc desc;
@@ -211,8 +219,10 @@ cudaError_t tc_init(ace_layer* L);
 // Packs W_gate / W_up / W_down into the tiled, pre-swizzled layouts of w_gu and w_down.
 cudaError_t tc_pack_weights(ace_layer* L, const void* w_gate, const void* w_up, const void* w_down, cudaStream_t s);
 // ev (nullable): recorded after gather, after gate/up, after down, after combine.
+// next (nullable, T > 256 only): the following layer of a stack; the combine
+// then also writes that layer's RMSNorm of `out` into next->ws.h.
 cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int T, ace_skip_ctl ctl, cudaStream_t s,
-                              cudaEvent_t* ev);
+                              cudaEvent_t* ev, const ace_layer* next = nullptr);
 // Router logits on the tensor cores (T > kTcSmallT): z = (h W_r^T + b) / temp.
 // With router_splits(L, T) > 1 it writes raw partial sums [splits, T, N] into
 // ws.act_bf16 and the top-k kernel forms the logits.

@@ -38,13 +38,18 @@ __device__ __forceinline__ void rmsnorm_row(const T* __restrict__ xr, const T* _
         const int c = lane + 32 * i;
         xs[i] = c < nvec ? xv[c] : make_uint4(0, 0, 0, 0);
     }
+    // sum of squares: one partial per 16-byte chunk (an fma chain from 0),
+    // the lane's partials added in chunk order, then the warp butterfly --
+    // the order every RMSNorm of the library uses
     float ss = 0.f;
 #pragma unroll
     for (int i = 0; i < NV; ++i) {
         float f[V];
         Vec16<T>::to_float(xs[i], f);
+        float part = 0.f;
 #pragma unroll
-        for (int j = 0; j < V; ++j) ss = fmaf(f[j], f[j], ss);
+        for (int j = 0; j < V; ++j) part = fmaf(f[j], f[j], part);
+        ss += part;
     }
     ss = warp_sum(ss);
     const float inv = 1.0f / sqrtf(ss / (float)d + rms_eps);
@@ -1047,13 +1052,15 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         if (warp < nt) {
             // h = x / sqrt(mean(x^2) + eps) * gamma, rounded to T (the stored h feeds the router)
             uint4* xr = reinterpret_cast<uint4*>(xs + (size_t)warp * rs);
-            float ss = 0.f;
+            float ss = 0.f;                                   // chunk partials, as rmsnorm_row
 #pragma unroll 1
             for (int c = lane; c < nvec; c += 32) {
                 float f[V];
                 Vec16<T>::to_float(xr[c], f);
+                float part = 0.f;
 #pragma unroll
-                for (int j = 0; j < V; ++j) ss = fmaf(f[j], f[j], ss);
+                for (int j = 0; j < V; ++j) part = fmaf(f[j], f[j], part);
+                ss += part;
             }
             ss = warp_sum(ss);
             const float inv = 1.0f / sqrtf(ss / (float)d + a.rms_eps);

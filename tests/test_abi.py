@@ -88,3 +88,14 @@ def test_unknown_fusion_rejected_on_host(libace):
     with pytest.raises(ValueError):
         ace._ctl("ratio", 0.5, "median")
     assert ace._ctl("ratio", 0.5, "score").fusion == ace.ACE_FUSION_SCORE
+
+
+def test_stack_argument_checks_on_host(libace):
+    ace._lib = None
+    L = ace.lib()
+    out = ctypes.c_void_p(7)
+    assert L.ace_stack_create(None, 2, ctypes.byref(out)) == 1 and out.value is None
+    arr = (ctypes.c_void_p * 1)(None)
+    assert L.ace_stack_create(arr, 1, ctypes.byref(out)) == 1
+    assert L.ace_stack_forward(None, None, None, 1, ace.ace_skip_ctl(0, 0.1, 0), None) == 1
+    L.ace_stack_destroy(None)

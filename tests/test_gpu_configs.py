@@ -154,3 +154,36 @@ def test_large_layer_tables_device():
     np.testing.assert_allclose(a[idx] / a[idx[0]], sub / sub[0], rtol=3e-5)
     r_ref = O.rcr_table(w.router_w, w.gamma, w.w_gate, w.w_up, w.w_down, w.spec.eps)
     np.testing.assert_allclose(r, r_ref, rtol=3e-5)
+
+
+@pytest.mark.parametrize("T", [32, 300, 4096])
+def test_stack_api_matches_chained_layers(T):
+    """ace_stack_forward (the prefill path computes each next layer's RMSNorm
+    inside the combine) gives the same bits as chaining the layers' forwards,
+    and leaves each layer's decision readable."""
+    ws, layers = _stack()
+    spec = ws[0].spec
+    x = _dev(synth.make_tokens(spec, T, seed=3))
+    cur = x
+    for layer in layers:
+        nxt = torch.empty_like(cur)
+        layer.forward(cur, nxt, T, "ratio", 0.5)
+        cur = nxt
+    torch.cuda.synchronize()
+    want = cur.view(torch.int16).cpu().numpy()
+    masks = [ace.ace_last_skip_mask(layer.handle, T, spec.top_k)[0].copy() for layer in layers]
+    st = ace.ace_stack_create([layer.handle for layer in layers])
+    try:
+        out = torch.empty_like(x)
+        for _ in range(2):
+            ace.ace_stack_forward(st, x, out, T, "ratio", 0.5)
+            torch.cuda.synchronize()
+            assert (out.view(torch.int16).cpu().numpy() == want).all()
+        for layer, m in zip(layers, masks):
+            assert (ace.ace_last_skip_mask(layer.handle, T, spec.top_k)[0] == m).all()
+        with pytest.raises(ace.AceError):
+            ace.ace_stack_forward(st, x, x, T, "ratio", 0.5)            # out aliases x
+    finally:
+        ace.ace_stack_destroy(st)
+    with pytest.raises(ace.AceError):
+        ace.ace_stack_create([layers[0].handle, layers[0].handle])      # the same layer twice
