@@ -176,8 +176,14 @@ void ace_stack_destroy(ace_stack* stack);
  * ace_moe_forward_host — the same forward from HOST buffers: copies x to a
  * layer-owned device buffer, runs ace_moe_forward, copies the result back
  * and synchronises `stream` before returning.
- *   x_host   [T, d] host, dtype (pinned memory gives the fastest copies)
+ *   x_host   [T, d] host, dtype
  *   out_host [T, d] host, dtype
+ * With page-locked (pinned) host buffers the copy-in, forward and copy-out
+ * are captured once as a CUDA graph and replayed while the stream, the host
+ * pointers, T and ctl stay the same (one launch per call). Calls on the
+ * legacy default stream (NULL) run on a blocking stream of the layer, which
+ * is ordered with it. The call cannot be made while `stream` is being
+ * captured (INVALID_ARG).
  */
 ace_status ace_moe_forward_host(ace_layer* layer, const void* x_host, void* out_host, int T,
                                 ace_skip_ctl ctl, void* stream);

@@ -47,7 +47,89 @@ void free_layer(ace_layer* L) {
         if (p) cudaFree(p);
     for (cudaEvent_t e : L->ev)
         if (e) cudaEventDestroy(e);
+    if (L->hg.exec) cudaGraphExecDestroy(L->hg.exec);
+    if (L->hg.own) cudaStreamDestroy(L->hg.own);
+    if (L->hg.err_host) cudaFreeHost(L->hg.err_host);
     delete L;
+}
+
+bool pinned_host(const void* p) {
+    cudaPointerAttributes a{};
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return a.type == cudaMemoryTypeHost;
+}
+
+// Runs `body(stream, err_host)` -- which enqueues the copy-in, the forward,
+// the copy-out and copies of the layers' device error words into err_host --
+// through a CUDA graph captured on the first call and replayed while the
+// stream, the host buffers, T, the skip control and the profiling switch stay
+// the same; then synchronises. Pageable host buffers are enqueued directly
+// (they cannot be captured). Calls on the legacy default stream use a
+// blocking stream owned by g (ordered with the default stream).
+template <typename Body>
+ace_status run_host_graph(AceHostGraph& g, cudaStream_t user, const void* xh, void* oh, int T, ace_skip_ctl ctl,
+                          bool profiling, int n_err, Body body) {
+    cudaStream_t s = user;
+    if (!s) {
+        if (!g.own) ACE_CUDA(cudaStreamCreate(&g.own), "create stream");
+        s = g.own;
+    }
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    ACE_CUDA(cudaStreamIsCapturing(s, &cs), "query capture");
+    if (cs != cudaStreamCaptureStatusNone) return fail(ACE_ERR_INVALID_ARG, "host-buffer calls synchronise and cannot be captured");
+    if (g.n_err < n_err) {
+        if (g.exec) {
+            cudaGraphExecDestroy(g.exec);
+            g.exec = nullptr;
+        }
+        if (g.err_host) cudaFreeHost(g.err_host);
+        g.err_host = nullptr;
+        g.n_err = 0;
+        ACE_CUDA(cudaMallocHost(&g.err_host, n_err * sizeof(int)), "allocate pinned error words");
+        g.n_err = n_err;
+    }
+    const bool same = g.exec && g.stream == s && g.x_host == xh && g.out_host == oh && g.T == T &&
+                      g.ctl.mode == ctl.mode && g.ctl.value == ctl.value && g.ctl.fusion == ctl.fusion &&
+                      g.profiling == profiling;
+    if (!same) {
+        if (g.exec) {
+            cudaGraphExecDestroy(g.exec);
+            g.exec = nullptr;
+        }
+        if (!pinned_host(xh) || !pinned_host(oh)) {
+            ace_status st = body(s, g.err_host);
+            if (st != ACE_OK) return st;
+            ACE_CUDA(cudaStreamSynchronize(s), "forward_host: synchronize");
+            return ACE_OK;
+        }
+        ACE_CUDA(cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal), "begin capture");
+        ace_status st = body(s, g.err_host);
+        cudaGraph_t graph = nullptr;
+        const cudaError_t ce = cudaStreamEndCapture(s, &graph);
+        if (st != ACE_OK) {
+            if (graph) cudaGraphDestroy(graph);
+            return st;
+        }
+        if (ce != cudaSuccess) return cuda_fail(ce, "end capture");
+        const cudaError_t ie = cudaGraphInstantiate(&g.exec, graph, 0);
+        cudaGraphDestroy(graph);
+        if (ie != cudaSuccess) {
+            g.exec = nullptr;
+            return cuda_fail(ie, "instantiate graph");
+        }
+        g.stream = s;
+        g.x_host = xh;
+        g.out_host = oh;
+        g.T = T;
+        g.ctl = ctl;
+        g.profiling = profiling;
+    }
+    ACE_CUDA(cudaGraphLaunch(g.exec, s), "graph launch");
+    ACE_CUDA(cudaStreamSynchronize(s), "forward_host: synchronize");
+    return ACE_OK;
 }
 
 bool tables_ok(const float* t, int n) {
@@ -56,9 +138,7 @@ bool tables_ok(const float* t, int n) {
     return true;
 }
 
-ace_status check_device_word(ace_layer* L) {
-    int err = 0;
-    ACE_CUDA(cudaMemcpy(&err, L->ws.err, sizeof(int), cudaMemcpyDeviceToHost), "read device error word");
+ace_status report_error_word(ace_layer* L, int err) {
     if (err) {
         ACE_CUDA(cudaMemset(L->ws.err, 0, sizeof(int)), "clear device error word");
         if (err & ace::kErrTimeout) return fail(ACE_ERR_TIMEOUT, "a bounded device wait ran out");
@@ -66,6 +146,12 @@ ace_status check_device_word(ace_layer* L) {
         if (err & ace::kErrBounds) return fail(ACE_ERR_CUDA, "a device index check failed");
     }
     return ACE_OK;
+}
+
+ace_status check_device_word(ace_layer* L) {
+    int err = 0;
+    ACE_CUDA(cudaMemcpy(&err, L->ws.err, sizeof(int), cudaMemcpyDeviceToHost), "read device error word");
+    return report_error_word(L, err);
 }
 
 ace_status check_ctl(ace_skip_ctl ctl) {
@@ -388,6 +474,9 @@ void ace_stack_destroy(ace_stack* st) {
     cudaDeviceSynchronize();
     for (void* b : st->buf)
         if (b) cudaFree(b);
+    if (st->hg.exec) cudaGraphExecDestroy(st->hg.exec);
+    if (st->hg.own) cudaStreamDestroy(st->hg.own);
+    if (st->hg.err_host) cudaFreeHost(st->hg.err_host);
     delete st;
 }
 
@@ -396,19 +485,32 @@ ace_status ace_stack_forward_host(ace_stack* st, const void* x_host, void* out_h
     if (!st) return fail(ACE_ERR_INVALID_ARG, "stack is NULL");
     if (T < 0 || T > st->max_tokens) return fail(ACE_ERR_INVALID_ARG, "T out of range [0, max_tokens]");
     if (T > 0 && (!x_host || !out_host)) return fail(ACE_ERR_INVALID_ARG, "x_host and out_host must be non-NULL");
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    ace_status rc = check_ctl(ctl);
+    if (rc != ACE_OK) return rc;
+    if (T == 0) return ACE_OK;
     ace_layer* first = st->layers.front();
     ace_layer* last = st->layers.back();
     const size_t bytes = (size_t)T * st->hidden * 2;
-    if (T > 0)
-        ACE_CUDA(cudaMemcpyAsync(first->ws.x_stage, x_host, bytes, cudaMemcpyHostToDevice, s), "copy x to device");
-    ace_status rc = ace_stack_forward(st, first->ws.x_stage, last->ws.out_stage, T, ctl, stream);
+    bool profiling = false;
+    for (ace_layer* L : st->layers) profiling = profiling || L->profiling;
+    const int n = (int)st->layers.size();
+    rc = run_host_graph(st->hg, static_cast<cudaStream_t>(stream), x_host, out_host, T, ctl, profiling, n,
+                        [&](cudaStream_t s, int* err_host) -> ace_status {
+                            ACE_CUDA(cudaMemcpyAsync(first->ws.x_stage, x_host, bytes, cudaMemcpyHostToDevice, s),
+                                     "copy x to device");
+                            ace_status r = ace_stack_forward(st, first->ws.x_stage, last->ws.out_stage, T, ctl, s);
+                            if (r != ACE_OK) return r;
+                            ACE_CUDA(cudaMemcpyAsync(out_host, last->ws.out_stage, bytes, cudaMemcpyDeviceToHost, s),
+                                     "copy out to host");
+                            for (int l = 0; l < n; ++l)
+                                ACE_CUDA(cudaMemcpyAsync(err_host + l, st->layers[l]->ws.err, sizeof(int),
+                                                         cudaMemcpyDeviceToHost, s),
+                                         "copy error word");
+                            return ACE_OK;
+                        });
     if (rc != ACE_OK) return rc;
-    if (T > 0)
-        ACE_CUDA(cudaMemcpyAsync(out_host, last->ws.out_stage, bytes, cudaMemcpyDeviceToHost, s), "copy out to host");
-    ACE_CUDA(cudaStreamSynchronize(s), "stack forward_host: synchronize");
-    for (ace_layer* L : st->layers) {
-        rc = check_device_word(L);
+    for (int l = 0; l < n; ++l) {
+        rc = report_error_word(st->layers[l], st->hg.err_host[l]);
         if (rc != ACE_OK) return rc;
     }
     return ACE_OK;
@@ -438,15 +540,24 @@ ace_status ace_moe_forward_host(ace_layer* L, const void* x_host, void* out_host
     if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
     if (T < 0 || T > L->desc.max_tokens) return fail(ACE_ERR_INVALID_ARG, "T out of range [0, max_tokens]");
     if (T > 0 && (!x_host || !out_host)) return fail(ACE_ERR_INVALID_ARG, "x_host and out_host must be non-NULL");
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const size_t bytes = (size_t)T * L->desc.hidden * L->elem;
-    if (T > 0) ACE_CUDA(cudaMemcpyAsync(L->ws.x_stage, x_host, bytes, cudaMemcpyHostToDevice, s), "copy x to device");
-    ace_status st = ace_moe_forward(L, L->ws.x_stage, L->ws.out_stage, T, ctl, stream);
+    ace_status st = check_ctl(ctl);
     if (st != ACE_OK) return st;
-    if (T > 0)
-        ACE_CUDA(cudaMemcpyAsync(out_host, L->ws.out_stage, bytes, cudaMemcpyDeviceToHost, s), "copy out to host");
-    ACE_CUDA(cudaStreamSynchronize(s), "forward_host: synchronize");
-    return check_device_word(L);
+    if (T == 0) return ace_moe_forward(L, L->ws.x_stage, L->ws.out_stage, 0, ctl, stream);
+    const size_t bytes = (size_t)T * L->desc.hidden * L->elem;
+    st = run_host_graph(L->hg, static_cast<cudaStream_t>(stream), x_host, out_host, T, ctl, L->profiling, 1,
+                        [&](cudaStream_t s, int* err_host) -> ace_status {
+                            ACE_CUDA(cudaMemcpyAsync(L->ws.x_stage, x_host, bytes, cudaMemcpyHostToDevice, s),
+                                     "copy x to device");
+                            ace_status r = forward_impl(L, L->ws.x_stage, L->ws.out_stage, T, ctl, s, nullptr, false);
+                            if (r != ACE_OK) return r;
+                            ACE_CUDA(cudaMemcpyAsync(out_host, L->ws.out_stage, bytes, cudaMemcpyDeviceToHost, s),
+                                     "copy out to host");
+                            ACE_CUDA(cudaMemcpyAsync(err_host, L->ws.err, sizeof(int), cudaMemcpyDeviceToHost, s),
+                                     "copy error word");
+                            return ACE_OK;
+                        });
+    if (st != ACE_OK) return st;
+    return report_error_word(L, L->hg.err_host[0]);
 }
 
 ace_status ace_layer_sync(ace_layer* L) {

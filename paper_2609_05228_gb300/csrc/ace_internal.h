@@ -88,7 +88,23 @@ struct TcMaps {
 
 }  // namespace ace
 
+// A host-buffer forward (copy in, forward, copy out) captured as a CUDA
+// graph and replayed while the call's arguments stay the same.
+struct AceHostGraph {
+    cudaGraphExec_t exec = nullptr;
+    cudaStream_t own = nullptr;          // used for calls on the legacy default stream
+    cudaStream_t stream = nullptr;       // the stream the graph was captured for
+    const void* x_host = nullptr;
+    void* out_host = nullptr;
+    int T = -1;
+    ace_skip_ctl ctl{0, 0.f, 0};
+    bool profiling = false;
+    int* err_host = nullptr;             // pinned copies of the device error words, written by the graph
+    int n_err = 0;
+};
+
 struct ace_stack {
+    AceHostGraph hg;
     std::vector<ace_layer*> layers;
     void* buf[2] = {nullptr, nullptr};   // [max_tokens, d] bf16: alternating layer outputs
     int max_tokens = 0;
@@ -125,6 +141,7 @@ struct ace_layer {
     cudaEvent_t ev[10] = {};
     int n_stages = 0;
     int last_launches = 0;       // kernels launched by the last forward / route call
+    AceHostGraph hg;             // ace_moe_forward_host
 };
 
 namespace ace {

@@ -181,6 +181,11 @@ def test_stack_api_matches_chained_layers(T):
             assert (out.view(torch.int16).cpu().numpy() == want).all()
         for layer, m in zip(layers, masks):
             assert (ace.ace_last_skip_mask(layer.handle, T, spec.top_k)[0] == m).all()
+        xp = x.cpu().pin_memory()
+        op = torch.empty_like(xp).pin_memory()
+        for _ in range(2):                                               # capture, then replay
+            ace.ace_stack_forward_host(st, xp, op, T, "ratio", 0.5)
+            assert (op.view(torch.int16).numpy() == want).all()
         with pytest.raises(ace.AceError):
             ace.ace_stack_forward(st, x, x, T, "ratio", 0.5)            # out aliases x
     finally:

@@ -398,3 +398,23 @@ def test_calibrated_threshold_reproduces_ratio(T):
         got = ace.ace_last_skip_mask(layer.handle, T, w.spec.top_k)
         assert (got[0] == ref[0]).all() and (got[2].view(np.uint32) == ref[2].view(np.uint32)).all()
         assert got[4] == ref[4]
+
+
+def test_forward_host_graph_replay():
+    """Pinned host buffers: the host call replays a captured graph; results
+    equal the device-buffer forward, also after the host buffers, T or the
+    skip control change (re-capture)."""
+    w, layer = _layer("qwen")
+    for T, mode, val in [(64, "ratio", 0.5), (64, "ratio", 0.5), (32, "threshold", 0.11), (300, "ratio", 0.25)]:
+        xh = synth.make_tokens(w.spec, T, seed=5 + T)
+        x = _dev(xh)
+        o = torch.empty_like(x)
+        layer.forward(x, o, T, mode, val)
+        want = o.view(torch.int16).cpu().numpy().view(np.uint16)
+        for _ in range(2):
+            xp = torch.from_numpy(xh.view(np.int16)).pin_memory()
+            op = torch.empty_like(xp).pin_memory()
+            ace.ace_moe_forward_host(layer.handle, xp, op, T, mode, val)
+            assert (op.numpy().view(np.uint16) == want).all(), (T, mode, val)
+            ace.ace_moe_forward_host(layer.handle, xp, op, T, mode, val)     # replay
+            assert (op.numpy().view(np.uint16) == want).all(), (T, mode, val)
