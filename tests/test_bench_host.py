@@ -1,0 +1,59 @@
+"""Host-side pieces of bench.py that need no GPU: the reference arm's JSON
+line (the oracle on a bounded sample), the ncu traffic record guard, and the
+algorithmic byte counts of the roofline."""
+import json
+import os
+import shutil
+import subprocess
+import sys
+
+import numpy as np
+
+import bench
+from paper_2609_05228_gb300 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def test_recorded_traffic_follows_the_kernel_sources(tmp_path, monkeypatch):
+    rec = os.path.join("profiles", "decode_T64_q0.5_expert_decode_full.md")
+    value = bench._recorded_traffic(rec)
+    assert isinstance(value, int) and 1.0e9 < value < 1.1e9
+    # a record whose source hash no longer matches reads as "no traffic figure"
+    text = open(os.path.join(ROOT, rec)).read().replace("source_sha256=", "source_sha256=0")
+    bad = tmp_path / "bad.md"
+    bad.write_text(text)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    os.makedirs(tmp_path / "paper_2609_05228_gb300" / "csrc", exist_ok=True)
+    for src in ("ace_expert_tc.cu", "ace_tc.cuh", "ace_device.cuh"):
+        shutil.copy(os.path.join(ROOT, "paper_2609_05228_gb300", "csrc", src),
+                    tmp_path / "paper_2609_05228_gb300" / "csrc" / src)
+    assert bench._recorded_traffic("bad.md") is None
+    assert bench._recorded_traffic("missing.md") is None
+
+
+def test_algorithmic_bytes_of_the_decode_layer():
+    """Retained-expert weight bytes: 3 matrices of d x m bf16 per distinct expert."""
+    w = synth.LayerWeights(synth.spec_qwen(), None, None, None, None, None, None)
+    d, m, N = 2048, 768, 128
+    total, flops, gu, down = bench.algorithmic(w, 64, 256, 110)
+    assert total == 3 * d * m * 2 * 110 + N * d * 2 + 2 * 64 * d * 2
+    assert flops == 6 * d * m * 256 + 2 * d * N * 64
+    assert gu == 2 * d * m * 2 * 110 + 256 * d * 2 + 256 * m * 2
+    assert down == d * m * 2 * 110 + 256 * m * 2 + 256 * d * 4
+
+
+def test_reference_arm_json_line():
+    """`bench.py --impl reference` prints one JSON line with the contract's
+    keys, timing the oracle on the host (tokens per step sized to the steps)."""
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "2",
+                        "--warmup", "1"], capture_output=True, text=True, cwd=ROOT, timeout=900)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.strip()]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["unit"] == "tokens/s" and d["value"] > 0
+    assert d["steps"] == 2 and d["warmup"] >= 3 and d["higher_is_better"] is True
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
+    assert d["e2e"] == {"value": d["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    assert 1 <= d["config"]["tokens_per_step"] <= 64
