@@ -210,9 +210,17 @@ def _layer(kind):
         elif kind == "qwen_temp":
             # router temperature != 1 and m_min = 2 (Algorithm 4's restore)
             spec, seed = dataclasses.replace(synth.spec_qwen(zipf=True), router_temp=1.3, min_active=2), 7
+        elif kind == "wide":
+            # the widest routing the library takes: 1024 experts, top-16 (a token's
+            # 16 slots in the combine, 32 logits per lane in the top-k)
+            spec, seed = synth.LayerSpec(256, 1024, 16, 128, dtype="bf16"), 11
         else:
             raise KeyError(kind)
         w = synth.make_layer(spec, seed)
+        if kind == "wide":
+            # 4x router scale: with 1024 logits per token the default scale leaves
+            # most top-16 boundaries within rounding distance
+            w.router_w = synth.bf16_bits(synth.bf16_to_f32(w.router_w) * 4.0)
         a_gsp, a_rcr = offline.tables(w)
         w.extra["a_gsp"], w.extra["a_rcr"] = a_gsp, a_rcr
         _LAYERS[kind] = (w, ace.AceLayer(w, a_gsp, a_rcr, max_tokens=4096))
@@ -273,6 +281,8 @@ FORWARD_CASES = [
     ("qwen", 17, "threshold", 0.11), ("qwen", 129, "ratio", 0.5), ("qwen", 1000, "ratio", 0.625),
     ("qwen_zipf", 4096, "ratio", 0.0), ("qwen_zipf", 4096, "ratio", 0.5),
     ("qwen_temp", 64, "ratio", 0.5), ("qwen_temp", 600, "ratio", 0.625), ("qwen_temp", 48, "threshold", 0.1),
+    ("qwen", 256, "ratio", 0.5), ("qwen", 257, "ratio", 0.5),          # both sides of the small-batch path
+    ("wide", 40, "ratio", 0.5), ("wide", 700, "ratio", 0.5), ("wide", 256, "threshold", 0.05),
 ]
 
 
@@ -295,8 +305,11 @@ def _check_forward(kind, T, mode, val, fusion):
     w, spec, x, y_gpu, y_ref, dec, z_ref, (skip, ids, gh, tau, R) = _run_layer(kind, T, mode, val, fusion=fusion)
     k = spec.top_k
     margin = 1e-4 if spec.dtype == "f32" else None
-    clear = _clear_tokens(dec, z_ref, k, margin or 6e-3, margin or 8e-3, spec.min_active)
-    assert clear.mean() >= 0.4, clear.mean()
+    # the wide layer's logits are 4x the scale (so is their rounding), and its
+    # 1024 candidates put more top-16 boundaries within that distance
+    dz = 4 * 6e-3 if kind == "wide" else (margin or 6e-3)
+    clear = _clear_tokens(dec, z_ref, k, dz, margin or 8e-3, spec.min_active)
+    assert clear.mean() >= (0.2 if kind == "wide" else 0.4), clear.mean()
     # decisions agree on every clear token (compared per expert id)
     for t in np.nonzero(clear)[0]:
         gpu = {int(ids[t, i]): bool(skip[t, i]) for i in range(k)}
