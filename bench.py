@@ -68,8 +68,16 @@ class L2Flush:
         self.sink.copy_(self.r.sum().reshape(1))
 
 
+# ncu summaries whose machine-read record gives roofline.traffic, per workload
+TRAFFIC_RECORDS = {
+    "decode": "profiles/decode_T64_q0.5_expert_decode_full.md",
+    "prefill": "profiles/prefill_T4096_q0.5_expert_tc_full.md",
+    "stack_prefill": "profiles/stack_prefill_T16384_q0.5_expert_pair_full.md",
+}
+
+
 def _recorded_traffic(path="profiles/decode_T64_q0.5_expert_decode_full.md"):
-    """DRAM bytes per launch of the gate/up kernel from the committed ncu
+    """DRAM bytes per launch of the dominant kernel from a committed ncu
     summary, or None when the kernel source has changed since the capture."""
     import hashlib
     try:
@@ -413,20 +421,23 @@ def run_ours(args, rank, world, torch, dist):
         kname = "k_expert_pair gate/up (tcgen05 cta_group::2)" if pair else "k_expert_tc gate/up (tcgen05)"
         roof = {"bound": "tensor", "kernel": kname, "achieved": round(achieved, 1),
                 "peak": bf16_sust, "unit": "TFLOP/s", "frac": round(achieved / bf16_sust, 4),
-                "peak_source": peak_kind + " (sustained bf16)", "traffic": None,
+                "peak_source": peak_kind + " (sustained bf16)",
+                "traffic": _recorded_traffic(TRAFFIC_RECORDS[args.workload]) if args.workload in TRAFFIC_RECORDS else None,
                 "algorithmic_flops": gu_flops, "kernel_us": round(gu_ms * 1e3, 2)}
     elif T <= 256:
         kb = gu_bytes + down_bytes
         achieved = kb / (gu_ms * 1e-3) / 1e9
         roof = {"bound": "hbm", "kernel": "k_expert_decode gate/up + down (tcgen05, one launch)",
                 "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s", "frac": round(achieved / hbm, 4),
-                "peak_source": peak_kind, "traffic": _recorded_traffic() if args.workload == "decode" else None,
+                "peak_source": peak_kind,
+                "traffic": _recorded_traffic(TRAFFIC_RECORDS[args.workload]) if args.workload in TRAFFIC_RECORDS else None,
                 "algorithmic_bytes": kb, "kernel_us": round(gu_ms * 1e3, 2)}
     else:
         achieved = gu_bytes / (gu_ms * 1e-3) / 1e9
         roof = {"bound": "hbm", "kernel": "k_expert_tc gate/up (tcgen05)",
                 "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s", "frac": round(achieved / hbm, 4),
-                "peak_source": peak_kind, "traffic": None,
+                "peak_source": peak_kind,
+                "traffic": _recorded_traffic(TRAFFIC_RECORDS[args.workload]) if args.workload in TRAFFIC_RECORDS else None,
                 "algorithmic_bytes": gu_bytes, "kernel_us": round(gu_ms * 1e3, 2)}
 
     result = {
