@@ -167,6 +167,8 @@ class Stack:
     """The workload's layers on one device; a step chains their forwards.
     In a stack every layer adds its input back (out = x + MoE(x))."""
 
+    fusion = "max"     # skip rule of every forward (ace_skip_ctl.fusion); "max" is ACE
+
     def __init__(self, wl, max_tokens):
         from paper_2609_05228_gb300 import ace, offline, synth
         spec = synth.spec_qwen(zipf=wl["zipf"]) if wl["spec"] == "qwen" else synth.spec_large(zipf=wl["zipf"])
@@ -192,25 +194,25 @@ class Stack:
     def forward(self, x, bufs, T, q, stream=None):
         from paper_2609_05228_gb300 import ace
         if self.stack:
-            ace.ace_stack_forward(self.stack, x, bufs[-1], T, "ratio", q, stream)
+            ace.ace_stack_forward(self.stack, x, bufs[-1], T, "ratio", q, stream, self.fusion)
             return
         cur = x
         for layer, out in zip(self.layers, bufs):
-            ace.ace_moe_forward(layer.handle, cur, out, T, "ratio", q, stream)
+            ace.ace_moe_forward(layer.handle, cur, out, T, "ratio", q, stream, self.fusion)
             cur = out
 
     def forward_host(self, xp, op, T, q):
         from paper_2609_05228_gb300 import ace
         if self.stack:
-            ace.ace_stack_forward_host(self.stack, xp, op, T, "ratio", q)
+            ace.ace_stack_forward_host(self.stack, xp, op, T, "ratio", q, None, self.fusion)
         else:
-            ace.ace_moe_forward_host(self.layers[0].handle, xp, op, T, "ratio", q)
+            ace.ace_moe_forward_host(self.layers[0].handle, xp, op, T, "ratio", q, None, self.fusion)
 
     def forward_threshold(self, x, bufs, T, taus, stream=None):
         from paper_2609_05228_gb300 import ace
         cur = x
         for layer, out, tau in zip(self.layers, bufs, taus):
-            ace.ace_moe_forward(layer.handle, cur, out, T, "threshold", tau, stream)
+            ace.ace_moe_forward(layer.handle, cur, out, T, "threshold", tau, stream, self.fusion)
             cur = out
 
     def close(self):
@@ -337,6 +339,7 @@ def run_ours(args, rank, world, torch, dist):
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
     model = Stack(wl, max_tokens=max(T, 64))
+    model.fusion = args.fusion
     spec, w, layer = model.spec, model.ws[0], model.layers[0]
     xh = synth.make_tokens(spec, T, seed=1 + rank)
     x = torch.from_numpy(xh.view(np.int16)).view(torch.bfloat16).to(dev)
@@ -375,7 +378,7 @@ def run_ours(args, rank, world, torch, dist):
     # threshold mode with tau calibrated on a separate seed-2 batch (App. B.1 mapping)
     from paper_2609_05228_gb300 import calibrate
     xc = torch.from_numpy(synth.make_tokens(spec, T, seed=2).view(np.int16)).view(torch.bfloat16).to(dev)
-    taus = [calibrate.calibrate_taus(l, xc, T, [q])[float(q)] for l in model.layers]
+    taus = [calibrate.calibrate_taus(l, xc, T, [q], fusion=args.fusion)[float(q)] for l in model.layers]
     thr_ms = time_threshold(torch, model, x, bufs, T, taus, max(10, min(args.steps // 2, 200)), 3, flush)
     model.forward_threshold(x, bufs, T, taus)
     _, _, _, _, R_thr = ace.ace_last_skip_mask(layer.handle, T, spec.top_k)
@@ -456,6 +459,7 @@ def run_ours(args, rank, world, torch, dist):
                 ("offline GSP/RCR tables from the host library)" if wl["tables"] == "offline"
                  else "offline GSP/RCR tables computed on the GPU)"),
         "config": {"workload": wl["name"], "tokens_per_step": T, "layers": n_layers, "skip_ratio": q,
+                   "skip_rule": args.fusion,
                    "parallelism": f"replicas{world}" if world > 1 else "single GPU",
                    "l2": "flushed between timed steps (512 MB write, then a 256 MB read)", "graph": "CUDA graph replay"},
         "realised_skip_ratio": round((T * spec.top_k - R) / (T * spec.top_k), 6),
@@ -480,7 +484,7 @@ def run_ours(args, rank, world, torch, dist):
         "offline_tables": time_tables(torch, w) if rank == 0 else None,
     }
     if rank == 0 and not args.no_cpu_baseline:
-        result["cpu_baseline"] = cpu_baseline(model.ws, wl, budget_s=args.cpu_seconds)
+        result["cpu_baseline"] = cpu_baseline(model.ws, wl, budget_s=args.cpu_seconds, fusion=args.fusion)
     if rank == 0 and args.sweep:
         result["sweep"] = sweep(torch, args)
     model.close()
@@ -502,6 +506,7 @@ def sweep(torch, args):
     pts = []
     for wlname, Ts, qs in plan:
         model = Stack(WORKLOADS[wlname], max_tokens=max(Ts))
+        model.fusion = args.fusion
         flush = L2Flush(torch, "cuda")
         for T in Ts:
             xh = synth.make_tokens(model.spec, T, seed=1)
@@ -548,7 +553,7 @@ def time_tables(torch, w, reps=3):
             "note": "whole call: scratch allocation, packing, GSP GEMM, norms, RCR GEMV, normalisation"}
 
 
-def cpu_baseline(ws, wl, budget_s=12.0):
+def cpu_baseline(ws, wl, budget_s=12.0, fusion="max"):
     """The CPU oracle (fp64) on a bounded sample of the same workload: the
     stacked layers over a sample of tokens (64, or 256 for prefill)."""
     import oracle as O
@@ -560,7 +565,7 @@ def cpu_baseline(ws, wl, budget_s=12.0):
     while True:
         cur = O.to_f64(x)
         for i, w in enumerate(ws):
-            y = O.moe_forward(cur, w, "ratio", wl["q"])
+            y = O.moe_forward(cur, w, "ratio", wl["q"], fusion=fusion)
             cur = cur + y if len(ws) > 1 else y
         n += 1
         if time.perf_counter() - t0 > budget_s:
@@ -591,7 +596,7 @@ def run_reference(args):
     def step(T):
         cur = O.to_f64(xall[:T])
         for w in ws:
-            y = O.moe_forward(cur, w, "ratio", wl["q"])
+            y = O.moe_forward(cur, w, "ratio", wl["q"], fusion=args.fusion)
             cur = cur + y if len(ws) > 1 else y
 
     # tokens per step: the whole run (warm-up + steps) is sized to about two
@@ -614,7 +619,8 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(st * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": {"workload": wl["name"], "tokens_per_step": T, "layers": len(ws),
-                                            "skip_ratio": wl["q"], "sample": f"{T} tokens per step"},
+                                            "skip_ratio": wl["q"], "skip_rule": args.fusion,
+                                            "sample": f"{T} tokens per step"},
             "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                              "sample": f"{args.steps} steps of {T} tokens"},
             "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -629,6 +635,8 @@ def main():
     ap.add_argument("--workload", default="decode", choices=sorted(WORKLOADS))
     ap.add_argument("--sweep", action="store_true", help="add decode/prefill sweep points")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--fusion", default="max", choices=["max", "min", "mean", "gsp", "rcr", "score"],
+                    help="skip rule (max = ACE; the others are the paper's ablation variants and router-score skipping)")
     ap.add_argument("--tables-only", action="store_true",
                     help="time only the GPU offline tables (ace_offline_tables_device) of the workload's layer")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)

@@ -12,13 +12,14 @@ from __future__ import annotations
 from . import ace
 
 
-def calibrate_taus(layer: "ace.AceLayer", x_calib, T: int, qs, stream=None) -> dict:
-    """{q: tau} for the layer from the device tokens x_calib [T, d]."""
+def calibrate_taus(layer: "ace.AceLayer", x_calib, T: int, qs, stream=None, fusion="max") -> dict:
+    """{q: tau} for the layer from the device tokens x_calib [T, d] (under the
+    given skip rule: tau is a threshold on that rule's score)."""
     import torch
     out = torch.empty_like(x_calib)
     taus = {}
     for q in qs:
-        ace.ace_moe_forward(layer.handle, x_calib, out, T, "ratio", float(q), stream)
+        ace.ace_moe_forward(layer.handle, x_calib, out, T, "ratio", float(q), stream, fusion)
         _, _, _, tau, _ = ace.ace_last_skip_mask(layer.handle, T, layer.spec.top_k)
         taus[float(q)] = float(tau)
     return taus
