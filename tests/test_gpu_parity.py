@@ -431,3 +431,24 @@ def test_forward_host_graph_replay():
             assert (op.numpy().view(np.uint16) == want).all(), (T, mode, val)
             ace.ace_moe_forward_host(layer.handle, xp, op, T, mode, val)     # replay
             assert (op.numpy().view(np.uint16) == want).all(), (T, mode, val)
+
+
+@pytest.mark.parametrize("T", [64, 300])
+def test_non_finite_logits_reported(T):
+    """A NaN router logit ranks last in the top-k, and the next call that
+    synchronises reports ACE_ERR_NUMERIC once (the device word is cleared)."""
+    N, k = 128, 8
+    tables = synth.make_tables(N, seed=3, spread=0.2)
+    layer = _route_layer(N, k, T, 1, tables)
+    z = synth.make_logits(T, N, seed=17)
+    bad = z.copy()
+    bad[3, 5] = np.nan
+    ace.ace_route_logits(layer.handle, torch.from_numpy(bad).cuda(), T, "ratio", 0.5)
+    with pytest.raises(ace.AceError) as e:
+        ace.ace_last_skip_mask(layer.handle, T, k)
+    assert e.value.status == 6
+    skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, k)    # word cleared: no error now
+    assert 5 not in ids[3].tolist()                                         # NaN ranks last
+    ace.ace_route_logits(layer.handle, torch.from_numpy(z).cuda(), T, "ratio", 0.5)
+    ace.ace_last_skip_mask(layer.handle, T, k)
+    layer.close()
