@@ -160,13 +160,45 @@ __device__ __forceinline__ Tile tile_at(const TcParams& p, int tile, int n_base,
 // TMEM at tbase): EPI 0 writes SiLU(gate) * up as bf16 act (gate and up
 // columns interleaved in blocks of 16); EPI 1 writes the g_hat-scaled output
 // row of the slot, rounded to bf16, at its expert-grouped row (the combine
-// sums a token's rows in rank order). `row` is the token row in the tile.
+// sums a token's rows in rank order). The calling warp holds tile rows
+// [row_base, row_base + 32), one per lane; `gh` is the lane's g_hat (EPI 1,
+// loaded before the accumulator wait so its latency overlaps the MMAs).
+//
+// EPI 1 writes twice the bytes per tile of EPI 0 after a K loop of m instead
+// of d, so its stores bound the down GEMM. TMEM hands each lane one row, so
+// the warp's values pass through `stg` (32 rows x 128 B of this warp's shared
+// memory, 16-byte chunks XOR-swizzled by row so both the row-wise writes and
+// the column-wise reads are free of bank conflicts) and leave as 128-byte row
+// segments: each store instruction writes four whole lines instead of 32
+// separate 16-byte pieces.
+__device__ __forceinline__ void stage_chunk(unsigned char* stg, int lane, const uint4 (&v)[8]) {
+#pragma unroll
+    for (int g = 0; g < 8; ++g)
+        *reinterpret_cast<uint4*>(stg + lane * 128 + ((g ^ (lane & 7)) << 4)) = v[g];
+    __syncwarp();
+}
+
+// Rows [row_base, row_base + 32) of `stg`, 128 bytes each, to dst0 + row * ld_bytes.
+__device__ __forceinline__ void store_chunk(const unsigned char* stg, int lane, unsigned char* dst0, size_t ld_bytes,
+                                            int row_base, int nrows) {
+    const int gg = lane & 7;
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+        const int r = it * 4 + (lane >> 3);
+        const uint4 v = *reinterpret_cast<const uint4*>(stg + r * 128 + ((gg ^ (r & 7)) << 4));
+        if (row_base + r < nrows) *reinterpret_cast<uint4*>(dst0 + (size_t)(row_base + r) * ld_bytes + gg * 16) = v;
+    }
+    __syncwarp();                                        // stg is rewritten by the next chunk
+}
+
 template <int EPI>
-__device__ __forceinline__ void epilogue_wide(const TcParams& p, const Tile& t, uint32_t tbase, int row) {
+__device__ __forceinline__ void epilogue_wide(const TcParams& p, const Tile& t, uint32_t tbase, int row_base,
+                                              int lane, float gh, unsigned char* stg) {
     constexpr int WT = 256;
-    const bool valid = row < t.nrows;
-    const size_t orow = (size_t)(t.row0 + row);
     if (EPI == 0) {
+        // direct 32-byte stores per row: staging these through shared memory
+        // measured slower (the MMAs, not the stores, bound this GEMM)
+        const int row = row_base + lane;
         __nv_bfloat16* act = static_cast<__nv_bfloat16*>(p.out);
 #pragma unroll 1
         for (int blk = 0; blk < WT / 32; ++blk) {
@@ -174,43 +206,49 @@ __device__ __forceinline__ void epilogue_wide(const TcParams& p, const Tile& t, 
             tmem_ld16(tbase + blk * 32, g);
             tmem_ld16(tbase + blk * 32 + 16, u);
             tmem_ld_wait();
-            if (valid) {
+            if (row < t.nrows) {
                 __align__(16) __nv_bfloat16 o[16];
 #pragma unroll
                 for (int i = 0; i < 16; ++i)
                     o[i] = __float2bfloat16_rn(silu(__uint_as_float(g[i])) * __uint_as_float(u[i]));
                 const int j0 = (t.wt * (WT / 32) + blk) * 16;
-                uint4* dst = reinterpret_cast<uint4*>(act + orow * p.out_ld + j0);
+                uint4* dst = reinterpret_cast<uint4*>(act + (size_t)(t.row0 + row) * p.out_ld + j0);
                 dst[0] = reinterpret_cast<const uint4*>(o)[0];
                 dst[1] = reinterpret_cast<const uint4*>(o)[1];
             }
         }
     } else {
-        __nv_bfloat16* y = static_cast<__nv_bfloat16*>(p.out);
-        const float gh = valid ? p.ghat[p.perm[orow]] : 0.f;
-        uint4* dst = reinterpret_cast<uint4*>(y + orow * p.out_ld + t.wt * WT);
+        unsigned char* y = static_cast<unsigned char*>(p.out) + (size_t)t.row0 * p.out_ld * 2;
 #pragma unroll 1
         for (int c0 = 0; c0 < WT; c0 += 64) {
             uint32_t r[4][16];
 #pragma unroll
             for (int q = 0; q < 4; ++q) tmem_ld16(tbase + c0 + 16 * q, r[q]);
             tmem_ld_wait();
-            if (valid) {
+            uint4 v[8];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    uint32_t w[8];
+            for (int q = 0; q < 4; ++q) {
+                uint32_t w[8];
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const __nv_bfloat162 b2 = __floats2bfloat162_rn(gh * __uint_as_float(r[q][2 * i]),
-                                                                        gh * __uint_as_float(r[q][2 * i + 1]));
-                        w[i] = *reinterpret_cast<const uint32_t*>(&b2);
-                    }
-                    dst[(c0 + 16 * q) / 8] = make_uint4(w[0], w[1], w[2], w[3]);
-                    dst[(c0 + 16 * q) / 8 + 1] = make_uint4(w[4], w[5], w[6], w[7]);
+                for (int i = 0; i < 8; ++i) {
+                    const __nv_bfloat162 b2 = __floats2bfloat162_rn(gh * __uint_as_float(r[q][2 * i]),
+                                                                    gh * __uint_as_float(r[q][2 * i + 1]));
+                    w[i] = *reinterpret_cast<const uint32_t*>(&b2);
                 }
+                v[2 * q] = make_uint4(w[0], w[1], w[2], w[3]);
+                v[2 * q + 1] = make_uint4(w[4], w[5], w[6], w[7]);
             }
+            stage_chunk(stg, lane, v);
+            store_chunk(stg, lane, y + (size_t)(t.wt * WT + c0) * 2, (size_t)p.out_ld * 2, row_base, t.nrows);
         }
     }
+}
+
+// g_hat of a wide tile's row for EPI 1 (0 for rows past the tile's end).
+template <int EPI>
+__device__ __forceinline__ float wide_row_ghat(const TcParams& p, const Tile& t, int row) {
+    if (EPI != 1 || row >= t.nrows) return 0.f;
+    return p.ghat[p.perm[t.row0 + row]];
 }
 
 // ---------------------------------------------------------------- kernel
@@ -233,7 +271,8 @@ struct TcCfg {
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int ACC_COLS = BN;                       // fp32 columns per accumulator
     static constexpr int TMEM_COLS = (2 * ACC_COLS) < 32 ? 32 : 2 * ACC_COLS;
-    static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+    static constexpr int STG_BYTES = (!SWAP && EPI == 1) ? 4 * 4096 : 0;   // EPI 1 staging, 4 KB per warp
+    static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/ + STG_BYTES;
 };
 
 template <bool SWAP, int EPI, int STAGES>
@@ -368,15 +407,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
     } else {
         // ------------------------------------------------ epilogue (warps 2..5)
         const int quad = warp & 3;                       // TMEM lane quadrant of this warp
+        unsigned char* stg = smem + STAGES * C::STAGE_BYTES + 256 + quad * 4096;
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+            // the tile's rows and g_hat are read while its MMAs still run
+            const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile, n_base, kblocks);
+            const float gh = SWAP ? 0.f : wide_row_ghat<EPI>(p, t, quad * 32 + lane);
             bool ok = true;
             if (lane == 0) ok = mbar_wait(&acc_full[acc], acc_phase, p.err) && !*abort_flag;
             ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
             if (!ok) break;
             tc_fence_after();
-            const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile, n_base, kblocks);
             const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * C::ACC_COLS);
             if (SWAP) {
                 // lane = weight row (32 per warp), columns = TOKTILE (16) tokens
@@ -424,7 +466,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                 const bool valid = row < t.nrows;
                 const size_t orow = (size_t)(t.row0 + row);
                 if (EPI != 2) {
-                    epilogue_wide<EPI>(p, t, tbase, row);
+                    epilogue_wide<EPI>(p, t, tbase, quad * 32, lane, gh, stg);
                 } else {
                     // split-K: raw partial sums per slice (bias and temperature added by the consumer)
                     float* z = static_cast<float*>(p.out) + (size_t)t.split * p.split_stride;
@@ -738,7 +780,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
 constexpr int kPairStages = 6;
 constexpr int kPairHalf = 128 * kBK * 2;                   // 16 KB: 128 rows x 64 bf16
 constexpr int kPairStage = 2 * kPairHalf;                  // this CTA's A + B halves
-constexpr int kPairSmem = kPairStages * kPairStage + 1024 + 256;
+constexpr int kPairSmem = kPairStages * kPairStage + 1024 + 256 + 4 * 4096;   // + epilogue staging
 
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1) k_expert_pair(const __grid_constant__ TcParams p) {
@@ -845,18 +887,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_pair(const __grid_consta
     } else {
         // ------------------------------------------------ epilogue (warps 2..5, both CTAs)
         const int quad = warp & 3;
+        const int row_base = 128 * (int)rank + quad * 32;
+        unsigned char* stg = smem + kPairStages * kPairStage + 256 + quad * 4096;
         const uint32_t acc_empty_leader[2] = {mapa_shared(&acc_empty[0], 0), mapa_shared(&acc_empty[1], 0)};
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int tile = unit; tile < n_tiles; tile += n_units) {
+            // the tile's rows and g_hat are read while its MMAs still run
+            const Tile t = tile_at<256, 256>(p, tile, n_tiles, kblocks);
+            const float gh = wide_row_ghat<EPI>(p, t, row_base + lane);
             bool ok = true;
             if (lane == 0) ok = mbar_wait(&acc_full[acc], acc_phase, p.err) && !*abort_flag;
             ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
             if (!ok) break;
             tc_fence_after();
-            const Tile t = tile_at<256, 256>(p, tile, n_tiles, kblocks);
             const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * 256);
-            epilogue_wide<EPI>(p, t, tbase, 128 * (int)rank + quad * 32 + lane);
+            epilogue_wide<EPI>(p, t, tbase, row_base, lane, gh, stg);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(acc_empty_leader[acc]);
