@@ -672,10 +672,11 @@ __device__ __forceinline__ int block_exscan_1024(int v, int* wtot, int& total) {
 //   k_topk_score  adds the digit-1 histogram (4096 bins, hist1);
 //   k_sel_collect (many blocks) finds digit 1 from hist1 (every block, the
 //                 same way), appends the keys inside it to cand and adds
-//                 their digit-2 histogram (1024 bins, hist2);
+//                 their digit-2 histogram (1024 bins, hist2); KPT keys per
+//                 thread, chosen so the grid spans the SMs (its time is the
+//                 latency of the hist1 and key loads, not bandwidth);
 //   k_sel_final   (one block) finds digit 2, then digit 3 over cand, writes
 //                 tau and re-zeroes hist1, hist2 and the candidate count.
-constexpr int kSelKeysPerThread = 8;
 
 // Block-wide digit search over `bins` = 1024 * per counts held per thread:
 // the owner of rank `want` records prefix | digit << shift in S.
@@ -704,6 +705,7 @@ __device__ __forceinline__ void find_digit(const int (&b)[PER], int want, uint32
     __syncthreads();
 }
 
+template <int KPT>
 __global__ void __launch_bounds__(1024) k_sel_collect(const uint32_t* __restrict__ keys, int n, int m,
                                                       const int32_t* __restrict__ hist1,
                                                       int32_t* __restrict__ hist2, uint32_t* __restrict__ cand,
@@ -723,21 +725,21 @@ __global__ void __launch_bounds__(1024) k_sel_collect(const uint32_t* __restrict
         meta[kMetaSelWant] = S.want;
         meta[kMetaSelBelow] = S.below;
     }
-    // this block's keys: kSelKeysPerThread per thread, 16-byte loads
-    const int base = (blockIdx.x * 1024 + tid) * kSelKeysPerThread;
-    uint32_t kv[kSelKeysPerThread];
-    if (base + kSelKeysPerThread <= n) {
+    // this block's keys: KPT per thread (16-byte loads when KPT is a multiple of 4)
+    const int base = (blockIdx.x * 1024 + tid) * KPT;
+    uint32_t kv[KPT];
+    if (KPT % 4 == 0 && base + KPT <= n) {
 #pragma unroll
-        for (int j = 0; j < kSelKeysPerThread; j += 4) {
+        for (int j = 0; j + 3 < KPT; j += 4) {
             const uint4 v = __ldcg(reinterpret_cast<const uint4*>(keys + base + j));
             kv[j] = v.x; kv[j + 1] = v.y; kv[j + 2] = v.z; kv[j + 3] = v.w;
         }
     } else {
 #pragma unroll
-        for (int j = 0; j < kSelKeysPerThread; ++j) kv[j] = base + j < n ? __ldcg(keys + base + j) : 0xffffffffu;
+        for (int j = 0; j < KPT; ++j) kv[j] = base + j < n ? __ldcg(keys + base + j) : 0xffffffffu;
     }
 #pragma unroll
-    for (int j = 0; j < kSelKeysPerThread; ++j) {
+    for (int j = 0; j < KPT; ++j) {
         const bool in = kv[j] != 0xffffffffu && (kv[j] & 0xFFF00000u) == prefix;
         const unsigned bal = __ballot_sync(0xffffffffu, in);
         if (!bal) continue;
@@ -806,11 +808,14 @@ __global__ void __launch_bounds__(1024) k_sel_final(int m, int32_t* __restrict__
 // slots grouped by expert, tokens increasing inside a group.
 // Pass A (k_compact_count): per-chunk per-expert counts, stored expert-major
 //   (counts[e * n_chunks + c]).
-// Pass B (k_compact_scan, one block): exclusive scan of the counts in that
-//   order, so counts[e][c] becomes the first row of chunk c's expert-e slots;
-//   offsets[N+1], the distinct-expert list and the token-tile table.
-// Pass C (k_compact_place): each chunk places its slots: rank within
-//   (chunk, expert) from a per-expert token bitmap, so the order is deterministic.
+// Pass B (k_compact_scan, a block per expert): exclusive scan of expert e's
+//   row, so counts[e][c] becomes the first row of chunk c's expert-e slots
+//   within the expert's group; the last block to finish (atomic ticket) scans
+//   the row totals into offsets[N+1], the distinct-expert list and the
+//   token-tile table.
+// Pass C (k_compact_place): each chunk places its slots at offsets[e] +
+//   counts[e][c] + rank, the rank within (chunk, expert) from a per-expert
+//   token bitmap, so the order is deterministic.
 // With DECIDE (ratio mode) pass A first takes each token's decision from the
 // stored g, c and the device tau (decide_token).
 template <bool DECIDE>
@@ -839,63 +844,79 @@ __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, i
         chunk_counts[(size_t)e * n_chunks + blockIdx.x] = cnt[e];
 }
 
-constexpr int kScanPer = 8;   // counts per thread per round of k_compact_scan
+constexpr int kScanThreads = 256;   // k_compact_scan block: 4 counts per thread per round
 
-// Rounds of 8192 counts: coalesced load into shared memory, each thread
-// scans its 8 consecutive counts, block scan of the thread sums, coalesced
-// store of the exclusive prefixes.
-__global__ void __launch_bounds__(1024) k_compact_scan(int n_exp, int n_chunks, int32_t* __restrict__ counts,
-                                                       int32_t* __restrict__ offsets, int32_t* __restrict__ dlist,
-                                                       int32_t* __restrict__ meta, int tok_tile,
-                                                       int32_t* __restrict__ tt_off, int4* __restrict__ tt_tab) {
+// Exclusive prefix of v over the block (thread order, blockDim.x a multiple
+// of 32); total = the block's sum. wtot: 32 ints of shared memory.
+__device__ __forceinline__ int block_exscan(int v, int* wtot, int& total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    int inc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+    }
+    if (lane == 31) wtot[warp] = inc;
+    __syncthreads();
+    if (warp == 0) {
+        int wi = lane < nw ? wtot[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += y;
+        }
+        wtot[lane] = wi;
+    }
+    __syncthreads();
+    const int exc = inc - v + (warp ? wtot[warp - 1] : 0);
+    total = wtot[nw - 1];
+    __syncthreads();
+    return exc;
+}
+
+// Block e: exclusive scan of counts[e][0 .. n_chunks) in place, row total to
+// offsets[e]. The last block (ticket in meta) turns the totals into
+// offsets[N+1], the distinct-expert list, the meta totals and the token-tile
+// table, and re-zeroes the ticket.
+__global__ void __launch_bounds__(kScanThreads) k_compact_scan(int n_exp, int n_chunks, int32_t* __restrict__ counts,
+                                                               int32_t* __restrict__ offsets,
+                                                               int32_t* __restrict__ dlist,
+                                                               int32_t* __restrict__ meta, int tok_tile,
+                                                               int32_t* __restrict__ tt_off, int4* __restrict__ tt_tab) {
     __shared__ int wtot[32];
     __shared__ int wsum[96];
     __shared__ int cnt[kMaxExperts];
-    __shared__ __align__(16) int buf[1024 * kScanPer];
+    __shared__ int s_last;
     pdl_wait();
-    const int n = n_exp * n_chunks;
     const int tid = threadIdx.x;
+    int32_t* row = counts + (size_t)blockIdx.x * n_chunks;
     int carry = 0;
-    for (int r0 = 0; r0 < n; r0 += 1024 * kScanPer) {
+    for (int c0 = 0; c0 < n_chunks; c0 += 4 * kScanThreads) {
+        int v[4];
 #pragma unroll
-        for (int j = 0; j < kScanPer; ++j) {
-            const int i = r0 + j * 1024 + tid;
-            buf[j * 1024 + tid] = i < n ? __ldcg(counts + i) : 0;
+        for (int j = 0; j < 4; ++j) {
+            const int c = c0 + 4 * tid + j;
+            v[j] = c < n_chunks ? __ldcg(row + c) : 0;
         }
-        __syncthreads();
-        int v[kScanPer];
-        const int4* b4 = reinterpret_cast<const int4*>(buf + tid * kScanPer);
-#pragma unroll
-        for (int q = 0; q < kScanPer / 4; ++q) {
-            const int4 x = b4[q];
-            v[4 * q] = x.x; v[4 * q + 1] = x.y; v[4 * q + 2] = x.z; v[4 * q + 3] = x.w;
-        }
-        int loc = 0;
-#pragma unroll
-        for (int j = 0; j < kScanPer; ++j) loc += v[j];
         int total;
-        int run = carry + block_exscan_1024(loc, wtot, total);   // (its barriers also order buf)
+        int run = carry + block_exscan(v[0] + v[1] + v[2] + v[3], wtot, total);
 #pragma unroll
-        for (int j = 0; j < kScanPer; ++j) {
-            buf[tid * kScanPer + j] = run;
+        for (int j = 0; j < 4; ++j) {
+            const int c = c0 + 4 * tid + j;
+            if (c < n_chunks) row[c] = run;
             run += v[j];
         }
-        __syncthreads();
-#pragma unroll
-        for (int j = 0; j < kScanPer; ++j) {
-            const int i = r0 + j * 1024 + tid;
-            if (i < n) {
-                const int b = buf[j * 1024 + tid];
-                counts[i] = b;
-                if (i % n_chunks == 0) offsets[i / n_chunks] = b;
-            }
-        }
-        __syncthreads();
         carry += total;
     }
-    if (tid == 0) offsets[n_exp] = carry;
+    if (tid == 0) offsets[blockIdx.x] = carry;
+    __threadfence();
     __syncthreads();
-    for (int e = tid; e < n_exp; e += blockDim.x) cnt[e] = __ldcg(offsets + e + 1) - __ldcg(offsets + e);
+    if (tid == 0) s_last = atomicAdd(&meta[kMetaTicket], 1) == (int)gridDim.x - 1;
+    __syncthreads();
+    if (!s_last) return;
+    if (tid == 0) meta[kMetaTicket] = 0;
+    __threadfence();
+    for (int e = tid; e < n_exp; e += blockDim.x) cnt[e] = __ldcg(offsets + e);
     __syncthreads();
     scan_counts_block(cnt, n_exp, offsets, dlist, meta, nullptr, tok_tile, tt_off, wsum);
     __syncthreads();
@@ -905,6 +926,7 @@ __global__ void __launch_bounds__(1024) k_compact_scan(int n_exp, int n_chunks, 
 __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, int n_exp, int n_chunks,
                                                           const int32_t* __restrict__ ids,
                                                           const uint8_t* __restrict__ skip,
+                                                          const int32_t* __restrict__ offsets,
                                                           const int32_t* __restrict__ chunk_base,
                                                           int32_t* __restrict__ perm,
                                                           int32_t* __restrict__ slot_pos) {
@@ -929,7 +951,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
             const int e = ids[s];
             int rank = __popc(bm[e * W + w] & lt);
             for (int ww = 0; ww < w; ++ww) rank += __popc(bm[e * W + ww]);
-            const int r = __ldcg(chunk_base + (size_t)e * n_chunks + blockIdx.x) + rank;
+            const int r = __ldcg(offsets + e) + __ldcg(chunk_base + (size_t)e * n_chunks + blockIdx.x) + rank;
             perm[r] = (int32_t)s;
             slot_pos[s] = r;
         }
@@ -1465,9 +1487,16 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     if (e != cudaSuccess) return e;
     if (mode == ACE_SKIP_RATIO) {
         const int nk = T * k;
-        e = launch_pdl(k_sel_collect, dim3(cdiv(nk, 1024 * kSelKeysPerThread)), dim3(1024), 0, s,
-                       (const uint32_t*)W.keys, nk, m_q, (const int32_t*)W.sel_hist, W.sel_hist + kHistBins,
-                       W.sel_cand, W.meta);
+        // fewest keys per thread that keep the grid within two 1024-thread blocks per SM
+#define ACE_COLLECT(KPT)                                                                                          \
+    launch_pdl(k_sel_collect<KPT>, dim3(cdiv(nk, 1024 * KPT)), dim3(1024), 0, s, (const uint32_t*)W.keys, nk, m_q, \
+               (const int32_t*)W.sel_hist, W.sel_hist + kHistBins, W.sel_cand, W.meta)
+        const long long slots = 2LL * 1024 * L->num_sms;
+        if (nk <= slots) e = ACE_COLLECT(1);
+        else if (nk <= 2 * slots) e = ACE_COLLECT(2);
+        else if (nk <= 4 * slots) e = ACE_COLLECT(4);
+        else e = ACE_COLLECT(8);
+#undef ACE_COLLECT
         if (e != cudaSuccess) return e;
         e = launch_pdl(k_sel_final, dim3(1), dim3(1024), 0, s, m_q, W.sel_hist, W.sel_hist + kHistBins,
                        (const uint32_t*)W.sel_cand, W.meta, W.tau);
@@ -1479,11 +1508,12 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
                    n_chunks, (const int32_t*)W.ids, W.skip, (const float*)W.gates, (const float*)W.cval,
                    (const float*)W.tau, D.min_active, D.eps, W.ghat, W.chunk_counts);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k_compact_scan, dim3(1), dim3(1024), 0, s, n, n_chunks, W.chunk_counts, W.offsets, W.dlist, W.meta,
-                   tok_tile, W.tt_off, W.tt_tab);
+    e = launch_pdl(k_compact_scan, dim3(n), dim3(kScanThreads), 0, s, n, n_chunks, W.chunk_counts, W.offsets, W.dlist,
+                   W.meta, tok_tile, W.tt_off, W.tt_tab);
     if (e != cudaSuccess) return e;
     return launch_pdl(k_compact_place, dim3(n_chunks), dim3(kChunk), 0, s, T, k, n, n_chunks, (const int32_t*)W.ids,
-                      (const uint8_t*)W.skip, (const int32_t*)W.chunk_counts, W.perm, W.slot_pos);
+                      (const uint8_t*)W.skip, (const int32_t*)W.offsets, (const int32_t*)W.chunk_counts, W.perm,
+                      W.slot_pos);
 }
 
 int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl) {
