@@ -116,11 +116,11 @@ def _large():
         # the GPU tables (checked against the oracle in test_large_layer_tables_device)
         w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables_device(w)
         _LARGE["w"] = w
-        _LARGE["layer"] = ace.AceLayer(w, w.extra["a_gsp"], w.extra["a_rcr"], max_tokens=2048)
+        _LARGE["layer"] = ace.AceLayer(w, w.extra["a_gsp"], w.extra["a_rcr"], max_tokens=8192)
     return _LARGE["w"], _LARGE["layer"]
 
 
-@pytest.mark.parametrize("T,q", [(1, 0.5), (16, 0.25), (128, 0.5), (2048, 0.5)])
+@pytest.mark.parametrize("T,q", [(1, 0.5), (16, 0.25), (128, 0.5), (128, 0.625), (2048, 0.5), (8192, 0.5)])
 def test_large_layer(T, q):
     w, layer = _large()
     spec = w.spec

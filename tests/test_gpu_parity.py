@@ -279,7 +279,8 @@ FORWARD_CASES = [
     ("qwen", 1, "ratio", 0.5), ("qwen", 8, "ratio", 0.25), ("qwen", 32, "ratio", 0.5),
     ("qwen", 64, "ratio", 0.0), ("qwen", 64, "ratio", 0.25), ("qwen", 64, "ratio", 0.5),
     ("qwen", 17, "threshold", 0.11), ("qwen", 129, "ratio", 0.5), ("qwen", 1000, "ratio", 0.625),
-    ("qwen_zipf", 4096, "ratio", 0.0), ("qwen_zipf", 4096, "ratio", 0.5),
+    ("qwen_zipf", 4096, "ratio", 0.0), ("qwen_zipf", 4096, "ratio", 0.25), ("qwen_zipf", 4096, "ratio", 0.5),
+    ("qwen_zipf", 4096, "ratio", 0.625),
     ("qwen_temp", 64, "ratio", 0.5), ("qwen_temp", 600, "ratio", 0.625), ("qwen_temp", 48, "threshold", 0.1),
     ("qwen", 256, "ratio", 0.5), ("qwen", 257, "ratio", 0.5),          # both sides of the small-batch path
     ("wide", 40, "ratio", 0.5), ("wide", 700, "ratio", 0.5), ("wide", 256, "threshold", 0.05),
