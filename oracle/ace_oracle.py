@@ -33,8 +33,10 @@ router translation invariance (App. A.2.2), the closed-form table means and
 scaling laws, the realised skip count of the quantile rule, the exp error
 bound against math.exp, and for the skip-rule variants a hand-worked example
 (tests/golden/fusion_worked.json), the nesting Max within Mean within Min,
-Max / Min as intersection / union of the single views, and router-score
-skipping as the GSP view with unit tables.
+Max / Min as intersection / union of the single views, router-score
+skipping as the GSP view with unit tables, and for the layer stack the
+identity when every down projection is zero and a dense evaluation of its one
+non-zero layer.
 
 Readings where the paper is silent (each also listed in the design notes):
   * gates g are the softmax over the top-k logits (softmax over all experts

@@ -459,6 +459,35 @@ def test_exp32_error_bound():
     assert O.exp32(np.array([-90.0], np.float32))[0] == 0.0
 
 
+def test_stack_residual_structure():
+    """The stack reading x_{l+1} = x_l + y_l(x_l), each layer with its own
+    RMSNorm: experts with zero down projections make every layer the
+    identity, and a stack whose only non-zero layer is the second one equals
+    x plus that layer's output on x, computed densely over all experts."""
+    layers = [_tiny_layer(s) for s in (11, 12, 13)]
+    x = np.random.Generator(np.random.PCG64(14)).standard_normal((20, layers[0].spec.hidden)) * 3.0
+    for w in layers:
+        w.w_down = np.zeros_like(w.w_down)
+    assert np.array_equal(O.moe_stack_forward(x, layers, "ratio", 0.5), x)
+    live = _tiny_layer(15)
+    layers[1] = live
+    got = O.moe_stack_forward(x, layers, "threshold", 0.3)
+    # dense reference for the live layer: every expert on every token, weighted by kept g_hat
+    h = x / np.sqrt((x * x).mean(axis=1, keepdims=True) + live.spec.rms_eps) * live.gamma
+    z = h @ live.router_w.T + live.router_b
+    dec = O.ace_decide(z, live.spec.top_k, live.extra["a_gsp"], live.extra["a_rcr"], "threshold", 0.3)
+    y = np.zeros_like(x)
+    for t in range(x.shape[0]):
+        for i in range(live.spec.top_k):
+            if dec["skip"][t, i]:
+                continue
+            e = dec["ids"][t, i]
+            u, v = live.w_gate[e] @ h[t], live.w_up[e] @ h[t]
+            y[t] += dec["g_hat"][t, i] * (live.w_down[e] @ (u / (1 + np.exp(-u)) * v))
+    np.testing.assert_allclose(got, x + y, rtol=1e-12, atol=1e-12)
+    assert np.abs(y).max() > 1e-2                      # the live layer really contributes
+
+
 def test_permutation_bruteforce():
     rng = np.random.Generator(np.random.PCG64(15))
     T, N, k = 50, 12, 4
