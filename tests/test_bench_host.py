@@ -32,6 +32,19 @@ def test_recorded_traffic_follows_the_kernel_sources(tmp_path, monkeypatch):
     assert bench._recorded_traffic("missing.md") is None
 
 
+def test_clock_records_that_disqualify_a_timed_region():
+    ok = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [], "samples": 17}
+    capped = {"sm_mhz": 1850.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 30}
+    assert bench.clocks_rejected(ok) is None
+    assert bench.clocks_rejected(capped) is None          # power cap under load is kept
+    assert bench.clocks_rejected(None) is None            # no nvidia-smi: nothing to judge
+    for r in ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"):
+        assert r in bench.clocks_rejected(dict(ok, reasons=[r, "sw_power_cap"]))
+    locked = dict(ok, sm_mhz=1200.0)                      # held low with no reason: a clock lock
+    assert bench.clocks_rejected(locked) is not None
+    assert bench.clocks_rejected(dict(locked, reasons=["sw_power_cap"])) is None
+
+
 def test_algorithmic_bytes_of_the_decode_layer():
     """Retained-expert weight bytes: 3 matrices of d x m bf16 per distinct expert."""
     w = synth.LayerWeights(synth.spec_qwen(), None, None, None, None, None, None)
