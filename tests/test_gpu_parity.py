@@ -279,6 +279,7 @@ FORWARD_CASES = [
     ("qwen", 1, "ratio", 0.5), ("qwen", 8, "ratio", 0.25), ("qwen", 32, "ratio", 0.5),
     ("qwen", 64, "ratio", 0.0), ("qwen", 64, "ratio", 0.25), ("qwen", 64, "ratio", 0.5),
     ("qwen", 17, "threshold", 0.11), ("qwen", 129, "ratio", 0.5), ("qwen", 1000, "ratio", 0.625),
+    ("qwen", 1000, "ratio", 1.0),                                      # every non-top-1 slot skipped
     ("qwen_zipf", 4096, "ratio", 0.0), ("qwen_zipf", 4096, "ratio", 0.25), ("qwen_zipf", 4096, "ratio", 0.5),
     ("qwen_zipf", 4096, "ratio", 0.625),
     ("qwen_temp", 64, "ratio", 0.5), ("qwen_temp", 600, "ratio", 0.625), ("qwen_temp", 48, "threshold", 0.1),
