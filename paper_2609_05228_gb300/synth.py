@@ -32,10 +32,15 @@ import numpy as np
 # Elements per generation chunk. Fixed: changing it changes every value.
 _CHUNK = 1 << 22
 
-# Zipf router-bias scale. The routed-count slope over the popularity ranks
-# 1..N/2 that this produces is checked by the tests (target slope -1.1).
+# Zipf router-bias profile b_e = -beta * ZIPF_S * log(r_e). beta depends on
+# the layer shape (the logit noise grows with the hidden size, the ranks with
+# the expert count), so each named shape carries its own value, found by a 1-D
+# search with the CPU oracle's routing (tests/golden/derive_zipf_beta.py) so
+# that the routed-slot counts, sorted, fall with log-log slope -1.1 +- 0.05
+# over the popularity ranks 1..N/2; the tests check that slope per shape.
 ZIPF_S = 1.1
-ZIPF_BETA = 0.59
+ZIPF_BETA = 0.59          # hidden 2048, 128 experts, top-8 (4096 tokens: -1.10)
+ZIPF_BETA_LARGE = 0.70    # hidden 4096, 256 experts, top-8 (8192 tokens: -1.105; 2048: -1.08)
 
 
 def bf16_bits(a: np.ndarray) -> np.ndarray:
@@ -91,6 +96,7 @@ class LayerSpec:
     eps: float = 1e-6            # the paper's numerical constant epsilon
     router_temp: float = 1.0
     min_active: int = 1
+    zipf_beta: float = ZIPF_BETA  # scale of the Zipf router bias (used when zipf)
 
 
 @dataclass
@@ -134,7 +140,7 @@ def make_layer(spec: LayerSpec, seed: int) -> LayerWeights:
     if spec.zipf:
         gz = np.random.Generator(np.random.PCG64(s_zipf))
         ranks = gz.permutation(n) + 1
-        b = -ZIPF_BETA * ZIPF_S * np.log(ranks.astype(np.float64))
+        b = -spec.zipf_beta * ZIPF_S * np.log(ranks.astype(np.float64))
         b -= b.mean()
         router_b = b.astype(np.float32)
     return LayerWeights(spec, router_w, router_b, w_gate, w_up, w_down, gamma, seed)
@@ -184,4 +190,4 @@ def spec_qwen(zipf: bool = False) -> LayerSpec:
 
 
 def spec_large(zipf: bool = True) -> LayerSpec:
-    return LayerSpec(4096, 256, 8, 2048, dtype="bf16", zipf=zipf)
+    return LayerSpec(4096, 256, 8, 2048, dtype="bf16", zipf=zipf, zipf_beta=ZIPF_BETA_LARGE)
