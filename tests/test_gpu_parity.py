@@ -4,10 +4,15 @@ the same seeded inputs.
 * exp32 and the whole decision (top-k ids, skip mask, g_hat, tau, retained
   count, offsets, permutation) are bit-exact against the oracle's float32
   decision spec, given the same float32 logits from the input generator.
-* The full layer is compared with the fp64 oracle: rel-L2 <= 5e-3 and
-  max-abs <= 3e-2 * max|ref| (bf16), on every token whose routing is not
-  within rounding distance of a decision boundary (top-k logit gap and
-  |c - tau|); those boundary tokens are counted and must stay a minority.
+* Every forward is checked in replay mode: its own float32 router logits
+  (compared with the fp64 oracle's logits from x) are fed to the float32
+  decision spec, which must reproduce the forward's decision bit for bit;
+  the fp64 oracle then evaluates the layer under that decision and every
+  token's output is compared: rel-L2 <= 5e-3 and max-abs <= 3e-2 * max|ref|
+  (bf16), rel-L2 <= 1e-5 (fp32 layer).
+* The independent fp64 decision is checked on the tokens whose routing is
+  clear of every boundary by more than the GPU's rounding can move it, and
+  its disagreement rate with the replayed decision is reported.
 """
 import dataclasses
 import math
@@ -17,14 +22,11 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
+import _replay as RP
 import oracle as O
 from paper_2609_05228_gb300 import ace, offline, synth
 
 pytestmark = pytest.mark.gpu
-
-RTOL_L2 = 5e-3
-RTOL_MAX = 3e-2
-RTOL_L2_F32 = 1e-5
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -176,6 +178,31 @@ def test_decision_degenerate_scores(T, pattern):
     layer.close()
 
 
+@pytest.mark.parametrize("T", [5, 700])
+def test_decision_signed_zero_and_tied_logits(T):
+    """Exact logit ties, including -0.0 against +0.0 (equal logits): the
+    lower expert index ranks first, through the small-batch fused route and
+    the large-batch chain, bit-exact with the fp32 decision spec."""
+    N, k = 64, 6
+    g = np.random.Generator(np.random.PCG64(41))
+    z = np.zeros((T, N), np.float32)
+    z[:, :] = np.where(g.random((T, N)) < 0.5, np.float32(-0.0), np.float32(0.0))
+    hot = g.random((T, N)) < 0.1                     # a few higher logits, some tied among themselves
+    z[hot] = g.choice(np.array([0.5, 0.5, 1.0], np.float32), size=int(hot.sum()))
+    tables = synth.make_tables(N, seed=4, spread=0.2)
+    layer = _route_layer(N, k, T, 1, tables)
+    zd = torch.from_numpy(z).cuda()
+    ids_ref, g_ref = O.route_fp32(z, k)
+    for mode, val in [("threshold", 0.1), ("ratio", 0.5)]:
+        ace.ace_route_logits(layer.handle, zd, T, mode, val)
+        skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, k)
+        ref = O.decide_fp32(ids_ref, g_ref, tables[0], tables[1], mode, val, 1, 1e-6)
+        assert (ids == ids_ref).all(), mode
+        assert (skip.astype(bool) == ref["skip"]).all(), mode
+        assert (gh.view(np.uint32) == ref["g_hat"].view(np.uint32)).all(), mode
+    layer.close()
+
+
 def test_decision_repeatable():
     T, N, k = 4096, 128, 8
     z = synth.make_logits(T, N, seed=3)
@@ -265,18 +292,13 @@ def _run_layer(kind, T, mode, val, x_seed=1, fusion="max"):
     out = torch.empty_like(xd)
     layer.forward(xd, out, T, mode, val, fusion=fusion)
     torch.cuda.synchronize()
-    skip, ids, gh, tau, R = ace.ace_last_skip_mask(layer.handle, T, spec.top_k)
-    y_gpu = _host(out).astype(np.float64)
-    y_ref, dec = O.moe_forward(x, w, mode, val, return_decision=True, fusion=fusion)
-    h = O.rmsnorm(x, w.gamma, spec.rms_eps)
-    z_ref = O.router_logits(h, w.router_w, w.router_b, spec.router_temp)
-    return w, spec, x, y_gpu, y_ref, dec, z_ref, (skip, ids, gh, tau, R)
+    return w, layer, spec, x, _host(out).astype(np.float64)
 
 
 FORWARD_CASES = [
     ("tiny", 64, "ratio", 0.0), ("tiny", 64, "ratio", 0.25), ("tiny", 64, "ratio", 0.5),
     ("tiny", 64, "threshold", 0.2), ("tiny", 5, "ratio", 0.5),
-    ("qwen", 1, "ratio", 0.5), ("qwen", 8, "ratio", 0.25), ("qwen", 32, "ratio", 0.5),
+    ("qwen", 1, "ratio", 0.5), ("qwen", 1, "ratio", 0.0), ("qwen", 8, "ratio", 0.0), ("qwen", 8, "ratio", 0.25), ("qwen", 32, "ratio", 0.5),
     ("qwen", 64, "ratio", 0.0), ("qwen", 64, "ratio", 0.25), ("qwen", 64, "ratio", 0.5),
     ("qwen", 17, "threshold", 0.11), ("qwen", 129, "ratio", 0.5), ("qwen", 1000, "ratio", 0.625),
     ("qwen", 1000, "ratio", 1.0),                                      # every non-top-1 slot skipped
@@ -304,31 +326,54 @@ def test_forward_parity_fusion(fusion, kind, T, mode, val):
 
 
 def _check_forward(kind, T, mode, val, fusion):
-    w, spec, x, y_gpu, y_ref, dec, z_ref, (skip, ids, gh, tau, R) = _run_layer(kind, T, mode, val, fusion=fusion)
+    w, layer, spec, x, y_gpu = _run_layer(kind, T, mode, val, fusion=fusion)
     k = spec.top_k
-    margin = 1e-4 if spec.dtype == "f32" else None
+    f32 = spec.dtype == "f32"
+    # replay: the forward's own logits through the fp32 decision spec, bit-exact
+    dec, z_gpu = RP.replay_decision(layer.handle, spec, w.extra["a_gsp"], w.extra["a_rcr"], T, mode, val, fusion)
+    if mode == "ratio":
+        m_q = min(O.llround_pos(float(np.float32(val)) * T * k), T * (k - max(spec.min_active, 1)))
+        assert dec["count"] == m_q
+    # the logits themselves against the fp64 oracle, then every token's output
+    z_ref = RP.check_logits(z_gpu, x, w, f32=f32)
+    y_ref = O.moe_forward(x, w, decision=dec)
+    RP.compare(y_gpu, y_ref, f32=f32)
+    # the independent fp64 decision: equal on every token clear of a boundary
+    dec64 = O.ace_decide(z_ref, k, w.extra["a_gsp"], w.extra["a_rcr"], mode, val, spec.min_active, spec.eps, fusion)
+    margin = 1e-4 if f32 else None
     # the wide layer's logits are 4x the scale (so is their rounding), and its
     # 1024 candidates put more top-16 boundaries within that distance
     dz = 4 * 6e-3 if kind == "wide" else (margin or 6e-3)
-    clear = _clear_tokens(dec, z_ref, k, dz, margin or 8e-3, spec.min_active)
+    clear = _clear_tokens(dec64, z_ref, k, dz, margin or 8e-3, spec.min_active)
     assert clear.mean() >= (0.2 if kind == "wide" else 0.4), clear.mean()
-    # decisions agree on every clear token (compared per expert id)
     for t in np.nonzero(clear)[0]:
-        gpu = {int(ids[t, i]): bool(skip[t, i]) for i in range(k)}
-        ref = {int(dec["ids"][t, i]): bool(dec["skip"][t, i]) for i in range(k)}
+        gpu = {int(dec["ids"][t, i]): bool(dec["skip"][t, i]) for i in range(k)}
+        ref = {int(dec64["ids"][t, i]): bool(dec64["skip"][t, i]) for i in range(k)}
         assert gpu == ref, t
-    if mode == "ratio":
-        n_all = T * k
-        m_q = min(O.llround_pos(float(np.float32(val)) * n_all), T * (k - max(spec.min_active, 1)))
-        assert n_all - R == m_q
-    yr, yg = y_ref[clear], y_gpu[clear]
-    rel = np.linalg.norm(yg - yr) / max(np.linalg.norm(yr), 1e-30)
-    mx = np.abs(yg - yr).max() / max(np.abs(yr).max(), 1e-30)
-    if spec.dtype == "f32":
-        assert rel <= RTOL_L2_F32, rel
-    else:
-        assert rel <= RTOL_L2, rel
-        assert mx <= RTOL_MAX, mx
+    RP.note_disagreement(f"{kind} T={T} {mode}={val} {fusion}", dec, dec64)
+
+
+def test_layers_of_different_shapes_coexist():
+    """A layer created after another with a smaller shape must not lower the
+    kernels' shared-memory limits the first one needs: its forwards keep
+    working and give the same bits (decode and prefill paths)."""
+    w, layer = _layer("qwen")
+    outs = {}
+    for T in (64, 300):
+        x = _dev(synth.make_tokens(w.spec, T, seed=21))
+        o = torch.empty_like(x)
+        layer.forward(x, o, T, "ratio", 0.5)
+        outs[T] = (x, o)
+    torch.cuda.synchronize()
+    small = _route_layer(16, 4, 8, 1, synth.make_tables(16, seed=2))
+    small_f32 = ace.AceLayer(synth.make_layer(synth.spec_tiny(), 3), *synth.make_tables(16, seed=3), max_tokens=8)
+    for T, (x, o) in outs.items():
+        o2 = torch.empty_like(x)
+        layer.forward(x, o2, T, "ratio", 0.5)
+        torch.cuda.synchronize()
+        assert torch.equal(o, o2), T
+    small.close()
+    small_f32.close()
 
 
 def test_forward_q0_matches_threshold0():
