@@ -2,15 +2,18 @@
 """Benchmark of the ACE MoE-layer forward (token-adaptive expert skipping) on
 GB300, one process per GPU.
 
-Default workload: the Qwen3-30B-A3B-shaped MoE layer (hidden 2048, 128
-experts, top-8, expert FFN 768, bf16) decoding a batch of 64 tokens at target
-skip ratio 0.5 (per-batch threshold, App. B.1). A step is one full layer
-forward: RMSNorm, router, top-k, skip decision, threshold, compaction,
-experts and combine. Inputs are synthetic (seeded N(0,1) tokens, N(0, 0.02^2)
-weights) and resident in HBM; the forward is replayed from a CUDA graph and
-each step is timed with CUDA events; L2 is flushed between steps (a 512 MB
-write, then a 256 MB read so dirty lines are written back), outside the
-timed events.
+Default workload: the large MoE layer (hidden 4096, 256 experts, top-8,
+expert FFN 2048, bf16; 12.9 GB of expert weights) prefilling 8192 tokens with
+Zipf(1.1)-skewed routing at target skip ratio 0.5 (per-batch threshold,
+App. B.1). A step is one full layer forward: RMSNorm, router, top-k, skip
+decision, threshold, compaction, experts and combine. Inputs are synthetic
+(seeded N(0,1) tokens, N(0, 0.02^2) weights) and resident in HBM; the
+forward is replayed from a CUDA graph and each step is timed with CUDA
+events; L2 is flushed between steps (a 512 MB write, then a 256 MB read so
+dirty lines are written back), outside the timed events. The line also
+carries per-point records (`points`) for the decode batches 1, 8 and 64 and
+the 4096-token Zipf prefill of the hidden-2048 layer, its 4-layer stack
+prefilling 16384 tokens and the large layer decoding 128 tokens.
 
 Prints one JSON line (rank 0). `--impl reference` times the CPU oracle
 instead, on a bounded sample of the same workload.
@@ -31,24 +34,33 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
+QWEN = "d=2048 N=128 top-8 m=768 bf16"
+LARGE = "d=4096 N=256 top-8 m=2048 bf16"
 WORKLOADS = {
     "decode": dict(spec="qwen", zipf=False, T=64, q=0.5, layers=1, tables="offline",
-                   name="ACE MoE layer decode: d=2048 N=128 top-8 m=768 bf16, batch 64 tokens, skip ratio 0.5"),
+                   shape=f"ACE MoE layer decode: {QWEN}"),
     "prefill": dict(spec="qwen", zipf=True, T=4096, q=0.5, layers=1, tables="offline",
-                    name="ACE MoE layer prefill: d=2048 N=128 top-8 m=768 bf16, 4096 tokens Zipf(1.1) routing, "
-                         "skip ratio 0.5"),
+                    shape=f"ACE MoE layer prefill: {QWEN}, Zipf(1.1) routing"),
     "stack_prefill": dict(spec="qwen", zipf=False, T=16384, q=0.5, layers=4, tables="offline",
-                          name="4-layer stack of the d=2048 N=128 top-8 m=768 layer (residual), prefill 16384 tokens, "
-                               "skip ratio 0.5"),
+                          shape=f"4-layer stack of the {QWEN} layer (residual), prefill"),
     "stack_decode": dict(spec="qwen", zipf=False, T=32, q=0.5, layers=4, tables="offline",
-                         name="4-layer stack of the d=2048 N=128 top-8 m=768 layer (residual), decode 32 tokens, "
-                              "skip ratio 0.5"),
+                         shape=f"4-layer stack of the {QWEN} layer (residual), decode"),
     "large_prefill": dict(spec="large", zipf=True, T=8192, q=0.5, layers=1, tables="gpu",
-                          name="large MoE layer d=4096 N=256 top-8 m=2048 bf16, prefill 8192 tokens Zipf routing, "
-                               "skip ratio 0.5"),
+                          shape=f"large MoE layer {LARGE}, prefill, Zipf(1.1) routing"),
     "large_decode": dict(spec="large", zipf=True, T=128, q=0.5, layers=1, tables="gpu",
-                         name="large MoE layer d=4096 N=256 top-8 m=2048 bf16, decode 128 tokens, skip ratio 0.5"),
+                         shape=f"large MoE layer {LARGE}, decode, Zipf(1.1) routing"),
 }
+
+
+def wl_name(wl, T=None, q=None):
+    """A workload named by what it is, with its sizes."""
+    T = wl["T"] if T is None else T
+    q = wl["q"] if q is None else q
+    return f"{wl['shape']}, {T} tokens, skip ratio {q}"
+
+
+for _wl in WORKLOADS.values():
+    _wl["name"] = wl_name(_wl)
 METRIC = "ACE MoE-layer tokens/s (prefill, decode) + speedup vs skip=0; % of roofline"
 # The paper's own speedups (§4 efficiency, Tab. latency): whole-model TTFT and TPOT
 # with and without skipping, on an A100 in bf16 at a 60% skip ratio, five
@@ -139,18 +151,38 @@ def _peaks():
         return 6800.0, 1900.0, "fallback"
 
 
+def smi_gpu_id(props):
+    """The nvidia-smi --id of the GPU behind a CUDA device, from its device
+    properties (UUID, else PCI address), never from the CUDA ordinal: under
+    CUDA_VISIBLE_DEVICES the ordinal names another physical GPU in
+    nvidia-smi's numbering. None when the properties carry neither."""
+    u = getattr(props, "uuid", None)
+    if u is not None and str(u):
+        u = str(u)
+        return u if u.startswith(("GPU-", "MIG-")) else "GPU-" + u
+    bus = getattr(props, "pci_bus_id", None)
+    if bus is not None:
+        dom = getattr(props, "pci_domain_id", 0) or 0
+        dev = getattr(props, "pci_device_id", 0) or 0
+        return f"{int(dom):08X}:{int(bus):02X}:{int(dev):02X}.0"
+    return None
+
+
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 100 ms."""
+    """nvidia-smi clocks and throttle reasons of one GPU (named by UUID or PCI
+    address, see smi_gpu_id) sampled every 100 ms."""
 
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_id):
         self.proc = None
-        self.gpu = gpu_index
+        self.gpu = gpu_id
+        if gpu_id is None:
+            return
         try:
-            self.proc = subprocess.Popen(["nvidia-smi", f"--id={gpu_index}", f"--query-gpu={self.Q}",
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={gpu_id}", f"--query-gpu={self.Q}",
                                           "--format=csv,noheader,nounits", "-lms", "100"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except Exception:
@@ -183,7 +215,7 @@ class ClockSampler:
         if not sm:
             return None
         return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), "gpu": self.gpu}
 
 
 class Stack:
@@ -192,14 +224,14 @@ class Stack:
 
     fusion = "max"     # skip rule of every forward (ace_skip_ctl.fusion); "max" is ACE
 
-    def __init__(self, wl, max_tokens):
+    def __init__(self, wl, max_tokens, tables=None):
         from paper_2609_05228_gb300 import ace, offline, synth
         spec = synth.spec_qwen(zipf=wl["zipf"]) if wl["spec"] == "qwen" else synth.spec_large(zipf=wl["zipf"])
         self.ws, self.layers = [], []
         n = wl["layers"]
         for l in range(n):
             w = synth.make_layer(spec, seed=0 if n == 1 else 100 + l)
-            if wl["tables"] == "offline":     # host library (fp64)
+            if (tables or wl["tables"]) == "offline":     # host library (fp64)
                 w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables(w)
             else:                             # the GPU tables (ace_offline_tables_device)
                 w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables_device(w)
@@ -383,7 +415,7 @@ def run_ours(args, rank, world, torch, dist):
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize()
-        clocks = ClockSampler(dev.index)
+        clocks = ClockSampler(smi_gpu_id(torch.cuda.get_device_properties(dev)))
         t_wall = time.perf_counter()
         ms = time_point(torch, model, x, bufs, T, q, args.steps, args.warmup, flush)
         torch.cuda.synchronize()
@@ -396,6 +428,8 @@ def run_ours(args, rank, world, torch, dist):
             dist.all_reduce(flag, op=dist.ReduceOp.MAX)
             bad = bool(flag.item())
             dist.barrier()
+        # the reported attempt's own verdict (any rank's), null when clean
+        clock_rejected = (why or "another rank's clocks") if bad else None
         if not bad or attempt == 1:
             break
         retry = {"first_clocks": clk, "reason": why or "another rank's clocks"}
@@ -517,14 +551,102 @@ def run_ours(args, rank, world, torch, dist):
         "gpu_launches": args.steps * launches,
         "clocks": clk,
         "clock_retry": retry,
+        "clock_rejected": clock_rejected,
         "offline_tables": time_tables(torch, w) if rank == 0 else None,
     }
     if rank == 0 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(model.ws, wl, budget_s=args.cpu_seconds, fusion=args.fusion)
+    if rank == 0 and not args.no_points:
+        result["points"] = measure_points(torch, args, {"large_decode": model} if args.workload == "large_prefill"
+                                          else None)
     if rank == 0 and args.sweep:
         result["sweep"] = sweep(torch, args)
     model.close()
     return result
+
+
+# Per-point records of the default run: the other batch sizes and workloads
+# (tokens/s, retained slots R, distinct retained experts D, fractions of the
+# binding roofline, speedup over the same kernels at skip ratio 0).
+POINTS = [("decode", 1), ("decode", 8), ("decode", 64), ("prefill", 4096), ("stack_prefill", 16384),
+          ("large_decode", 128)]
+
+
+def layer_roofline(spec, T, R, D, n_layers=1):
+    """Algorithmic bytes and FLOPs of a forward (retained work only), summed
+    over layers: B = 6 d m D + 2 d N + 4 d T per layer (bf16 weights of the
+    distinct retained experts, the router, tokens in and out), F = 6 d m R +
+    2 d N T. R and D are lists (one entry per layer)."""
+    d, m, N = spec.hidden, spec.ffn, spec.n_experts
+    B = sum(6 * d * m * Dl + 2 * d * N + 4 * d * T for Dl in D)
+    F = sum(6 * d * m * Rl + 2 * d * N * T for Rl in R)
+    return B, F
+
+
+def roofline_point(spec, T, R, D, ms, hbm_gbs, tensor_tflops):
+    """Fractions of the HBM and tensor rooflines for one step of `ms` ms, and
+    of t* = max(B / BW, F / P), the binding one."""
+    B, F = layer_roofline(spec, T, R, D)
+    t_hbm = B / (hbm_gbs * 1e9)
+    t_tc = F / (tensor_tflops * 1e12)
+    t = ms * 1e-3
+    tstar = max(t_hbm, t_tc)
+    return {"bytes": B, "flops": F, "bound": "hbm" if t_hbm >= t_tc else "tensor",
+            "tstar_us": round(tstar * 1e6, 2), "frac_of_tstar": round(tstar / t, 4),
+            "hbm_frac": round(t_hbm / t, 4), "tensor_frac": round(t_tc / t, 4)}
+
+
+def decision_stats(model, T):
+    """Retained slots and distinct retained experts of each layer's last forward."""
+    from paper_2609_05228_gb300 import ace
+    spec = model.spec
+    R, D = [], []
+    for layer in model.layers:
+        _, _, _, _, r = ace.ace_last_skip_mask(layer.handle, T, spec.top_k)
+        off, _ = ace.ace_last_permutation(layer.handle, spec.n_experts, r)
+        R.append(int(r))
+        D.append(int((np.diff(off) > 0).sum()))
+    return R, D
+
+
+def measure_points(torch, args, models=None):
+    """The POINTS at skip ratio 0.5 and 0, each timed as in the main line
+    (graph replay, L2 flushed between steps, median of the replays). Layers are
+    built per workload and freed after it (the GPU tables, as the large layer
+    uses); `models` maps a workload to a Stack that is already built."""
+    from paper_2609_05228_gb300 import synth
+    hbm, _, _ = _peaks()
+    sust = _peak_sustained()
+    flush = L2Flush(torch, "cuda")
+    groups = {}
+    for wl, T in POINTS:
+        groups.setdefault(wl, []).append(T)
+    out = []
+    for wl, Ts in groups.items():
+        own = not (models and wl in models)
+        model = Stack(WORKLOADS[wl], max_tokens=max(Ts), tables="gpu") if own else models[wl]
+        model.fusion = args.fusion
+        q = WORKLOADS[wl]["q"]
+        for T in Ts:
+            xh = synth.make_tokens(model.spec, T, seed=1)
+            x = torch.from_numpy(xh.view(np.int16)).view(torch.bfloat16).cuda()
+            bufs = model.buffers(torch, x)
+            ms = float(np.median(time_point(torch, model, x, bufs, T, q, 30, 3, flush)))
+            model.forward(x, bufs, T, q)
+            R, D = decision_stats(model, T)
+            ms0 = float(np.median(time_point(torch, model, x, bufs, T, 0.0, 15, 3, flush)))
+            rec = {"workload": wl_name(WORKLOADS[wl], T), "tokens": T, "layers": len(model.layers), "skip_ratio": q,
+                   "tokens_per_s": round(T / (ms * 1e-3), 1), "us_per_step": round(ms * 1e3, 2),
+                   "retained_slots": R, "distinct_experts": D,
+                   "speedup_vs_q0": round(ms0 / ms, 4), "q0_us_per_step": round(ms0 * 1e3, 2)}
+            rec.update(roofline_point(model.spec, T, R, D, ms, hbm, sust))
+            out.append(rec)
+            del x, bufs
+        if own:
+            model.close()
+            del model
+            torch.cuda.empty_cache()
+    return out
 
 
 def sweep(torch, args):
@@ -616,16 +738,17 @@ def cpu_baseline(ws, wl, budget_s=12.0, fusion="max"):
 def run_reference(args):
     """The reference arm: the CPU oracle on a bounded sample, per step."""
     import oracle as O
-    from paper_2609_05228_gb300 import offline, synth
+    from oracle import seeded_tables
+    from paper_2609_05228_gb300 import synth
     wl = WORKLOADS[args.workload]
     spec = synth.spec_qwen(zipf=wl["zipf"]) if wl["spec"] == "qwen" else synth.spec_large(zipf=wl["zipf"])
     ws = []
     for l in range(wl["layers"]):
-        w = synth.make_layer(spec, seed=0 if wl["layers"] == 1 else 100 + l)
-        if wl["tables"] == "offline":
-            w.extra["a_gsp"], w.extra["a_rcr"] = offline.tables(w)
-        else:   # the arm stays on the host: seeded positive tables stand in for the GPU tables
-            w.extra["a_gsp"], w.extra["a_rcr"] = synth.make_tables(spec.n_experts, seed=5, spread=0.1)
+        seed = 0 if wl["layers"] == 1 else 100 + l
+        w = synth.make_layer(spec, seed=seed)
+        # the oracle's own tables (Algorithms 2 and 3): stored by oracle/seeded_tables.py, else computed here
+        tabs = seeded_tables.load(spec, seed)
+        w.extra["a_gsp"], w.extra["a_rcr"] = tabs if tabs is not None else seeded_tables.compute(w)
         ws.append(w)
     xall = synth.make_tokens(spec, min(wl["T"], 256), seed=1)
 
@@ -668,7 +791,9 @@ def main():
     ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="decode", choices=sorted(WORKLOADS))
+    ap.add_argument("--workload", default="large_prefill", choices=sorted(WORKLOADS))
+    ap.add_argument("--no-points", action="store_true",
+                    help="skip the per-point records (other batch sizes and workloads) of the default run")
     ap.add_argument("--sweep", action="store_true", help="add decode/prefill sweep points")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--fusion", default="max", choices=["max", "min", "mean", "gsp", "rcr", "score"],

@@ -59,8 +59,8 @@ def test_algorithmic_bytes_of_the_decode_layer():
 def test_reference_arm_json_line():
     """`bench.py --impl reference` prints one JSON line with the contract's
     keys, timing the oracle on the host (tokens per step sized to the steps)."""
-    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "2",
-                        "--warmup", "1"], capture_output=True, text=True, cwd=ROOT, timeout=900)
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload", "decode",
+                        "--steps", "2", "--warmup", "1"], capture_output=True, text=True, cwd=ROOT, timeout=900)
     assert r.returncode == 0, r.stderr[-2000:]
     lines = [l for l in r.stdout.splitlines() if l.strip()]
     assert len(lines) == 1
@@ -70,3 +70,39 @@ def test_reference_arm_json_line():
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
     assert d["e2e"] == {"value": d["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
     assert 1 <= d["config"]["tokens_per_step"] <= 64
+    assert "libace" not in r.stderr
+
+
+def test_smi_gpu_id_names_the_device_not_the_ordinal():
+    """nvidia-smi is pointed at the GPU by UUID (else PCI address) from the
+    device's properties; the CUDA ordinal is never used."""
+    class P:
+        uuid = "1a2b3c4d-0000-1111-2222-333344445555"
+        pci_bus_id, pci_domain_id, pci_device_id = 0x41, 0, 0
+    assert bench.smi_gpu_id(P()) == "GPU-1a2b3c4d-0000-1111-2222-333344445555"
+
+    class Q:
+        pci_bus_id, pci_domain_id, pci_device_id = 0x41, 2, 0
+    assert bench.smi_gpu_id(Q()) == "00000002:41:00.0"
+    assert bench.smi_gpu_id(object()) is None
+    assert bench.ClockSampler(None).stop() is None        # unknown GPU: no samples rather than another GPU's
+
+
+def test_reference_arm_reads_oracle_tables_only():
+    """The reference arm's tables are the oracle's (Algorithms 2 and 3), stored
+    by oracle/seeded_tables.py for every benchmark layer: check one stored
+    entry against a fresh oracle computation on a subset of experts."""
+    import oracle as O
+    from oracle import seeded_tables
+    spec = synth.spec_qwen()
+    for seed in (0, 100, 101, 102, 103):
+        assert seeded_tables.load(spec, seed) is not None, seed
+    assert seeded_tables.load(synth.spec_large(), 0) is not None
+    a, r = seeded_tables.load(spec, 0)
+    w = synth.make_layer(spec, seed=0)
+    # the normalisation is one constant per table, so ratios of entries are those of the raw scores
+    idx = [0, 5, 77]
+    sub = O.gsp_table(w.gamma, w.w_gate[idx], w.w_up[idx], w.w_down[idx], 0.0)
+    np.testing.assert_allclose(a[idx] / a[idx[0]], sub / sub[0], rtol=1e-6)
+    r_full = O.rcr_table(w.router_w, w.gamma, w.w_gate, w.w_up, w.w_down, spec.eps)
+    np.testing.assert_allclose(r, r_full.astype(np.float32), rtol=1e-6)
