@@ -279,11 +279,15 @@ ace_status ace_last_launch_count(const ace_layer* layer, int* n_kernels);
  * The results are bit-identical to ace_route_logits on the same inputs.
  * The first call on a device (with that device current) looks up the array's
  * device address; make that first call before any stream capture. All calls
- * share the one array and it keeps the last call's contents (the kernel's
- * counters are cleared at the start of every call): calls that overlap on
- * the GPU, on different streams or devices sharing the library state per
- * device, race. Asynchronous on `stream`; errors found by the kernel (NaN
- * logits) are not reported by this entry point.
+ * on a device share that device's one array, and it keeps the last call's
+ * contents (the kernel's counters are cleared at the start of every call):
+ * calls on one device that overlap on the GPU (on different streams, or from
+ * different host threads) race. Calls on different devices use different
+ * copies of the array and do not. The decision kernel's shared-memory limit
+ * is only ever raised, by this call and by ace_layer_create alike, so a
+ * layer created on another host thread cannot make this launch fail.
+ * Asynchronous on `stream`; errors found by the kernel (NaN logits) are not
+ * reported by this entry point.
  */
 ace_status ace_route_decide_noalloc(const float* logits, int T, int n_experts, int top_k,
                                     const float* a_gsp, const float* a_rcr, float eps, int min_active,

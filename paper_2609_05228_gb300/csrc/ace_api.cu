@@ -4,6 +4,8 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <map>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -55,13 +57,23 @@ void free_layer(ace_layer* L) {
 
 // Device-accessible address of page-locked host memory (nullptr if `p` is
 // not page-locked and mapped).
-void* mapped_host(const void* p) {
+void* mapped_host_byte(const void* p) {
     cudaPointerAttributes a{};
     if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
         cudaGetLastError();
         return nullptr;
     }
     return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
+}
+
+// Device address of a page-locked host buffer of `bytes` bytes, or NULL when
+// it is pageable or not mapped as one range (its last byte must map to the
+// same offset as its first).
+void* mapped_host(const void* p, size_t bytes = 1) {
+    void* m = mapped_host_byte(p);
+    if (!m || bytes <= 1) return m;
+    void* e = mapped_host_byte(static_cast<const char*>(p) + bytes - 1);
+    return e == static_cast<char*>(m) + bytes - 1 ? m : nullptr;
 }
 
 // Host <-> device copies for the host-buffer calls. Transfers of a few MB are
@@ -105,8 +117,11 @@ ace_status copy_async(void* dst, const void* src, void* dst_mapped, const void* 
 // and copies of the device error words `errs` into g.err_host, through a
 // CUDA graph captured on the first call and replayed while the stream, the
 // host buffers, T, the skip control and the profiling switch stay the same;
-// then synchronises. Pageable host buffers cannot be captured and are
-// enqueued directly. Calls on the legacy default stream use a blocking
+// then synchronises. The host buffers are looked up on every call: the graph
+// is replayed only while both are still page-locked and mapped at the device
+// addresses it was captured with (a buffer freed and its address reused, or
+// registered again, is captured anew). Pageable host buffers cannot be
+// captured and are enqueued directly. Calls on the legacy default stream use a blocking
 // stream owned by g (ordered with the default stream).
 template <typename Body>
 ace_status run_host_graph(AceHostGraph& g, cudaStream_t user, const void* xh, void* oh, void* dev_in,
@@ -131,17 +146,17 @@ ace_status run_host_graph(AceHostGraph& g, cudaStream_t user, const void* xh, vo
         ACE_CUDA(cudaMallocHost(&g.err_host, n_err * sizeof(int)), "allocate pinned error words");
         g.n_err = n_err;
     }
-    const bool same = g.exec && g.stream == s && g.x_host == xh && g.out_host == oh && g.T == T &&
-                      g.ctl.mode == ctl.mode && g.ctl.value == ctl.value && g.ctl.fusion == ctl.fusion &&
-                      g.profiling == profiling;
+    const void* xh_m = mapped_host(xh, bytes);
+    void* oh_m = mapped_host(oh, bytes);
+    const bool same = g.exec && xh_m && oh_m && g.stream == s && g.x_host == xh && g.out_host == oh &&
+                      g.x_mapped == xh_m && g.out_mapped == oh_m && g.T == T && g.ctl.mode == ctl.mode &&
+                      g.ctl.value == ctl.value && g.ctl.fusion == ctl.fusion && g.profiling == profiling;
     if (!same) {
         if (g.exec) {
             cudaGraphExecDestroy(g.exec);
             g.exec = nullptr;
         }
-        const void* xh_m = mapped_host(xh);
-        void* oh_m = mapped_host(oh);
-        void* err_m = mapped_host(g.err_host);
+        void* err_m = mapped_host(g.err_host, n_err * sizeof(int));
         auto enqueue = [&](cudaStream_t st) -> ace_status {
             ace_status r = copy_async(dev_in, xh, nullptr, xh_m, bytes, cudaMemcpyHostToDevice, num_sms, st);
             if (r != ACE_OK) return r;
@@ -186,6 +201,8 @@ ace_status run_host_graph(AceHostGraph& g, cudaStream_t user, const void* xh, vo
         g.stream = s;
         g.x_host = xh;
         g.out_host = oh;
+        g.x_mapped = xh_m;
+        g.out_mapped = oh_m;
         g.T = T;
         g.ctl = ctl;
         g.profiling = profiling;
@@ -235,6 +252,20 @@ ace_status check_ctl(ace_skip_ctl ctl) {
 
 namespace ace {
 void set_last_error(const char* msg) { g_last_error = msg; }
+
+cudaError_t raise_smem_limit(const void* kernel, int bytes) {
+    static std::mutex mu;
+    static std::map<std::pair<int, const void*>, int> limits;   // (device, kernel) -> limit set
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    int& cur = limits[{dev, kernel}];
+    if (bytes <= cur) return cudaSuccess;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) cur = bytes;
+    return e;
+}
 }  // namespace ace
 
 extern "C" {

@@ -262,17 +262,13 @@ cudaError_t gemv_init(const ace_layer* L) {
     const int d = L->desc.hidden, m = L->desc.ffn;
     cudaError_t e;
     if (L->desc.dtype == ACE_BF16) {
-        e = cudaFuncSetAttribute(k_gemv_gateup<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)(kTC * d * sizeof(__nv_bfloat16)));
+        e = raise_smem_limit(k_gemv_gateup<__nv_bfloat16>, (int)(kTC * d * sizeof(__nv_bfloat16)));
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(k_gemv_down<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)(kTC * m * sizeof(float)));
+        e = raise_smem_limit(k_gemv_down<__nv_bfloat16>, (int)(kTC * m * sizeof(float)));
     } else {
-        e = cudaFuncSetAttribute(k_gemv_gateup<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)(kTC * d * sizeof(float)));
+        e = raise_smem_limit(k_gemv_gateup<float>, (int)(kTC * d * sizeof(float)));
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(k_gemv_down<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)(kTC * m * sizeof(float)));
+        e = raise_smem_limit(k_gemv_down<float>, (int)(kTC * m * sizeof(float)));
     }
     return e;
 }

@@ -96,6 +96,8 @@ struct AceHostGraph {
     cudaStream_t stream = nullptr;       // the stream the graph was captured for
     const void* x_host = nullptr;
     void* out_host = nullptr;
+    const void* x_mapped = nullptr;      // device addresses of the page-locked host buffers at capture
+    void* out_mapped = nullptr;
     int T = -1;
     ace_skip_ctl ctl{0, 0.f, 0};
     bool profiling = false;
@@ -212,6 +214,17 @@ inline cudaError_t record_stage(cudaEvent_t ev, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     return st == cudaStreamCaptureStatusActive ? cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal)
                                                : cudaEventRecord(ev, s);
+}
+
+// Raise a kernel's dynamic shared-memory limit on the current device to at
+// least `bytes`, never lowering it: layers of different shapes (and the
+// no-allocation entry point) share the kernels, so a limit set for one must
+// not drop below what another, created or launched earlier or on another
+// host thread, still needs. Serialised by a process-wide mutex.
+cudaError_t raise_smem_limit(const void* kernel, int bytes);
+template <typename K>
+inline cudaError_t raise_smem_limit(K* kernel, int bytes) {
+    return raise_smem_limit(reinterpret_cast<const void*>(kernel), bytes);
 }
 
 // Prefer the largest shared-memory carveout (all kernels share one L1/shared split).

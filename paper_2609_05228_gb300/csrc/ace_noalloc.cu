@@ -105,7 +105,7 @@ extern "C" ace_status ace_route_decide_noalloc(const float* logits, int T, int n
     sc.tile_cnt = sc.meta + ace::kMetaCount;
     sc.err = sc.tile_cnt + kNaMaxTokens / 8 + 1;
     // shared-memory limit of the decision kernel for the largest accepted shape
-    // (set on every call: creating a layer may lower it for its own shape)
+    // (only ever raised; a no-op after the first call on the device)
     e = ace::route_decide_attr((int)ace::route_decide_smem(kNaMaxTokens, kNaMaxSlots / kNaMaxTokens, kNaMaxExperts));
     if (e != cudaSuccess) return na_fail(ACE_ERR_CUDA, std::string("kernel attribute: ") + cudaGetErrorString(e));
     cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -1321,9 +1321,9 @@ cudaError_t router_launch(const ace_layer* L, const void* src, int T_, cudaStrea
 
 template <typename T>
 cudaError_t set_router_attrs(size_t smem) {
-    cudaError_t e = cudaFuncSetAttribute(k_router<T, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = raise_smem_limit(k_router<T, true>, (int)smem);
     if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(k_router<T, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    return raise_smem_limit(k_router<T, false>, (int)smem);
 }
 
 int select_mq(const ace_layer* L, int T, ace_skip_ctl ctl, float* tau, bool* need_select) {
@@ -1364,7 +1364,7 @@ cudaError_t fused_dispatch(const ace_layer* L, const FusedArgs& a, int n_tok, cu
 
 template <typename T, int NPL, bool LOGITS>
 cudaError_t fused_attr(int smem) {
-    return cudaFuncSetAttribute(k_route_fused<T, NPL, LOGITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    return raise_smem_limit(k_route_fused<T, NPL, LOGITS>, smem);
 }
 
 template <typename T>
@@ -1549,14 +1549,9 @@ size_t route_decide_smem(int T, int k, int n_exp) { return fused_phase_c_bytes(T
 
 cudaError_t route_decide_attr(int smem_bytes) {
     cudaError_t e;
-    if ((e = cudaFuncSetAttribute(k_route_fused<__nv_bfloat16, 4, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  smem_bytes)) != cudaSuccess)
-        return e;
-    if ((e = cudaFuncSetAttribute(k_route_fused<__nv_bfloat16, 8, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  smem_bytes)) != cudaSuccess)
-        return e;
-    return cudaFuncSetAttribute(k_route_fused<__nv_bfloat16, 32, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                smem_bytes);
+    if ((e = raise_smem_limit(k_route_fused<__nv_bfloat16, 4, false>, smem_bytes)) != cudaSuccess) return e;
+    if ((e = raise_smem_limit(k_route_fused<__nv_bfloat16, 8, false>, smem_bytes)) != cudaSuccess) return e;
+    return raise_smem_limit(k_route_fused<__nv_bfloat16, 32, false>, smem_bytes);
 }
 
 cudaError_t launch_route_decide_scratch(const float* logits, int T, int n_exp, int k, const float* a_gsp,

@@ -549,8 +549,8 @@ extern "C" ace_status ace_offline_tables_device(int d, int N, int m, const void*
         }                                                                                                 \
     } while (0)
     TAB_CK(cudaFuncSetAttribute(k_gsp_frob, cudaFuncAttributeMaxDynamicSharedMemorySize, kTabSmem));
-    TAB_CK(cudaFuncSetAttribute(k_rcr_gateup, cudaFuncAttributeMaxDynamicSharedMemorySize, d * 4));
-    TAB_CK(cudaFuncSetAttribute(k_rcr_down, cudaFuncAttributeMaxDynamicSharedMemorySize, m * 4));
+    TAB_CK(ace::raise_smem_limit(k_rcr_gateup, d * 4));
+    TAB_CK(ace::raise_smem_limit(k_rcr_down, m * 4));
     TAB_CK(cudaMemsetAsync(err, 0, 4, s));
     k_gamma2<<<(d + 255) / 256, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(gamma), g2, d);
     TAB_CK(cudaGetLastError());
