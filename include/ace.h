@@ -235,6 +235,20 @@ ace_status ace_layer_sync(ace_layer* layer);
 ace_status ace_debug_exp32(const float* x, float* y, int n, void* stream);
 
 /*
+ * ace_debug_set_wait_budget — test hook for the bounded device waits (the
+ * paper has no counterpart). With cycles > 0, the decode expert kernel
+ * (batches of at most 256 tokens on the tensor-core path) waits for a token
+ * tile's gate/up results with a target that is never reached and gives up
+ * after `cycles` SM clock cycles: it sets the layer's error word, lets the
+ * copies it has issued land, frees its tensor memory and returns, and the
+ * next synchronising call reports ACE_ERR_TIMEOUT. The kernel's other waits
+ * keep their normal bound (about 2 s), so such a forward takes a few seconds
+ * and its output is not valid. cycles = 0 restores normal operation. Only
+ * forwards launched (or graphs captured) while it is set are affected.
+ */
+ace_status ace_debug_set_wait_budget(ace_layer* layer, long long cycles);
+
+/*
  * Stage timing (instrumentation; the paper has no counterpart). When enabled,
  * each ace_moe_forward records CUDA events on its stream around its stages:
  *   0 RMSNorm (T > 256), 1 router logits (T <= 256: the whole fused

@@ -67,6 +67,7 @@ def lib() -> ctypes.CDLL:
             "ace_last_permutation": (_S, [_P, _P, _P]),
             "ace_layer_sync": (_S, [_P]),
             "ace_debug_exp32": (_S, [_P, _P, _I, _P]),
+            "ace_debug_set_wait_budget": (_S, [_P, ctypes.c_longlong]),
             "ace_layer_get_desc": (_S, [_P, ctypes.POINTER(ace_layer_desc)]),
             "ace_layer_set_profiling": (_S, [_P, _I]),
             "ace_last_stage_times": (_S, [_P, _P, _I, _P]),
@@ -208,6 +209,10 @@ def ace_last_permutation(layer: int, N: int, R: int):
 
 def ace_layer_sync(layer: int) -> None:
     _check(lib().ace_layer_sync(layer))
+
+
+def ace_debug_set_wait_budget(layer: int, cycles: int) -> None:
+    _check(lib().ace_debug_set_wait_budget(layer, int(cycles)))
 
 
 def ace_debug_exp32(x, y, n: int, stream=None) -> None:

@@ -720,6 +720,13 @@ ace_status ace_last_launch_count(const ace_layer* L, int* n_kernels) {
     return ACE_OK;
 }
 
+ace_status ace_debug_set_wait_budget(ace_layer* L, long long cycles) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    if (cycles < 0) return fail(ACE_ERR_INVALID_ARG, "cycles must be >= 0");
+    L->dbg_ready_spin = cycles;
+    return ACE_OK;
+}
+
 ace_status ace_debug_exp32(const float* x, float* y, int n, void* stream) {
     if (n < 0 || (n > 0 && (!x || !y))) return fail(ACE_ERR_INVALID_ARG, "bad arguments");
     if (n == 0) return ACE_OK;

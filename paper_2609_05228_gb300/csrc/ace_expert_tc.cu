@@ -548,6 +548,8 @@ struct DecParams {
     int* done;                          // [token tiles] gate/up epilogue warps finished (zeroed by the gather)
     int* err;
     int d, m, k;
+    long long ready_spin;               // bound (SM clock cycles) on the wait for a token tile's act rows
+    int ready_extra;                    // added to that wait's target: 0, or unreachable (a test of the bound)
 };
 
 constexpr int kDecStages = 8;
@@ -633,7 +635,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
     const int ntt = p.meta[kMetaTokTiles];
     const int wt1 = 2 * p.m / 128;
     const int n1 = ntt * wt1, n_tiles = n1 + ntt * (p.d / 128);
-    const int done_target = 4 * wt1;
+    const int done_target = 4 * wt1 + p.ready_extra;
 
     if (warp == 0) {
         // ------------------------------------------------ producer
@@ -649,7 +651,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
                     if (ld_acquire(p.done + t.tt) < done_target) {
                         const long long t0 = clock64();
                         while (ld_acquire(p.done + t.tt) < done_target) {
-                            if (clock64() - t0 > kSpinCycles || *abort_flag) {
+                            if (clock64() - t0 > p.ready_spin || *abort_flag) {
                                 atomicOr(p.err, kErrTimeout);
                                 ok = false;
                                 break;
@@ -1365,6 +1367,8 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
         q.d = d;
         q.m = m;
         q.k = k;
+        q.ready_spin = L->dbg_ready_spin > 0 ? L->dbg_ready_spin : kSpinCycles;
+        q.ready_extra = L->dbg_ready_spin > 0 ? (1 << 30) : 0;
         e = launch_pdl(k_expert_decode, dim3(L->num_sms), dim3(kThreads), kDecSmem, s, q);
         if (e != cudaSuccess) return e;
         if (ev) {                           // gate/up and down share one launch: the down stage reads 0

@@ -144,6 +144,7 @@ struct ace_layer {
     int n_stages = 0;
     int last_launches = 0;       // kernels launched by the last forward / route call
     AceHostGraph hg;             // ace_moe_forward_host
+    long long dbg_ready_spin = 0;  // ace_debug_set_wait_budget: 0 = off
 };
 
 namespace ace {
