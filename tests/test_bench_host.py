@@ -3,6 +3,7 @@ line (the oracle on a bounded sample), the ncu traffic record guard, and the
 algorithmic byte counts of the roofline."""
 import json
 import os
+import re
 import shutil
 import subprocess
 import sys
@@ -16,20 +17,37 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 def test_recorded_traffic_follows_the_kernel_sources(tmp_path, monkeypatch):
-    rec = os.path.join("profiles", "decode_T64_q0.5_expert_decode_full.md")
-    value = bench._recorded_traffic(rec)
-    assert isinstance(value, int) and 1.0e9 < value < 1.1e9
-    # a record whose source hash no longer matches reads as "no traffic figure"
-    text = open(os.path.join(ROOT, rec)).read().replace("source_sha256=", "source_sha256=0")
-    bad = tmp_path / "bad.md"
-    bad.write_text(text)
-    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    """A record gives its DRAM bytes only while the hash of its listed sources
+    matches; a stale hash, a missing file or a missing source gives None."""
+    import hashlib
+    srcs = ("ace_expert_tc.cu", "ace_tc.cuh", "ace_device.cuh")
     os.makedirs(tmp_path / "paper_2609_05228_gb300" / "csrc", exist_ok=True)
-    for src in ("ace_expert_tc.cu", "ace_tc.cuh", "ace_device.cuh"):
-        shutil.copy(os.path.join(ROOT, "paper_2609_05228_gb300", "csrc", src),
-                    tmp_path / "paper_2609_05228_gb300" / "csrc" / src)
+    h = hashlib.sha256()
+    for src in srcs:
+        path = os.path.join(ROOT, "paper_2609_05228_gb300", "csrc", src)
+        shutil.copy(path, tmp_path / "paper_2609_05228_gb300" / "csrc" / src)
+        h.update(open(path, "rb").read())
+    listed = ",".join("paper_2609_05228_gb300/csrc/" + s for s in srcs)
+    record = ("Machine-read record:\n\n"
+              "    kernel=k_expert_decode\n"
+              f"    source={listed}\n"
+              f"    source_sha256={h.hexdigest()}\n"
+              "    dram_bytes_per_launch=1044777984\n")
+    (tmp_path / "good.md").write_text(record)
+    (tmp_path / "bad.md").write_text(record.replace("source_sha256=", "source_sha256=0"))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench._recorded_traffic("good.md") == 1044777984
     assert bench._recorded_traffic("bad.md") is None
     assert bench._recorded_traffic("missing.md") is None
+    os.remove(tmp_path / "paper_2609_05228_gb300" / "csrc" / "ace_tc.cuh")
+    assert bench._recorded_traffic("good.md") is None
+    # every committed record names the files it hashes, and those files exist
+    monkeypatch.setattr(bench, "ROOT", ROOT)
+    for rec in bench.TRAFFIC_RECORDS.values():
+        text = open(os.path.join(ROOT, rec)).read()
+        listed = re.search(r"source=(\S+)", text).group(1).split(",")
+        assert all(os.path.exists(os.path.join(ROOT, s)) for s in listed)
+        assert re.search(r"dram_bytes_per_launch=\d+", text)
 
 
 def test_clock_records_that_disqualify_a_timed_region():
