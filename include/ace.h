@@ -249,6 +249,29 @@ ace_status ace_debug_exp32(const float* x, float* y, int n, void* stream);
 ace_status ace_debug_set_wait_budget(ace_layer* layer, long long cycles);
 
 /*
+ * Debug build (the paper has no counterpart). libace_debug.so is the same
+ * library compiled with ACE_DEBUG_CHECKS:
+ *   - the routing, compaction, gather and combine kernels check every index
+ *     they compute (expert ids, permutation rows, tile-table entries, slot
+ *     rows) before using it; a failed check sets the layer's error word and
+ *     the access is skipped, and the next synchronising call (ace_layer_sync,
+ *     ace_last_*) returns ACE_ERR_CUDA;
+ *   - every device array of a layer is allocated with 256 extra bytes of a
+ *     known pattern (canary words), which the synchronising calls compare;
+ *     a difference returns ACE_ERR_CUDA naming the array.
+ * It is a stand-in for a memory checker on the hand-indexed kernels; the
+ * release library compiles the checks away.
+ *
+ * ace_debug_checks_enabled returns 1 for the debug build, else 0.
+ * ace_debug_poke_canary (test hook) overwrites one byte of the canary words
+ * of the layer's array number `index` (allocation order), as a kernel that
+ * wrote past that array would; ACE_ERR_UNSUPPORTED in the release build,
+ * ACE_ERR_INVALID_ARG for an index out of range. It synchronises the device.
+ */
+int ace_debug_checks_enabled(void);
+ace_status ace_debug_poke_canary(ace_layer* layer, int index);
+
+/*
  * Stage timing (instrumentation; the paper has no counterpart). When enabled,
  * each ace_moe_forward records CUDA events on its stream around its stages:
  *   0 RMSNorm (T > 256), 1 router logits (T <= 256: the whole fused

@@ -13,7 +13,10 @@ import os
 
 import numpy as np
 
-LIBPATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libace.so")
+_LIBDIR = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib")
+# ACE_LIB_VARIANT=debug loads libace_debug.so (index guards and canary words)
+LIBNAME = "libace_debug.so" if os.environ.get("ACE_LIB_VARIANT") == "debug" else "libace.so"
+LIBPATH = os.path.join(_LIBDIR, LIBNAME)
 
 ACE_BF16, ACE_F32 = 0, 1
 ACE_SKIP_THRESHOLD, ACE_SKIP_RATIO = 0, 1
@@ -52,7 +55,7 @@ def lib() -> ctypes.CDLL:
     global _lib
     if _lib is None:
         if not os.path.exists(LIBPATH):
-            raise AceError(4, f"libace.so not found at {LIBPATH}; build it with "
+            raise AceError(4, f"{LIBNAME} not found at {LIBPATH}; build it with "
                               "`python -m paper_2609_05228_gb300.build`")
         L = ctypes.CDLL(LIBPATH)
         sig = {
@@ -68,6 +71,8 @@ def lib() -> ctypes.CDLL:
             "ace_layer_sync": (_S, [_P]),
             "ace_debug_exp32": (_S, [_P, _P, _I, _P]),
             "ace_debug_set_wait_budget": (_S, [_P, ctypes.c_longlong]),
+            "ace_debug_checks_enabled": (_I, []),
+            "ace_debug_poke_canary": (_S, [_P, _I]),
             "ace_layer_get_desc": (_S, [_P, ctypes.POINTER(ace_layer_desc)]),
             "ace_layer_set_profiling": (_S, [_P, _I]),
             "ace_last_stage_times": (_S, [_P, _P, _I, _P]),
@@ -213,6 +218,14 @@ def ace_layer_sync(layer: int) -> None:
 
 def ace_debug_set_wait_budget(layer: int, cycles: int) -> None:
     _check(lib().ace_debug_set_wait_budget(layer, int(cycles)))
+
+
+def ace_debug_checks_enabled() -> bool:
+    return bool(lib().ace_debug_checks_enabled())
+
+
+def ace_debug_poke_canary(layer: int, index: int) -> None:
+    _check(lib().ace_debug_poke_canary(layer, int(index)))
 
 
 def ace_debug_exp32(x, y, n: int, stream=None) -> None:

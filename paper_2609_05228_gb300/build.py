@@ -1,5 +1,6 @@
 """Builds libace.so in-tree (paper_2609_05228_gb300/_lib/) with nvcc for sm_103a,
-and libace_offline.so (the host-only offline table tool) with g++.
+its debug variant libace_debug.so (-DACE_DEBUG_CHECKS: index guards and
+canary words), and libace_offline.so (the host-only offline table tool) with g++.
 
 Each .cu file under csrc/ is compiled in parallel, then linked into one
 shared library (CUDA runtime linked statically). Run as
@@ -55,32 +56,46 @@ def build_offline() -> str:
     return OFFLINE_LIB
 
 
-def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
-    os.makedirs(OBJDIR, exist_ok=True)
-    cc = nvcc()
-    flags = NVCC_FLAGS + (extra_flags or [])
+DEBUG_LIBPATH = os.path.join(LIBDIR, "libace_debug.so")
+# the debug variant: index guards in the routing, compaction, gather and
+# combine kernels, canary words past every device array of a layer
+DEBUG_FLAGS = ["-DACE_DEBUG_CHECKS"]
 
-    def compile_one(src: str) -> str:
-        obj = os.path.join(OBJDIR, os.path.basename(src)[:-3] + ".o")
+
+def build(verbose: bool = False, extra_flags: list[str] | None = None, debug: bool = True) -> str:
+    """Compile every .cu file for both variants in parallel and link
+    libace.so (and libace_debug.so unless debug=False). Returns libace.so's path."""
+    cc = nvcc()
+    variants = [("release", NVCC_FLAGS + (extra_flags or []), LIBPATH)]
+    if debug:
+        variants.append(("debug", NVCC_FLAGS + DEBUG_FLAGS + (extra_flags or []), DEBUG_LIBPATH))
+    for name, _, _ in variants:
+        os.makedirs(os.path.join(OBJDIR, name), exist_ok=True)
+
+    def compile_one(job) -> str:
+        src, name, flags = job
+        obj = os.path.join(OBJDIR, name, os.path.basename(src)[:-3] + ".o")
         cmd = [cc, *ARCH, *flags, "-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
-            raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
+            raise RuntimeError(f"nvcc failed for {src} ({name}):\n{r.stdout}\n{r.stderr}")
         if verbose and (r.stdout or r.stderr):
             print(r.stdout + r.stderr, file=sys.stderr)
         return obj
 
     srcs = sources()
-    with ThreadPoolExecutor(max(1, min(len(srcs) + 1, os.cpu_count() or 1))) as ex:
+    jobs = [(src, name, flags) for name, flags, _ in variants for src in srcs]
+    with ThreadPoolExecutor(max(1, min(len(jobs) + 1, os.cpu_count() or 1))) as ex:
         host = ex.submit(build_offline)
-        objs = list(ex.map(compile_one, srcs))
+        objs = list(ex.map(compile_one, jobs))
         host.result()
-    tmp = LIBPATH + ".tmp"
-    cmd = [cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs]
-    r = subprocess.run(cmd, capture_output=True, text=True)
-    if r.returncode != 0:
-        raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIBPATH)
+    for i, (name, _, path) in enumerate(variants):
+        tmp = path + ".tmp"
+        cmd = [cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs[i * len(srcs):(i + 1) * len(srcs)]]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"link failed ({name}):\n{r.stdout}\n{r.stderr}")
+        os.replace(tmp, path)
     return LIBPATH
 
 

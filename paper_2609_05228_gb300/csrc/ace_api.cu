@@ -223,7 +223,20 @@ ace_status report_error_word(ace_layer* L, int err) {
         ACE_CUDA(cudaMemset(L->ws.err, 0, sizeof(int)), "clear device error word");
         if (err & ace::kErrTimeout) return fail(ACE_ERR_TIMEOUT, "a bounded device wait ran out");
         if (err & ace::kErrNumeric) return fail(ACE_ERR_NUMERIC, "non-finite router logits were seen");
-        if (err & ace::kErrBounds) return fail(ACE_ERR_CUDA, "a device index check failed");
+        if (err & ace::kErrBounds) return fail(ACE_ERR_CUDA, "a device index check failed (debug build)");
+    }
+    return ACE_OK;
+}
+
+// Debug build: the canary words past every array of the layer (a kernel
+// that wrote past an array's end shows here; the first one found is named).
+ace_status check_canaries(ace_layer* L) {
+    unsigned char buf[ace::kCanaryBytes];
+    for (const ace::Canary& c : L->canaries) {
+        ACE_CUDA(cudaMemcpy(buf, c.at, sizeof(buf), cudaMemcpyDeviceToHost), "read canary");
+        for (size_t i = 0; i < sizeof(buf); ++i)
+            if (buf[i] != ace::kCanaryByte)
+                return fail(ACE_ERR_CUDA, std::string("device memory past the end of ") + c.name + " was overwritten");
     }
     return ACE_OK;
 }
@@ -231,7 +244,9 @@ ace_status report_error_word(ace_layer* L, int err) {
 ace_status check_device_word(ace_layer* L) {
     int err = 0;
     ACE_CUDA(cudaMemcpy(&err, L->ws.err, sizeof(int), cudaMemcpyDeviceToHost), "read device error word");
-    return report_error_word(L, err);
+    ace_status st = report_error_word(L, err);
+    if (st != ACE_OK) return st;
+    return check_canaries(L);
 }
 
 ace_status check_ctl(ace_skip_ctl ctl) {
@@ -334,14 +349,35 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     const int n_chunks = (int)((T + ace::kChunk - 1) / ace::kChunk);
     ace::Workspace& W = L->ws;
     cudaError_t e = cudaSuccess;
+#ifdef ACE_DEBUG_CHECKS
+    // canary words past the end of every array (checked by the synchronising calls)
+#define ACE_CANARY(ptr, bytes)                                                                    \
+    do {                                                                                          \
+        const size_t nb_ = (bytes) < 16 ? 16 : (bytes);                                          \
+        unsigned char* at_ = reinterpret_cast<unsigned char*>(ptr) + nb_;                         \
+        e = cudaMemset(at_, ace::kCanaryByte, ace::kCanaryBytes);                                \
+        if (e != cudaSuccess) {                                                                   \
+            free_layer(L);                                                                        \
+            return cuda_fail(e, "canary fill");                                                   \
+        }                                                                                         \
+        L->canaries.push_back(ace::Canary{#ptr, at_});                                            \
+    } while (0)
+    constexpr size_t kPad = ace::kCanaryBytes;
+#else
+#define ACE_CANARY(ptr, bytes) \
+    do {                       \
+    } while (0)
+    constexpr size_t kPad = 0;
+#endif
 #define ALLOC(ptr, bytes)                                                   \
     do {                                                                    \
-        e = dalloc(&(ptr), (bytes));                                        \
+        e = dalloc(&(ptr), ((bytes) < 16 ? 16 : (bytes)) + kPad);           \
         if (e != cudaSuccess) {                                             \
             free_layer(L);                                                  \
             cudaGetLastError();                                             \
             return fail(ACE_ERR_OOM, std::string("cudaMalloc failed for ") + #ptr); \
         }                                                                   \
+        ACE_CANARY(ptr, bytes);                                             \
     } while (0)
     L->tc = ace::tc_supported(L);
     ALLOC(L->router_w, n_pad * d * E);
@@ -378,7 +414,8 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
         ALLOC(W.h_perm, slots * d * E);
         ALLOC(W.act_bf16, slots * m * E);
         ALLOC(W.tt_off, (n + 1) * sizeof(int32_t));
-        ALLOC(W.tt_tab, (n + slots / 16 + 1) * sizeof(int4));
+        L->tt_cap = (int)(n + slots / 16 + 1);
+        ALLOC(W.tt_tab, (size_t)L->tt_cap * sizeof(int4));
         ALLOC(W.dec_done, (n + slots / 16 + 1) * sizeof(int32_t));
     } else {
         ALLOC(W.act, slots * m * sizeof(float));
@@ -391,6 +428,7 @@ ace_status ace_layer_create(const ace_layer_desc* desc_in, const void* router_w,
     ALLOC(W.x_stage, T * d * E);
     ALLOC(W.out_stage, T * d * E);
 #undef ALLOC
+#undef ACE_CANARY
 #define CK(call, where)                       \
     do {                                      \
         e = (call);                           \
@@ -724,6 +762,23 @@ ace_status ace_debug_set_wait_budget(ace_layer* L, long long cycles) {
     if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
     if (cycles < 0) return fail(ACE_ERR_INVALID_ARG, "cycles must be >= 0");
     L->dbg_ready_spin = cycles;
+    return ACE_OK;
+}
+
+int ace_debug_checks_enabled(void) {
+#ifdef ACE_DEBUG_CHECKS
+    return 1;
+#else
+    return 0;
+#endif
+}
+
+ace_status ace_debug_poke_canary(ace_layer* L, int index) {
+    if (!L) return fail(ACE_ERR_INVALID_ARG, "layer is NULL");
+    if (L->canaries.empty()) return fail(ACE_ERR_UNSUPPORTED, "canary words exist in the debug build only");
+    if (index < 0 || index >= (int)L->canaries.size()) return fail(ACE_ERR_INVALID_ARG, "canary index out of range");
+    ACE_CUDA(cudaDeviceSynchronize(), "synchronize");
+    ACE_CUDA(cudaMemset(L->canaries[index].at + 7, 0x5A, 1), "overwrite canary byte");
     return ACE_OK;
 }
 

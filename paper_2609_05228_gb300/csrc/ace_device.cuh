@@ -9,6 +9,16 @@
 
 namespace ace {
 
+// Index guards of the debug build (compiled with ACE_DEBUG_CHECKS): a
+// computed index that falls outside its array sets kErrBounds in the layer's
+// error word and the caller skips (or neutralises) the access; no trap. The
+// release build compiles every guard to `true`.
+#ifdef ACE_DEBUG_CHECKS
+#define ACE_IDX_OK(cond, err) ((cond) ? true : (atomicOr((err), ::ace::kErrBounds), false))
+#else
+#define ACE_IDX_OK(cond, err) true
+#endif
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

@@ -929,7 +929,8 @@ __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __rest
                                                      const int32_t* __restrict__ perm,
                                                      const int32_t* __restrict__ meta,
                                                      __nv_bfloat16* __restrict__ h_perm,
-                                                     int d, int k, int* __restrict__ done) {
+                                                     int d, int k, int* __restrict__ done, int n_slots,
+                                                     int* __restrict__ err) {
     pdl_wait();
     if (done && blockIdx.x == 0)                 // the decode kernel's per-token-tile counters
         for (int i = threadIdx.x; i < meta[kMetaTokTiles]; i += blockDim.x) done[i] = 0;
@@ -941,7 +942,9 @@ __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __rest
     // them in L2; the h_perm rows are read once, by GEMM 1's TMA: stream them
     const uint64_t keep = l2_policy_evict_last();
     for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < R; r += gridDim.x * wpb) {
-        const int tok = perm[r] / k;
+        const int slot = perm[r];
+        if (!ACE_IDX_OK(r < n_slots && slot >= 0 && slot < n_slots, err)) continue;
+        const int tok = slot / k;
         const uint4* src = reinterpret_cast<const uint4*>(h + (size_t)tok * d);
         uint4* dst = reinterpret_cast<uint4*>(h_perm + (size_t)r * d);
         uint4 v[16];
@@ -992,7 +995,8 @@ struct Row8<__nv_bfloat16> {
 template <typename Y, int KMAX>
 __global__ void __launch_bounds__(256) k_combine_bf16(const Y* __restrict__ y, const int32_t* __restrict__ slot_pos,
                                                       const __nv_bfloat16* __restrict__ resid,
-                                                      __nv_bfloat16* __restrict__ out, int n_tokens, int d, int k) {
+                                                      __nv_bfloat16* __restrict__ out, int n_tokens, int d, int k,
+                                                      int y_rows, int* __restrict__ err) {
     pdl_wait();
     const int nq = d / 8;
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
@@ -1000,7 +1004,10 @@ __global__ void __launch_bounds__(256) k_combine_bf16(const Y* __restrict__ y, c
     const int t = (int)(idx / nq), c8 = (int)(idx % nq);
     int r[KMAX];
 #pragma unroll
-    for (int i = 0; i < KMAX; ++i) r[i] = i < k ? __ldg(slot_pos + (size_t)t * k + i) : -1;
+    for (int i = 0; i < KMAX; ++i) {
+        r[i] = i < k ? __ldg(slot_pos + (size_t)t * k + i) : -1;
+        if (!ACE_IDX_OK(r[i] >= -1 && r[i] < y_rows, err)) r[i] = -1;
+    }
     Row8<Y> v[KMAX];
 #pragma unroll
     for (int i = 0; i < KMAX; ++i)
@@ -1037,14 +1044,17 @@ __global__ void __launch_bounds__(512) k_combine_norm(const __nv_bfloat16* __res
                                                       __nv_bfloat16* __restrict__ out,
                                                       const __nv_bfloat16* __restrict__ gamma_next,
                                                       __nv_bfloat16* __restrict__ h_next, float eps_next, int d,
-                                                      int k) {
+                                                      int k, int y_rows, int* __restrict__ err) {
     __shared__ float part_s[512];
     __shared__ float inv_s;
     pdl_wait();
     const int t = blockIdx.x, c8 = threadIdx.x;
     int r[KMAX];
 #pragma unroll
-    for (int i = 0; i < KMAX; ++i) r[i] = i < k ? __ldg(slot_pos + (size_t)t * k + i) : -1;
+    for (int i = 0; i < KMAX; ++i) {
+        r[i] = i < k ? __ldg(slot_pos + (size_t)t * k + i) : -1;
+        if (!ACE_IDX_OK(r[i] >= -1 && r[i] < y_rows, err)) r[i] = -1;
+    }
     Row8<__nv_bfloat16> v[KMAX];
 #pragma unroll
     for (int i = 0; i < KMAX; ++i)
@@ -1087,11 +1097,12 @@ __global__ void __launch_bounds__(512) k_combine_norm(const __nv_bfloat16* __res
 
 template <int KMAX>
 cudaError_t launch_combine_norm(const __nv_bfloat16* y, const int32_t* sp, const __nv_bfloat16* resid,
-                                __nv_bfloat16* out, const ace_layer* next, int T, int d, int k, cudaStream_t s) {
+                                __nv_bfloat16* out, const ace_layer* next, int T, int d, int k, int y_rows, int* err,
+                                cudaStream_t s) {
     // d is a multiple of 256 (tensor-core layers) and at most 4096: d / 8 threads, whole warps
     return launch_pdl(k_combine_norm<KMAX>, dim3(T), dim3(d / 8), 0, s, y, sp, resid, out,
                       static_cast<const __nv_bfloat16*>(next->gamma), static_cast<__nv_bfloat16*>(next->ws.h),
-                      next->desc.rms_eps, d, k);
+                      next->desc.rms_eps, d, k, y_rows, err);
 }
 
 // ---------------------------------------------------------------- host side
@@ -1345,7 +1356,7 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     {
         e = launch_pdl(k_gather_rows, dim3(L->num_sms * 4), dim3(256), 0, s, (const __nv_bfloat16*)W.h,
                        (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k,
-                       small ? W.dec_done : (int*)nullptr);
+                       small ? W.dec_done : (int*)nullptr, T * k, W.err);
         if (e != cudaSuccess) return e;
     }
     if (small) {
@@ -1377,10 +1388,11 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
         }
         const long long nthreads = (long long)T * (d / 8);
         const dim3 grid((unsigned)((nthreads + 255) / 256));
+        const int yr = T * k;                 // fp32 slot rows of this batch
         e = k <= 8 ? launch_pdl(k_combine_bf16<float, 8>, grid, dim3(256), 0, s, (const float*)W.yslot,
-                                (const int32_t*)W.slot_pos, resid, (__nv_bfloat16*)out, T, d, k)
+                                (const int32_t*)W.slot_pos, resid, (__nv_bfloat16*)out, T, d, k, yr, W.err)
                    : launch_pdl(k_combine_bf16<float, kMaxTopK>, grid, dim3(256), 0, s, (const float*)W.yslot,
-                                (const int32_t*)W.slot_pos, resid, (__nv_bfloat16*)out, T, d, k);
+                                (const int32_t*)W.slot_pos, resid, (__nv_bfloat16*)out, T, d, k, yr, W.err);
         if (ev) ace::record_stage(ev[3], s);
         return e;
     }
@@ -1437,18 +1449,22 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     const dim3 grid((unsigned)((nthreads + 255) / 256));
     const int32_t* sp = W.slot_pos;
     __nv_bfloat16* o = static_cast<__nv_bfloat16*>(out);
+    const int yr = T * k;                     // slot rows of this batch
     if (small) {
         const float* y = W.yslot;
-        e = k <= 8 ? launch_pdl(k_combine_bf16<float, 8>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k)
-                   : launch_pdl(k_combine_bf16<float, kMaxTopK>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k);
+        e = k <= 8 ? launch_pdl(k_combine_bf16<float, 8>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k, yr, W.err)
+                   : launch_pdl(k_combine_bf16<float, kMaxTopK>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k, yr,
+                                W.err);
     } else if (next) {
         const __nv_bfloat16* y = static_cast<const __nv_bfloat16*>(W.h_perm);
-        e = k <= 8 ? launch_combine_norm<8>(y, sp, resid, o, next, T, d, k, s)
-                   : launch_combine_norm<kMaxTopK>(y, sp, resid, o, next, T, d, k, s);
+        e = k <= 8 ? launch_combine_norm<8>(y, sp, resid, o, next, T, d, k, yr, W.err, s)
+                   : launch_combine_norm<kMaxTopK>(y, sp, resid, o, next, T, d, k, yr, W.err, s);
     } else {
         const __nv_bfloat16* y = static_cast<const __nv_bfloat16*>(W.h_perm);
-        e = k <= 8 ? launch_pdl(k_combine_bf16<__nv_bfloat16, 8>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k)
-                   : launch_pdl(k_combine_bf16<__nv_bfloat16, kMaxTopK>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k);
+        e = k <= 8 ? launch_pdl(k_combine_bf16<__nv_bfloat16, 8>, grid, dim3(256), 0, s, y, sp, resid, o, T, d, k, yr,
+                                W.err)
+                   : launch_pdl(k_combine_bf16<__nv_bfloat16, kMaxTopK>, grid, dim3(256), 0, s, y, sp, resid, o, T, d,
+                                k, yr, W.err);
     }
     if (ev) ace::record_stage(ev[3], s);
     return e;

@@ -113,11 +113,25 @@ struct ace_stack {
     int hidden = 0;
 };
 
+// Debug build (ACE_DEBUG_CHECKS): every device array of a layer is
+// allocated kCanaryBytes longer and the tail filled with kCanaryByte; the
+// synchronising calls check that no kernel wrote past an array's end.
+namespace ace {
+constexpr size_t kCanaryBytes = 256;
+constexpr unsigned char kCanaryByte = 0xA5;
+struct Canary {
+    const char* name;   // the array's field name
+    unsigned char* at;  // first byte past the array
+};
+}  // namespace ace
+
 struct ace_layer {
     ace_layer_desc desc;
     int device = 0;
     int num_sms = 0;
     int pair_clusters = 0;       // CTA pairs of the wide-tile expert kernel resident at once
+    int tt_cap = 0;              // entries allocated in ws.tt_tab
+    std::vector<ace::Canary> canaries;   // debug build only
     size_t elem = 2;             // bytes per element of dtype
     // layer-owned weights
     void* router_w = nullptr;    // [N, d]

@@ -539,15 +539,19 @@ __device__ void scan_counts_block(const int* cnt, int n_exp, int32_t* __restrict
 
 // After scan_counts_block and a block barrier: the flat token-tile table of
 // the tensor-core experts, tt_tab[tt] = (expert, first row, rows, 0).
+// tt_cap: entries allocated in tt_tab (checked by the debug build).
 __device__ void fill_tile_table(const int32_t* offsets, const int32_t* dlist, const int32_t* tt_off,
-                                const int32_t* meta, int tok_tile, int4* tt_tab) {
+                                const int32_t* meta, int tok_tile, int4* tt_tab, int n_exp, int tt_cap, int* err) {
     if (tok_tile <= 0) return;
     const int D = meta[kMetaDistinct];
     for (int j = threadIdx.x; j < D; j += blockDim.x) {
         const int e = dlist[j];
+        if (!ACE_IDX_OK((unsigned)e < (unsigned)n_exp, err)) continue;
         const int beg = offsets[e], cnt = offsets[e + 1] - beg, base = tt_off[j];
-        for (int b = 0; b * tok_tile < cnt; ++b)
+        for (int b = 0; b * tok_tile < cnt; ++b) {
+            if (!ACE_IDX_OK(base + b >= 0 && base + b < tt_cap, err)) break;
             tt_tab[base + b] = make_int4(e, beg + b * tok_tile, min(tok_tile, cnt - b * tok_tile), 0);
+        }
     }
 }
 
@@ -603,6 +607,7 @@ __global__ void __launch_bounds__(kTopkWarps * 32) k_topk_score(float* __restric
         float zv;
         bool nan;
         warp_topk<NPL>(logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
+        if (lane < k && !ACE_IDX_OK((unsigned)id < (unsigned)n_exp, err)) id = 0;   // tables are read at id
         const float z0 = __shfl_sync(0xffffffffu, zv, 0);
         if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(err, kErrNumeric);
         const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a_gsp, a_rcr, eps, fusion);
@@ -709,7 +714,7 @@ template <int KPT>
 __global__ void __launch_bounds__(1024) k_sel_collect(const uint32_t* __restrict__ keys, int n, int m,
                                                       const int32_t* __restrict__ hist1,
                                                       int32_t* __restrict__ hist2, uint32_t* __restrict__ cand,
-                                                      int32_t* __restrict__ meta) {
+                                                      int32_t* __restrict__ meta, int* err) {
     __shared__ SelShared S;
     __shared__ int h2[1024];
     const int tid = threadIdx.x, lane = tid & 31;
@@ -746,7 +751,7 @@ __global__ void __launch_bounds__(1024) k_sel_collect(const uint32_t* __restrict
         int pos = 0;
         if (lane == 0) pos = atomicAdd(&meta[kMetaSelCount], __popc(bal));
         pos = __shfl_sync(0xffffffffu, pos, 0) + __popc(bal & lanemask_lt());
-        if (in) {
+        if (in && ACE_IDX_OK(pos < n, err)) {
             cand[pos] = kv[j];
             const int bin = (int)((kv[j] >> 10) & 1023u);
             const unsigned peers = __match_any_sync(bal, bin);
@@ -826,7 +831,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, i
                                                           const float* __restrict__ cval,
                                                           const float* __restrict__ tau_dev, int m_min, float eps,
                                                           float* __restrict__ ghat,
-                                                          int32_t* __restrict__ chunk_counts) {
+                                                          int32_t* __restrict__ chunk_counts, int* err) {
     __shared__ int cnt[kMaxExperts];
     for (int e = threadIdx.x; e < n_exp; e += blockDim.x) cnt[e] = 0;
     __syncthreads();
@@ -836,8 +841,10 @@ __global__ void __launch_bounds__(kChunk) k_compact_count(int n_tokens, int k, i
         const size_t base = (size_t)t * k;
         if (DECIDE)
             decide_token(gates + base, cval + base, k, __ldcg(tau_dev), m_min, eps, skip + base, ghat + base, nullptr);
-        for (int i = 0; i < k; ++i)
-            if (!skip[base + i]) atomicAdd(&cnt[ids[base + i]], 1);
+        for (int i = 0; i < k; ++i) {
+            const int e = ids[base + i];
+            if (!skip[base + i] && ACE_IDX_OK((unsigned)e < (unsigned)n_exp, err)) atomicAdd(&cnt[e], 1);
+        }
     }
     __syncthreads();
     for (int e = threadIdx.x; e < n_exp; e += blockDim.x)
@@ -882,7 +889,8 @@ __global__ void __launch_bounds__(kScanThreads) k_compact_scan(int n_exp, int n_
                                                                int32_t* __restrict__ offsets,
                                                                int32_t* __restrict__ dlist,
                                                                int32_t* __restrict__ meta, int tok_tile,
-                                                               int32_t* __restrict__ tt_off, int4* __restrict__ tt_tab) {
+                                                               int32_t* __restrict__ tt_off, int4* __restrict__ tt_tab,
+                                                               int tt_cap, int* err) {
     __shared__ int wtot[32];
     __shared__ int wsum[96];
     __shared__ int cnt[kMaxExperts];
@@ -920,7 +928,7 @@ __global__ void __launch_bounds__(kScanThreads) k_compact_scan(int n_exp, int n_
     __syncthreads();
     scan_counts_block(cnt, n_exp, offsets, dlist, meta, nullptr, tok_tile, tt_off, wsum);
     __syncthreads();
-    fill_tile_table(offsets, dlist, tt_off, meta, tok_tile, tt_tab);
+    fill_tile_table(offsets, dlist, tt_off, meta, tok_tile, tt_tab, n_exp, tt_cap, err);
 }
 
 __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, int n_exp, int n_chunks,
@@ -929,7 +937,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
                                                           const int32_t* __restrict__ offsets,
                                                           const int32_t* __restrict__ chunk_base,
                                                           int32_t* __restrict__ perm,
-                                                          int32_t* __restrict__ slot_pos) {
+                                                          int32_t* __restrict__ slot_pos, int* err) {
     constexpr int W = kChunk / 32;
     __shared__ uint32_t bm[kMaxExperts * W];
     for (int i = threadIdx.x; i < n_exp * W; i += blockDim.x) bm[i] = 0u;
@@ -939,8 +947,10 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
     const int w = threadIdx.x >> 5;
     const unsigned bit = 1u << (threadIdx.x & 31);
     if (t < n_tokens) {
-        for (int i = 0; i < k; ++i)
-            if (!skip[(size_t)t * k + i]) atomicOr(&bm[ids[(size_t)t * k + i] * W + w], bit);
+        for (int i = 0; i < k; ++i) {
+            const int e = ids[(size_t)t * k + i];
+            if (!skip[(size_t)t * k + i] && ACE_IDX_OK((unsigned)e < (unsigned)n_exp, err)) atomicOr(&bm[e * W + w], bit);
+        }
     }
     __syncthreads();
     if (t < n_tokens) {
@@ -949,9 +959,11 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
             const size_t s = (size_t)t * k + i;
             if (skip[s]) { slot_pos[s] = -1; continue; }
             const int e = ids[s];
+            if (!ACE_IDX_OK((unsigned)e < (unsigned)n_exp, err)) { slot_pos[s] = -1; continue; }
             int rank = __popc(bm[e * W + w] & lt);
             for (int ww = 0; ww < w; ++ww) rank += __popc(bm[e * W + ww]);
             const int r = __ldcg(offsets + e) + __ldcg(chunk_base + (size_t)e * n_chunks + blockIdx.x) + rank;
+            if (!ACE_IDX_OK(r >= 0 && (size_t)r < (size_t)n_tokens * k, err)) { slot_pos[s] = -1; continue; }
             perm[r] = (int32_t)s;
             slot_pos[s] = r;
         }
@@ -1011,6 +1023,7 @@ struct FusedArgs {
     int tok_tile;
     int32_t* tt_off;
     int4* tt_tab;
+    int tt_cap;                 // entries allocated in tt_tab
     int32_t* tile_cnt;
     const uint8_t* pf_base;     // expert weights to start pulling into L2 while routing runs
     long long pf_bytes;         // (a multiple of 256 bytes; 0 = none)
@@ -1204,6 +1217,7 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         float zv;
         bool nan;
         warp_topk<NPL>(a.logits + (size_t)t * n_exp, n_exp, k, lane, id, zv, nan);
+        if (lane < k && !ACE_IDX_OK((unsigned)id < (unsigned)n_exp, a.err)) id = 0;
         const float z0 = __shfl_sync(0xffffffffu, zv, 0);
         if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(a.err, kErrNumeric);
         const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a.a_gsp, a.a_rcr, a.eps, a.fusion);
@@ -1274,19 +1288,22 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
     for (int s = threadIdx.x; s < ns; s += blockDim.x) {
         if (skip_s[s]) continue;
         const int e = id_s[s], t = s / k;
+        if (!ACE_IDX_OK((unsigned)e < (unsigned)n_exp && (t >> 5) < 8, a.err)) continue;
         atomicAdd(&cnt[e], 1);
         atomicOr(&bm[e * 8 + (t >> 5)], 1u << (t & 31));
     }
     __syncthreads();
     scan_counts_block(cnt, n_exp, a.offsets, a.dlist, a.meta, off_s, a.tok_tile, a.tt_off, S.hist);
     __syncthreads();
-    fill_tile_table(a.offsets, a.dlist, a.tt_off, a.meta, a.tok_tile, a.tt_tab);
+    fill_tile_table(a.offsets, a.dlist, a.tt_off, a.meta, a.tok_tile, a.tt_tab, n_exp, a.tt_cap, a.err);
     for (int s = threadIdx.x; s < ns; s += blockDim.x) {
         if (skip_s[s]) { a.slot_pos[s] = -1; continue; }
         const int e = id_s[s], t = s / k, w = t >> 5;
+        if (!ACE_IDX_OK((unsigned)e < (unsigned)n_exp && w < 8, a.err)) { a.slot_pos[s] = -1; continue; }
         int rank = __popc(bm[e * 8 + w] & ((1u << (t & 31)) - 1u));
         for (int ww = 0; ww < w; ++ww) rank += __popc(bm[e * 8 + ww]);
         const int r = off_s[e] + rank;
+        if (!ACE_IDX_OK(r >= 0 && r < ns, a.err)) { a.slot_pos[s] = -1; continue; }
         a.perm[r] = s;
         a.slot_pos[s] = r;
     }
@@ -1424,6 +1441,7 @@ cudaError_t launch_route_fused(const ace_layer* L, const void* x, const float* l
     a.tok_tile = L->tc ? tc_token_tile(L, T, ctl) : 0;
     a.tt_off = W.tt_off;
     a.tt_tab = W.tt_tab;
+    a.tt_cap = L->tt_cap;
     a.tile_cnt = W.tile_cnt;
     if (x && L->tc && L->w_gu) {
         const long long gu_bytes = 2LL * D.ffn * D.hidden * 2 * D.n_experts;
@@ -1490,7 +1508,7 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
         // fewest keys per thread that keep the grid within two 1024-thread blocks per SM
 #define ACE_COLLECT(KPT)                                                                                          \
     launch_pdl(k_sel_collect<KPT>, dim3(cdiv(nk, 1024 * KPT)), dim3(1024), 0, s, (const uint32_t*)W.keys, nk, m_q, \
-               (const int32_t*)W.sel_hist, W.sel_hist + kHistBins, W.sel_cand, W.meta)
+               (const int32_t*)W.sel_hist, W.sel_hist + kHistBins, W.sel_cand, W.meta, W.err)
         const long long slots = 2LL * 1024 * L->num_sms;
         if (nk <= slots) e = ACE_COLLECT(1);
         else if (nk <= 2 * slots) e = ACE_COLLECT(2);
@@ -1506,14 +1524,14 @@ cudaError_t launch_route(const ace_layer* L, const float* logits, int T, ace_ski
     const bool dec = mode == ACE_SKIP_RATIO;
     e = launch_pdl(dec ? k_compact_count<true> : k_compact_count<false>, dim3(n_chunks), dim3(kChunk), 0, s, T, k, n,
                    n_chunks, (const int32_t*)W.ids, W.skip, (const float*)W.gates, (const float*)W.cval,
-                   (const float*)W.tau, D.min_active, D.eps, W.ghat, W.chunk_counts);
+                   (const float*)W.tau, D.min_active, D.eps, W.ghat, W.chunk_counts, W.err);
     if (e != cudaSuccess) return e;
     e = launch_pdl(k_compact_scan, dim3(n), dim3(kScanThreads), 0, s, n, n_chunks, W.chunk_counts, W.offsets, W.dlist,
-                   W.meta, tok_tile, W.tt_off, W.tt_tab);
+                   W.meta, tok_tile, W.tt_off, W.tt_tab, L->tt_cap, W.err);
     if (e != cudaSuccess) return e;
     return launch_pdl(k_compact_place, dim3(n_chunks), dim3(kChunk), 0, s, T, k, n, n_chunks, (const int32_t*)W.ids,
                       (const uint8_t*)W.skip, (const int32_t*)W.offsets, (const int32_t*)W.chunk_counts, W.perm,
-                      W.slot_pos);
+                      W.slot_pos, W.err);
 }
 
 int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl) {

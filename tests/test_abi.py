@@ -99,3 +99,19 @@ def test_stack_argument_checks_on_host(libace):
     assert L.ace_stack_create(arr, 1, ctypes.byref(out)) == 1
     assert L.ace_stack_forward(None, None, None, 1, ace.ace_skip_ctl(0, 0.1, 0), None) == 1
     L.ace_stack_destroy(None)
+
+
+def test_debug_library_exports_the_same_boundary():
+    """libace_debug.so (index guards, canary words) exports every declared
+    symbol too; the two builds report which one they are, and the canary hook
+    rejects a NULL layer before touching a device."""
+    if not os.path.exists(build.DEBUG_LIBPATH):
+        build.build()
+    dbg = ctypes.CDLL(build.DEBUG_LIBPATH)
+    rel = ctypes.CDLL(ace.LIBPATH)
+    missing = [n for n in declared_functions() if not hasattr(dbg, n)]
+    assert not missing, missing
+    assert dbg.ace_debug_checks_enabled() == 1
+    assert rel.ace_debug_checks_enabled() == 0
+    dbg.ace_debug_poke_canary.argtypes = [ctypes.c_void_p, ctypes.c_int]
+    assert dbg.ace_debug_poke_canary(None, 0) == 1          # ACE_ERR_INVALID_ARG
