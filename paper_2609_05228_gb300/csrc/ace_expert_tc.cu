@@ -552,11 +552,24 @@ struct DecParams {
     int ready_extra;                    // added to that wait's target: 0, or unreachable (a test of the bound)
 };
 
-constexpr int kDecStages = 8;
-constexpr int kDecA = 128 * kBK * 2;
-constexpr int kDecB = 16 * kBK * 2;
-constexpr int kDecStage = kDecA + kDecB;
-constexpr int kDecSmem = kDecStages * kDecStage + 1024 + 256;
+// A stage holds KBS K blocks: the KBS weight tiles of one (expert, weight
+// tile) are adjacent in the tiled layout, so they arrive with one bulk copy
+// of KBS x 16 KB, followed by KBS token boxes. Each stage costs a fixed
+// producer / MMA / barrier round trip (measured about 0.2 us on one SM), so a
+// lone SM streams about twice as fast with 36 KB stages as with 18 KB ones:
+// batches that retain few experts, where few SMs have work, take KBS = 2;
+// larger ones keep KBS = 1 (8 stages), which every SM streams at its share of
+// the HBM bandwidth.
+template <int KBS>
+struct DecCfg {
+    static constexpr int STAGES = KBS == 1 ? 8 : 6;
+    static constexpr int A = KBS * 128 * kBK * 2;             // weight tiles
+    static constexpr int B1 = 16 * kBK * 2;                   // one token box (16 rows x 64 bf16)
+    static constexpr int STAGE = A + KBS * B1;
+    static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
+};
+// Decode batches that take 2 K blocks per stage: few distinct retained experts.
+constexpr int kDecWideStageTokens = 16;
 
 __device__ __forceinline__ int ld_acquire(const int* p) {
     int v;
@@ -598,7 +611,10 @@ __device__ __forceinline__ DecTile dec_tile(const DecParams& p, int tile, int n1
     return t;
 }
 
+template <int KBS>
 __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_constant__ DecParams p) {
+    using C = DecCfg<KBS>;
+    constexpr int kDecStages = C::STAGES, kDecStage = C::STAGE, kDecA = C::A;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + kDecStages * kDecStage);
@@ -663,13 +679,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
                 }
                 const uint8_t* wbase = t.phase == 0 ? p.w_gu : p.w_down;
                 const int wrows = t.phase == 0 ? 2 * p.m : p.d;
-                for (int kb = 0; kb < t.kblocks; ++kb) {
+                for (int kb = 0; kb < t.kblocks; kb += KBS) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
                     unsigned char* sa = smem + stage * kDecStage;
                     mbar_expect_tx(&full[stage], kDecStage);
-                    bulk_g2s(sa, wbase + (((size_t)t.e * (wrows / 128) + t.wt) * t.kblocks + kb) * 16384, 16384,
-                             &full[stage]);
-                    tma_load_2d(sa + kDecA, t.phase == 0 ? &p.tm_h : &p.tm_act, &full[stage], kb * kBK, t.row0);
+                    bulk_g2s(sa, wbase + (((size_t)t.e * (wrows / 128) + t.wt) * t.kblocks + kb) * 16384,
+                             KBS * 16384, &full[stage]);
+#pragma unroll
+                    for (int j = 0; j < KBS; ++j)
+                        tma_load_2d(sa + kDecA + j * C::B1, t.phase == 0 ? &p.tm_h : &p.tm_act, &full[stage],
+                                    (kb + j) * kBK, t.row0);
                     ++issued;
                     if (++stage == kDecStages) { stage = 0; phase ^= 1u; }
                 }
@@ -695,15 +714,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
                 if (!mbar_wait(&acc_empty[acc], acc_phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 16);
-                for (int kb = 0; kb < t.kblocks; ++kb) {
+                for (int kb = 0; kb < t.kblocks; kb += KBS) {
                     if (!mbar_wait(&full[stage], phase, p.err) || *abort_flag) { ok = false; break; }
                     tc_fence_after();
-                    const uint32_t a_addr = smem_u32(smem + stage * kDecStage);
-                    const uint32_t b_addr = a_addr + kDecA;
+                    const uint32_t s_addr = smem_u32(smem + stage * kDecStage);
 #pragma unroll
-                    for (int kk = 0; kk < kBK / kUmmaK; ++kk)
-                        mma_bf16(d_tmem, smem_desc_sw128(a_addr + kk * kUmmaK * 2), smem_desc_sw128(b_addr + kk * kUmmaK * 2),
-                                 idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                    for (int j = 0; j < KBS; ++j) {
+                        const uint32_t a_addr = s_addr + j * 16384;               // weight tile kb + j
+                        const uint32_t b_addr = s_addr + kDecA + j * C::B1;       // its token box
+#pragma unroll
+                        for (int kk = 0; kk < kBK / kUmmaK; ++kk)
+                            mma_bf16(d_tmem, smem_desc_sw128(a_addr + kk * kUmmaK * 2),
+                                     smem_desc_sw128(b_addr + kk * kUmmaK * 2), idesc,
+                                     (kb + j > 0 || kk > 0) ? 1u : 0u);
+                    }
                     mma_commit(&empty[stage]);
                     if (++stage == kDecStages) { stage = 0; phase ^= 1u; }
                 }
@@ -1275,9 +1299,14 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = set_attr<false, 0>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 1>()) != cudaSuccess) return e;
     if ((e = set_attr<false, 2>()) != cudaSuccess) return e;
-    if ((e = cudaFuncSetAttribute(k_expert_decode, cudaFuncAttributeMaxDynamicSharedMemorySize, kDecSmem)) != cudaSuccess)
+    if ((e = cudaFuncSetAttribute(k_expert_decode<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  DecCfg<1>::SMEM)) != cudaSuccess)
         return e;
-    if ((e = prefer_shared(k_expert_decode)) != cudaSuccess) return e;
+    if ((e = prefer_shared(k_expert_decode<1>)) != cudaSuccess) return e;
+    if ((e = cudaFuncSetAttribute(k_expert_decode<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  DecCfg<2>::SMEM)) != cudaSuccess)
+        return e;
+    if ((e = prefer_shared(k_expert_decode<2>)) != cudaSuccess) return e;
     if ((e = set_pair_attr((const void*)k_expert_pair<0>)) != cudaSuccess) return e;
     if ((e = set_pair_attr((const void*)k_expert_pair<1>)) != cudaSuccess) return e;
     int c0 = 0, c1 = 0;
@@ -1380,7 +1409,10 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
         q.k = k;
         q.ready_spin = L->dbg_ready_spin > 0 ? L->dbg_ready_spin : kSpinCycles;
         q.ready_extra = L->dbg_ready_spin > 0 ? (1 << 30) : 0;
-        e = launch_pdl(k_expert_decode, dim3(L->num_sms), dim3(kThreads), kDecSmem, s, q);
+        // K blocks are even: d is a multiple of 256 and m of 128 on this path
+        e = T <= kDecWideStageTokens
+                ? launch_pdl(k_expert_decode<2>, dim3(L->num_sms), dim3(kThreads), DecCfg<2>::SMEM, s, q)
+                : launch_pdl(k_expert_decode<1>, dim3(L->num_sms), dim3(kThreads), DecCfg<1>::SMEM, s, q);
         if (e != cudaSuccess) return e;
         if (ev) {                           // gate/up and down share one launch: the down stage reads 0
             ace::record_stage(ev[1], s);
