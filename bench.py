@@ -47,6 +47,11 @@ WORKLOADS = {
                          shape=f"4-layer stack of the {QWEN} layer (residual), decode"),
     "large_prefill": dict(spec="large", zipf=True, T=8192, q=0.5, layers=1, tables="gpu",
                           shape=f"large MoE layer {LARGE}, prefill, Zipf(1.1) routing"),
+    # the large layer's expert shape with 32 experts (1.6 GB): a case small enough for an
+    # ncu --set full capture of the large prefill's GEMMs (traffic scaled to the full layer)
+    "large_prefill_e32": dict(spec="large32", zipf=True, T=1024, q=0.5, layers=1, tables="gpu",
+                              shape="large MoE layer shape d=4096 top-8 m=2048 bf16 with 32 experts, prefill, "
+                                    "Zipf(1.1) routing"),
     "large_decode": dict(spec="large", zipf=True, T=128, q=0.5, layers=1, tables="gpu",
                          shape=f"large MoE layer {LARGE}, decode, Zipf(1.1) routing"),
 }
@@ -92,12 +97,16 @@ TRAFFIC_RECORDS = {
     "decode": "profiles/decode_T64_q0.5_expert_decode_full.md",
     "prefill": "profiles/prefill_T4096_q0.5_expert_tc_full.md",
     "stack_prefill": "profiles/stack_prefill_T16384_q0.5_expert_pair_full.md",
+    "large_prefill": "profiles/large_prefill_e32_T1024_q0.5_expert_tc_full.md",
 }
 
 
-def _recorded_traffic(path="profiles/decode_T64_q0.5_expert_decode_full.md"):
+def _recorded_traffic(path="profiles/decode_T64_q0.5_expert_decode_full.md", alg_bytes=None):
     """DRAM bytes per launch of the dominant kernel from a committed ncu
-    summary, or None when the kernel source has changed since the capture."""
+    summary, or None when the kernel source has changed since the capture.
+    A record taken on a smaller case of the workload (it then states
+    algorithmic_bytes_per_launch) is scaled by the algorithmic bytes of the
+    launch being reported, `alg_bytes`."""
     import hashlib
     try:
         rec = {}
@@ -113,6 +122,10 @@ def _recorded_traffic(path="profiles/decode_T64_q0.5_expert_decode_full.md"):
                 h.update(f.read())
         if h.hexdigest() != rec["source_sha256"]:
             return None
+        if "algorithmic_bytes_per_launch" in rec:
+            if alg_bytes is None:
+                return None
+            return int(round(int(rec["dram_bytes_per_launch"]) * alg_bytes / int(rec["algorithmic_bytes_per_launch"])))
         return int(rec["dram_bytes_per_launch"])
     except Exception:
         return None
@@ -226,7 +239,8 @@ class Stack:
 
     def __init__(self, wl, max_tokens, tables=None):
         from paper_2609_05228_gb300 import ace, offline, synth
-        spec = synth.spec_qwen(zipf=wl["zipf"]) if wl["spec"] == "qwen" else synth.spec_large(zipf=wl["zipf"])
+        spec = (synth.spec_qwen(zipf=wl["zipf"]) if wl["spec"] == "qwen" else
+                synth.spec_large(zipf=wl["zipf"], n_experts=32 if wl["spec"] == "large32" else 256))
         self.ws, self.layers = [], []
         n = wl["layers"]
         for l in range(n):
@@ -508,7 +522,8 @@ def run_ours(args, rank, world, torch, dist):
         roof = {"bound": "hbm", "kernel": "k_expert_tc gate/up (tcgen05)",
                 "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s", "frac": round(achieved / hbm, 4),
                 "peak_source": peak_kind,
-                "traffic": _recorded_traffic(TRAFFIC_RECORDS[args.workload]) if args.workload in TRAFFIC_RECORDS else None,
+                "traffic": _recorded_traffic(TRAFFIC_RECORDS[args.workload], gu_bytes)
+                if args.workload in TRAFFIC_RECORDS else None,
                 "algorithmic_bytes": gu_bytes, "kernel_us": round(gu_ms * 1e3, 2)}
 
     result = {
@@ -817,7 +832,8 @@ def main():
         if rank == 0:
             from paper_2609_05228_gb300 import synth
             wl = WORKLOADS[args.workload]
-            spec = synth.spec_qwen(zipf=wl["zipf"]) if wl["spec"] == "qwen" else synth.spec_large(zipf=wl["zipf"])
+            spec = (synth.spec_qwen(zipf=wl["zipf"]) if wl["spec"] == "qwen" else
+                synth.spec_large(zipf=wl["zipf"], n_experts=32 if wl["spec"] == "large32" else 256))
             w = synth.make_layer(spec, seed=0)
             print(json.dumps({"workload": wl["name"], "offline_tables": time_tables(torch, w, reps=args.steps)}),
                   flush=True)

@@ -189,5 +189,7 @@ def spec_qwen(zipf: bool = False) -> LayerSpec:
     return LayerSpec(2048, 128, 8, 768, dtype="bf16", zipf=zipf)
 
 
-def spec_large(zipf: bool = True) -> LayerSpec:
-    return LayerSpec(4096, 256, 8, 2048, dtype="bf16", zipf=zipf, zipf_beta=ZIPF_BETA_LARGE)
+def spec_large(zipf: bool = True, n_experts: int = 256) -> LayerSpec:
+    """The large layer; n_experts < 256 gives a smaller case with the same
+    expert shape (for profiler captures that must stay a few GB)."""
+    return LayerSpec(4096, n_experts, 8, 2048, dtype="bf16", zipf=zipf, zipf_beta=ZIPF_BETA_LARGE)
