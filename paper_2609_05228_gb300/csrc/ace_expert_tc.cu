@@ -333,7 +333,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
             const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile, n_base, kblocks);
             for (int kb = 0; kb < kblocks; ++kb) {
                 int go = 1;
-                if (lane == 0) go = mbar_wait(&empty[stage], phase ^ 1u, p.err) && !*abort_flag;
+                if (lane == 0) go = mbar_wait_or_abort(&empty[stage], phase ^ 1u, p.err, abort_flag);
                 if (!__shfl_sync(0xffffffffu, go, 0)) { ok = false; break; }
                 unsigned char* sa = smem + stage * C::STAGE_BYTES;
                 unsigned char* sb = sa + C::A_BYTES;
@@ -381,20 +381,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
             uint32_t acc_phase = 0;
             bool ok = true;
             for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-                if (!mbar_wait(&acc_empty[acc], acc_phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                if (!mbar_wait_or_abort(&acc_empty[acc], acc_phase ^ 1u, p.err, abort_flag)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * C::ACC_COLS);
                 for (int kb = 0; kb < kblocks; ++kb) {
-                    if (!mbar_wait(&full[stage], phase, p.err) || *abort_flag) { ok = false; break; }
+                    if (!mbar_wait_or_abort(&full[stage], phase, p.err, abort_flag)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t a_addr = smem_u32(smem + stage * C::STAGE_BYTES);
                     const uint32_t b_addr = a_addr + C::A_BYTES;
+                    // descriptors of the stage's first K step; a K step of 16 bf16 (32 B)
+                    // adds 2 to the 14-bit start-address field
+                    const uint64_t ad = smem_desc_sw128(a_addr), bd = smem_desc_sw128(b_addr);
 #pragma unroll
-                    for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
-                        const uint64_t ad = smem_desc_sw128(a_addr + kk * kUmmaK * 2);
-                        const uint64_t bd = smem_desc_sw128(b_addr + kk * kUmmaK * 2);
-                        mma_bf16(d_tmem, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
-                    }
+                    for (int kk = 0; kk < kBK / kUmmaK; ++kk)
+                        mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
                     mma_commit(&empty[stage]);           // frees the stage when these MMAs finish
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
@@ -415,7 +415,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
             const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile, n_base, kblocks);
             const float gh = SWAP ? 0.f : wide_row_ghat<EPI>(p, t, quad * 32 + lane);
             bool ok = true;
-            if (lane == 0) ok = mbar_wait(&acc_full[acc], acc_phase, p.err) && !*abort_flag;
+            if (lane == 0) ok = mbar_wait_or_abort(&acc_full[acc], acc_phase, p.err, abort_flag);
             ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
             if (!ok) break;
             tc_fence_after();
@@ -680,7 +680,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
                 const uint8_t* wbase = t.phase == 0 ? p.w_gu : p.w_down;
                 const int wrows = t.phase == 0 ? 2 * p.m : p.d;
                 for (int kb = 0; kb < t.kblocks; kb += KBS) {
-                    if (!mbar_wait(&empty[stage], phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                    if (!mbar_wait_or_abort(&empty[stage], phase ^ 1u, p.err, abort_flag)) { ok = false; break; }
                     unsigned char* sa = smem + stage * kDecStage;
                     mbar_expect_tx(&full[stage], kDecStage);
                     bulk_g2s(sa, wbase + (((size_t)t.e * (wrows / 128) + t.wt) * t.kblocks + kb) * 16384,
@@ -711,22 +711,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
             bool ok = true;
             for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
                 const DecTile t = dec_tile(p, tile, n1);
-                if (!mbar_wait(&acc_empty[acc], acc_phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                if (!mbar_wait_or_abort(&acc_empty[acc], acc_phase ^ 1u, p.err, abort_flag)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 16);
                 for (int kb = 0; kb < t.kblocks; kb += KBS) {
-                    if (!mbar_wait(&full[stage], phase, p.err) || *abort_flag) { ok = false; break; }
+                    if (!mbar_wait_or_abort(&full[stage], phase, p.err, abort_flag)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t s_addr = smem_u32(smem + stage * kDecStage);
 #pragma unroll
                     for (int j = 0; j < KBS; ++j) {
                         const uint32_t a_addr = s_addr + j * 16384;               // weight tile kb + j
                         const uint32_t b_addr = s_addr + kDecA + j * C::B1;       // its token box
+                        const uint64_t ad = smem_desc_sw128(a_addr), bd = smem_desc_sw128(b_addr);
 #pragma unroll
                         for (int kk = 0; kk < kBK / kUmmaK; ++kk)
-                            mma_bf16(d_tmem, smem_desc_sw128(a_addr + kk * kUmmaK * 2),
-                                     smem_desc_sw128(b_addr + kk * kUmmaK * 2), idesc,
-                                     (kb + j > 0 || kk > 0) ? 1u : 0u);
+                            mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, (kb + j > 0 || kk > 0) ? 1u : 0u);
                     }
                     mma_commit(&empty[stage]);
                     if (++stage == kDecStages) { stage = 0; phase ^= 1u; }
@@ -744,7 +743,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
         uint32_t acc_phase = 0;
         for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
             bool ok = true;
-            if (lane == 0) ok = mbar_wait(&acc_full[acc], acc_phase, p.err) && !*abort_flag;
+            if (lane == 0) ok = mbar_wait_or_abort(&acc_full[acc], acc_phase, p.err, abort_flag);
             ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
             if (!ok) break;
             tc_fence_after();
@@ -860,7 +859,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_pair(const __grid_consta
             for (int tile = unit; tile < n_tiles && ok; tile += n_units) {
                 const Tile t = tile_at<256, 256>(p, tile, n_tiles, kblocks);
                 for (int kb = 0; kb < kblocks; ++kb) {
-                    if (!mbar_wait(&empty[stage], phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                    if (!mbar_wait_or_abort(&empty[stage], phase ^ 1u, p.err, abort_flag)) { ok = false; break; }
                     unsigned char* sa = smem + stage * kPairStage;
                     unsigned char* sb = sa + kPairHalf;
                     const uint32_t bar = mapa_shared(&full[stage], 0);
@@ -889,18 +888,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_pair(const __grid_consta
             uint32_t acc_phase = 0;
             bool ok = true;
             for (int tile = unit; tile < n_tiles && ok; tile += n_units) {
-                if (!mbar_wait(&acc_empty[acc], acc_phase ^ 1u, p.err) || *abort_flag) { ok = false; break; }
+                if (!mbar_wait_or_abort(&acc_empty[acc], acc_phase ^ 1u, p.err, abort_flag)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 256);
                 for (int kb = 0; kb < kblocks; ++kb) {
-                    if (!mbar_wait(&full[stage], phase, p.err) || *abort_flag) { ok = false; break; }
+                    if (!mbar_wait_or_abort(&full[stage], phase, p.err, abort_flag)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t a_addr = smem_u32(smem + stage * kPairStage);
                     const uint32_t b_addr = a_addr + kPairHalf;
+                    const uint64_t ad = smem_desc_sw128(a_addr), bd = smem_desc_sw128(b_addr);
 #pragma unroll
                     for (int kk = 0; kk < kBK / kUmmaK; ++kk)
-                        mma_bf16_pair(d_tmem, smem_desc_sw128(a_addr + kk * kUmmaK * 2),
-                                      smem_desc_sw128(b_addr + kk * kUmmaK * 2), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                        mma_bf16_pair(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
                     mma_commit_pair(&empty[stage]);      // both CTAs may refill this stage
                     if (++stage == kPairStages) { stage = 0; phase ^= 1u; }
                 }
@@ -923,7 +922,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_pair(const __grid_consta
             const Tile t = tile_at<256, 256>(p, tile, n_tiles, kblocks);
             const float gh = wide_row_ghat<EPI>(p, t, row_base + lane);
             bool ok = true;
-            if (lane == 0) ok = mbar_wait(&acc_full[acc], acc_phase, p.err) && !*abort_flag;
+            if (lane == 0) ok = mbar_wait_or_abort(&acc_full[acc], acc_phase, p.err, abort_flag);
             ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
             if (!ok) break;
             tc_fence_after();
