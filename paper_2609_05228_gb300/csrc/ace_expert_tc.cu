@@ -61,6 +61,7 @@ struct TcParams {
     long long split_stride;
     const float* ghat;                  // [T*k] g_hat by slot (GEMM 2 reads ghat[perm[r]])
     int k;
+    const __nv_bfloat16* h_src;         // GEMM 1 of a prefill batch: h [T, K], rows gathered by the kernel
 };
 
 // ---------------------------------------------------------------- CTA-pair (cta_group::2) helpers
@@ -273,10 +274,27 @@ struct TcCfg {
     static constexpr int TMEM_COLS = (2 * ACC_COLS) < 32 ? 32 : 2 * ACC_COLS;
     static constexpr int STG_BYTES = (!SWAP && EPI == 1) ? 4 * 4096 : 0;   // EPI 1 staging, 4 KB per warp
     static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/ + STG_BYTES;
+    // GEMM 1 of a prefill batch gathers its token rows itself: four more
+    // warps copy them from h with 16-byte cp.async (no h_perm round trip)
+    static constexpr bool GATHER = !SWAP && EPI == 0;
+    static constexpr int THREADS = GATHER ? kThreads + 32 * 4 : kThreads;
 };
+constexpr int kGatherWarp0 = kThreads / 32;      // first token-gather warp (warps 6..9)
+
+// 16-byte copy global -> shared through the L2 (cp.async.cg); src_bytes 0
+// writes zeros without reading.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+
+// Arrives on `bar` once this thread's earlier cp.async copies have landed
+// (the barrier's expected count includes this arrival).
+__device__ __forceinline__ void cp_async_arrive_noinc(uint64_t* bar) {
+    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
 
 template <bool SWAP, int EPI, int STAGES>
-__global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant__ TcParams p) {
+__global__ void __launch_bounds__(TcCfg<SWAP, EPI, STAGES>::THREADS, 1) k_expert_tc(const __grid_constant__ TcParams p) {
     using C = TcCfg<SWAP, EPI, STAGES>;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -297,7 +315,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
-            mbar_init(&full[s], 1);
+            mbar_init(&full[s], C::GATHER ? 1 + 128 : 1);     // + one arrival per gather thread
             mbar_init(&empty[s], 1);
         }
         for (int a = 0; a < 2; ++a) {
@@ -338,7 +356,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                 unsigned char* sa = smem + stage * C::STAGE_BYTES;
                 unsigned char* sb = sa + C::A_BYTES;
                 if (lane == 0) {
-                    mbar_expect_tx(&full[stage], C::STAGE_BYTES);
+                    // the gather threads' copies complete on this barrier by their own arrivals
+                    mbar_expect_tx(&full[stage], C::GATHER ? C::B_BYTES : C::STAGE_BYTES);
                     const int kx = (t.kb0 + kb) * kBK;
                     if (SWAP) {
                         if (p.w_tiles_hbm)
@@ -348,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                             tma_load_2d(sa, &p.tm_w, &full[stage], kx, t.wrow0);
                         tma_load_2d(sb, &p.tm_tok, &full[stage], kx, t.row0);
                     } else {
-                        tma_load_2d(sa, &p.tm_tok, &full[stage], kx, t.row0);
+                        if (!C::GATHER) tma_load_2d(sa, &p.tm_tok, &full[stage], kx, t.row0);
                         if (p.w_tiles_hbm) {
                             const unsigned char* wt0 =
                                 p.w_tiles_hbm + (((size_t)t.e * (p.w_rows / 128) + 2 * t.wt) * p.w_kb + (t.kb0 + kb)) * 16384;
@@ -386,6 +405,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * C::ACC_COLS);
                 for (int kb = 0; kb < kblocks; ++kb) {
                     if (!mbar_wait_or_abort(&full[stage], phase, p.err, abort_flag)) { ok = false; break; }
+                    // gathered rows were written by cp.async (generic proxy); the MMA reads
+                    // them through the async proxy
+                    if (C::GATHER) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                     tc_fence_after();
                     const uint32_t a_addr = smem_u32(smem + stage * C::STAGE_BYTES);
                     const uint32_t b_addr = a_addr + C::A_BYTES;
@@ -403,6 +425,45 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_tc(const __grid_constant
                 if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
             }
             if (!ok) *abort_flag = 1;
+        }
+    } else if (warp >= kGatherWarp0) {
+        // ------------------------------------------------ token-row gather (GATHER: warps 6..9)
+        // Thread g * 8 + c copies 16-byte chunk c of tile rows g, g + 16, ..., g + 112 for each
+        // K block, into the 128-byte-swizzled layout the TMA would write (row r at 128 r, chunk
+        // c at chunk c ^ (r & 7)); rows past the tile's end are zero-filled.
+        if (C::GATHER) {
+            const int gt = threadIdx.x - 32 * kGatherWarp0;
+            const int c = gt & 7, g = gt >> 3;
+            const uint32_t cx = (uint32_t)((c ^ (g & 7)) << 4);
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+                const Tile t = tile_at<C::TOKTILE, C::WTILE>(p, tile, n_base, kblocks);
+                const __nv_bfloat16* src[8];
+                uint32_t nb[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const int row = g + 16 * j;
+                    const bool in = row < t.nrows;
+                    const int tok = in ? p.perm[t.row0 + row] / p.k : 0;
+                    src[j] = p.h_src + (size_t)tok * p.K + c * 8;
+                    nb[j] = in ? 16u : 0u;
+                }
+                for (int kb = 0; kb < kblocks; ++kb) {
+                    int go = 1;
+                    if (lane == 0) go = mbar_wait_or_abort(&empty[stage], phase ^ 1u, p.err, abort_flag);
+                    if (!__shfl_sync(0xffffffffu, go, 0)) { ok = false; break; }
+                    const uint32_t sa = smem_u32(smem + stage * C::STAGE_BYTES) + (uint32_t)g * 128u + cx;
+                    const int kx = (t.kb0 + kb) * kBK;
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) cp_async16(sa + (uint32_t)j * 2048u, src[j] + kx, nb[j]);
+                    cp_async_arrive_noinc(&full[stage]);
+                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                }
+            }
+            if (!ok) *abort_flag = 1;
+            asm volatile("cp.async.wait_all;" ::: "memory");    // no copy in flight at exit
         }
     } else {
         // ------------------------------------------------ epilogue (warps 2..5)
@@ -1219,7 +1280,8 @@ cudaError_t set_attr() {
 template <bool SWAP, int EPI>
 cudaError_t launch_gemm(const ace_layer* L, const TcParams& p, cudaStream_t s) {
     constexpr int S = stages_for<SWAP, EPI>();
-    return launch_pdl(k_expert_tc<SWAP, EPI, S>, dim3(L->num_sms), dim3(kThreads), TcCfg<SWAP, EPI, S>::SMEM, s, p);
+    return launch_pdl(k_expert_tc<SWAP, EPI, S>, dim3(L->num_sms), dim3(TcCfg<SWAP, EPI, S>::THREADS),
+                      TcCfg<SWAP, EPI, S>::SMEM, s, p);
 }
 
 // Expert weights as tiles in HBM: block (e, t, kb) holds weight rows
@@ -1379,9 +1441,10 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     const int d = D.hidden, m = D.ffn, k = D.top_k;
     const bool small = T <= kTcSmallT;
     cudaError_t e = cudaSuccess;
-    // token rows in expert-grouped order for GEMM 1's TMA tiles (16 or 128 rows);
-    // loading them one row per TMA box from h instead measured slower
-    {
+    // token rows in expert-grouped order for GEMM 1's TMA tiles (16 or 256-row pair
+    // tiles); loading them one row per TMA box from h instead measured slower. The
+    // single-CTA prefill GEMM 1 gathers its rows itself.
+    if (small || pair) {
         e = launch_pdl(k_gather_rows, dim3(L->num_sms * 4), dim3(256), 0, s, (const __nv_bfloat16*)W.h,
                        (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k,
                        small ? W.dec_done : (int*)nullptr, T * k, W.err);
@@ -1440,6 +1503,7 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     p1.ghat = W.ghat;
     p1.k = k;
     p1.out = W.act_bf16;
+    p1.h_src = static_cast<const __nv_bfloat16*>(W.h);
     p1.K = d;
     p1.w_rows = 2 * m;
     p1.w_tiles = 2 * m / (small ? 128 : 256);
