@@ -541,7 +541,7 @@ ace_status forward_impl(ace_layer* L, const void* x, void* out, int T, ace_skip_
     }
     L->n_stages = ev ? ace::kNumStages : 0;
     L->last_launches = (small ? 1 : (h_ready ? 1 : 2) + ace::route_launch_count(L, T, ctl)) +
-                       (L->tc ? (small ? 3 : 4) : 3);
+                       (L->tc ? (small ? 2 : (ace::tc_use_pair(L, T, ctl) ? 4 : 3)) : 3);
     return ACE_OK;
 }
 

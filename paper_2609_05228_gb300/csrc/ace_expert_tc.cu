@@ -606,9 +606,10 @@ struct DecParams {
     const float* ghat;
     __nv_bfloat16* act;                 // [R, m]
     float* y;                           // [R, d]
-    int* done;                          // [token tiles] gate/up epilogue warps finished (zeroed by the gather)
+    int* done;                          // [token tiles] gate/up epilogue warps finished (zeroed by the routing)
     int* err;
     int d, m, k;
+    const __nv_bfloat16* h;             // [T, d] normalised rows: gate/up token rows are gathered from here
     long long ready_spin;               // bound (SM clock cycles) on the wait for a token tile's act rows
     int ready_extra;                    // added to that wait's target: 0, or unreachable (a test of the bound)
 };
@@ -623,6 +624,10 @@ struct DecParams {
 // the HBM bandwidth.
 template <int KBS>
 struct DecCfg {
+    // warps 0-5 as in k_expert_tc; warps 6-9 gather the gate/up tiles' token
+    // rows from h with cp.async (one 16-byte chunk of each row per thread and
+    // K block) and arrive on every stage's full barrier
+    static constexpr int THREADS = kThreads + 32 * 4;
     static constexpr int STAGES = KBS == 1 ? 8 : 6;
     static constexpr int A = KBS * 128 * kBK * 2;             // weight tiles
     static constexpr int B1 = 16 * kBK * 2;                   // one token box (16 rows x 64 bf16)
@@ -673,7 +678,7 @@ __device__ __forceinline__ DecTile dec_tile(const DecParams& p, int tile, int n1
 }
 
 template <int KBS>
-__global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_constant__ DecParams p) {
+__global__ void __launch_bounds__(DecCfg<KBS>::THREADS, 1) k_expert_decode(const __grid_constant__ DecParams p) {
     using C = DecCfg<KBS>;
     constexpr int kDecStages = C::STAGES, kDecStage = C::STAGE, kDecA = C::A;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -689,7 +694,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_h)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_act)) : "memory");
         for (int s = 0; s < kDecStages; ++s) {
-            mbar_init(&full[s], 1);
+            mbar_init(&full[s], 1 + 128);           // the producer's arrival + one per gather thread
             mbar_init(&empty[s], 1);
         }
         for (int a = 0; a < 2; ++a) {
@@ -743,13 +748,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
                 for (int kb = 0; kb < t.kblocks; kb += KBS) {
                     if (!mbar_wait_or_abort(&empty[stage], phase ^ 1u, p.err, abort_flag)) { ok = false; break; }
                     unsigned char* sa = smem + stage * kDecStage;
-                    mbar_expect_tx(&full[stage], kDecStage);
+                    // gate/up: the gather warps copy the token rows (their own arrivals)
+                    mbar_expect_tx(&full[stage], t.phase == 0 ? kDecA : kDecStage);
                     bulk_g2s(sa, wbase + (((size_t)t.e * (wrows / 128) + t.wt) * t.kblocks + kb) * 16384,
                              KBS * 16384, &full[stage]);
+                    if (t.phase == 1) {
 #pragma unroll
-                    for (int j = 0; j < KBS; ++j)
-                        tma_load_2d(sa + kDecA + j * C::B1, t.phase == 0 ? &p.tm_h : &p.tm_act, &full[stage],
-                                    (kb + j) * kBK, t.row0);
+                        for (int j = 0; j < KBS; ++j)
+                            tma_load_2d(sa + kDecA + j * C::B1, &p.tm_act, &full[stage], (kb + j) * kBK, t.row0);
+                    }
                     ++issued;
                     if (++stage == kDecStages) { stage = 0; phase ^= 1u; }
                 }
@@ -777,6 +784,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 16);
                 for (int kb = 0; kb < t.kblocks; kb += KBS) {
                     if (!mbar_wait_or_abort(&full[stage], phase, p.err, abort_flag)) { ok = false; break; }
+                    // gathered token rows were written by cp.async (generic proxy)
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                     tc_fence_after();
                     const uint32_t s_addr = smem_u32(smem + stage * kDecStage);
 #pragma unroll
@@ -797,6 +806,38 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_decode(const __grid_cons
             }
             if (!ok) *abort_flag = 1;
         }
+    } else if (warp >= kGatherWarp0) {
+        // ------------------------------------------------ token-row gather (warps 6..9)
+        // Gate/up tiles: thread r * 8 + c copies chunk c of token row r (r < 16) of each K
+        // block into the stage's token box, in the 128-byte-swizzled layout the TMA would
+        // write; rows past the tile's end are zero-filled. Down tiles (act rows by TMA): the
+        // threads only arrive, after the stage's slot is free, so every phase of the full
+        // barrier gets its 128 arrivals.
+        const int gt = threadIdx.x - 32 * kGatherWarp0;
+        const int r = gt >> 3, c = gt & 7;
+        const uint32_t off = (uint32_t)r * 128u + (uint32_t)((c ^ (r & 7)) << 4);
+        int stage = 0;
+        uint32_t phase = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+            const DecTile t = dec_tile(p, tile, n1);
+            const bool in = t.phase == 0 && r < t.nrows;
+            const __nv_bfloat16* src = p.h + (size_t)(in ? p.perm[t.row0 + r] / p.k : 0) * p.d + c * 8;
+            for (int kb = 0; kb < t.kblocks; kb += KBS) {
+                int go = 1;
+                if (lane == 0) go = mbar_wait_or_abort(&empty[stage], phase ^ 1u, p.err, abort_flag);
+                if (!__shfl_sync(0xffffffffu, go, 0)) { ok = false; break; }
+                if (t.phase == 0) {
+                    const uint32_t sb = smem_u32(smem + stage * kDecStage + kDecA) + off;
+#pragma unroll
+                    for (int j = 0; j < KBS; ++j) cp_async16(sb + j * C::B1, src + (kb + j) * kBK, in ? 16u : 0u);
+                }
+                cp_async_arrive_noinc(&full[stage]);
+                if (++stage == kDecStages) { stage = 0; phase ^= 1u; }
+            }
+        }
+        if (!ok) *abort_flag = 1;
+        asm volatile("cp.async.wait_all;" ::: "memory");    // no copy in flight at exit
     } else {
         // ------------------------------------------------ epilogue (warps 2..5)
         const int quad = warp & 3;
@@ -1441,13 +1482,12 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     const int d = D.hidden, m = D.ffn, k = D.top_k;
     const bool small = T <= kTcSmallT;
     cudaError_t e = cudaSuccess;
-    // token rows in expert-grouped order for GEMM 1's TMA tiles (16 or 256-row pair
-    // tiles); loading them one row per TMA box from h instead measured slower. The
-    // single-CTA prefill GEMM 1 gathers its rows itself.
-    if (small || pair) {
+    // token rows in expert-grouped order for the CTA-pair GEMM 1's 256-row TMA tiles;
+    // the decode kernel and the single-CTA prefill GEMM 1 gather their rows themselves
+    if (pair) {
         e = launch_pdl(k_gather_rows, dim3(L->num_sms * 4), dim3(256), 0, s, (const __nv_bfloat16*)W.h,
                        (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k,
-                       small ? W.dec_done : (int*)nullptr, T * k, W.err);
+                       (int*)nullptr, T * k, W.err);
         if (e != cudaSuccess) return e;
     }
     if (small) {
@@ -1465,6 +1505,7 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
         q.act = static_cast<__nv_bfloat16*>(W.act_bf16);
         q.y = W.yslot;
         q.done = W.dec_done;
+        q.h = static_cast<const __nv_bfloat16*>(W.h);
         q.err = W.err;
         q.d = d;
         q.m = m;
@@ -1473,8 +1514,8 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
         q.ready_extra = L->dbg_ready_spin > 0 ? (1 << 30) : 0;
         // K blocks are even: d is a multiple of 256 and m of 128 on this path
         e = T <= kDecWideStageTokens
-                ? launch_pdl(k_expert_decode<2>, dim3(L->num_sms), dim3(kThreads), DecCfg<2>::SMEM, s, q)
-                : launch_pdl(k_expert_decode<1>, dim3(L->num_sms), dim3(kThreads), DecCfg<1>::SMEM, s, q);
+                ? launch_pdl(k_expert_decode<2>, dim3(L->num_sms), dim3(DecCfg<2>::THREADS), DecCfg<2>::SMEM, s, q)
+                : launch_pdl(k_expert_decode<1>, dim3(L->num_sms), dim3(DecCfg<1>::THREADS), DecCfg<1>::SMEM, s, q);
         if (e != cudaSuccess) return e;
         if (ev) {                           // gate/up and down share one launch: the down stage reads 0
             ace::record_stage(ev[1], s);

@@ -1027,6 +1027,7 @@ struct FusedArgs {
     int32_t* tile_cnt;
     const uint8_t* pf_base;     // expert weights to start pulling into L2 while routing runs
     long long pf_bytes;         // (a multiple of 256 bytes; 0 = none)
+    int* dec_done;              // the decode expert kernel's per-token-tile counters, zeroed here (or nullptr)
 };
 
 __host__ __device__ inline size_t fused_phase_c_bytes(int T, int k, int n_exp) {
@@ -1295,6 +1296,8 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
     __syncthreads();
     scan_counts_block(cnt, n_exp, a.offsets, a.dlist, a.meta, off_s, a.tok_tile, a.tt_off, S.hist);
     __syncthreads();
+    if (a.dec_done)                       // the decode expert kernel counts up from zero
+        for (int i = threadIdx.x; i < a.meta[kMetaTokTiles]; i += blockDim.x) a.dec_done[i] = 0;
     fill_tile_table(a.offsets, a.dlist, a.tt_off, a.meta, a.tok_tile, a.tt_tab, n_exp, a.tt_cap, a.err);
     for (int s = threadIdx.x; s < ns; s += blockDim.x) {
         if (skip_s[s]) { a.slot_pos[s] = -1; continue; }
@@ -1443,6 +1446,7 @@ cudaError_t launch_route_fused(const ace_layer* L, const void* x, const float* l
     a.tt_tab = W.tt_tab;
     a.tt_cap = L->tt_cap;
     a.tile_cnt = W.tile_cnt;
+    if (x && L->tc) a.dec_done = W.dec_done;
     if (x && L->tc && L->w_gu) {
         const long long gu_bytes = 2LL * D.ffn * D.hidden * 2 * D.n_experts;
         const long long want = kRoutePrefetchBytes;
