@@ -19,9 +19,15 @@
 // Warp roles (192 threads): warp 0 issues TMA loads into a STAGES-deep ring,
 // warp 1 owns TMEM and issues the MMAs (one thread), warps 2..5 run the
 // epilogue from TMEM (each warp reads its 32-lane quadrant). Two accumulator
-// buffers let the epilogue of one tile overlap the MMAs of the next. Every
-// mbarrier wait is bounded; on expiry the kernel sets kErrTimeout, stops
-// issuing work and releases TMEM before returning.
+// buffers let the epilogue of one tile overlap the MMAs of the next. GEMM 1
+// of a prefill batch on one CTA per tile and the decode kernel have four more
+// warps (320 threads) that gather their token rows from h with 16-byte
+// cp.async straight into the stage, so no permuted copy of h is written and
+// read back; the CTA-pair GEMM 1 still loads rows gathered by k_gather_rows
+// (gathering there was measured 2x slower: the partner CTA's rows need a
+// relayed arrival per stage). Every mbarrier wait is bounded; on expiry the
+// kernel sets kErrTimeout, stops issuing work and releases TMEM before
+// returning.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <math.h>
@@ -596,7 +602,6 @@ __global__ void __launch_bounds__(TcCfg<SWAP, EPI, STAGES>::THREADS, 1) k_expert
 // its tiles in index order and issues all its gate/up tiles before any down
 // tile can wait, so the waits cannot form a cycle.
 struct DecParams {
-    CUtensorMap tm_h;                   // h_perm rows, 16-row boxes
     CUtensorMap tm_act;                 // act rows, 16-row boxes
     const uint8_t* w_gu;                // tiled W_gu
     const uint8_t* w_down;              // tiled W_down
@@ -691,7 +696,6 @@ __global__ void __launch_bounds__(DecCfg<KBS>::THREADS, 1) k_expert_decode(const
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
-        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_h)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_act)) : "memory");
         for (int s = 0; s < kDecStages; ++s) {
             mbar_init(&full[s], 1 + 128);           // the producer's arrival + one per gather thread
@@ -1054,11 +1058,8 @@ __global__ void __launch_bounds__(256) k_gather_rows(const __nv_bfloat16* __rest
                                                      const int32_t* __restrict__ perm,
                                                      const int32_t* __restrict__ meta,
                                                      __nv_bfloat16* __restrict__ h_perm,
-                                                     int d, int k, int* __restrict__ done, int n_slots,
-                                                     int* __restrict__ err) {
+                                                     int d, int k, int n_slots, int* __restrict__ err) {
     pdl_wait();
-    if (done && blockIdx.x == 0)                 // the decode kernel's per-token-tile counters
-        for (int i = threadIdx.x; i < meta[kMetaTokTiles]; i += blockDim.x) done[i] = 0;
     const int R = meta[kMetaRetained];
     const int nvec = d / 8;
     const int lane = threadIdx.x & 31;
@@ -1487,14 +1488,13 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
     if (pair) {
         e = launch_pdl(k_gather_rows, dim3(L->num_sms * 4), dim3(256), 0, s, (const __nv_bfloat16*)W.h,
                        (const int32_t*)W.perm, (const int32_t*)W.meta, (__nv_bfloat16*)W.h_perm, d, k,
-                       (int*)nullptr, T * k, W.err);
+                       T * k, W.err);
         if (e != cudaSuccess) return e;
     }
     if (small) {
         // both GEMMs in one persistent launch (k_expert_decode), then the combine
         if (ev) ace::record_stage(ev[0], s);
         DecParams q{};
-        q.tm_h = L->tcm.tok1_small;
         q.tm_act = L->tcm.tok2_small;
         q.w_gu = static_cast<const uint8_t*>(L->w_gu);
         q.w_down = static_cast<const uint8_t*>(L->w_down);
