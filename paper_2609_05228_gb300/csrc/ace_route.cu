@@ -465,6 +465,38 @@ __device__ float block_select_tau(const uint32_t* keys, int n, int m, SelectSmem
     return tau;
 }
 
+// The same threshold for at most blockDim.x keys, by counting ranks: key i
+// (not protected) is v when lt_i <= m < le_i, with lt_i = #{keys < key i} and
+// le_i = #{keys <= key i} (a protected 0xffffffff key is above every
+// candidate, so it counts in neither); then lo = lt_i and hi = le_i. One pass
+// over the keys and one barrier, against the radix select's four passes of
+// five barriers each: faster up to about 128 keys. The caller sets S.prefix /
+// S.below / S.last_cnt beforehand and synchronises (the values stay if no key
+// qualifies, which 0 < m < #candidates rules out).
+template <int NW>
+__device__ float block_select_tau_rank(const uint32_t* keys, int n, int m, SelectSmem<NW>& S) {
+    const int i = threadIdx.x;
+    const uint32_t ki = i < n ? keys[i] : 0xffffffffu;
+    int lt = 0, le = 0;
+#pragma unroll 8
+    for (int j = 0; j < n; ++j) {
+        const uint32_t kj = keys[j];
+        lt += kj < ki;
+        le += kj <= ki;
+    }
+    if (ki != 0xffffffffu && lt <= m && m < le) {
+        S.prefix = ki;
+        S.below = lt;
+        S.last_cnt = le - lt;
+    }
+    __syncthreads();
+    const uint32_t v = S.prefix;
+    const int lo = S.below, hi = S.below + S.last_cnt;
+    float tau = __uint_as_float(v);
+    if (!(lo == m || (m - lo) <= (hi - m))) tau = __uint_as_float(v + 1u);
+    return tau;
+}
+
 // Exclusive scan of cnt[0..n_exp) by the whole block (called by every
 // thread; blockDim.x a multiple of 32, at most 1024): offsets[e],
 // offsets[n_exp] = total, the distinct-expert list (increasing) and the meta
@@ -986,6 +1018,7 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
 constexpr int kFuseTok = 8;
 constexpr int kFuseWarps = 8;
 constexpr int kRowPad = 16;    // bytes appended to each row staged by phase A
+constexpr int kRankSelectMax = 128;   // slots up to which phase C counts ranks instead of a radix select
 static_assert(kFuseTok == 8 && kFuseWarps == 8, "phase A's MMA takes 8 token rows x 8 router rows");
 constexpr long long kRoutePrefetchBytes = 48LL << 20;   // decode: leading W_gu bytes pulled towards L2 while routing
 
@@ -1040,10 +1073,38 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ SelectSmem<kFuseWarps> S;
     __shared__ int s_last;
+    __shared__ float s_tab[LOGITS ? 2 * kMaxExperts : 1];   // the layer's GSP / RCR tables (phase B)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int t0 = blockIdx.x * kFuseTok;
     const int nt = min(kFuseTok, a.n_tokens - t0);
     const int n_exp = a.n_exp, k = a.k;
+    // the expert kernel may launch now: its prologue (TMEM, barriers) overlaps the
+    // routing, and it reads nothing of ours before its griddepcontrol.wait
+    pdl_trigger();
+    // one token tile: phases B and C run in the same block, which hands phase B's
+    // results to phase C in shared memory (no fence, ticket or reload)
+    const bool solo = gridDim.x == 1;
+    const float* tab_gsp = a.a_gsp;
+    const float* tab_rcr = a.a_rcr;
+    if (LOGITS) {
+        // A layer's tables were written when it was created: every block copies them
+        // into shared memory before the dependency wait, so that phase B (whichever
+        // block runs it) reads its experts' entries without a dependent global load.
+        for (int i = threadIdx.x; i < n_exp; i += blockDim.x) {
+            s_tab[i] = __ldg(a.a_gsp + i);
+            s_tab[kMaxExperts + i] = __ldg(a.a_rcr + i);
+        }
+        tab_gsp = s_tab;
+        tab_rcr = s_tab + kMaxExperts;
+    } else if (blockIdx.y == 0) {
+        // caller-owned tables (read after the wait): pull their lines towards L2
+        const int lines = (n_exp + 31) / 32;
+        if ((int)threadIdx.x < 2 * lines) {
+            const float* tab = (int)threadIdx.x < lines ? a.a_gsp : a.a_rcr;
+            const int l = (int)threadIdx.x % lines;
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(tab + min(l * 32, n_exp - 1)) : "memory");
+        }
+    }
     if (LOGITS) {
         // ---------------- phase A: RMSNorm + logits for 8 tokens x 8 experts.
         // Warp 0 bulk-copies gamma and the block's 8 router rows (layer
@@ -1064,6 +1125,11 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         float* red = reinterpret_cast<float*>(wsm + (size_t)kFuseWarps * rs);   // [warps][8][8] partial logits
         const int e0 = blockIdx.y * kFuseWarps;
         const int ne = min(kFuseWarps, n_exp - e0);
+        const bool mma_path = sizeof(T) == 2 && d % (16 * kFuseWarps) == 0;
+        // the router bias of this thread's output column (MMA path: column tid & 7 of
+        // the 8 x 8 block; FMA path: the warp's expert), read before the dependency wait
+        const int bj = mma_path ? (int)(threadIdx.x & 7) : warp;
+        const float bias = bj < ne ? __ldg(a.b_r + e0 + bj) : 0.f;
         if (threadIdx.x == 0) {
             mbar_init(bar, 1);
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -1117,7 +1183,7 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         }
         __syncthreads();
         if (threadIdx.x == 0) mbar_inval(bar);
-        if (sizeof(T) == 2 && d % (16 * kFuseWarps) == 0) {
+        if (mma_path) {
             // bf16: warp w takes K slice w and runs mma.sync m16n8k16 over it
             // (A = the 8 token rows, zero-padded to 16; B = the 8 router rows;
             // products exact, fp32 accumulation); the 8 partial 8 x 8 blocks
@@ -1150,7 +1216,7 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
 #pragma unroll
                 for (int w = 0; w < kFuseWarps; ++w) v += red[(w * 8 + r) * 8 + j];
                 if (r < nt && j < ne) {
-                    v = v + a.b_r[e0 + j];
+                    v = v + bias;
                     if (a.use_temp) v = v * a.inv_temp;
                     a.logits[(size_t)(t0 + r) * n_exp + e0 + j] = v;
                 }
@@ -1179,7 +1245,7 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
                 float v = acc[0];
 #pragma unroll
                 for (int r = 1; r < kFuseTok; ++r) if (lane == r) v = acc[r];
-                v = v + a.b_r[e];
+                v = v + bias;
                 if (a.use_temp) v = v * a.inv_temp;
                 a.logits[(size_t)(t0 + lane) * n_exp + e] = v;
             }
@@ -1210,6 +1276,18 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
     } else {
         pdl_wait();                                               // logits are the predecessor's output
     }
+    // phase C's shared arrays (over phase A's staging rows, which no warp reads past the
+    // ticket's barrier)
+    const int n_tokens = a.n_tokens;
+    const int ns = n_tokens * k;
+    float* g_s = reinterpret_cast<float*>(smem_raw + 16);
+    float* c_s = g_s + ns;
+    uint32_t* key_s = reinterpret_cast<uint32_t*>(c_s + ns);
+    int* id_s = reinterpret_cast<int*>(key_s + ns);
+    int* cnt = id_s + ns;                                            // [n_exp]
+    int* off_s = cnt + n_exp;                                        // [n_exp + 1]
+    uint32_t* bm = reinterpret_cast<uint32_t*>(off_s + n_exp + 1);   // [n_exp * 8]
+    uint8_t* skip_s = reinterpret_cast<uint8_t*>(bm + n_exp * 8);    // [ns]
     // ---------------- phase B: top-k, gates, c for this token tile
     const bool ratio = a.mode == ACE_SKIP_RATIO;
     for (int r = warp; r < nt; r += kFuseWarps) {
@@ -1221,12 +1299,17 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
         if (lane < k && !ACE_IDX_OK((unsigned)id < (unsigned)n_exp, a.err)) id = 0;
         const float z0 = __shfl_sync(0xffffffffu, zv, 0);
         if (__any_sync(0xffffffffu, nan) && lane == 0) atomicOr(a.err, kErrNumeric);
-        const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, a.a_gsp, a.a_rcr, a.eps, a.fusion);
+        const SlotScore sc = score_slot(lane, k, zv, z0, lane < k ? id : 0, tab_gsp, tab_rcr, a.eps, a.fusion);
         const size_t base = (size_t)t * k;
         if (lane < k) {
             a.ids[base + lane] = id;
             a.gates[base + lane] = sc.g;
             a.cval[base + lane] = sc.c;
+            if (solo) {
+                id_s[base + lane] = id;
+                g_s[base + lane] = sc.g;
+                c_s[base + lane] = sc.c;
+            }
         }
         if (!ratio) {
             bool sk;
@@ -1235,47 +1318,52 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
             if (lane < k) {
                 a.skip[base + lane] = sk ? 1 : 0;
                 a.ghat[base + lane] = gh;
+                if (solo) skip_s[base + lane] = sk ? 1 : 0;
             }
         } else {
             const bool prot = slot_protected(lane, k, sc.c, a.m_min);
-            if (lane < k) a.keys[base + lane] = prot ? 0xffffffffu : __float_as_uint(sc.c);
+            const uint32_t key = prot ? 0xffffffffu : __float_as_uint(sc.c);
+            if (lane < k) {
+                a.keys[base + lane] = key;
+                if (solo) key_s[base + lane] = key;
+            }
         }
     }
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        s_last = atomicAdd(&a.meta[kMetaTicket2], 1) == (int)gridDim.x - 1;
-        if (s_last) a.meta[kMetaTicket2] = 0;
+    if (!solo) {
+        __threadfence();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            s_last = atomicAdd(&a.meta[kMetaTicket2], 1) == (int)gridDim.x - 1;
+            if (s_last) a.meta[kMetaTicket2] = 0;
+        }
+        __syncthreads();
+        if (!s_last) return;
+        __threadfence();
     }
-    __syncthreads();
-    if (!s_last) return;
-    __threadfence();
     // ---------------- phase C: threshold, decision, compaction (all tokens)
-    const int n_tokens = a.n_tokens;
-    const int ns = n_tokens * k;
-    float* g_s = reinterpret_cast<float*>(smem_raw + 16);
-    float* c_s = g_s + ns;
-    uint32_t* key_s = reinterpret_cast<uint32_t*>(c_s + ns);
-    int* id_s = reinterpret_cast<int*>(key_s + ns);
-    int* cnt = id_s + ns;                                            // [n_exp]
-    int* off_s = cnt + n_exp;                                        // [n_exp + 1]
-    uint32_t* bm = reinterpret_cast<uint32_t*>(off_s + n_exp + 1);   // [n_exp * 8]
-    uint8_t* skip_s = reinterpret_cast<uint8_t*>(bm + n_exp * 8);    // [ns]
     for (int i = threadIdx.x; i < n_exp; i += blockDim.x) cnt[i] = 0;
     for (int i = threadIdx.x; i < n_exp * 8; i += blockDim.x) bm[i] = 0u;
-    for (int i = threadIdx.x; i < ns; i += blockDim.x) {
-        id_s[i] = __ldcg(a.ids + i);
-        if (ratio) {
-            g_s[i] = __ldcg(a.gates + i);
-            c_s[i] = __ldcg(a.cval + i);
-            key_s[i] = __ldcg(a.keys + i);
-        } else {
-            skip_s[i] = __ldcg(a.skip + i);
+    if (!solo) {
+        for (int i = threadIdx.x; i < ns; i += blockDim.x) {
+            id_s[i] = __ldcg(a.ids + i);
+            if (ratio) {
+                g_s[i] = __ldcg(a.gates + i);
+                c_s[i] = __ldcg(a.cval + i);
+                key_s[i] = __ldcg(a.keys + i);
+            } else {
+                skip_s[i] = __ldcg(a.skip + i);
+            }
         }
+    }
+    if (threadIdx.x == 0) {
+        S.prefix = 0u;
+        S.below = 0;
+        S.last_cnt = 0;
     }
     __syncthreads();
     if (ratio) {
-        const float tau = block_select_tau(key_s, ns, a.m_q, S);
+        const float tau = ns <= kRankSelectMax ? block_select_tau_rank(key_s, ns, a.m_q, S)
+                                               : block_select_tau(key_s, ns, a.m_q, S);
         if (threadIdx.x == 0) *a.tau_out = tau;
         for (int t = threadIdx.x; t < n_tokens; t += blockDim.x) {
             const int base = t * k;

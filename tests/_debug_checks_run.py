@@ -33,15 +33,16 @@ def host(t):
 
 def main():
     assert ace.LIBNAME == "libace_debug.so" and ace.ace_debug_checks_enabled(), "debug library not loaded"
+    # the last spec (hidden 512, 24 experts) adds a second tensor-core shape at decode batch sizes
     specs = [synth.LayerSpec(256, 20, 4, 128, dtype="bf16"), synth.LayerSpec(256, 100, 8, 128, dtype="bf16"),
-             synth.LayerSpec(256, 20, 4, 128, dtype="f32")]
+             synth.LayerSpec(256, 20, 4, 128, dtype="f32"), synth.LayerSpec(512, 24, 4, 256, dtype="bf16")]
     runs = 0
     for si, spec in enumerate(specs):
         w = synth.make_layer(spec, seed=11 + si)
         a_gsp, a_rcr = offline.tables(w)
         layer = ace.AceLayer(w, a_gsp, a_rcr, max_tokens=300)
         bf = spec.dtype == "bf16"
-        for T in (1, 3, 17, 129, 300):
+        for T in ((1, 3, 8, 9, 129) if spec.hidden == 512 else (1, 3, 17, 129, 300)):
             x = synth.make_tokens(spec, T, seed=T)
             xd = dev(x, bf)
             out = torch.empty_like(xd)

@@ -301,6 +301,8 @@ FORWARD_CASES = [
     ("qwen", 1, "ratio", 0.5), ("qwen", 1, "ratio", 0.0), ("qwen", 8, "ratio", 0.0), ("qwen", 8, "ratio", 0.25), ("qwen", 32, "ratio", 0.5),
     ("qwen", 64, "ratio", 0.0), ("qwen", 64, "ratio", 0.25), ("qwen", 64, "ratio", 0.5),
     ("qwen", 17, "threshold", 0.11), ("qwen", 129, "ratio", 0.5), ("qwen", 1000, "ratio", 0.625),
+    ("qwen", 3, "threshold", 0.11), ("qwen", 8, "ratio", 0.5), ("qwen", 9, "ratio", 0.5),   # decode stages of
+    ("qwen", 12, "ratio", 0.5),                                        # two K blocks (up to 16 tokens)
     ("qwen", 1000, "ratio", 1.0),                                      # every non-top-1 slot skipped
     ("qwen_zipf", 4096, "ratio", 0.0), ("qwen_zipf", 4096, "ratio", 0.25), ("qwen_zipf", 4096, "ratio", 0.5),
     ("qwen_zipf", 4096, "ratio", 0.625),
