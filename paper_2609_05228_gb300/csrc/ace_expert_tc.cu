@@ -595,12 +595,16 @@ __global__ void __launch_bounds__(TcCfg<SWAP, EPI, STAGES>::THREADS, 1) k_expert
 // finish their gate/up tiles start on down tiles instead of idling through
 // the tail of a separate launch. Tiles 0 .. n1-1 are gate/up (token-tile
 // major, so one token tile's gate/up tiles run together), n1 .. are down. A
-// down tile's weights load at once; its act rows load after done[tt] shows
-// that every gate/up epilogue warp of that token tile has written its act
-// columns (release: store, proxy fence, fence, atomic; acquire: bounded spin
-// on an acquiring load, then a proxy fence before the TMA). Each CTA takes
-// its tiles in index order and issues all its gate/up tiles before any down
-// tile can wait, so the waits cannot form a cycle.
+// down tile's weights and act rows load after done[tt] shows that every
+// gate/up epilogue warp of that token tile has written its act columns
+// (release: store, proxy fence, fence, atomic; acquire: bounded spin on an
+// acquiring load, then a proxy fence before the TMA). The producer takes the
+// tiles from a counter (zeroed by the routing), so CTAs that drew light tiles
+// draw more, and hands each index to the MMA, epilogue and gather warps
+// through a ring in shared memory. Tiles leave the counter in index order and
+// a CTA issues every stage of a tile before it takes the next, so a down
+// tile's wait is on gate/up tiles already taken, whose MMAs and epilogues
+// finish without their producers: the waits cannot form a cycle.
 struct DecParams {
     CUtensorMap tm_act;                 // act rows, 16-row boxes
     const uint8_t* w_gu;                // tiled W_gu
@@ -612,6 +616,7 @@ struct DecParams {
     __nv_bfloat16* act;                 // [R, m]
     float* y;                           // [R, d]
     int* done;                          // [token tiles] gate/up epilogue warps finished (zeroed by the routing)
+    int* tile_next;                     // the next tile to take (zeroed by the routing)
     int* err;
     int d, m, k;
     const __nv_bfloat16* h;             // [T, d] normalised rows: gate/up token rows are gathered from here
@@ -637,8 +642,10 @@ struct DecCfg {
     static constexpr int A = KBS * 128 * kBK * 2;             // weight tiles
     static constexpr int B1 = 16 * kBK * 2;                   // one token box (16 rows x 64 bf16)
     static constexpr int STAGE = A + KBS * B1;
-    static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
+    static constexpr int SMEM = STAGES * STAGE + 1024 + 512;
 };
+constexpr int kDecRing = 8;             // tile indices in flight from the producer to the other roles
+constexpr int kDecRingTakers = 1 + 4 + 4;   // the MMA thread, the epilogue and the gather warps
 // Decode batches that take 2 K blocks per stage: few distinct retained experts.
 constexpr int kDecWideStageTokens = 16;
 
@@ -692,8 +699,11 @@ __global__ void __launch_bounds__(DecCfg<KBS>::THREADS, 1) k_expert_decode(const
     uint64_t* empty = full + kDecStages;
     uint64_t* acc_full = empty + kDecStages;
     uint64_t* acc_empty = acc_full + 2;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+    uint64_t* ring_full = acc_empty + 2;
+    uint64_t* ring_empty = ring_full + kDecRing;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ring_empty + kDecRing);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    volatile int* ring = abort_flag + 1;        // [kDecRing] tile indices, -1 = no more
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_act)) : "memory");
@@ -704,6 +714,10 @@ __global__ void __launch_bounds__(DecCfg<KBS>::THREADS, 1) k_expert_decode(const
         for (int a = 0; a < 2; ++a) {
             mbar_init(&acc_full[a], 1);
             mbar_init(&acc_empty[a], 4);
+        }
+        for (int r = 0; r < kDecRing; ++r) {
+            mbar_init(&ring_full[r], 1);
+            mbar_init(&ring_empty[r], kDecRingTakers);
         }
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -730,7 +744,16 @@ __global__ void __launch_bounds__(DecCfg<KBS>::THREADS, 1) k_expert_decode(const
             uint32_t phase = 0;
             bool ok = true;
             long long issued = 0;
-            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+            int ri = 0;
+            uint32_t rph = 0;
+            int tile = atomicAdd(p.tile_next, 1);
+            while (ok) {
+                // hand the tile (or the end) to the other roles
+                if (!mbar_wait_or_abort(&ring_empty[ri], rph ^ 1u, p.err, abort_flag)) { ok = false; break; }
+                ring[ri] = tile < n_tiles ? tile : -1;
+                mbar_arrive(&ring_full[ri]);
+                if (++ri == kDecRing) { ri = 0; rph ^= 1u; }
+                if (tile >= n_tiles) break;
                 const DecTile t = dec_tile(p, tile, n1);
                 if (t.phase == 1) {
                     // the token tile's act rows: every gate/up epilogue warp has written
@@ -764,6 +787,9 @@ __global__ void __launch_bounds__(DecCfg<KBS>::THREADS, 1) k_expert_decode(const
                     ++issued;
                     if (++stage == kDecStages) { stage = 0; phase ^= 1u; }
                 }
+                // the next tile, taken once this one's stages are out (its latency hides
+                // behind the stages in flight)
+                if (ok) tile = atomicAdd(p.tile_next, 1);
             }
             if (!ok) {
                 *abort_flag = 1;
@@ -781,7 +807,14 @@ __global__ void __launch_bounds__(DecCfg<KBS>::THREADS, 1) k_expert_decode(const
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+            int ri = 0;
+            uint32_t rph = 0;
+            while (ok) {
+                if (!mbar_wait_or_abort(&ring_full[ri], rph, p.err, abort_flag)) { ok = false; break; }
+                const int tile = ring[ri];
+                mbar_arrive(&ring_empty[ri]);
+                if (++ri == kDecRing) { ri = 0; rph ^= 1u; }
+                if (tile < 0) break;
                 const DecTile t = dec_tile(p, tile, n1);
                 if (!mbar_wait_or_abort(&acc_empty[acc], acc_phase ^ 1u, p.err, abort_flag)) { ok = false; break; }
                 tc_fence_after();
@@ -823,7 +856,20 @@ __global__ void __launch_bounds__(DecCfg<KBS>::THREADS, 1) k_expert_decode(const
         int stage = 0;
         uint32_t phase = 0;
         bool ok = true;
-        for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+        int ri = 0;
+        uint32_t rph = 0;
+        while (ok) {
+            int tile = -1, go = 1;
+            if (lane == 0) {
+                go = mbar_wait_or_abort(&ring_full[ri], rph, p.err, abort_flag);
+                if (go) tile = ring[ri];
+            }
+            go = __shfl_sync(0xffffffffu, go, 0);
+            tile = __shfl_sync(0xffffffffu, tile, 0);
+            if (!go) { ok = false; break; }
+            if (lane == 0) mbar_arrive(&ring_empty[ri]);
+            if (++ri == kDecRing) { ri = 0; rph ^= 1u; }
+            if (tile < 0) break;
             const DecTile t = dec_tile(p, tile, n1);
             const bool in = t.phase == 0 && r < t.nrows;
             const __nv_bfloat16* src = p.h + (size_t)(in ? p.perm[t.row0 + r] / p.k : 0) * p.d + c * 8;
@@ -847,7 +893,20 @@ __global__ void __launch_bounds__(DecCfg<KBS>::THREADS, 1) k_expert_decode(const
         const int quad = warp & 3;
         int acc = 0;
         uint32_t acc_phase = 0;
-        for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+        int ri = 0;
+        uint32_t rph = 0;
+        while (true) {
+            int tile = -1, go = 1;
+            if (lane == 0) {
+                go = mbar_wait_or_abort(&ring_full[ri], rph, p.err, abort_flag);
+                if (go) tile = ring[ri];
+            }
+            go = __shfl_sync(0xffffffffu, go, 0);
+            tile = __shfl_sync(0xffffffffu, tile, 0);
+            if (!go) break;
+            if (lane == 0) mbar_arrive(&ring_empty[ri]);
+            if (++ri == kDecRing) { ri = 0; rph ^= 1u; }
+            if (tile < 0) break;
             bool ok = true;
             if (lane == 0) ok = mbar_wait_or_abort(&acc_full[acc], acc_phase, p.err, abort_flag);
             ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
@@ -1505,6 +1564,7 @@ cudaError_t launch_experts_tc(const ace_layer* L, const void* x, void* out, int 
         q.act = static_cast<__nv_bfloat16*>(W.act_bf16);
         q.y = W.yslot;
         q.done = W.dec_done;
+        q.tile_next = W.meta + kMetaDecNext;
         q.h = static_cast<const __nv_bfloat16*>(W.h);
         q.err = W.err;
         q.d = d;

@@ -37,6 +37,7 @@ enum : int {
     kMetaSelPrefix = 10,   //   first digit, as the key prefix
     kMetaSelWant = 11,     //   rank still wanted inside the first digit
     kMetaSelBelow = 12,    //   candidates below the first digit
+    kMetaDecNext = 13,     // decode expert kernel: the next tile to take (zeroed by the routing)
     kMetaCount = 16,
 };
 

@@ -1384,8 +1384,10 @@ __global__ void __launch_bounds__(kFuseWarps * 32) k_route_fused(const __grid_co
     __syncthreads();
     scan_counts_block(cnt, n_exp, a.offsets, a.dlist, a.meta, off_s, a.tok_tile, a.tt_off, S.hist);
     __syncthreads();
-    if (a.dec_done)                       // the decode expert kernel counts up from zero
+    if (a.dec_done) {                     // the decode expert kernel counts up from zero
         for (int i = threadIdx.x; i < a.meta[kMetaTokTiles]; i += blockDim.x) a.dec_done[i] = 0;
+        if (threadIdx.x == 0) a.meta[kMetaDecNext] = 0;
+    }
     fill_tile_table(a.offsets, a.dlist, a.tt_off, a.meta, a.tok_tile, a.tt_tab, n_exp, a.tt_cap, a.err);
     for (int s = threadIdx.x; s < ns; s += blockDim.x) {
         if (skip_s[s]) { a.slot_pos[s] = -1; continue; }
