@@ -1221,7 +1221,10 @@ __global__ void __launch_bounds__(256) k_combine_bf16(const Y* __restrict__ y, c
 // then adds, for lane l, the partials of chunks l, l + 32, l + 64, ... in that
 // order and reduces across lanes by the butterfly -- the order of the
 // stand-alone RMSNorm, so h_next = out / sqrt(mean(out^2) + eps) * gamma_next
-// has the same bits as that kernel applied to the output.
+// has the same bits as that kernel applied to the output. A thread's 16-byte
+// chunks of the slot rows come through shared memory by cp.async (k x d x 2
+// bytes of dynamic shared memory per block), so no registers are held per
+// load: more blocks, and so more tokens' rows, are in flight per SM.
 template <int KMAX>
 __global__ void __launch_bounds__(512) k_combine_norm(const __nv_bfloat16* __restrict__ y,
                                                       const int32_t* __restrict__ slot_pos,
@@ -1230,6 +1233,7 @@ __global__ void __launch_bounds__(512) k_combine_norm(const __nv_bfloat16* __res
                                                       const __nv_bfloat16* __restrict__ gamma_next,
                                                       __nv_bfloat16* __restrict__ h_next, float eps_next, int d,
                                                       int k, int y_rows, int* __restrict__ err) {
+    extern __shared__ __align__(16) unsigned char cn_rows[];   // [k][blockDim.x] 16-byte chunks
     __shared__ float part_s[512];
     __shared__ float inv_s;
     pdl_wait();
@@ -1240,14 +1244,21 @@ __global__ void __launch_bounds__(512) k_combine_norm(const __nv_bfloat16* __res
         r[i] = i < k ? __ldg(slot_pos + (size_t)t * k + i) : -1;
         if (!ACE_IDX_OK(r[i] >= -1 && r[i] < y_rows, err)) r[i] = -1;
     }
-    Row8<__nv_bfloat16> v[KMAX];
+    const uint32_t sb = smem_u32(cn_rows) + (uint32_t)c8 * 16u;
 #pragma unroll
     for (int i = 0; i < KMAX; ++i)
-        if (r[i] >= 0) v[i].load(y + (size_t)r[i] * d + 8 * c8);
+        if (r[i] >= 0) cp_async16(sb + (uint32_t)(i * blockDim.x) * 16u, y + (size_t)r[i] * d + 8 * c8, 16u);
+    asm volatile("cp.async.wait_all;" ::: "memory");   // each thread reads back only its own chunks
     float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int i = 0; i < KMAX; ++i)
-        if (r[i] >= 0) v[i].add_to(acc);
+        if (r[i] >= 0) {
+            float f[8];
+            Vec16<__nv_bfloat16>::to_float(
+                *reinterpret_cast<const uint4*>(cn_rows + ((size_t)i * blockDim.x + c8) * 16), f);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[j] += f[j];
+        }
     if (resid) {
         float xr[8];
         Vec16<__nv_bfloat16>::to_float(reinterpret_cast<const uint4*>(resid + (size_t)t * d)[c8], xr);
@@ -1285,7 +1296,7 @@ cudaError_t launch_combine_norm(const __nv_bfloat16* y, const int32_t* sp, const
                                 __nv_bfloat16* out, const ace_layer* next, int T, int d, int k, int y_rows, int* err,
                                 cudaStream_t s) {
     // d is a multiple of 256 (tensor-core layers) and at most 4096: d / 8 threads, whole warps
-    return launch_pdl(k_combine_norm<KMAX>, dim3(T), dim3(d / 8), 0, s, y, sp, resid, out,
+    return launch_pdl(k_combine_norm<KMAX>, dim3(T), dim3(d / 8), (size_t)k * d * 2, s, y, sp, resid, out,
                       static_cast<const __nv_bfloat16*>(next->gamma), static_cast<__nv_bfloat16*>(next->ws.h),
                       next->desc.rms_eps, d, k, y_rows, err);
 }
@@ -1476,6 +1487,11 @@ cudaError_t tc_init(ace_layer* L) {
     if ((e = max_pair_clusters((const void*)k_expert_pair<1>, &c1)) != cudaSuccess) return e;
     L->pair_clusters = c0 < c1 ? c0 : c1;
     if ((e = prefer_shared(k_gather_rows)) != cudaSuccess) return e;
+    // the stack's combine stages k slot-row chunks per thread: k x d x 2 bytes per block
+    if ((e = raise_smem_limit(k_combine_norm<8>, 8 * D.hidden * 2)) != cudaSuccess) return e;
+    if ((e = raise_smem_limit(k_combine_norm<kMaxTopK>, kMaxTopK * D.hidden * 2)) != cudaSuccess) return e;
+    if ((e = prefer_shared(k_combine_norm<8>)) != cudaSuccess) return e;
+    if ((e = prefer_shared(k_combine_norm<kMaxTopK>)) != cudaSuccess) return e;
 
     // row counts as allocated at create time (padded to at least 256 rows)
     const uint64_t rows = (uint64_t)D.max_tokens * D.top_k < 256 ? 256 : (uint64_t)D.max_tokens * D.top_k;
