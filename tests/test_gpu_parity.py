@@ -154,11 +154,14 @@ def test_decision_bitexact_fusion(T, N, k, m_min, fusion):
     layer.close()
 
 
-@pytest.mark.parametrize("T,pattern", [(16384, "equal"), (8192, "two_values"), (300, "equal")])
+@pytest.mark.parametrize("T,pattern", [(16384, "equal"), (8192, "two_values"), (300, "equal"), (1, "equal"),
+                                       (8, "equal"), (12, "two_values"), (16, "equal"), (17, "two_values")])
 def test_decision_degenerate_scores(T, pattern):
     """Every candidate score equal (or only two distinct values): the
     threshold select meets one value held by far more keys than the select
-    stages in shared memory (and the App. B.1 tie rule decides tau)."""
+    stages in shared memory (and the App. B.1 tie rule decides tau). Up to
+    128 slots (16 tokens of top-8) the small-batch route selects by counting
+    ranks; 17 tokens is the first size on its radix select."""
     N, k = 128, 8
     z = np.zeros((T, N), np.float32)
     if pattern == "two_values":
