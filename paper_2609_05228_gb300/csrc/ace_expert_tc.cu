@@ -99,8 +99,13 @@ __device__ __forceinline__ void tma_load_2d_pair(void* smem_dst, const CUtensorM
         : "memory");
 }
 
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+// A remote arrival that orders no memory operations: for a barrier whose waiter
+// reads nothing the arriving threads wrote. An epilogue warp frees an
+// accumulator this way once tcgen05.wait::ld has completed its TMEM loads
+// (and tcgen05.fence::before_thread_sync has ordered them before the arrival),
+// without first waiting for its own global stores of output rows.
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint32_t bar_cluster) {
+    asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
 
 __device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
@@ -1095,7 +1100,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expert_pair(const __grid_consta
             epilogue_wide<EPI>(p, t, tbase, row_base, lane, gh, stg);
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive_cluster(acc_empty_leader[acc]);
+            if (lane == 0) mbar_arrive_cluster_relaxed(acc_empty_leader[acc]);
             if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
         }
     }
