@@ -442,7 +442,7 @@ def run_ours(args, rank, world, torch, dist):
             dist.all_reduce(flag, op=dist.ReduceOp.MAX)
             bad = bool(flag.item())
             dist.barrier()
-        # the reported attempt's own verdict (any rank's), null when clean
+        # why the reported attempt's own clock record was rejected (any rank's), null when clean
         clock_rejected = (why or "another rank's clocks") if bad else None
         if not bad or attempt == 1:
             break

@@ -55,7 +55,7 @@ def test_clock_records_that_disqualify_a_timed_region():
     capped = {"sm_mhz": 1850.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 30}
     assert bench.clocks_rejected(ok) is None
     assert bench.clocks_rejected(capped) is None          # power cap under load is kept
-    assert bench.clocks_rejected(None) is None            # no nvidia-smi: nothing to judge
+    assert bench.clocks_rejected(None) is None            # no nvidia-smi: nothing to reject
     for r in ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"):
         assert r in bench.clocks_rejected(dict(ok, reasons=[r, "sw_power_cap"]))
     locked = dict(ok, sm_mhz=1200.0)                      # held low with no reason: a clock lock
