@@ -668,8 +668,12 @@ def sweep(torch, args):
     """Tokens/s and speedup vs q=0 over the configurations' batch sizes and
     skip ratios: the d=2048 layer (decode batches, 4096-token prefill), or the
     large layer (decode 1/16/128, prefill 2048/8192; q from 0 to 0.625 in
-    steps of 0.125) when the workload is a large-layer one."""
+    steps of 0.125) when the workload is a large-layer one. Each point also
+    carries its retained slots, distinct retained experts and roofline
+    fractions, as the main line's points do."""
     from paper_2609_05228_gb300 import synth
+    hbm, _, _ = _peaks()
+    sust = _peak_sustained()
     if args.workload.startswith("large"):
         qs = [0.0, 0.125, 0.25, 0.375, 0.5, 0.625]
         plan = [("large_prefill", [1, 16, 128, 2048, 8192], qs)]
@@ -690,9 +694,14 @@ def sweep(torch, args):
                 ms = time_point(torch, model, x, bufs, T, q, 20, 3, flush)
                 t = float(np.median(ms))
                 base = t if q == 0.0 else base
-                pts.append({"workload": wlname, "T": T, "q": q, "us": round(t * 1e3, 2),
-                            "tokens_per_s": round(T / (t * 1e-3), 1),
-                            "speedup_vs_q0": round(base / t, 4) if base else None})
+                model.forward(x, bufs, T, q)
+                R, D = decision_stats(model, T)
+                rec = {"workload": wlname, "T": T, "q": q, "us": round(t * 1e3, 2),
+                       "tokens_per_s": round(T / (t * 1e-3), 1),
+                       "speedup_vs_q0": round(base / t, 4) if base else None,
+                       "retained_slots": R, "distinct_experts": D}
+                rec.update(roofline_point(model.spec, T, R, D, t, hbm, sust))
+                pts.append(rec)
         model.close()
     return pts
 
