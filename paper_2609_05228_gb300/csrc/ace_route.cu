@@ -1011,9 +1011,14 @@ __global__ void __launch_bounds__(kChunk) k_compact_place(int n_tokens, int k, i
 //     [8 by, 8 by + 8), one expert row per warp;
 //   phase B (last block of each token tile, by an atomic ticket): top-k,
 //     gates and c for the tile's tokens (and the decision in threshold mode);
-//   phase C (the globally last block): the App. B.1 threshold in ratio mode,
+//   phase C (the globally last block): the App. B.1 threshold in ratio mode
+//     (by counting ranks up to kRankSelectMax slots, else a radix select),
 //     the decision, and the compaction of retained slots.
-// Tickets are reset by the block that consumed them. No block waits on another.
+// With one token tile (T <= 8) phases B and C run in the same block, which
+// passes phase B's results to phase C in shared memory. Tickets are reset by
+// the block that consumed them. No block waits on another. The kernel lets
+// its dependent launch at entry; that kernel reads nothing of this one before
+// its own griddepcontrol.wait.
 // --------------------------------------------------------------------------
 constexpr int kFuseTok = 8;
 constexpr int kFuseWarps = 8;
