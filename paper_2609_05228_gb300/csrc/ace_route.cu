@@ -68,15 +68,64 @@ __device__ __forceinline__ void rmsnorm_row(const T* __restrict__ xr, const T* _
     }
 }
 
-// NV = 16-byte vectors per lane, sized to the row so that short rows hold
-// fewer registers and more rows (more loads in flight) fit on an SM.
+__device__ __forceinline__ void cp_async16_row(uint32_t dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+
+// A warp per row. The row comes into shared memory by cp.async (d x sizeof(T)
+// bytes per warp of dynamic shared memory), so no registers are held per load
+// and more rows are in flight per SM; each lane reads back only its own
+// 16-byte chunks (lane + 32 i), in the order and with the arithmetic of
+// rmsnorm_row, so the bits are the same. NV bounds the chunks per lane.
 template <typename T, int NV>
 __global__ void __launch_bounds__(256) k_rmsnorm(const T* __restrict__ x, const T* __restrict__ gamma,
                                                  T* __restrict__ h, int n_tokens, int d, float rms_eps) {
+    extern __shared__ __align__(16) unsigned char rn_rows[];      // [warps][d] staged rows
     pdl_wait();
-    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    if (warp >= n_tokens) return;
-    rmsnorm_row<T, NV>(x + (size_t)warp * d, gamma, h + (size_t)warp * d, d, rms_eps, threadIdx.x & 31);
+    const int wib = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int row = blockIdx.x * (blockDim.x >> 5) + wib;
+    if (row >= n_tokens) return;
+    constexpr int V = Vec16<T>::N;
+    const int nvec = d / V;
+    const uint4* xv = reinterpret_cast<const uint4*>(x + (size_t)row * d);
+    const uint4* rs = reinterpret_cast<const uint4*>(rn_rows + (size_t)wib * d * sizeof(T));
+    const uint32_t rs_addr = (uint32_t)__cvta_generic_to_shared(rs);
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        const int c = lane + 32 * i;
+        if (c < nvec) cp_async16_row(rs_addr + (uint32_t)c * 16u, xv + c);
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        const int c = lane + 32 * i;
+        if (c < nvec) {
+            float f[V];
+            Vec16<T>::to_float(rs[c], f);
+            float part = 0.f;
+#pragma unroll
+            for (int j = 0; j < V; ++j) part = fmaf(f[j], f[j], part);
+            ss += part;
+        }
+    }
+    ss = warp_sum(ss);
+    const float inv = 1.0f / sqrtf(ss / (float)d + rms_eps);
+    const uint4* gv = reinterpret_cast<const uint4*>(gamma);
+    uint4* hv = reinterpret_cast<uint4*>(h + (size_t)row * d);
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        const int c = lane + 32 * i;
+        if (c < nvec) {
+            float f[V], gm[V];
+            Vec16<T>::to_float(rs[c], f);
+            Vec16<T>::to_float(gv[c], gm);
+            T o[V];
+#pragma unroll
+            for (int j = 0; j < V; ++j) o[j] = from_f32<T>(f[j] * inv * gm[j]);
+            hv[c] = *reinterpret_cast<const uint4*>(o);
+        }
+    }
 }
 
 // --------------------------------------------------------------------------
@@ -1562,9 +1611,10 @@ cudaError_t launch_rmsnorm_t(const ace_layer* L, const void* x, int T, cudaStrea
     const E* g = static_cast<const E*>(L->gamma);
     E* h = static_cast<E*>(L->ws.h);
     const float eps = L->desc.rms_eps;
-    if (nv <= 4) return launch_pdl(k_rmsnorm<E, 4>, dim3(blocks), dim3(256), 0, s, xt, g, h, T, d, eps);
-    if (nv <= 8) return launch_pdl(k_rmsnorm<E, 8>, dim3(blocks), dim3(256), 0, s, xt, g, h, T, d, eps);
-    return launch_pdl(k_rmsnorm<E, kNormVec>, dim3(blocks), dim3(256), 0, s, xt, g, h, T, d, eps);
+    const size_t sm = (size_t)8 * d * sizeof(E);      // one staged row per warp
+    if (nv <= 4) return launch_pdl(k_rmsnorm<E, 4>, dim3(blocks), dim3(256), sm, s, xt, g, h, T, d, eps);
+    if (nv <= 8) return launch_pdl(k_rmsnorm<E, 8>, dim3(blocks), dim3(256), sm, s, xt, g, h, T, d, eps);
+    return launch_pdl(k_rmsnorm<E, kNormVec>, dim3(blocks), dim3(256), sm, s, xt, g, h, T, d, eps);
 }
 
 cudaError_t launch_rmsnorm(const ace_layer* L, const void* x, int T, cudaStream_t s) {
@@ -1644,6 +1694,13 @@ int route_launch_count(const ace_layer* L, int T, ace_skip_ctl ctl) {
 cudaError_t route_init(const ace_layer* L) {
     cudaError_t e = set_router_attrs<__nv_bfloat16>(router_smem(L));
     if (e != cudaSuccess) return e;
+    // k_rmsnorm stages one row per warp: 8 x d x element bytes
+    const int rn = 8 * L->desc.hidden * (int)L->elem;
+    const void* norms[] = {(const void*)k_rmsnorm<__nv_bfloat16, 4>, (const void*)k_rmsnorm<__nv_bfloat16, 8>,
+                           (const void*)k_rmsnorm<__nv_bfloat16, kNormVec>, (const void*)k_rmsnorm<float, 4>,
+                           (const void*)k_rmsnorm<float, 8>, (const void*)k_rmsnorm<float, kNormVec>};
+    for (const void* kf : norms)
+        if ((e = raise_smem_limit(kf, rn)) != cudaSuccess) return e;
     e = set_router_attrs<float>(router_smem(L));
     if (e != cudaSuccess) return e;
     const int sm = (int)fused_smem_bytes(L, kSmallT);
