@@ -113,6 +113,42 @@ def test_tau_ties_worked_example(fp32):
             assert tau == ftype(float(want))
 
 
+@pytest.mark.parametrize("fp32", [False, True])
+def test_tau_bruteforce_heavy_ties(fp32):
+    """App. B.1 against an enumeration: every count a threshold can realise
+    over the candidates is #{c < u} or #{c <= u} for some candidate value u;
+    the mapping takes the one closest to m_q (the lower on a tie), with tau
+    the largest threshold realising a count below or at m_q (the next
+    candidate value) or the smallest realising one above it (just above the
+    last counted value). Scores come from a small set, so ties are common."""
+    ftype = np.float32 if fp32 else np.float64
+    fn = O.tau_from_ratio_fp32 if fp32 else O.tau_from_ratio
+    rng = np.random.Generator(np.random.PCG64(77))
+    values = np.array([0.05, 0.2, 0.2, 0.35, 0.5, 0.5, 0.5, 0.9], dtype=ftype)
+    for trial in range(600):
+        n = int(rng.integers(1, 41))
+        c = rng.choice(values, size=n).astype(ftype)
+        prot = rng.random(n) < 0.2
+        q = float(rng.random())
+        cand = np.sort(c[~prot])
+        nc = cand.size
+        m = min(max(int(math.floor(q * n + 0.5)), 0), nc)
+        tau, m_q, cnt = fn(c, prot, q)
+        assert m_q == m, (trial, m_q, m)
+        if m == 0:
+            assert tau == 0 and cnt == 0
+            continue
+        if m == nc:
+            assert math.isinf(tau) and cnt == nc
+            continue
+        counts = sorted({int(np.sum(cand < u)) for u in cand} | {int(np.sum(cand <= u)) for u in cand})
+        best = min(counts, key=lambda x: (abs(x - m), x))
+        want = cand[best] if best <= m else np.nextafter(cand[best - 1], ftype(np.inf))
+        assert cnt == best, (trial, cnt, best, m)
+        assert ftype(tau) == want, (trial, tau, want)
+        assert int(np.sum(cand < ftype(tau))) == best
+
+
 def test_tables_worked_example():
     ex = _load("tables_worked.json")
     gs = ex["gsp"]
